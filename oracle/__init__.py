@@ -1,0 +1,192 @@
+"""fp64 CPU oracle for the QUASAR reconstruction (test infrastructure only).
+
+Only ``tests/``, ``__graft_entry__.smoke()`` and the CPU-baseline leg of
+``bench.py`` may import this package.  The CUDA library never does, and this
+package never imports the CUDA library: the two share no code.
+
+The arithmetic lives in ``quasar_oracle.c`` (plain C, fp64, OpenMP over
+groups); this module only compiles it with gcc and marshals numpy arrays.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import subprocess
+import threading
+
+import numpy as np
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+_SRC = os.path.join(_HERE, "quasar_oracle.c")
+_BUILD = os.path.join(_HERE, "_build")
+_LIB_PATH = os.path.join(_BUILD, "libquasar_oracle.so")
+_lib = None
+_lock = threading.Lock()
+
+
+def build(force: bool = False) -> str:
+    """Compile the oracle with gcc (no FMA contraction, so x86 and Arm agree)."""
+    os.makedirs(_BUILD, exist_ok=True)
+    if (not force and os.path.exists(_LIB_PATH)
+            and os.path.getmtime(_LIB_PATH) >= os.path.getmtime(_SRC)):
+        return _LIB_PATH
+    tmp = _LIB_PATH + f".tmp{os.getpid()}"
+    cmd = ["gcc", "-O2", "-std=c11", "-fPIC", "-shared", "-fopenmp",
+           "-ffp-contract=off", "-fno-fast-math", _SRC, "-o", tmp, "-lm"]
+    subprocess.run(cmd, check=True)
+    os.replace(tmp, _LIB_PATH)
+    return _LIB_PATH
+
+
+def _load():
+    global _lib
+    with _lock:
+        if _lib is not None:
+            return _lib
+        lib = ctypes.CDLL(build())
+        P = ctypes.c_void_p
+        i64, i32, f32, f64 = ctypes.c_int64, ctypes.c_int, ctypes.c_float, ctypes.c_double
+        lib.qo_ema.argtypes = [P, P, i64, f32, P]
+        lib.qo_ema.restype = None
+        lib.qo_recon_int.argtypes = [P, P, i64, i32, i32, P, i32] + [P] * 11
+        lib.qo_recon_int.restype = i32
+        lib.qo_refit_int.argtypes = [P, P, P, i32, i32, f32, P, P]
+        lib.qo_refit_int.restype = f64
+        lib.qo_codes_int.argtypes = [P, i32, i32, f32, P, P]
+        lib.qo_codes_int.restype = i32
+        lib.qo_tensor_scale.argtypes = [P, i64, P, P]
+        lib.qo_tensor_scale.restype = None
+        lib.qo_recon_nvfp4.argtypes = [P, P, i64, f32, P, i32] + [P] * 10
+        lib.qo_recon_nvfp4.restype = i32
+        lib.qo_e2m1_round.argtypes = [f64]
+        lib.qo_e2m1_round.restype = i32
+        lib.qo_e4m3_round.argtypes = [f64]
+        lib.qo_e4m3_round.restype = i32
+        lib.qo_e4m3_value.argtypes = [i32]
+        lib.qo_e4m3_value.restype = f64
+        lib.qo_set_threads.argtypes = [i32]
+        lib.qo_set_threads.restype = None
+        lib.qo_get_threads.argtypes = []
+        lib.qo_get_threads.restype = i32
+        _lib = lib
+        return lib
+
+
+def _ptr(a):
+    return None if a is None else ctypes.c_void_p(a.ctypes.data)
+
+
+def _c(a, dtype):
+    return np.ascontiguousarray(a, dtype=dtype)
+
+
+def set_threads(n: int) -> None:
+    _load().qo_set_threads(int(n))
+
+
+def get_threads() -> int:
+    return int(_load().qo_get_threads())
+
+
+def ema(v, g, beta2: float) -> np.ndarray:
+    """Saliency EMA: fl32(beta2*v + (1-beta2)*g^2) in fp64; g=None: no update."""
+    v = _c(v, np.float32).ravel()
+    gg = None if g is None else _c(g, np.float32).ravel()
+    out = np.empty_like(v)
+    _load().qo_ema(_ptr(v), _ptr(gg), v.size, ctypes.c_float(beta2), _ptr(out))
+    return out
+
+
+def recon_int(w, h, group_size: int, bits: int, clip) -> dict:
+    """Algorithm 1 with asymmetric integer codes, every group of a flat tensor."""
+    w = _c(w, np.float32).ravel()
+    h = _c(h, np.float32).ravel()
+    clip = _c(clip, np.float32).ravel()
+    G, K = int(group_size), clip.size
+    assert w.size == h.size and w.size % G == 0
+    n = w.size // G
+    out = dict(
+        idx=np.empty(n, np.int32), a=np.empty(n), b=np.empty(n),
+        codes=np.empty(w.size, np.uint8), r=np.empty(w.size), err=np.empty(n),
+        cand_err=np.empty(n * K), cand_a=np.empty(n * K), cand_b=np.empty(n * K),
+        m_round=np.empty(n), m_tie=np.empty(n))
+    rc = _load().qo_recon_int(
+        _ptr(w), _ptr(h), n, G, int(bits), _ptr(clip), K,
+        _ptr(out["idx"]), _ptr(out["a"]), _ptr(out["b"]), _ptr(out["codes"]),
+        _ptr(out["r"]), _ptr(out["err"]), _ptr(out["cand_err"]), _ptr(out["cand_a"]),
+        _ptr(out["cand_b"]), _ptr(out["m_round"]), _ptr(out["m_tie"]))
+    if rc != 0:
+        raise ValueError("qo_recon_int: bad arguments")
+    for key in ("cand_err", "cand_a", "cand_b"):
+        out[key] = out[key].reshape(n, K)
+    return out
+
+
+def codes_int(w_group, bits: int, f: float):
+    """Eq. 1 codes and per-element margins of one candidate for one group."""
+    w = _c(w_group, np.float32).ravel()
+    q = np.empty(w.size, np.uint8)
+    m = np.empty(w.size)
+    _load().qo_codes_int(_ptr(w), w.size, int(bits), ctypes.c_float(f), _ptr(q), _ptr(m))
+    return q, m
+
+
+def refit_int(w_group, h_group, codes, bits: int, f: float):
+    """Eq. 4 fit and Eq. 3 error for given codes; returns (s, z, err)."""
+    w = _c(w_group, np.float32).ravel()
+    h = _c(h_group, np.float32).ravel()
+    q = _c(codes, np.uint8).ravel()
+    s = ctypes.c_double()
+    z = ctypes.c_double()
+    e = _load().qo_refit_int(_ptr(w), _ptr(h), _ptr(q), w.size, int(bits), ctypes.c_float(f),
+                             ctypes.byref(s), ctypes.byref(z))
+    return s.value, z.value, float(e)
+
+
+def tensor_scale(w):
+    """NVFP4 per-tensor scale: (amax, s_T) as fp32 values."""
+    w = _c(w, np.float32).ravel()
+    amax = ctypes.c_float()
+    sT = ctypes.c_float()
+    _load().qo_tensor_scale(_ptr(w), w.size, ctypes.byref(amax), ctypes.byref(sT))
+    return np.float32(amax.value), np.float32(sT.value)
+
+
+def recon_nvfp4(w, h, s_T: float, clip) -> dict:
+    """NVFP4 QUASAR (Sec. 4.2) over every 16-element block of a flat tensor."""
+    w = _c(w, np.float32).ravel()
+    h = _c(h, np.float32).ravel()
+    clip = _c(clip, np.float32).ravel()
+    K = clip.size
+    assert w.size == h.size and w.size % 16 == 0
+    n = w.size // 16
+    out = dict(
+        idx=np.empty(n, np.int32), scale=np.empty(n, np.uint8), codes=np.empty(w.size, np.uint8),
+        r=np.empty(w.size), err=np.empty(n), cand_err=np.empty(n * K),
+        cand_scale=np.empty(n * K, np.uint8), m_round=np.empty(n), m_scale=np.empty(n),
+        m_tie=np.empty(n))
+    rc = _load().qo_recon_nvfp4(
+        _ptr(w), _ptr(h), n, ctypes.c_float(s_T), _ptr(clip), K,
+        _ptr(out["idx"]), _ptr(out["scale"]), _ptr(out["codes"]), _ptr(out["r"]),
+        _ptr(out["err"]), _ptr(out["cand_err"]), _ptr(out["cand_scale"]),
+        _ptr(out["m_round"]), _ptr(out["m_scale"]), _ptr(out["m_tie"]))
+    if rc != 0:
+        raise ValueError("qo_recon_nvfp4: bad arguments")
+    out["cand_err"] = out["cand_err"].reshape(n, K)
+    out["cand_scale"] = out["cand_scale"].reshape(n, K)
+    return out
+
+
+def e2m1_round(y: float) -> int:
+    return int(_load().qo_e2m1_round(float(y)))
+
+
+def e4m3_round(x: float) -> int:
+    return int(_load().qo_e4m3_round(float(x)))
+
+
+def e4m3_value(bits: int) -> float:
+    return float(_load().qo_e4m3_value(int(bits)))
+
+
+E2M1_MAGNITUDES = (0.0, 0.5, 1.0, 1.5, 2.0, 3.0, 4.0, 6.0)

@@ -1,0 +1,530 @@
+/*
+ * QUASAR reconstruction oracle: plain, slow, fp64 CPU code.
+ *
+ * TEST INFRASTRUCTURE ONLY.  Nothing in the product path (the CUDA library
+ * and its Python binding) includes, links or calls this file.  Only the
+ * tests, the smoke check and the CPU-baseline leg of the benchmark use it.
+ * It shares no code, header or table with the CUDA kernels.
+ *
+ * What it computes (paper: "QUASAR: Lowering the Loss Floor of
+ * Quantization-Aware Training with Loss-Aware Reconstruction"):
+ *
+ *   qo_ema          saliency EMA of squared gradients (Sec. 4.1.1: the Adam
+ *                   second moment as diagonal-Fisher saliency; App. A.2: an
+ *                   explicitly kept EMA of squared gradients).
+ *   qo_recon_int    Algorithm 1 on asymmetric integer codes: group range,
+ *                   per-candidate code assignment (Eq. 1), saliency-weighted
+ *                   least-squares dequantizer (Eq. 4), weighted error by
+ *                   direct summation (Eq. 3), argmin over the clip grid.
+ *   qo_refit_int    Eq. 4 + Eq. 3 for a caller-given code vector (checker).
+ *   qo_codes_int    Eq. 1 codes of one candidate range (checker).
+ *   qo_tensor_scale NVFP4 per-tensor FP32 scale from the tensor absmax
+ *                   (Sec. 4.2).
+ *   qo_recon_nvfp4  Sec. 4.2: per 16-element block, search scales -> E2M1
+ *                   codes, fit the FP8 (E4M3) dequantization scale under
+ *                   Eq. 3, keep the candidate with the lowest error.
+ *   qo_e4m3_round / qo_e2m1_round   the two codecs, by enumeration of the
+ *                   representable values.
+ *
+ * Everything is fp64 except values the method stores (the EMA state is
+ * rounded to fp32 because it is fp32 state; the NVFP4 tensor scale is an FP32
+ * number by the format's definition).  No FMA contraction is relied upon:
+ * build with -ffp-contract=off so x86 and Arm give identical bits.
+ *
+ * Readings of the paper taken where it is silent (listed with reasons in the
+ * design notes):
+ *   R1  rounding in Eq. 1 is round-half-to-even;
+ *   R3  the saliency is the post-update EMA, no bias correction;
+ *   R4  Eq. 4 as printed (no ridge term);
+ *   R6  argmin ties go to the lowest candidate index;
+ *   D1  zero-range group: codes 0, a = 0, b = w_0, r = w, error 0, index 0;
+ *   D2  all saliencies zero: the group is fitted with h = 1 everywhere;
+ *   D3  all h > 0 elements share one code: a = the candidate's grid step,
+ *       b = weighted mean - a*code, error = sum h (w - weighted mean)^2;
+ *   N1  s_T = fl32(amax / (6*448)); amax = 0 gives s_T = 1;
+ *   N2  codes come from the unquantized search scale f*amax_b/6;
+ *   N3  the FP8 scale is the E4M3 value nearest a* / s_T (RNE, saturating);
+ *   N4  zero block: all zero; sum h q^2 = 0: e = E4M3(sigma/s_T), error =
+ *       sum h w^2; all saliencies zero: h = 1;
+ *   N5  E2M1 rounding is nearest with ties to the even code; magnitude 0 is
+ *       stored as +0;
+ *   N6  the candidate error uses the E4M3-rounded scale.
+ */
+#include <math.h>
+#include <stdint.h>
+#include <stdlib.h>
+#include <string.h>
+
+#ifdef _OPENMP
+#include <omp.h>
+#endif
+
+#define QO_MAX_K 64
+
+/* Thread control for the OpenMP loops over groups (1 if built without it). */
+void qo_set_threads(int n)
+{
+#ifdef _OPENMP
+    if (n > 0) omp_set_num_threads(n);
+#else
+    (void)n;
+#endif
+}
+
+int qo_get_threads(void)
+{
+#ifdef _OPENMP
+    return omp_get_max_threads();
+#else
+    return 1;
+#endif
+}
+
+/* ------------------------------------------------------------------------ */
+/* Saliency EMA.                                                            */
+/* ------------------------------------------------------------------------ */
+
+/* v_out[i] = fl32(beta2*v[i] + (1-beta2)*g[i]^2), evaluated in fp64.
+ * g == NULL means no update (v_out = v).  v_out may equal v. */
+void qo_ema(const float* v, const float* g, int64_t n, float beta2, float* v_out)
+{
+    const double b2 = (double)beta2;
+    const double c1 = 1.0 - b2;
+    for (int64_t i = 0; i < n; ++i) {
+        if (g) {
+            const double gi = (double)g[i];
+            v_out[i] = (float)(b2 * (double)v[i] + c1 * gi * gi);
+        } else {
+            v_out[i] = v[i];
+        }
+    }
+}
+
+/* ------------------------------------------------------------------------ */
+/* Integer path (Sec. 3.1 Eq. 1, Sec. 4.1.2 Eq. 4, Eq. 3, Algorithm 1).      */
+/* ------------------------------------------------------------------------ */
+
+/* Saliency of one group with rule D2 applied: if every h is zero, h = 1. */
+static void group_saliency(const float* h, int G, double* hd)
+{
+    double sum = 0.0;
+    for (int i = 0; i < G; ++i) sum += (double)h[i];
+    for (int i = 0; i < G; ++i) hd[i] = (sum == 0.0) ? 1.0 : (double)h[i];
+}
+
+/* Eq. 1 on the range [c - f*rho, c + f*rho]:
+ *   z = c - f*rho, s = 2*f*rho/qmax, t = (w - z)/s,
+ *   q = clamp(round_half_even(t), 0, qmax).
+ * margin[i] (optional): distance of t to the nearest decision boundary
+ * j + 1/2 (j = 0..qmax-1), divided by qmax, i.e. the distance of w to the
+ * boundary as a fraction of the clipping range 2*f*rho. */
+static void int_codes(const float* w, int G, double c, double rho, double f, int qmax,
+                      uint8_t* q, double* margin)
+{
+    const double z = c - f * rho;
+    const double s = 2.0 * f * rho / (double)qmax;
+    for (int i = 0; i < G; ++i) {
+        const double t = ((double)w[i] - z) / s;
+        double k = nearbyint(t); /* default rounding mode: half to even */
+        if (k < 0.0) k = 0.0;
+        if (k > (double)qmax) k = (double)qmax;
+        q[i] = (uint8_t)k;
+        if (margin) {
+            double j = floor(t);
+            if (j < 0.0) j = 0.0;
+            if (j > (double)(qmax - 1)) j = (double)(qmax - 1);
+            margin[i] = fabs(t - (j + 0.5)) / (double)qmax;
+        }
+    }
+}
+
+/* Eq. 4 for fixed codes q and saliency hd (rule D2 already applied), then
+ * Eq. 3 by direct summation.  step is the candidate's grid step, used only by
+ * rule D3.  Returns the weighted error; writes s*, z*. */
+static double wls_fit(const float* w, const double* hd, const uint8_t* q, int G,
+                      double step, double* s_out, double* z_out)
+{
+    double sh = 0.0, shq = 0.0, shw = 0.0;
+    for (int i = 0; i < G; ++i) {
+        sh += hd[i];
+        shq += hd[i] * (double)q[i];
+        shw += hd[i] * (double)w[i];
+    }
+    const double qbar = shq / sh;
+    const double wbar = shw / sh;
+
+    /* D3: exact test on the codes of the elements that carry weight. */
+    int first = -1, one_code = 1;
+    for (int i = 0; i < G; ++i) {
+        if (hd[i] > 0.0) {
+            if (first < 0) first = q[i];
+            else if (q[i] != first) one_code = 0;
+        }
+    }
+
+    double s, z;
+    if (one_code) {
+        s = step;
+        z = wbar - step * (double)first;
+    } else {
+        double num = 0.0, den = 0.0;
+        for (int i = 0; i < G; ++i) {
+            const double dq = (double)q[i] - qbar;
+            num += hd[i] * dq * ((double)w[i] - wbar);
+            den += hd[i] * dq * dq;
+        }
+        s = num / den;
+        z = wbar - s * qbar;
+    }
+
+    double err = 0.0;
+    for (int i = 0; i < G; ++i) {
+        const double d = s * (double)q[i] + z - (double)w[i];
+        err += hd[i] * d * d;
+    }
+    *s_out = s;
+    *z_out = z;
+    return err;
+}
+
+/* Codes of one candidate for one group (for the parity checker).  Returns 0
+ * for a zero-range group (all codes 0, margins +inf). */
+int qo_codes_int(const float* w, int G, int bits, float f, uint8_t* q, double* margin)
+{
+    const int qmax = (1 << bits) - 1;
+    double mn = (double)w[0], mx = (double)w[0];
+    for (int i = 1; i < G; ++i) {
+        if ((double)w[i] < mn) mn = (double)w[i];
+        if ((double)w[i] > mx) mx = (double)w[i];
+    }
+    if (mx == mn) {
+        for (int i = 0; i < G; ++i) {
+            q[i] = 0;
+            if (margin) margin[i] = HUGE_VAL;
+        }
+        return 0;
+    }
+    const double c = 0.5 * (mn + mx), rho = 0.5 * (mx - mn);
+    int_codes(w, G, c, rho, (double)f, qmax, q, margin);
+    return 1;
+}
+
+/* Eq. 4 + Eq. 3 for caller-given codes (rule D2 applied to h; rule D3 uses
+ * the grid step of candidate f).  Returns the weighted error. */
+double qo_refit_int(const float* w, const float* h, const uint8_t* q, int G, int bits, float f,
+                    double* s_out, double* z_out)
+{
+    const int qmax = (1 << bits) - 1;
+    double mn = (double)w[0], mx = (double)w[0];
+    for (int i = 1; i < G; ++i) {
+        if ((double)w[i] < mn) mn = (double)w[i];
+        if ((double)w[i] > mx) mx = (double)w[i];
+    }
+    double* hd = (double*)malloc(sizeof(double) * (size_t)G);
+    group_saliency(h, G, hd);
+    const double step = (mx - mn) * (double)f / (double)qmax;
+    const double e = wls_fit(w, hd, q, G, step, s_out, z_out);
+    free(hd);
+    return e;
+}
+
+/* Algorithm 1 over n_groups consecutive groups of G elements.
+ *
+ * Inputs: w, h (fp32, n_groups*G), bits in [1,8], clip[K] (factors in (0,1],
+ * list order).  Every output pointer may be NULL.
+ *   idx[n_groups]      chosen candidate (lowest index on equal error)
+ *   a[n_groups], b[n_groups]   fitted s*, z* of the chosen candidate
+ *   codes[n_groups*G]  chosen codes
+ *   r[n_groups*G]      a*q + b in fp64
+ *   err[n_groups]      weighted error of the chosen candidate
+ *   cand_err/cand_a/cand_b[n_groups*K]   the same for every candidate
+ *   m_round[n_groups]  min over candidates and elements of the code margin
+ *   m_tie[n_groups]    (second-best error - best error)/best error, where
+ *                      second-best ranges over candidates whose code vector
+ *                      differs from the winner's (+inf if none)
+ * Returns 0 on success, -1 on bad arguments. */
+int qo_recon_int(const float* w, const float* h, int64_t n_groups, int G, int bits,
+                 const float* clip, int K,
+                 int32_t* idx, double* a, double* b, uint8_t* codes, double* r, double* err,
+                 double* cand_err, double* cand_a, double* cand_b,
+                 double* m_round, double* m_tie)
+{
+    if (G < 1 || bits < 1 || bits > 8 || K < 1 || K > QO_MAX_K || n_groups < 0) return -1;
+    const int qmax = (1 << bits) - 1;
+
+#pragma omp parallel for schedule(dynamic, 64)
+    for (int64_t grp = 0; grp < n_groups; ++grp) {
+        const float* wg = w + grp * G;
+        const float* hg = h + grp * G;
+        uint8_t* qk = (uint8_t*)malloc((size_t)K * (size_t)G);
+        double* hd = (double*)malloc(sizeof(double) * (size_t)G);
+        double* mg = (double*)malloc(sizeof(double) * (size_t)G);
+        double ek[QO_MAX_K], sk[QO_MAX_K], zk[QO_MAX_K];
+
+        double mn = (double)wg[0], mx = (double)wg[0];
+        for (int i = 1; i < G; ++i) {
+            if ((double)wg[i] < mn) mn = (double)wg[i];
+            if ((double)wg[i] > mx) mx = (double)wg[i];
+        }
+
+        int best = 0;
+        double mround = HUGE_VAL, mtie = HUGE_VAL;
+
+        if (mx == mn) {
+            /* D1: zero range. */
+            memset(qk, 0, (size_t)K * (size_t)G);
+            for (int k = 0; k < K; ++k) {
+                ek[k] = 0.0;
+                sk[k] = 0.0;
+                zk[k] = (double)wg[0];
+            }
+        } else {
+            const double c = 0.5 * (mn + mx);
+            const double rho = 0.5 * (mx - mn);
+            group_saliency(hg, G, hd);
+            for (int k = 0; k < K; ++k) {
+                const double f = (double)clip[k];
+                uint8_t* q = qk + (size_t)k * G;
+                int_codes(wg, G, c, rho, f, qmax, q, mg);
+                for (int i = 0; i < G; ++i)
+                    if (mg[i] < mround) mround = mg[i];
+                const double step = 2.0 * f * rho / (double)qmax;
+                ek[k] = wls_fit(wg, hd, q, G, step, &sk[k], &zk[k]);
+            }
+            for (int k = 1; k < K; ++k)
+                if (ek[k] < ek[best]) best = k;
+            double second = HUGE_VAL;
+            for (int k = 0; k < K; ++k) {
+                if (k == best) continue;
+                if (memcmp(qk + (size_t)k * G, qk + (size_t)best * G, (size_t)G) == 0) continue;
+                if (ek[k] < second) second = ek[k];
+            }
+            if (second < HUGE_VAL) {
+                const double denom = ek[best] > 1e-300 ? ek[best] : 1e-300;
+                mtie = (second - ek[best]) / denom;
+            }
+        }
+
+        if (idx) idx[grp] = best;
+        if (a) a[grp] = sk[best];
+        if (b) b[grp] = zk[best];
+        if (err) err[grp] = ek[best];
+        if (m_round) m_round[grp] = mround;
+        if (m_tie) m_tie[grp] = mtie;
+        for (int k = 0; k < K; ++k) {
+            if (cand_err) cand_err[grp * K + k] = ek[k];
+            if (cand_a) cand_a[grp * K + k] = sk[k];
+            if (cand_b) cand_b[grp * K + k] = zk[k];
+        }
+        const uint8_t* qb = qk + (size_t)best * G;
+        for (int i = 0; i < G; ++i) {
+            if (codes) codes[grp * G + i] = qb[i];
+            if (r) r[grp * G + i] = (mx == mn) ? (double)wg[i] : sk[best] * (double)qb[i] + zk[best];
+        }
+        free(qk);
+        free(hd);
+        free(mg);
+    }
+    return 0;
+}
+
+/* ------------------------------------------------------------------------ */
+/* NVFP4 path (Sec. 4.2).                                                   */
+/* ------------------------------------------------------------------------ */
+
+/* E2M1 magnitudes: 1 sign, 2 exponent, 1 mantissa bit (Sec. 4.2); code index
+ * m = 0..7, value 0, 0.5, 1, 1.5, 2, 3, 4, 6. */
+static const double e2m1_mag[8] = {0.0, 0.5, 1.0, 1.5, 2.0, 3.0, 4.0, 6.0};
+
+/* Nearest E2M1 magnitude to y >= 0, saturating at 6, ties to the even code
+ * index (even mantissa).  Returns the code index 0..7. */
+int qo_e2m1_round(double y)
+{
+    if (!(y < 6.0)) return 7;
+    int best = 0;
+    double bd = fabs(y - e2m1_mag[0]);
+    for (int m = 1; m < 8; ++m) {
+        const double d = fabs(y - e2m1_mag[m]);
+        if (d < bd || (d == bd && (m % 2) == 0)) {
+            best = m;
+            bd = d;
+        }
+    }
+    return best;
+}
+
+/* Value of a non-negative E4M3 (OCP FP8 e4m3fn) bit pattern 0x00..0x7E:
+ * exponent bias 7; exponent field 0 is subnormal (m/8 * 2^-6); 0x7F is NaN. */
+double qo_e4m3_value(int bits)
+{
+    const int e = (bits >> 3) & 0xF, m = bits & 7;
+    if (e == 0) return ldexp((double)m / 8.0, -6);
+    return ldexp(1.0 + (double)m / 8.0, e - 7);
+}
+
+/* Nearest non-negative finite E4M3 value to x >= 0: round to nearest, ties to
+ * the even mantissa, values above 448 saturate to 448 (satfinite).  Returns
+ * the bit pattern (0x00..0x7E). */
+int qo_e4m3_round(double x)
+{
+    if (!(x > 0.0)) return 0;
+    int best = 0;
+    double bd = fabs(x - qo_e4m3_value(0));
+    for (int c = 1; c <= 0x7E; ++c) {
+        const double d = fabs(x - qo_e4m3_value(c));
+        if (d < bd || (d == bd && (c % 2) == 0)) {
+            best = c;
+            bd = d;
+        }
+    }
+    return best;
+}
+
+/* Relative distance of x > 0 to the nearest decision boundary of E4M3
+ * rounding (midpoint between consecutive finite values; none above 448). */
+static double e4m3_margin(double x)
+{
+    double best = HUGE_VAL;
+    for (int c = 0; c < 0x7E; ++c) {
+        const double mid = 0.5 * (qo_e4m3_value(c) + qo_e4m3_value(c + 1));
+        const double d = fabs(x - mid) / mid;
+        if (d < best) best = d;
+    }
+    return best;
+}
+
+/* Relative distance of y >= 0 to the nearest E2M1 decision boundary. */
+static double e2m1_margin(double y)
+{
+    double best = HUGE_VAL;
+    for (int m = 0; m < 7; ++m) {
+        const double mid = 0.5 * (e2m1_mag[m] + e2m1_mag[m + 1]);
+        const double d = fabs(y - mid) / mid;
+        if (d < best) best = d;
+    }
+    return best;
+}
+
+/* Per-tensor scale from the tensor absmax (Sec. 4.2; reading N1):
+ * amax = max |w|, s_T = fl32(amax / (6*448)), s_T = 1 when amax = 0. */
+void qo_tensor_scale(const float* w, int64_t n, float* amax_out, float* s_T_out)
+{
+    double amax = 0.0;
+    for (int64_t i = 0; i < n; ++i) {
+        const double x = fabs((double)w[i]);
+        if (x > amax) amax = x;
+    }
+    if (amax_out) *amax_out = (float)amax;
+    if (s_T_out) *s_T_out = (amax == 0.0) ? 1.0f : (float)(amax / 2688.0);
+}
+
+/* NVFP4 QUASAR over n_blocks consecutive 16-element blocks (Sec. 4.2).
+ *
+ * For candidate f: sigma = f*amax_b/6, |q| = E2M1(min(|w|/sigma, 6)) with
+ * the sign of w; a* = sum h q w / sum h q^2 (symmetric weighted LS);
+ * e = E4M3(a* / s_T); error = sum h (s_T*e*q - w)^2; argmin over candidates.
+ * Outputs (each may be NULL):
+ *   idx[n_blocks], scale_bits[n_blocks] (E4M3 pattern of e),
+ *   codes[n_blocks*16] (sign<<3 | magnitude index; magnitude 0 stored as 0),
+ *   r[n_blocks*16] = s_T*e*q in fp64, err[n_blocks],
+ *   cand_err[n_blocks*K], cand_scale[n_blocks*K] (E4M3 patterns),
+ *   m_round (min relative distance of |w|/sigma to an E2M1 boundary),
+ *   m_scale (min relative distance of a* / s_T to an E4M3 boundary),
+ *   m_tie   (as in qo_recon_int; candidates with identical codes and scale
+ *            are not counted as competitors). */
+int qo_recon_nvfp4(const float* w, const float* h, int64_t n_blocks, float s_T,
+                   const float* clip, int K,
+                   int32_t* idx, uint8_t* scale_bits, uint8_t* codes, double* r, double* err,
+                   double* cand_err, uint8_t* cand_scale,
+                   double* m_round, double* m_scale, double* m_tie)
+{
+    if (K < 1 || K > QO_MAX_K || n_blocks < 0 || !(s_T > 0.0f)) return -1;
+    const double sT = (double)s_T;
+
+#pragma omp parallel for schedule(dynamic, 256)
+    for (int64_t blk = 0; blk < n_blocks; ++blk) {
+        const float* wb = w + blk * 16;
+        const float* hb = h + blk * 16;
+        double hd[16];
+        uint8_t qk[QO_MAX_K][16];
+        double ek[QO_MAX_K];
+        int sk[QO_MAX_K];
+
+        double amax_b = 0.0;
+        for (int i = 0; i < 16; ++i) {
+            const double x = fabs((double)wb[i]);
+            if (x > amax_b) amax_b = x;
+        }
+        group_saliency(hb, 16, hd);
+
+        int best = 0;
+        double mround = HUGE_VAL, mscale = HUGE_VAL, mtie = HUGE_VAL;
+        if (amax_b == 0.0) {
+            /* N4: zero block. */
+            for (int k = 0; k < K; ++k) {
+                memset(qk[k], 0, 16);
+                ek[k] = 0.0;
+                sk[k] = 0;
+            }
+        } else {
+            for (int k = 0; k < K; ++k) {
+                const double sigma = (double)clip[k] * amax_b / 6.0;
+                double s2 = 0.0, s3 = 0.0;
+                double qv[16];
+                for (int i = 0; i < 16; ++i) {
+                    const double y = fabs((double)wb[i]) / sigma;
+                    const int m = qo_e2m1_round(y);
+                    const double mg = e2m1_margin(y);
+                    if (mg < mround) mround = mg;
+                    const int neg = (wb[i] < 0.0f) && m != 0;
+                    qk[k][i] = (uint8_t)((neg << 3) | m);
+                    qv[i] = neg ? -e2m1_mag[m] : e2m1_mag[m];
+                    s2 += hd[i] * qv[i] * qv[i];
+                    s3 += hd[i] * qv[i] * (double)wb[i];
+                }
+                const double x = (s2 == 0.0) ? sigma / sT : (s3 / s2) / sT;
+                const double mgs = e4m3_margin(x);
+                if (mgs < mscale) mscale = mgs;
+                sk[k] = qo_e4m3_round(x);
+                const double alpha = sT * qo_e4m3_value(sk[k]);
+                double e = 0.0;
+                for (int i = 0; i < 16; ++i) {
+                    const double d = alpha * qv[i] - (double)wb[i];
+                    e += hd[i] * d * d;
+                }
+                ek[k] = e;
+            }
+            for (int k = 1; k < K; ++k)
+                if (ek[k] < ek[best]) best = k;
+            double second = HUGE_VAL;
+            for (int k = 0; k < K; ++k) {
+                if (k == best) continue;
+                if (sk[k] == sk[best] && memcmp(qk[k], qk[best], 16) == 0) continue;
+                if (ek[k] < second) second = ek[k];
+            }
+            if (second < HUGE_VAL) {
+                const double denom = ek[best] > 1e-300 ? ek[best] : 1e-300;
+                mtie = (second - ek[best]) / denom;
+            }
+        }
+
+        if (idx) idx[blk] = best;
+        if (scale_bits) scale_bits[blk] = (uint8_t)sk[best];
+        if (err) err[blk] = ek[best];
+        if (m_round) m_round[blk] = mround;
+        if (m_scale) m_scale[blk] = mscale;
+        if (m_tie) m_tie[blk] = mtie;
+        for (int k = 0; k < K; ++k) {
+            if (cand_err) cand_err[blk * K + k] = ek[k];
+            if (cand_scale) cand_scale[blk * K + k] = (uint8_t)sk[k];
+        }
+        const double alpha = sT * qo_e4m3_value(sk[best]);
+        for (int i = 0; i < 16; ++i) {
+            const int c = qk[best][i];
+            const double qv = (c & 8) ? -e2m1_mag[c & 7] : e2m1_mag[c & 7];
+            if (codes) codes[blk * 16 + i] = (uint8_t)c;
+            if (r) r[blk * 16 + i] = alpha * qv;
+        }
+    }
+    return 0;
+}

@@ -1,0 +1,103 @@
+"""Planted mistakes: each mutant of the oracle source must fail at least one pin.
+
+A mutant is a copy of ``oracle/quasar_oracle.c`` with one plausible slip
+(a dropped term, a wrong sign, a wrong rounding or tie rule, a transposed
+operand), compiled on the CPU into a temporary directory and swapped in for
+the real library while the pins of ``test_oracle_pins`` run against it.
+"""
+import ctypes
+import os
+import subprocess
+
+import pytest
+
+import oracle as oracle_mod
+from tests import test_oracle_pins as pins
+
+SRC = os.path.join(os.path.dirname(os.path.dirname(os.path.abspath(__file__))),
+                   "oracle", "quasar_oracle.c")
+
+MUTANTS = {
+    "round half up": ("nearbyint(t);", "floor(t + 0.5);"),
+    "offset sign": ("z = wbar - s * qbar;", "z = wbar + s * qbar;"),
+    "error sign": ("const double d = s * (double)q[i] + z - (double)w[i];",
+                   "const double d = s * (double)q[i] - z - (double)w[i];"),
+    "unweighted denominator": ("den += hd[i] * dq * dq;", "den += dq * dq;"),
+    "argmin ties to last": (
+        "if (ek[k] < ek[best]) best = k;\n            double second = HUGE_VAL;\n"
+        "            for (int k = 0; k < K; ++k) {\n                if (k == best) continue;\n"
+        "                if (memcmp(qk + (size_t)k",
+        "if (ek[k] <= ek[best]) best = k;\n            double second = HUGE_VAL;\n"
+        "            for (int k = 0; k < K; ++k) {\n                if (k == best) continue;\n"
+        "                if (memcmp(qk + (size_t)k"),
+    "NVFP4 argmin picks the largest error": (
+        "if (ek[k] < ek[best]) best = k;\n            double second = HUGE_VAL;\n"
+        "            for (int k = 0; k < K; ++k) {\n                if (k == best) continue;\n"
+        "                if (sk[k]",
+        "if (ek[k] > ek[best]) best = k;\n            double second = HUGE_VAL;\n"
+        "            for (int k = 0; k < K; ++k) {\n                if (k == best) continue;\n"
+        "                if (sk[k]"),
+    "center sign": ("const double c = 0.5 * (mn + mx);", "const double c = 0.5 * (mx - mn);"),
+    "clip ignored in offset": ("const double z = c - f * rho;", "const double z = c - rho;"),
+    "EMA drops square": ("c1 * gi * gi", "c1 * gi"),
+    "E4M3 subnormal exponent": ("ldexp((double)m / 8.0, -6)", "ldexp((double)m / 8.0, -7)"),
+    "NVFP4 search scale": ("(double)clip[k] * amax_b / 6.0", "(double)clip[k] * amax_b / 4.0"),
+    "NVFP4 error at unrounded scale": (
+        "const double alpha = sT * qo_e4m3_value(sk[k]);",
+        "const double alpha = (s2 == 0.0) ? sigma : s3 / s2;"),
+    "degenerate step dropped": ("s = step;", "s = 0.0;"),
+    "code margin not normalised": ("margin[i] = fabs(t - (j + 0.5)) / (double)qmax;",
+                                   "margin[i] = fabs(t - (j + 0.5));"),
+    "E2M1 ties to odd": ("if (d < bd || (d == bd && (m % 2) == 0)) {",
+                         "if (d < bd || (d == bd && (m % 2) == 1)) {"),
+}
+
+PIN_TESTS = [
+    (pins.test_int_worked_examples, {}),
+    (pins.test_nvfp4_worked_example, {}),
+    (pins.test_codes_are_nearest_grid_level, {"bits": 3}),
+    (pins.test_fit_matches_weighted_lstsq, {"bits": 3, "G": 128}),
+    (pins.test_fit_normal_equations, {}),
+    (pins.test_argmin_over_candidates, {}),
+    (pins.test_single_salient_element_rule, {}),
+    (pins.test_ema_special_cases, {}),
+    (pins.test_e4m3_values_match_torch, {}),
+    (pins.test_e2m1_grid_from_format, {}),
+    (pins.test_nvfp4_fit_and_scale_are_optimal, {}),
+]
+
+
+def _build_mutant(tmp_path, old, new):
+    src = open(SRC).read()
+    assert src.count(old) == 1, f"mutation anchor not unique: {old!r}"
+    path = tmp_path / "mutant.c"
+    path.write_text(src.replace(old, new))
+    so = tmp_path / "libmutant.so"
+    subprocess.run(["gcc", "-O1", "-std=c11", "-fPIC", "-shared", "-ffp-contract=off",
+                    str(path), "-o", str(so), "-lm"], check=True)
+    return str(so)
+
+
+@pytest.mark.parametrize("name", sorted(MUTANTS))
+def test_pins_catch_planted_mistake(oracle, tmp_path, name):
+    old, new = MUTANTS[name]
+    so = _build_mutant(tmp_path, old, new)
+    real = oracle_mod._load()
+    lib = ctypes.CDLL(so)
+    # give the mutant the same prototypes as the real library
+    for sym in ("qo_ema", "qo_recon_int", "qo_refit_int", "qo_codes_int", "qo_tensor_scale",
+                "qo_recon_nvfp4", "qo_e2m1_round", "qo_e4m3_round", "qo_e4m3_value",
+                "qo_set_threads", "qo_get_threads"):
+        f_real, f_mut = getattr(real, sym), getattr(lib, sym)
+        f_mut.argtypes, f_mut.restype = f_real.argtypes, f_real.restype
+    caught = []
+    oracle_mod._lib = lib
+    try:
+        for test, kw in PIN_TESTS:
+            try:
+                test(oracle_mod, **kw)
+            except (AssertionError, ValueError, ZeroDivisionError, FloatingPointError):
+                caught.append(test.__name__)
+    finally:
+        oracle_mod._lib = real
+    assert caught, f"no pin caught the planted mistake '{name}'"
