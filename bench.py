@@ -1,0 +1,457 @@
+#!/usr/bin/env python3
+"""Throughput of one QUASAR reconstruction step on GB300.
+
+A step is one pass of the whole hot path -- saliency EMA, clip-range search,
+code assignment, weighted least-squares fit and the write of r, v', a, b and
+the kept candidate -- over every linear weight of a 32-layer
+Llama-3.1-8B-shaped model (224 tensors, 6.98e9 weights, ~84 GB resident:
+fp32 w and v, bf16 g and r), with inputs already resident in HBM.  The
+headline format is INT3 with group 128 and 8 clip candidates; the other
+formats of the sweep (INT2, INT4, NVFP4) are timed after it and reported in
+"sweep".  Each step streams ~70 GB of inputs, far more than the 129 MB L2.
+
+Usage: python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+With N > 1 it runs under torchrun, one rank per GPU; every rank processes the
+whole model (independent replicas, weak scaling) and the slowest rank's time
+counts.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+import numpy as np
+import torch
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+from paper_2608_13966_gb300 import quasar as Q  # noqa: E402
+from paper_2608_13966_gb300 import workloads as WL  # noqa: E402
+
+METRIC = "reconstructed weights/sec and achieved HBM GB/s (fraction of ~8 TB/s) per QUASAR step"
+NOMINAL_HBM_GBS = 8000.0
+FALLBACK_HBM_GBS = 6800.0
+
+
+def peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(path):
+        with open(path) as f:
+            p = json.load(f)
+        return float(p["hbm_gbs"]), "measured"
+    return FALLBACK_HBM_GBS, "fallback"
+
+
+# ------------------------------------------------------------------ setup --
+
+def dist_setup(n_gpus):
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        torch.distributed.init_process_group("nccl" if torch.cuda.is_available() else "gloo")
+    if torch.cuda.is_available():
+        torch.cuda.set_device(local)
+    return world, rank
+
+
+def barrier(world):
+    if world > 1:
+        torch.distributed.barrier()
+
+
+def max_over_ranks(x, world):
+    if world == 1:
+        return x
+    t = torch.tensor([x], dtype=torch.float64, device="cuda")
+    torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+    return float(t.item())
+
+
+def bytes_per_step(wlo, elements):
+    """Algorithmic HBM bytes of one step: read w (4) + g (2) + v (4), write
+    v (4) + r (2) per weight; per group a, b (fp32) and the kept index (u8)
+    for integer codes; per 16-block the E4M3 scale and index for NVFP4, plus
+    the tensor-absmax pre-pass (one more read of w)."""
+    if wlo.fmt == "int":
+        return elements * 16 + (elements // wlo.group) * 9
+    return elements * 16 + (elements // 16) * 2 + elements * 4
+
+
+class Model:
+    """All tensors of a workload, resident on the device, with outputs."""
+
+    def __init__(self, wlo, device):
+        self.wlo = wlo
+        self.tensors = []
+        for spec in wlo.tensors:
+            d = WL.make_tensor(wlo, spec, device=device)
+            n = spec.numel
+            d["r"] = torch.empty((spec.rows, spec.cols), dtype=torch.bfloat16, device=device)
+            d["a"] = torch.empty(n // 128, dtype=torch.float32, device=device)
+            d["b"] = torch.empty(n // 128, dtype=torch.float32, device=device)
+            d["idx"] = torch.empty(n // 16, dtype=torch.uint8, device=device)
+            d["scale"] = torch.empty(n // 16, dtype=torch.uint8, device=device)
+            d["ts"] = torch.empty(1, dtype=torch.float32, device=device)
+            d["spec"] = spec
+            self.tensors.append(d)
+        self.elements = sum(t["spec"].numel for t in self.tensors)
+
+
+class Step:
+    """Pre-marshalled C-ABI calls of one step for one format."""
+
+    def __init__(self, model, wlo, stream):
+        import ctypes
+        self.lib = Q.load()
+        self.wlo = wlo
+        self.stream = stream.cuda_stream
+        self.clip = (ctypes.c_float * len(wlo.clip))(*wlo.clip)
+        self.calls = []
+        for d in model.tensors:
+            s = d["spec"]
+            if wlo.fmt == "int":
+                args = (d["w"].data_ptr(), d["g"].data_ptr(), Q.BF16, d["v"].data_ptr(), wlo.beta2,
+                        wlo.bits, wlo.group, self.clip, len(wlo.clip), s.rows, s.cols,
+                        d["r"].data_ptr(), Q.BF16, None, d["a"].data_ptr(), d["b"].data_ptr(),
+                        d["idx"].data_ptr(), self.stream)
+                self.calls.append((self.lib.quasar_recon_int, args, s.numel))
+            else:
+                args = (d["w"].data_ptr(), d["g"].data_ptr(), Q.BF16, d["v"].data_ptr(), wlo.beta2,
+                        self.clip, len(wlo.clip), s.rows, s.cols, None, d["r"].data_ptr(), Q.BF16,
+                        None, d["scale"].data_ptr(), d["ts"].data_ptr(), d["idx"].data_ptr(),
+                        self.stream)
+                self.calls.append((self.lib.quasar_recon_nvfp4, args, s.numel))
+        self.launches_per_call = 1 if wlo.fmt == "int" else 3
+
+    def run(self, events=None):
+        for i, (fn, args, _) in enumerate(self.calls):
+            if events is not None:
+                events[i][0].record()
+            st = fn(*args)
+            if st != 0:
+                raise Q.QuasarError(st)
+            if events is not None:
+                events[i][1].record()
+
+
+# ----------------------------------------------------------------- clocks --
+
+class ClockSampler:
+    QUERY = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+             "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+             "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, device_index):
+        self.dev = device_index
+        self.proc = None
+        self.path = None
+
+    def start(self):
+        try:
+            fd, self.path = tempfile.mkstemp(suffix=".csv")
+            os.close(fd)
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.dev), f"--query-gpu={self.QUERY}",
+                 "--format=csv,noheader,nounits", "-lms", "50"],
+                stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
+        except (OSError, FileNotFoundError):
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        rows = []
+        with open(self.path) as f:
+            for line in f:
+                parts = [x.strip() for x in line.split(",")]
+                if len(parts) >= 9:
+                    rows.append(parts)
+        os.unlink(self.path)
+        if not rows:
+            return None
+        sm = [float(r[1]) for r in rows if r[1].replace(".", "").isdigit()]
+        smax = [float(r[2]) for r in rows if r[2].replace(".", "").isdigit()]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[j] for r in rows for j in range(4)
+                          if r[5 + j].lower() in ("active", "1")})
+        power = [float(r[3]) for r in rows if r[3].replace(".", "").isdigit()]
+        return {"sm_mhz": statistics.median(sm) if sm else None,
+                "sm_max_mhz": max(smax) if smax else None,
+                "reasons": reasons, "samples": len(rows),
+                "power_w_max": max(power) if power else None}
+
+
+# ------------------------------------------------------------- CPU oracle --
+
+def cpu_oracle_rate(wlo, budget_s=12.0, seed=0):
+    """The fp64 oracle as it stands, on this host's cores, over a bounded
+    sample of the workload: the leading groups of each tensor of layer 0,
+    sized to take about budget_s seconds.  Returns (weights/s, cores, desc)."""
+    import oracle
+    oracle.build()
+    cores = oracle.get_threads()
+    specs = wlo.tensors[:7]
+    gsize = wlo.group if wlo.fmt == "int" else 16
+
+    def run(n_per_tensor):
+        total, t_run = 0, 0.0
+        for j, spec in enumerate(specs):
+            n = min(spec.numel, n_per_tensor) // gsize * gsize
+            d = WL.random_groups(n // gsize, gsize, seed=seed * 1000 + j, dist=wlo.w_dist,
+                                 g_dtype=wlo.g_dtype)
+            w = d["w"].numpy()
+            g = d["g"].float().numpy()
+            v = d["v"].numpy()
+            t0 = time.perf_counter()
+            h = oracle.ema(v, g, wlo.beta2)
+            if wlo.fmt == "int":
+                oracle.recon_int(w, h, wlo.group, wlo.bits, list(wlo.clip))
+            else:
+                _, sT = oracle.tensor_scale(w)
+                oracle.recon_nvfp4(w, h, sT, list(wlo.clip))
+            t_run += time.perf_counter() - t0
+            total += n
+        return total, t_run
+
+    n0 = 1 << 15
+    total, t = run(n0)
+    per = max(t / total, 1e-12)
+    n1 = int(min(budget_s / per / len(specs), 1 << 24))
+    n1 = max(n1, n0)
+    total, t = run(n1)
+    desc = (f"{n1 // gsize} groups per tensor shape of one layer, same value distributions, "
+            f"{total} weights in {t:.1f} s")
+    return total / t, cores, desc
+
+
+# ------------------------------------------------------------------- main --
+
+def kernel_source_hash():
+    h = hashlib.sha256()
+    csrc = os.path.join(ROOT, "paper_2608_13966_gb300", "csrc")
+    for name in sorted(os.listdir(csrc)):
+        with open(os.path.join(csrc, name), "rb") as f:
+            h.update(name.encode())
+            h.update(f.read())
+    return h.hexdigest()[:16]
+
+
+def profiled_traffic(kernel_tag):
+    """Per-launch DRAM bytes from the committed ncu summary, if it was taken
+    on the current kernel sources; else None."""
+    path = os.path.join(ROOT, "profiles", "traffic.txt")
+    if not os.path.exists(path):
+        return None
+    want = kernel_source_hash()
+    with open(path) as f:
+        for line in f:
+            parts = line.split()
+            if len(parts) >= 3 and parts[0] == kernel_tag and parts[1] == want:
+                return float(parts[2])
+    return None
+
+
+def timed_steps(step, n_launch_calls, steps, warmup, world):
+    for _ in range(warmup):
+        step.run()
+    torch.cuda.synchronize()
+    barrier(world)
+    events = [[(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+               for _ in range(n_launch_calls)] for _ in range(steps)]
+    start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    torch.cuda.synchronize()
+    start.record()
+    for k in range(steps):
+        step.run(events[k])
+    end.record()
+    torch.cuda.synchronize()
+    barrier(world)
+    total_ms = start.elapsed_time(end)
+    kernel_ms = sum(s.elapsed_time(e) for ev in events for (s, e) in ev)
+    return total_ms, kernel_ms
+
+
+def e2e_rate(wlo, steps, device, stream):
+    """Same metric through the C ABI with HOST buffers: every step copies each
+    tensor's w, g, v from pinned host memory, reconstructs, and reads r, v',
+    a, b and the kept index back.  The host and device staging buffers hold
+    one layer and are reused for each of the 32 layers (same bytes moved)."""
+    host, dev = [], []
+    for spec in wlo.tensors[:7]:
+        d = WL.make_tensor(wlo, spec, device=device)
+        n = spec.numel
+        h = {k: v.cpu().pin_memory() for k, v in d.items()}
+        del d
+        h["r"] = torch.empty((spec.rows, spec.cols), dtype=torch.bfloat16).pin_memory()
+        h["a"] = torch.empty(n // 128, dtype=torch.float32).pin_memory()
+        h["b"] = torch.empty(n // 128, dtype=torch.float32).pin_memory()
+        h["idx"] = torch.empty(n // 128, dtype=torch.uint8).pin_memory()
+        host.append(h)
+        dev.append({k: torch.empty_like(v, device=device) for k, v in h.items()})
+    n_layers = len(wlo.tensors) // 7
+    h2d = sum(h[k].numel() * h[k].element_size() for h in host for k in ("w", "g", "v")) * n_layers
+    d2h = sum(h[k].numel() * h[k].element_size() for h in host
+              for k in ("r", "v", "a", "b", "idx")) * n_layers
+    elements = sum(s.numel for s in wlo.tensors)
+
+    def one_step():
+        with torch.cuda.stream(stream):
+            for _ in range(n_layers):
+                for spec, h, d in zip(wlo.tensors[:7], host, dev):
+                    for k in ("w", "g", "v"):
+                        d[k].copy_(h[k], non_blocking=True)
+                    st = Q.quasar_recon_int(d["w"], d["g"], d["v"], wlo.beta2, wlo.bits, wlo.group,
+                                            list(wlo.clip), spec.rows, spec.cols, d["r"], None,
+                                            d["a"], d["b"], d["idx"], stream=stream)
+                    if st != 0:
+                        raise Q.QuasarError(st)
+                    for k in ("r", "v", "a", "b", "idx"):
+                        h[k].copy_(d[k], non_blocking=True)
+        stream.synchronize()
+
+    one_step()
+    t0 = time.perf_counter()
+    for _ in range(steps):
+        one_step()
+    dt = (time.perf_counter() - t0) / steps
+    return {"value": elements / dt, "unit": "weights/s", "h2d_bytes_per_step": int(h2d),
+            "d2h_bytes_per_step": int(d2h), "ms_per_step": dt * 1e3,
+            "how": "C-ABI calls on pinned host buffers, H2D of w/g/v and D2H of r/v/a/b/idx "
+                   "inside the timed region; one layer's buffers reused for all 32 layers"}
+
+
+def reference_arm(args, world, rank):
+    """The oracle, as it stands, on the host cores (rank 0 only)."""
+    if rank != 0:
+        return
+    wlo = WL.workload(args.workload)
+    rates = []
+    desc = cores = None
+    for i in range(args.warmup + args.steps):
+        rate, cores, desc = cpu_oracle_rate(wlo, budget_s=args.ref_budget)
+        if i >= args.warmup:
+            rates.append(rate)
+    value = statistics.median(rates)
+    n = sum(s.numel for s in wlo.tensors)
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": "weights/s",
+            "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": n / value * 1e3, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": {"workload": wlo.notes, "elements": n},
+            "cpu_baseline": {"value": value, "unit": "weights/s", "cores": cores, "kind": "oracle",
+                             "sample": desc},
+            "e2e": {"value": value, "unit": "weights/s", "h2d_bytes_per_step": 0,
+                    "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=30)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--workload", default="llama_int3")
+    ap.add_argument("--sweep", default="llama_int2,llama_int4,llama_nvfp4")
+    ap.add_argument("--sweep-steps", type=int, default=10)
+    ap.add_argument("--e2e-steps", type=int, default=2)
+    ap.add_argument("--cpu-budget", type=float, default=12.0)
+    ap.add_argument("--ref-budget", type=float, default=8.0)
+    args = ap.parse_args()
+
+    world, rank = dist_setup(args.gpus)
+    if args.impl == "reference":
+        reference_arm(args, world, rank)
+        return
+
+    device = torch.device("cuda", torch.cuda.current_device())
+    stream = torch.cuda.Stream()
+    hbm_peak, peak_kind = peaks()
+    wlo = WL.workload(args.workload)
+    model = Model(wlo, device)
+    torch.cuda.synchronize()
+    n_el = model.elements
+
+    clocks = ClockSampler(torch.cuda.current_device())
+    step = Step(model, wlo, stream)
+    with torch.cuda.stream(stream):
+        clocks.start()
+        total_ms, kernel_ms = timed_steps(step, len(step.calls), args.steps, args.warmup, world)
+        clk = clocks.stop()
+    total_ms = max_over_ranks(total_ms, world)
+    ms_per_step = total_ms / args.steps
+    step_bytes = bytes_per_step(wlo, n_el)
+    value = world * n_el / (ms_per_step / 1e3)
+    achieved = step_bytes * args.steps / (kernel_ms / 1e3) / 1e9
+    hbm_gbs = step_bytes / (ms_per_step / 1e3) / 1e9
+
+    sweep = {}
+    for name in [s for s in args.sweep.split(",") if s]:
+        sw = WL.workload(name)
+        st = Step(model, sw, stream)
+        with torch.cuda.stream(stream):
+            t_ms, k_ms = timed_steps(st, len(st.calls), args.sweep_steps, 2, world)
+        t_ms = max_over_ranks(t_ms, world)
+        b = bytes_per_step(sw, n_el)
+        sweep[name] = {"ms_per_step": t_ms / args.sweep_steps,
+                       "weights_per_s": world * n_el / (t_ms / args.sweep_steps / 1e3),
+                       "hbm_gbs": b / (t_ms / args.sweep_steps / 1e3) / 1e9,
+                       "kernel_gbs": b * args.sweep_steps / (k_ms / 1e3) / 1e9,
+                       "frac_of_measured": b / (t_ms / args.sweep_steps / 1e3) / 1e9 / hbm_peak,
+                       "bytes_per_weight": b / n_el}
+
+    e2e = None
+    if args.e2e_steps > 0 and rank == 0:
+        del model
+        torch.cuda.empty_cache()
+        e2e = e2e_rate(wlo, args.e2e_steps, device, stream)
+        e2e["value"] *= world
+
+    cpu = None
+    if rank == 0 and world == 1 and args.cpu_budget > 0:
+        rate, cores, desc = cpu_oracle_rate(wlo, budget_s=args.cpu_budget)
+        cpu = {"value": rate, "unit": "weights/s", "cores": cores, "kind": "oracle", "sample": desc}
+
+    if rank != 0:
+        return
+    traffic = profiled_traffic("k_recon_int_g128_k8" if wlo.fmt == "int" else "k_recon_nvfp4_k8")
+    line = {
+        "metric": METRIC, "value": value, "unit": "weights/s", "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_per_step,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
+        "data": "synthetic",
+        "config": {"workload": wlo.notes, "elements": n_el, "tensors": len(wlo.tensors),
+                   "bits": wlo.bits, "group": wlo.group, "clip_candidates": len(wlo.clip),
+                   "g_dtype": "bf16", "r_dtype": "bf16", "codes": "not written",
+                   "l2": "inputs larger than L2 (%.0f GB read per step)" % (n_el * 10 / 1e9),
+                   "parallelism": "replicas" if world > 1 else "single GPU"},
+        "hbm_gbs": hbm_gbs, "frac_of_8tbs": hbm_gbs / NOMINAL_HBM_GBS,
+        "frac_of_measured_copy": hbm_gbs / hbm_peak,
+        "roofline": {"bound": "hbm", "achieved": achieved, "peak": hbm_peak, "unit": "GB/s",
+                     "frac": achieved / hbm_peak, "traffic": traffic,
+                     "peak_kind": peak_kind,
+                     "kernel": "k_recon_int<16,1>" if wlo.fmt == "int" else "k_recon_nvfp4<1>",
+                     "bytes_per_weight": step_bytes / n_el},
+        "cpu_baseline": cpu, "e2e": e2e,
+        "gpu_launches": len(step.calls) * step.launches_per_call * args.steps,
+        "clocks": clk, "sweep": sweep,
+    }
+    print(json.dumps(line), flush=True)
+
+
+if __name__ == "__main__":
+    main()

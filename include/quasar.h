@@ -1,0 +1,175 @@
+/*
+ * quasar.h -- C ABI of the GB300 (sm_103a) QUASAR reconstruction library.
+ *
+ * QUASAR ("QUASAR: Lowering the Loss Floor of Quantization-Aware Training
+ * with Loss-Aware Reconstruction") rebuilds, at every training step, the
+ * quantized weights r that the forward pass uses from the latent weights w:
+ * for each group it updates the saliency EMA of squared gradients, searches
+ * a small grid of clipping ranges, assigns codes for each range, fits the
+ * dequantizer by saliency-weighted least squares, and keeps the range whose
+ * weighted reconstruction error is lowest (Algorithm 1; Sec. 4.2 for NVFP4).
+ *
+ * Conventions shared by every entry point:
+ *  - All tensor arguments are DEVICE pointers into memory owned by the caller
+ *    (cudaMalloc / a framework allocator).  The library allocates nothing on
+ *    these paths and keeps no per-call state.
+ *  - Calls are asynchronous on `stream` (NULL = legacy default stream).
+ *    Arguments are validated on the host first; on any error a status is
+ *    returned and nothing is launched.  A failed launch returns
+ *    QUASAR_ERR_CUDA.
+ *  - Tensors are row-major [rows, cols].  Groups of `group_size` consecutive
+ *    elements of a row share one dequantizer (rows of an nn.Linear weight
+ *    [out, in] are split along `in`), so the tensor is a flat sequence of
+ *    rows*cols/group_size groups.
+ *  - Device pointers to tensors must be 16-byte aligned.  Outputs must not
+ *    overlap the inputs w, g or v (checked by address range).
+ *  - Inputs holding NaN or Inf give unspecified outputs but never fault.
+ *  - A device-side wait that runs out (a shared-memory pipeline stage that
+ *    never arrives) does not hang: the kernel records QUASAR_ERR_TIMEOUT in
+ *    a per-device status word and returns; quasar_get_device_status reports
+ *    and clears it.
+ */
+#ifndef QUASAR_H
+#define QUASAR_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* Same type as cudaStream_t; declared here so C callers need no CUDA headers. */
+struct CUstream_st;
+typedef struct CUstream_st* quasar_stream_t;
+
+typedef enum {
+    QUASAR_OK = 0,
+    QUASAR_ERR_INVALID_ARG = 1, /* a NULL, out-of-range, misaligned or aliasing argument */
+    QUASAR_ERR_UNSUPPORTED = 2, /* a valid request this build has no kernel for           */
+    QUASAR_ERR_CUDA = 3,        /* a CUDA runtime call or a launch failed                */
+    QUASAR_ERR_TIMEOUT = 4      /* a device-side wait ran out (see quasar_get_device_status) */
+} quasar_status;
+
+typedef enum { QUASAR_F32 = 0, QUASAR_BF16 = 1 } quasar_dtype;
+
+/*
+ * quasar_recon_int -- QUASAR reconstruction with asymmetric b-bit integer
+ * codes (Algorithm 1; code assignment Eq. 1; dequantizer fit Eq. 4; error
+ * Eq. 3; saliency EMA Sec. 4.1.1 / App. A.2).
+ *
+ * For every group of `group_size` consecutive elements:
+ *   1. v' = beta2*v + (1-beta2)*g^2 is written back to v, and h = v' is the
+ *      saliency.  g == NULL skips the update (h = v, v untouched).
+ *   2. c = (min w + max w)/2, rho = (max w - min w)/2.
+ *   3. For each factor f = clip[k]: codes q = clamp(round_half_even((w - z)/s),
+ *      0, 2^bits - 1) with z = c - f*rho, s = 2*f*rho/(2^bits - 1); the
+ *      weighted least-squares (a_k, b_k) minimising sum h (a q + b - w)^2;
+ *      its error.
+ *   4. The candidate with the lowest error is kept (ties: lowest k);
+ *      r = a*q + b.
+ *   Degenerate groups: zero range gives q = 0, a = 0, b = w[0], r = w,
+ *   k = 0.  All h = 0 in a group: the group is fitted with h = 1.  If every
+ *   h > 0 element of a candidate shares one code, that candidate's error is
+ *   sum h (w - mean_h(w))^2 and a = its grid step, b = mean_h(w) - a*code.
+ *
+ * Arguments:
+ *   w          [rows, cols] fp32 latent weights (read).
+ *   g          [rows, cols] gradient, dtype g_dtype (read), or NULL.
+ *   v          [rows, cols] fp32 EMA state (read; overwritten with v').
+ *   beta2      EMA decay, 0 <= beta2 < 1.
+ *   bits       1..8.
+ *   group_size 32, 64, 128 or 256; cols % group_size == 0.
+ *   clip       HOST array of n_clip factors, each in (0, 1], in search order;
+ *              copied before the call returns.  1 <= n_clip <= 32.
+ *   r          [rows, cols] reconstruction, dtype r_dtype (written).
+ *   codes      [rows, cols] uint8 codes of the kept candidate, or NULL.
+ *   a, b       [rows*cols/group_size] fp32 scale and offset (written).
+ *   cand_idx   [rows*cols/group_size] uint8 index into clip[] of the kept
+ *              candidate, or NULL.
+ * Returns QUASAR_OK, or INVALID_ARG / UNSUPPORTED / CUDA with nothing done
+ * (CUDA: a launch failure after validation).  rows*cols == 0 is a no-op.
+ */
+quasar_status quasar_recon_int(const float* w, const void* g, quasar_dtype g_dtype, float* v,
+                               float beta2, int bits, int group_size, const float* clip,
+                               int n_clip, int64_t rows, int64_t cols, void* r,
+                               quasar_dtype r_dtype, uint8_t* codes, float* a, float* b,
+                               uint8_t* cand_idx, quasar_stream_t stream);
+
+/*
+ * quasar_recon_nvfp4 -- QUASAR for NVFP4 (Sec. 4.2): E2M1 codes, one FP8
+ * (E4M3) scale per 16 consecutive elements, one FP32 scale per tensor.
+ *
+ *   s_T = amax / (6*448) from the tensor absmax (amax = 0 gives s_T = 1);
+ *   the tensor scale is not optimised.  For each 16-element block and each
+ *   factor f = clip[k]: search scale sigma = f*max|w_block|/6; codes
+ *   q = sign(w) * E2M1_rne(min(|w|/sigma, 6)); least-squares slope
+ *   a* = sum h q w / sum h q^2; E4M3 scale e = E4M3_rne_satfinite(a* / s_T);
+ *   error sum h (s_T*e*q - w)^2.  The candidate with the lowest error is
+ *   kept (ties: lowest k) and r = s_T*e*q.  The saliency update is the same
+ *   as in quasar_recon_int.  A zero block gives q = 0, e = 0, r = 0; a
+ *   candidate whose weighted codes are all zero takes e = E4M3(sigma/s_T).
+ *
+ * Arguments as in quasar_recon_int, plus:
+ *   cols        cols % 16 == 0.
+ *   tensor_amax device pointer to max|w| of this tensor (fp32), or NULL to
+ *               have the library compute it (one extra read of w).
+ *   codes       [rows, cols] uint8, one E2M1 nibble per byte
+ *               (sign << 3 | magnitude index 0..7; magnitude 0 is +0), or NULL.
+ *   block_scale [rows*cols/16] uint8 E4M3 bit patterns (written).
+ *   tensor_scale device pointer to one fp32, receives s_T (written).
+ *   cand_idx    [rows*cols/16] uint8, or NULL.
+ */
+quasar_status quasar_recon_nvfp4(const float* w, const void* g, quasar_dtype g_dtype, float* v,
+                                 float beta2, const float* clip, int n_clip, int64_t rows,
+                                 int64_t cols, const float* tensor_amax, void* r,
+                                 quasar_dtype r_dtype, uint8_t* codes, uint8_t* block_scale,
+                                 float* tensor_scale, uint8_t* cand_idx,
+                                 quasar_stream_t stream);
+
+/*
+ * quasar_tensor_amax -- amax_out[0] = max |w[i]| over n fp32 elements (the
+ * NVFP4 tensor statistic of Sec. 4.2).  amax_out is a device pointer; it is
+ * overwritten.  n == 0 writes 0.
+ */
+quasar_status quasar_tensor_amax(const float* w, int64_t n, float* amax_out,
+                                 quasar_stream_t stream);
+
+/*
+ * quasar_get_device_status -- synchronises `stream`, then returns
+ * QUASAR_ERR_TIMEOUT if any kernel of this library on the current device
+ * recorded a timed-out wait since the previous query (and clears the record),
+ * QUASAR_ERR_CUDA if the synchronisation failed, else QUASAR_OK.
+ */
+quasar_status quasar_get_device_status(quasar_stream_t stream);
+
+/*
+ * quasar_debug_force_timeout -- testing hook for the failure path.  While
+ * set (nanoseconds > 0), the next kernels of this library on the calling
+ * host thread's current device also wait, for that many nanoseconds, on a
+ * pipeline barrier that nothing ever signals; the wait runs out, the kernel
+ * records QUASAR_ERR_TIMEOUT, drains its own copies in flight and returns.
+ * 0 turns the hook off.  Never needed in normal use.
+ */
+void quasar_debug_force_timeout(int64_t nanoseconds);
+
+/*
+ * quasar_debug_set_stats -- tuning hook.  While device_counters (a device
+ * array of at least 2 unsigned ints owned by the caller) is set, the
+ * reconstruction kernels atomically count [0] the groups/blocks whose
+ * candidates were re-evaluated exactly because of a near tie and [1] the
+ * integer groups whose kept fit was recomputed in two centred passes.  NULL
+ * turns counting off.  Process-wide; never needed in normal use.
+ */
+void quasar_debug_set_stats(unsigned int* device_counters);
+
+/* Static, human-readable name of a status code. */
+const char* quasar_status_string(quasar_status status);
+
+/* Library version as major*10000 + minor*100 + patch. */
+int quasar_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* QUASAR_H */

@@ -52,7 +52,7 @@ def _load():
         lib.qo_recon_int.restype = i32
         lib.qo_refit_int.argtypes = [P, P, P, i32, i32, f32, P, P]
         lib.qo_refit_int.restype = f64
-        lib.qo_codes_int.argtypes = [P, i32, i32, f32, P, P]
+        lib.qo_codes_int.argtypes = [P, i32, i32, f32, P, P, P]
         lib.qo_codes_int.restype = i32
         lib.qo_tensor_scale.argtypes = [P, i64, P, P]
         lib.qo_tensor_scale.restype = None
@@ -68,6 +68,12 @@ def _load():
         lib.qo_set_threads.restype = None
         lib.qo_get_threads.argtypes = []
         lib.qo_get_threads.restype = i32
+        lib.qo_codes_nvfp4.argtypes = [P, f32, P, P, P]
+        lib.qo_codes_nvfp4.restype = None
+        lib.qo_fit_nvfp4_scale.argtypes = [P, P, f32, f32, P, P]
+        lib.qo_fit_nvfp4_scale.restype = i32
+        lib.qo_eval_nvfp4.argtypes = [P, P, f32, P, i32]
+        lib.qo_eval_nvfp4.restype = f64
         _lib = lib
         return lib
 
@@ -122,13 +128,15 @@ def recon_int(w, h, group_size: int, bits: int, clip) -> dict:
     return out
 
 
-def codes_int(w_group, bits: int, f: float):
-    """Eq. 1 codes and per-element margins of one candidate for one group."""
+def codes_int(w_group, bits: int, f: float, with_t: bool = False):
+    """Eq. 1 codes and per-element margins of one candidate for one group
+    (and the unrounded positions t if with_t)."""
     w = _c(w_group, np.float32).ravel()
     q = np.empty(w.size, np.uint8)
     m = np.empty(w.size)
-    _load().qo_codes_int(_ptr(w), w.size, int(bits), ctypes.c_float(f), _ptr(q), _ptr(m))
-    return q, m
+    t = np.empty(w.size)
+    _load().qo_codes_int(_ptr(w), w.size, int(bits), ctypes.c_float(f), _ptr(q), _ptr(m), _ptr(t))
+    return (q, m, t) if with_t else (q, m)
 
 
 def refit_int(w_group, h_group, codes, bits: int, f: float):
@@ -175,6 +183,38 @@ def recon_nvfp4(w, h, s_T: float, clip) -> dict:
     out["cand_err"] = out["cand_err"].reshape(n, K)
     out["cand_scale"] = out["cand_scale"].reshape(n, K)
     return out
+
+
+def codes_nvfp4(w_block, f: float, with_y: bool = False):
+    """E2M1 codes and per-element boundary margins of one block for factor f
+    (and |w|/sigma if with_y)."""
+    w = _c(w_block, np.float32).ravel()
+    assert w.size == 16
+    q = np.empty(16, np.uint8)
+    m = np.empty(16)
+    y = np.empty(16)
+    _load().qo_codes_nvfp4(_ptr(w), ctypes.c_float(f), _ptr(q), _ptr(m), _ptr(y))
+    return (q, m, y) if with_y else (q, m)
+
+
+def fit_nvfp4_scale(w_block, h_block, s_T: float, f: float, codes):
+    """Fitted E4M3 scale bits of given codes and the E4M3 boundary margin."""
+    w = _c(w_block, np.float32).ravel()
+    h = _c(h_block, np.float32).ravel()
+    q = _c(codes, np.uint8).ravel()
+    m = ctypes.c_double()
+    bits = _load().qo_fit_nvfp4_scale(_ptr(w), _ptr(h), ctypes.c_float(s_T), ctypes.c_float(f),
+                                      _ptr(q), ctypes.byref(m))
+    return int(bits), m.value
+
+
+def eval_nvfp4(w_block, h_block, s_T: float, codes, scale_bits: int) -> float:
+    """Eq. 3 error of a block reconstructed as s_T * E4M3(scale_bits) * q."""
+    w = _c(w_block, np.float32).ravel()
+    h = _c(h_block, np.float32).ravel()
+    q = _c(codes, np.uint8).ravel()
+    return float(_load().qo_eval_nvfp4(_ptr(w), _ptr(h), ctypes.c_float(s_T), _ptr(q),
+                                       int(scale_bits)))
 
 
 def e2m1_round(y: float) -> int:

@@ -119,12 +119,13 @@ static void group_saliency(const float* h, int G, double* hd)
  * j + 1/2 (j = 0..qmax-1), divided by qmax, i.e. the distance of w to the
  * boundary as a fraction of the clipping range 2*f*rho. */
 static void int_codes(const float* w, int G, double c, double rho, double f, int qmax,
-                      uint8_t* q, double* margin)
+                      uint8_t* q, double* margin, double* t_out)
 {
     const double z = c - f * rho;
     const double s = 2.0 * f * rho / (double)qmax;
     for (int i = 0; i < G; ++i) {
         const double t = ((double)w[i] - z) / s;
+        if (t_out) t_out[i] = t;
         double k = nearbyint(t); /* default rounding mode: half to even */
         if (k < 0.0) k = 0.0;
         if (k > (double)qmax) k = (double)qmax;
@@ -187,9 +188,11 @@ static double wls_fit(const float* w, const double* hd, const uint8_t* q, int G,
     return err;
 }
 
-/* Codes of one candidate for one group (for the parity checker).  Returns 0
- * for a zero-range group (all codes 0, margins +inf). */
-int qo_codes_int(const float* w, int G, int bits, float f, uint8_t* q, double* margin)
+/* Codes of one candidate for one group (for the parity checker), with the
+ * margins and, if t_out is not NULL, the unrounded code positions t.
+ * Returns 0 for a zero-range group (all codes 0, margins +inf). */
+int qo_codes_int(const float* w, int G, int bits, float f, uint8_t* q, double* margin,
+                 double* t_out)
 {
     const int qmax = (1 << bits) - 1;
     double mn = (double)w[0], mx = (double)w[0];
@@ -201,11 +204,12 @@ int qo_codes_int(const float* w, int G, int bits, float f, uint8_t* q, double* m
         for (int i = 0; i < G; ++i) {
             q[i] = 0;
             if (margin) margin[i] = HUGE_VAL;
+            if (t_out) t_out[i] = 0.0;
         }
         return 0;
     }
     const double c = 0.5 * (mn + mx), rho = 0.5 * (mx - mn);
-    int_codes(w, G, c, rho, (double)f, qmax, q, margin);
+    int_codes(w, G, c, rho, (double)f, qmax, q, margin, t_out);
     return 1;
 }
 
@@ -285,7 +289,7 @@ int qo_recon_int(const float* w, const float* h, int64_t n_groups, int G, int bi
             for (int k = 0; k < K; ++k) {
                 const double f = (double)clip[k];
                 uint8_t* q = qk + (size_t)k * G;
-                int_codes(wg, G, c, rho, f, qmax, q, mg);
+                int_codes(wg, G, c, rho, f, qmax, q, mg, NULL);
                 for (int i = 0; i < G; ++i)
                     if (mg[i] < mround) mround = mg[i];
                 const double step = 2.0 * f * rho / (double)qmax;
@@ -362,16 +366,24 @@ double qo_e4m3_value(int bits)
     return ldexp(1.0 + (double)m / 8.0, e - 7);
 }
 
+/* The 127 finite non-negative E4M3 values, ascending with the bit pattern. */
+static double e4m3_tab[0x7F];
+
+static void e4m3_init(void)
+{
+    for (int c = 0; c < 0x7F; ++c) e4m3_tab[c] = qo_e4m3_value(c);
+}
+
 /* Nearest non-negative finite E4M3 value to x >= 0: round to nearest, ties to
  * the even mantissa, values above 448 saturate to 448 (satfinite).  Returns
- * the bit pattern (0x00..0x7E). */
-int qo_e4m3_round(double x)
+ * the bit pattern (0x00..0x7E).  Requires e4m3_init(). */
+static int e4m3_round(double x)
 {
     if (!(x > 0.0)) return 0;
     int best = 0;
-    double bd = fabs(x - qo_e4m3_value(0));
+    double bd = fabs(x - e4m3_tab[0]);
     for (int c = 1; c <= 0x7E; ++c) {
-        const double d = fabs(x - qo_e4m3_value(c));
+        const double d = fabs(x - e4m3_tab[c]);
         if (d < bd || (d == bd && (c % 2) == 0)) {
             best = c;
             bd = d;
@@ -380,13 +392,19 @@ int qo_e4m3_round(double x)
     return best;
 }
 
+int qo_e4m3_round(double x)
+{
+    e4m3_init();
+    return e4m3_round(x);
+}
+
 /* Relative distance of x > 0 to the nearest decision boundary of E4M3
  * rounding (midpoint between consecutive finite values; none above 448). */
 static double e4m3_margin(double x)
 {
     double best = HUGE_VAL;
     for (int c = 0; c < 0x7E; ++c) {
-        const double mid = 0.5 * (qo_e4m3_value(c) + qo_e4m3_value(c + 1));
+        const double mid = 0.5 * (e4m3_tab[c] + e4m3_tab[c + 1]);
         const double d = fabs(x - mid) / mid;
         if (d < best) best = d;
     }
@@ -440,6 +458,7 @@ int qo_recon_nvfp4(const float* w, const float* h, int64_t n_blocks, float s_T,
 {
     if (K < 1 || K > QO_MAX_K || n_blocks < 0 || !(s_T > 0.0f)) return -1;
     const double sT = (double)s_T;
+    e4m3_init();
 
 #pragma omp parallel for schedule(dynamic, 256)
     for (int64_t blk = 0; blk < n_blocks; ++blk) {
@@ -485,8 +504,8 @@ int qo_recon_nvfp4(const float* w, const float* h, int64_t n_blocks, float s_T,
                 const double x = (s2 == 0.0) ? sigma / sT : (s3 / s2) / sT;
                 const double mgs = e4m3_margin(x);
                 if (mgs < mscale) mscale = mgs;
-                sk[k] = qo_e4m3_round(x);
-                const double alpha = sT * qo_e4m3_value(sk[k]);
+                sk[k] = e4m3_round(x);
+                const double alpha = sT * e4m3_tab[sk[k]];
                 double e = 0.0;
                 for (int i = 0; i < 16; ++i) {
                     const double d = alpha * qv[i] - (double)wb[i];
@@ -518,7 +537,7 @@ int qo_recon_nvfp4(const float* w, const float* h, int64_t n_blocks, float s_T,
             if (cand_err) cand_err[blk * K + k] = ek[k];
             if (cand_scale) cand_scale[blk * K + k] = (uint8_t)sk[k];
         }
-        const double alpha = sT * qo_e4m3_value(sk[best]);
+        const double alpha = sT * e4m3_tab[sk[best]];
         for (int i = 0; i < 16; ++i) {
             const int c = qk[best][i];
             const double qv = (c & 8) ? -e2m1_mag[c & 7] : e2m1_mag[c & 7];
@@ -527,4 +546,75 @@ int qo_recon_nvfp4(const float* w, const float* h, int64_t n_blocks, float s_T,
         }
     }
     return 0;
+}
+
+/* ------------------------------------------------------------------------ */
+/* NVFP4 helpers for the parity checker (same definitions as above).        */
+/* ------------------------------------------------------------------------ */
+
+/* E2M1 codes of one 16-element block for search factor f, and per-element
+ * relative distance of |w|/sigma to the nearest E2M1 decision boundary
+ * (and, if y_out is not NULL, |w|/sigma itself). */
+void qo_codes_nvfp4(const float* w, float f, uint8_t* codes, double* margin, double* y_out)
+{
+    double amax_b = 0.0;
+    for (int i = 0; i < 16; ++i) {
+        const double x = fabs((double)w[i]);
+        if (x > amax_b) amax_b = x;
+    }
+    for (int i = 0; i < 16; ++i) {
+        if (amax_b == 0.0) {
+            codes[i] = 0;
+            if (margin) margin[i] = HUGE_VAL;
+            if (y_out) y_out[i] = 0.0;
+            continue;
+        }
+        const double sigma = (double)f * amax_b / 6.0;
+        const double y = fabs((double)w[i]) / sigma;
+        if (y_out) y_out[i] = y;
+        const int m = qo_e2m1_round(y);
+        const int neg = (w[i] < 0.0f) && m != 0;
+        codes[i] = (uint8_t)((neg << 3) | m);
+        if (margin) margin[i] = e2m1_margin(y);
+    }
+}
+
+/* Fitted E4M3 scale of given codes (Sec. 4.2 with Eq. 3): returns the bit
+ * pattern; *margin gets the relative distance of a* / s_T to an E4M3
+ * boundary.  Rule N4 (sum h q^2 = 0) uses the search scale of factor f. */
+int qo_fit_nvfp4_scale(const float* w, const float* h, float s_T, float f, const uint8_t* codes,
+                       double* margin)
+{
+    double hd[16], amax_b = 0.0, s2 = 0.0, s3 = 0.0;
+    group_saliency(h, 16, hd);
+    for (int i = 0; i < 16; ++i) {
+        const double x = fabs((double)w[i]);
+        if (x > amax_b) amax_b = x;
+        const double q = (codes[i] & 8) ? -e2m1_mag[codes[i] & 7] : e2m1_mag[codes[i] & 7];
+        s2 += hd[i] * q * q;
+        s3 += hd[i] * q * (double)w[i];
+    }
+    if (amax_b == 0.0) {
+        if (margin) *margin = HUGE_VAL;
+        return 0;
+    }
+    const double x = (s2 == 0.0) ? ((double)f * amax_b / 6.0) / (double)s_T : (s3 / s2) / (double)s_T;
+    e4m3_init();
+    if (margin) *margin = e4m3_margin(x);
+    return e4m3_round(x);
+}
+
+/* Eq. 3 error of a block reconstructed as s_T*e*q (rule D2 applied to h). */
+double qo_eval_nvfp4(const float* w, const float* h, float s_T, const uint8_t* codes, int scale_bits)
+{
+    double hd[16];
+    group_saliency(h, 16, hd);
+    const double alpha = (double)s_T * qo_e4m3_value(scale_bits);
+    double e = 0.0;
+    for (int i = 0; i < 16; ++i) {
+        const double q = (codes[i] & 8) ? -e2m1_mag[codes[i] & 7] : e2m1_mag[codes[i] & 7];
+        const double d = alpha * q - (double)w[i];
+        e += hd[i] * d * d;
+    }
+    return e;
 }

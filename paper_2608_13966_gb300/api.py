@@ -1,0 +1,83 @@
+"""Convenience layer over the C ABI: allocates the outputs with PyTorch and
+raises ``QuasarError`` on a non-OK status.  The computation itself is the
+library's; this module only allocates and marshals."""
+from __future__ import annotations
+
+import torch
+
+from .quasar import (QuasarError, QuasarStatus, quasar_recon_int, quasar_recon_nvfp4,
+                     quasar_tensor_amax)
+
+
+def _check(st):
+    if st != QuasarStatus.OK:
+        raise QuasarError(st)
+
+
+def _check_2d(w):
+    if w.dim() != 2:
+        raise ValueError("w must be a 2-D [rows, cols] tensor")
+    if not (w.is_cuda and w.dtype == torch.float32 and w.is_contiguous()):
+        raise ValueError("w must be a contiguous fp32 CUDA tensor")
+
+
+def recon_int(w, g, v, *, bits, group_size, clip, beta2=0.999, r_dtype=torch.bfloat16,
+              codes=True, cand_idx=True, stream=None, out=None):
+    """QUASAR integer reconstruction of one tensor; v is updated in place.
+
+    Returns a dict with r, a, b and (if requested) codes and cand_idx."""
+    _check_2d(w)
+    rows, cols = w.shape
+    dev = w.device
+    n_groups = rows * cols // group_size
+    o = out if out is not None else {}
+    r = o.get("r") if o.get("r") is not None else torch.empty((rows, cols), dtype=r_dtype, device=dev)
+    a = o.get("a") if o.get("a") is not None else torch.empty(n_groups, dtype=torch.float32, device=dev)
+    b = o.get("b") if o.get("b") is not None else torch.empty(n_groups, dtype=torch.float32, device=dev)
+    c = None
+    if codes:
+        c = o.get("codes") if o.get("codes") is not None else torch.empty((rows, cols), dtype=torch.uint8, device=dev)
+    k = None
+    if cand_idx:
+        k = o.get("cand_idx") if o.get("cand_idx") is not None else torch.empty(n_groups, dtype=torch.uint8, device=dev)
+    _check(quasar_recon_int(w, g, v, beta2, bits, group_size, clip, rows, cols, r, c, a, b, k,
+                            stream=stream))
+    res = {"r": r, "a": a, "b": b}
+    if c is not None:
+        res["codes"] = c
+    if k is not None:
+        res["cand_idx"] = k
+    return res
+
+
+def recon_nvfp4(w, g, v, *, clip, beta2=0.999, tensor_amax=None, r_dtype=torch.bfloat16,
+                codes=True, cand_idx=True, stream=None, out=None):
+    """QUASAR NVFP4 reconstruction of one tensor; v is updated in place."""
+    _check_2d(w)
+    rows, cols = w.shape
+    dev = w.device
+    n_blocks = rows * cols // 16
+    o = out if out is not None else {}
+    r = o.get("r") if o.get("r") is not None else torch.empty((rows, cols), dtype=r_dtype, device=dev)
+    sc = o.get("block_scale") if o.get("block_scale") is not None else torch.empty(n_blocks, dtype=torch.uint8, device=dev)
+    ts = o.get("tensor_scale") if o.get("tensor_scale") is not None else torch.empty(1, dtype=torch.float32, device=dev)
+    c = None
+    if codes:
+        c = o.get("codes") if o.get("codes") is not None else torch.empty((rows, cols), dtype=torch.uint8, device=dev)
+    k = None
+    if cand_idx:
+        k = o.get("cand_idx") if o.get("cand_idx") is not None else torch.empty(n_blocks, dtype=torch.uint8, device=dev)
+    _check(quasar_recon_nvfp4(w, g, v, beta2, clip, rows, cols, tensor_amax, r, c, sc, ts, k,
+                              stream=stream))
+    res = {"r": r, "block_scale": sc, "tensor_scale": ts}
+    if c is not None:
+        res["codes"] = c
+    if k is not None:
+        res["cand_idx"] = k
+    return res
+
+
+def tensor_amax(w, stream=None):
+    out = torch.empty(1, dtype=torch.float32, device=w.device)
+    _check(quasar_tensor_amax(w, w.numel(), out, stream=stream))
+    return out

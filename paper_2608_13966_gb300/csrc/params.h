@@ -1,0 +1,73 @@
+// Launch parameters of the QUASAR kernels (shared by host and device code).
+#pragma once
+
+#include <cstdint>
+
+namespace quasar {
+
+// Bit set in the per-device status word when a kernel gives up on a wait.
+constexpr unsigned kStatusTimeout = 1u;
+
+constexpr int kLanesPerGroup = 8;
+constexpr int kGroupsPerUnit = 4;
+constexpr int kMaxClip = 32;
+
+struct IntParams {
+    const float* w;
+    const void* g;
+    float* v;
+    void* r;
+    uint8_t* codes;
+    float* a;
+    float* b;
+    uint8_t* idx;
+    int64_t n_groups;
+    int g_kind;  // 0 none, 1 fp32, 2 bf16
+    int r_bf16;
+    int qmax;
+    int n_clip;
+    float beta2;
+    float c1;  // 1 - beta2
+    float tie_kappa;   // multiplier of the fp32 unit roundoff in the tie bound
+    float refit_cond;  // refit the kept candidate in two passes above this
+    int stages;
+    uint32_t stage_bytes;
+    uint64_t timeout_ns;
+    uint64_t force_timeout_ns;
+    unsigned int* status;  // per-device status word
+    unsigned int* stats;  // optional: [0] refined groups, [1] refitted groups
+    float f[kMaxClip];     // padded with the last factor
+    float invf[kMaxClip];  // fl32(1/f)
+};
+
+constexpr int kBlocksPerUnit = 32;
+
+struct Nvfp4Params {
+    const float* w;
+    const void* g;
+    float* v;
+    void* r;
+    uint8_t* codes;
+    uint8_t* scale;
+    uint8_t* idx;
+    const float* amax;     // device scalar (caller's, or the tensor_scale slot)
+    float* tensor_scale;   // written by block 0 when write_scale != 0
+    int write_scale;
+    int64_t n_blocks;
+    int g_kind;
+    int r_bf16;
+    int n_clip;
+    float beta2;
+    float c1;
+    float tie_kappa;
+    int stages;
+    uint32_t stage_bytes;
+    uint64_t timeout_ns;
+    uint64_t force_timeout_ns;
+    unsigned int* status;  // per-device status word
+    unsigned int* stats;
+    float f[kMaxClip];
+    float invf[kMaxClip];
+};
+
+}  // namespace quasar

@@ -1,0 +1,443 @@
+// C ABI of the QUASAR reconstruction library: argument validation, kernel
+// selection and launch configuration.  Declarations and contracts are in
+// include/quasar.h.
+#include <cuda_runtime.h>
+
+#include <algorithm>
+#include <atomic>
+#include <cmath>
+#include <cstdint>
+#include <cstdlib>
+#include <cstring>
+#include <mutex>
+
+#include "params.h"
+#include "quasar.h"
+
+namespace quasar {
+const void* int_kernel_nch1(int epl);
+const void* int_kernel_nch2(int epl);
+const void* int_kernel_nch4(int epl);
+const void* nvfp4_kernel(int nch);
+const void* amax_kernel();
+const void* amax_to_scale_kernel();
+}  // namespace quasar
+
+// Per-device status word (bit 0: a kernel timed out on a wait).
+__device__ unsigned int g_quasar_status_word;
+
+namespace {
+
+using namespace quasar;
+
+constexpr int kThreads = 256;
+constexpr int kWarps = kThreads / 32;
+constexpr uint64_t kDefaultTimeoutNs = 1000000000ull;  // 1 s per wait
+
+std::atomic<int64_t> g_force_timeout_ns{0};
+std::atomic<unsigned int*> g_stats{nullptr};
+
+struct Tuning {
+    int stages = 0;            // 0: chosen from the shared-memory budget
+    int smem_budget = 100 * 1024;
+    float tie_kappa = 16.0f;
+    float refit_cond = 8.0f;
+};
+
+const Tuning& tuning()
+{
+    static const Tuning t = [] {
+        Tuning x;
+        if (const char* s = std::getenv("QUASAR_STAGES")) x.stages = std::atoi(s);
+        if (const char* s = std::getenv("QUASAR_SMEM_BUDGET")) x.smem_budget = std::atoi(s);
+        if (const char* s = std::getenv("QUASAR_TIE_KAPPA")) x.tie_kappa = (float)std::atof(s);
+        if (const char* s = std::getenv("QUASAR_REFIT_COND")) x.refit_cond = (float)std::atof(s);
+        return x;
+    }();
+    return t;
+}
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+bool overlaps(const void* a, size_t na, const void* b, size_t nb)
+{
+    if (!a || !b || na == 0 || nb == 0) return false;
+    const uintptr_t x = reinterpret_cast<uintptr_t>(a), y = reinterpret_cast<uintptr_t>(b);
+    return x < y + nb && y < x + na;
+}
+
+size_t dtype_size(quasar_dtype d) { return d == QUASAR_BF16 ? 2 : 4; }
+
+bool valid_dtype(quasar_dtype d) { return d == QUASAR_F32 || d == QUASAR_BF16; }
+
+// Checks shared by both reconstruction entry points.  On success fills n.
+quasar_status check_common(const float* w, const void* g, quasar_dtype g_dtype, const float* v,
+                           float beta2, const float* clip, int n_clip, int64_t rows, int64_t cols,
+                           const void* r, quasar_dtype r_dtype, int64_t* n)
+{
+    if (rows < 0 || cols < 0) return QUASAR_ERR_INVALID_ARG;
+    if (rows != 0 && cols > (int64_t(1) << 62) / rows) return QUASAR_ERR_INVALID_ARG;
+    *n = rows * cols;
+    if (!(beta2 >= 0.0f && beta2 < 1.0f)) return QUASAR_ERR_INVALID_ARG;
+    if (!clip || n_clip < 1 || n_clip > kMaxClip) return QUASAR_ERR_INVALID_ARG;
+    for (int k = 0; k < n_clip; ++k)
+        if (!(clip[k] > 0.0f && clip[k] <= 1.0f)) return QUASAR_ERR_INVALID_ARG;
+    if (!valid_dtype(r_dtype) || (g && !valid_dtype(g_dtype))) return QUASAR_ERR_INVALID_ARG;
+    if (*n == 0) return QUASAR_OK;
+    if (!w || !v || !r) return QUASAR_ERR_INVALID_ARG;
+    if (!aligned16(w) || !aligned16(v) || !aligned16(r) || (g && !aligned16(g)))
+        return QUASAR_ERR_INVALID_ARG;
+    return QUASAR_OK;
+}
+
+// Output byte ranges must not overlap w, g or v.
+bool outputs_alias_inputs(const float* w, const void* g, quasar_dtype g_dtype, const float* v,
+                          int64_t n, const void* const* outs, const size_t* out_bytes, int n_out)
+{
+    const size_t nb = (size_t)n;
+    for (int i = 0; i < n_out; ++i) {
+        if (overlaps(outs[i], out_bytes[i], w, nb * 4)) return true;
+        if (overlaps(outs[i], out_bytes[i], v, nb * 4)) return true;
+        if (g && overlaps(outs[i], out_bytes[i], g, nb * dtype_size(g_dtype))) return true;
+    }
+    return false;
+}
+
+void fill_clip(const float* clip, int n_clip, float* f, float* invf)
+{
+    for (int k = 0; k < kMaxClip; ++k) {
+        const float fk = clip[std::min(k, n_clip - 1)];
+        f[k] = fk;
+        invf[k] = (float)(1.0 / (double)fk);
+    }
+}
+
+int nch_for(int n_clip) { return n_clip <= 8 ? 1 : (n_clip <= 16 ? 2 : 4); }
+
+struct Launch {
+    int stages;
+    uint32_t stage_bytes;
+    size_t smem;
+};
+
+Launch plan(uint32_t unit_bytes)
+{
+    const Tuning& t = tuning();
+    Launch L;
+    L.stage_bytes = (unit_bytes + 127u) & ~127u;
+    int s = t.stages;
+    if (s <= 0) {
+        s = 2;
+        while (s < 4 && (size_t)kWarps * (s + 1) * L.stage_bytes + kWarps * (s + 2) * 8 <=
+                            (size_t)t.smem_budget)
+            ++s;
+    }
+    L.stages = s;
+    L.smem = (size_t)kWarps * s * L.stage_bytes + (size_t)kWarps * (s + 1) * 8;
+    return L;
+}
+
+// Per-device facts looked up once: SM count and the status word's address.
+constexpr int kMaxDevices = 64;
+struct DeviceInfo {
+    std::atomic<int> ready{0};
+    int nsm = 0;
+    unsigned int* status = nullptr;
+};
+DeviceInfo g_dev[kMaxDevices];
+std::mutex g_mu;
+
+// Launch configuration of one kernel at one shared-memory size, per device.
+struct KernelConfig {
+    const void* fn = nullptr;
+    size_t smem = 0;
+    int dev = -1;
+    int occupancy = 0;
+};
+constexpr int kMaxConfigs = 256;
+KernelConfig g_cfg[kMaxConfigs];
+int g_ncfg = 0;
+
+quasar_status device_info(int* dev_out, const DeviceInfo** info)
+{
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return QUASAR_ERR_CUDA;
+    if (dev < 0 || dev >= kMaxDevices) return QUASAR_ERR_UNSUPPORTED;
+    DeviceInfo& d = g_dev[dev];
+    if (!d.ready.load(std::memory_order_acquire)) {
+        std::lock_guard<std::mutex> lock(g_mu);
+        if (!d.ready.load(std::memory_order_relaxed)) {
+            void* ptr = nullptr;
+            if (cudaDeviceGetAttribute(&d.nsm, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+                return QUASAR_ERR_CUDA;
+            if (cudaGetSymbolAddress(&ptr, g_quasar_status_word) != cudaSuccess)
+                return QUASAR_ERR_CUDA;
+            d.status = static_cast<unsigned int*>(ptr);
+            d.ready.store(1, std::memory_order_release);
+        }
+    }
+    *dev_out = dev;
+    *info = &d;
+    return QUASAR_OK;
+}
+
+quasar_status status_ptr(unsigned int** p)
+{
+    int dev;
+    const DeviceInfo* info;
+    const quasar_status st = device_info(&dev, &info);
+    if (st != QUASAR_OK) return st;
+    *p = info->status;
+    return QUASAR_OK;
+}
+
+// Resident CTAs per SM for (fn, smem) on device dev.  The kernel's dynamic
+// shared-memory limit only ever grows (to the largest size requested so far),
+// so a configuration cached earlier stays launchable.
+quasar_status occupancy(const void* fn, size_t smem, int dev, int* occ)
+{
+    std::lock_guard<std::mutex> lock(g_mu);
+    size_t limit = 0;
+    for (int i = 0; i < g_ncfg; ++i) {
+        if (g_cfg[i].fn != fn || g_cfg[i].dev != dev) continue;
+        if (g_cfg[i].smem == smem) {
+            *occ = g_cfg[i].occupancy;
+            return QUASAR_OK;
+        }
+        limit = std::max(limit, g_cfg[i].smem);
+    }
+    if (smem > limit &&
+        cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) !=
+            cudaSuccess)
+        return QUASAR_ERR_CUDA;
+    int o = 0;
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&o, fn, kThreads, smem) != cudaSuccess)
+        return QUASAR_ERR_CUDA;
+    if (g_ncfg < kMaxConfigs) g_cfg[g_ncfg++] = KernelConfig{fn, smem, dev, o};
+    *occ = o;
+    return QUASAR_OK;
+}
+
+// Persistent launch: at most (#SMs x resident CTAs) CTAs of 8 warps, no more
+// than there are units of work for the warps.
+quasar_status launch_persistent(const void* fn, void* params, size_t smem, int64_t n_units,
+                                cudaStream_t stream)
+{
+    int dev = 0, occ = 0;
+    const DeviceInfo* info = nullptr;
+    quasar_status st = device_info(&dev, &info);
+    if (st != QUASAR_OK) return st;
+    if ((st = occupancy(fn, smem, dev, &occ)) != QUASAR_OK) return st;
+    if (occ < 1) return QUASAR_ERR_UNSUPPORTED;
+    const int64_t want = (n_units + kWarps - 1) / kWarps;
+    const int grid = (int)std::max<int64_t>(1, std::min<int64_t>((int64_t)info->nsm * occ, want));
+    void* args[] = {params};
+    if (cudaLaunchKernel(fn, dim3(grid), dim3(kThreads), args, smem, stream) != cudaSuccess)
+        return QUASAR_ERR_CUDA;
+    return QUASAR_OK;
+}
+
+int g_kind_of(const void* g, quasar_dtype d) { return !g ? 0 : (d == QUASAR_BF16 ? 2 : 1); }
+
+}  // namespace
+
+extern "C" {
+
+quasar_status quasar_recon_int(const float* w, const void* g, quasar_dtype g_dtype, float* v,
+                               float beta2, int bits, int group_size, const float* clip,
+                               int n_clip, int64_t rows, int64_t cols, void* r,
+                               quasar_dtype r_dtype, uint8_t* codes, float* a, float* b,
+                               uint8_t* cand_idx, quasar_stream_t stream)
+{
+    int64_t n = 0;
+    quasar_status st = check_common(w, g, g_dtype, v, beta2, clip, n_clip, rows, cols, r, r_dtype, &n);
+    if (st != QUASAR_OK) return st;
+    if (bits < 1 || bits > 8) return QUASAR_ERR_INVALID_ARG;
+    if (group_size <= 0 || cols % group_size != 0) return QUASAR_ERR_INVALID_ARG;
+    if (group_size != 32 && group_size != 64 && group_size != 128 && group_size != 256)
+        return QUASAR_ERR_UNSUPPORTED;
+    if (n == 0) return QUASAR_OK;
+    if (!a || !b) return QUASAR_ERR_INVALID_ARG;
+    if (codes && !aligned16(codes)) return QUASAR_ERR_INVALID_ARG;
+    const int64_t n_groups = n / group_size;
+    {
+        const void* outs[] = {r, codes, a, b, cand_idx};
+        const size_t bytes[] = {(size_t)n * dtype_size(r_dtype), codes ? (size_t)n : 0,
+                                (size_t)n_groups * 4, (size_t)n_groups * 4,
+                                cand_idx ? (size_t)n_groups : 0};
+        if (outputs_alias_inputs(w, g, g_dtype, v, n, outs, bytes, 5)) return QUASAR_ERR_INVALID_ARG;
+    }
+
+    IntParams p{};
+    p.w = w;
+    p.g = g;
+    p.v = v;
+    p.r = r;
+    p.codes = codes;
+    p.a = a;
+    p.b = b;
+    p.idx = cand_idx;
+    p.n_groups = n_groups;
+    p.g_kind = g_kind_of(g, g_dtype);
+    p.r_bf16 = r_dtype == QUASAR_BF16;
+    p.qmax = (1 << bits) - 1;
+    p.n_clip = n_clip;
+    p.beta2 = beta2;
+    p.c1 = 1.0f - beta2;
+    p.tie_kappa = tuning().tie_kappa;
+    p.refit_cond = tuning().refit_cond;
+    p.timeout_ns = kDefaultTimeoutNs;
+    p.force_timeout_ns = (uint64_t)std::max<int64_t>(0, g_force_timeout_ns.load());
+    p.stats = g_stats.load();
+    fill_clip(clip, n_clip, p.f, p.invf);
+    if ((st = status_ptr(&p.status)) != QUASAR_OK) return st;
+
+    const int gbytes = p.g_kind == 2 ? 2 : (p.g_kind == 1 ? 4 : 0);
+    const Launch L = plan((uint32_t)(kGroupsPerUnit * group_size * (8 + gbytes)));
+    p.stages = L.stages;
+    p.stage_bytes = L.stage_bytes;
+
+    const int epl = group_size / kLanesPerGroup;
+    const int nch = nch_for(n_clip);
+    const void* fn = nch == 1 ? int_kernel_nch1(epl) : (nch == 2 ? int_kernel_nch2(epl) : int_kernel_nch4(epl));
+    if (!fn) return QUASAR_ERR_UNSUPPORTED;
+    const int64_t n_units = (n_groups + kGroupsPerUnit - 1) / kGroupsPerUnit;
+    return launch_persistent(fn, &p, L.smem, n_units, reinterpret_cast<cudaStream_t>(stream));
+}
+
+quasar_status quasar_tensor_amax(const float* w, int64_t n, float* amax_out, quasar_stream_t stream)
+{
+    if (n < 0 || !amax_out) return QUASAR_ERR_INVALID_ARG;
+    if (n > 0 && (!w || !aligned16(w))) return QUASAR_ERR_INVALID_ARG;
+    if ((reinterpret_cast<uintptr_t>(amax_out) & 3u) != 0) return QUASAR_ERR_INVALID_ARG;
+    cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+    if (cudaMemsetAsync(amax_out, 0, sizeof(float), s) != cudaSuccess) return QUASAR_ERR_CUDA;
+    if (n == 0) return QUASAR_OK;
+    int dev = 0;
+    const DeviceInfo* info = nullptr;
+    const quasar_status st = device_info(&dev, &info);
+    if (st != QUASAR_OK) return st;
+    const int64_t want = (n / 4 + kThreads - 1) / kThreads;
+    const int grid = (int)std::max<int64_t>(1, std::min<int64_t>((int64_t)info->nsm * 8, want));
+    unsigned int* out = reinterpret_cast<unsigned int*>(amax_out);
+    void* args[] = {(void*)&w, (void*)&n, (void*)&out};
+    if (cudaLaunchKernel(amax_kernel(), dim3(grid), dim3(kThreads), args, 0, s) != cudaSuccess)
+        return QUASAR_ERR_CUDA;
+    return QUASAR_OK;
+}
+
+quasar_status quasar_recon_nvfp4(const float* w, const void* g, quasar_dtype g_dtype, float* v,
+                                 float beta2, const float* clip, int n_clip, int64_t rows,
+                                 int64_t cols, const float* tensor_amax, void* r,
+                                 quasar_dtype r_dtype, uint8_t* codes, uint8_t* block_scale,
+                                 float* tensor_scale, uint8_t* cand_idx, quasar_stream_t stream)
+{
+    int64_t n = 0;
+    quasar_status st = check_common(w, g, g_dtype, v, beta2, clip, n_clip, rows, cols, r, r_dtype, &n);
+    if (st != QUASAR_OK) return st;
+    if (cols % 16 != 0) return QUASAR_ERR_INVALID_ARG;
+    if (!tensor_scale || (reinterpret_cast<uintptr_t>(tensor_scale) & 3u) != 0)
+        return QUASAR_ERR_INVALID_ARG;
+    if (tensor_amax && (reinterpret_cast<uintptr_t>(tensor_amax) & 3u) != 0)
+        return QUASAR_ERR_INVALID_ARG;
+    const int64_t n_blocks = n / 16;
+    if (n > 0) {
+        if (!block_scale) return QUASAR_ERR_INVALID_ARG;
+        if (codes && !aligned16(codes)) return QUASAR_ERR_INVALID_ARG;
+        const void* outs[] = {r, codes, block_scale, tensor_scale, cand_idx};
+        const size_t bytes[] = {(size_t)n * dtype_size(r_dtype), codes ? (size_t)n : 0,
+                                (size_t)n_blocks, 4, cand_idx ? (size_t)n_blocks : 0};
+        if (outputs_alias_inputs(w, g, g_dtype, v, n, outs, bytes, 5)) return QUASAR_ERR_INVALID_ARG;
+        if (tensor_amax && overlaps(tensor_amax, 4, tensor_scale, 4)) return QUASAR_ERR_INVALID_ARG;
+    }
+    cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+    if (n == 0) {
+        // empty tensor: amax = 0, so s_T = 1
+        if (cudaMemsetAsync(tensor_scale, 0, sizeof(float), s) != cudaSuccess) return QUASAR_ERR_CUDA;
+        void* args[] = {(void*)&tensor_scale};
+        if (cudaLaunchKernel(amax_to_scale_kernel(), dim3(1), dim3(1), args, 0, s) != cudaSuccess)
+            return QUASAR_ERR_CUDA;
+        return QUASAR_OK;
+    }
+
+    Nvfp4Params p{};
+    p.w = w;
+    p.g = g;
+    p.v = v;
+    p.r = r;
+    p.codes = codes;
+    p.scale = block_scale;
+    p.idx = cand_idx;
+    p.tensor_scale = tensor_scale;
+    p.n_blocks = n_blocks;
+    p.g_kind = g_kind_of(g, g_dtype);
+    p.r_bf16 = r_dtype == QUASAR_BF16;
+    p.n_clip = n_clip;
+    p.beta2 = beta2;
+    p.c1 = 1.0f - beta2;
+    p.tie_kappa = tuning().tie_kappa;
+    p.timeout_ns = kDefaultTimeoutNs;
+    p.force_timeout_ns = (uint64_t)std::max<int64_t>(0, g_force_timeout_ns.load());
+    p.stats = g_stats.load();
+    fill_clip(clip, n_clip, p.f, p.invf);
+    if ((st = status_ptr(&p.status)) != QUASAR_OK) return st;
+
+    if (tensor_amax) {
+        p.amax = tensor_amax;
+        p.write_scale = 1;
+    } else {
+        // amax is accumulated in the tensor_scale slot, then converted.
+        if ((st = quasar_tensor_amax(w, n, tensor_scale, stream)) != QUASAR_OK) return st;
+        p.amax = tensor_scale;
+        p.write_scale = 0;
+    }
+
+    const int gbytes = p.g_kind == 2 ? 2 : (p.g_kind == 1 ? 4 : 0);
+    const Launch L = plan((uint32_t)(kBlocksPerUnit * 16 * (8 + gbytes)));
+    p.stages = L.stages;
+    p.stage_bytes = L.stage_bytes;
+    const void* fn = nvfp4_kernel(nch_for(n_clip));
+    if (!fn) return QUASAR_ERR_UNSUPPORTED;
+    const int64_t n_units = (n_blocks + kBlocksPerUnit - 1) / kBlocksPerUnit;
+    if ((st = launch_persistent(fn, &p, L.smem, n_units, s)) != QUASAR_OK) return st;
+    if (!tensor_amax) {
+        void* args[] = {(void*)&tensor_scale};
+        if (cudaLaunchKernel(amax_to_scale_kernel(), dim3(1), dim3(1), args, 0, s) != cudaSuccess)
+            return QUASAR_ERR_CUDA;
+    }
+    return QUASAR_OK;
+}
+
+quasar_status quasar_get_device_status(quasar_stream_t stream)
+{
+    if (cudaStreamSynchronize(reinterpret_cast<cudaStream_t>(stream)) != cudaSuccess)
+        return QUASAR_ERR_CUDA;
+    unsigned int word = 0;
+    if (cudaMemcpyFromSymbol(&word, g_quasar_status_word, sizeof(word)) != cudaSuccess)
+        return QUASAR_ERR_CUDA;
+    if (word == 0) return QUASAR_OK;
+    const unsigned int zero = 0;
+    if (cudaMemcpyToSymbol(g_quasar_status_word, &zero, sizeof(zero)) != cudaSuccess)
+        return QUASAR_ERR_CUDA;
+    return (word & kStatusTimeout) ? QUASAR_ERR_TIMEOUT : QUASAR_OK;
+}
+
+void quasar_debug_force_timeout(int64_t nanoseconds) { g_force_timeout_ns.store(nanoseconds); }
+
+void quasar_debug_set_stats(unsigned int* device_counters) { g_stats.store(device_counters); }
+
+const char* quasar_status_string(quasar_status status)
+{
+    switch (status) {
+    case QUASAR_OK: return "QUASAR_OK";
+    case QUASAR_ERR_INVALID_ARG: return "QUASAR_ERR_INVALID_ARG";
+    case QUASAR_ERR_UNSUPPORTED: return "QUASAR_ERR_UNSUPPORTED";
+    case QUASAR_ERR_CUDA: return "QUASAR_ERR_CUDA";
+    case QUASAR_ERR_TIMEOUT: return "QUASAR_ERR_TIMEOUT";
+    default: return "QUASAR_ERR_UNKNOWN";
+    }
+}
+
+int quasar_version(void) { return 100; }
+
+}  // extern "C"

@@ -1,0 +1,160 @@
+"""ctypes binding of ``libquasar.so`` (declared in ``include/quasar.h``).
+
+Functions carry the C names and only marshal arguments: tensors become
+device pointers, the clip list becomes a host float array, the stream
+becomes its ``cudaStream_t`` handle.  Every step of the reconstruction runs
+in the library's CUDA kernels; there is no Python or CPU fallback, and the
+module raises at import-time use if the library cannot be loaded.
+"""
+from __future__ import annotations
+
+import ctypes
+import enum
+import os
+import threading
+
+from . import build as _build
+
+_lib = None
+_lock = threading.Lock()
+
+
+class QuasarStatus(enum.IntEnum):
+    OK = 0
+    ERR_INVALID_ARG = 1
+    ERR_UNSUPPORTED = 2
+    ERR_CUDA = 3
+    ERR_TIMEOUT = 4
+
+
+class QuasarError(RuntimeError):
+    def __init__(self, status):
+        self.status = QuasarStatus(status)
+        super().__init__(quasar_status_string(status))
+
+
+F32, BF16 = 0, 1
+
+# Every function declared in include/quasar.h, with its ctypes prototype.
+_P, _I, _I64, _F = ctypes.c_void_p, ctypes.c_int, ctypes.c_int64, ctypes.c_float
+PROTOTYPES = {
+    "quasar_recon_int": (_I, [_P, _P, _I, _P, _F, _I, _I, _P, _I, _I64, _I64, _P, _I, _P, _P, _P,
+                              _P, _P]),
+    "quasar_recon_nvfp4": (_I, [_P, _P, _I, _P, _F, _P, _I, _I64, _I64, _P, _P, _I, _P, _P, _P,
+                                _P, _P]),
+    "quasar_tensor_amax": (_I, [_P, _I64, _P, _P]),
+    "quasar_get_device_status": (_I, [_P]),
+    "quasar_debug_force_timeout": (None, [_I64]),
+    "quasar_debug_set_stats": (None, [_P]),
+    "quasar_status_string": (ctypes.c_char_p, [_I]),
+    "quasar_version": (_I, []),
+}
+
+
+def library_path() -> str:
+    return _build.LIB
+
+
+def load(build_if_missing: bool = True):
+    """Load libquasar.so (building it first if asked and needed)."""
+    global _lib
+    with _lock:
+        if _lib is not None:
+            return _lib
+        path = _build.LIB
+        if build_if_missing:
+            path = _build.build()
+        if not os.path.exists(path):
+            raise OSError(f"libquasar.so not found at {path}; run paper_2608_13966_gb300.build")
+        lib = ctypes.CDLL(path)
+        for name, (res, args) in PROTOTYPES.items():
+            fn = getattr(lib, name)
+            fn.restype = res
+            fn.argtypes = args
+        _lib = lib
+        return lib
+
+
+def _ptr(x):
+    """Device pointer of a tensor, an int, or None."""
+    if x is None:
+        return None
+    if isinstance(x, int):
+        return x
+    return x.data_ptr()
+
+
+def _dtype_code(t, default=F32):
+    if t is None:
+        return default
+    if isinstance(t, int):
+        return default
+    import torch
+    if t.dtype == torch.bfloat16:
+        return BF16
+    if t.dtype == torch.float32:
+        return F32
+    raise TypeError(f"unsupported dtype {t.dtype}")
+
+
+def _stream(stream):
+    if stream is None:
+        import torch
+        return torch.cuda.current_stream().cuda_stream
+    if isinstance(stream, int):
+        return stream
+    return stream.cuda_stream
+
+
+def _clip_array(clip):
+    arr = (ctypes.c_float * len(clip))(*[float(c) for c in clip])
+    return arr, len(clip)
+
+
+def quasar_recon_int(w, g, v, beta2, bits, group_size, clip, rows, cols, r, codes, a, b,
+                     cand_idx=None, stream=None, g_dtype=None, r_dtype=None) -> QuasarStatus:
+    lib = load()
+    carr, nclip = _clip_array(clip)
+    gd = g_dtype if g_dtype is not None else _dtype_code(g)
+    rd = r_dtype if r_dtype is not None else _dtype_code(r)
+    st = lib.quasar_recon_int(_ptr(w), _ptr(g), gd, _ptr(v), beta2, bits, group_size, carr, nclip,
+                              rows, cols, _ptr(r), rd, _ptr(codes), _ptr(a), _ptr(b),
+                              _ptr(cand_idx), _stream(stream))
+    return QuasarStatus(st)
+
+
+def quasar_recon_nvfp4(w, g, v, beta2, clip, rows, cols, tensor_amax, r, codes, block_scale,
+                       tensor_scale, cand_idx=None, stream=None, g_dtype=None,
+                       r_dtype=None) -> QuasarStatus:
+    lib = load()
+    carr, nclip = _clip_array(clip)
+    gd = g_dtype if g_dtype is not None else _dtype_code(g)
+    rd = r_dtype if r_dtype is not None else _dtype_code(r)
+    st = lib.quasar_recon_nvfp4(_ptr(w), _ptr(g), gd, _ptr(v), beta2, carr, nclip, rows, cols,
+                                _ptr(tensor_amax), _ptr(r), rd, _ptr(codes), _ptr(block_scale),
+                                _ptr(tensor_scale), _ptr(cand_idx), _stream(stream))
+    return QuasarStatus(st)
+
+
+def quasar_tensor_amax(w, n, amax_out, stream=None) -> QuasarStatus:
+    return QuasarStatus(load().quasar_tensor_amax(_ptr(w), n, _ptr(amax_out), _stream(stream)))
+
+
+def quasar_get_device_status(stream=None) -> QuasarStatus:
+    return QuasarStatus(load().quasar_get_device_status(_stream(stream)))
+
+
+def quasar_debug_force_timeout(nanoseconds: int) -> None:
+    load().quasar_debug_force_timeout(int(nanoseconds))
+
+
+def quasar_debug_set_stats(counters) -> None:
+    load().quasar_debug_set_stats(_ptr(counters))
+
+
+def quasar_status_string(status) -> str:
+    return load().quasar_status_string(int(status)).decode()
+
+
+def quasar_version() -> int:
+    return int(load().quasar_version())

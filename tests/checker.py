@@ -1,0 +1,287 @@
+"""Parity checker: CUDA outputs against the fp64 oracle.
+
+Acceptance (stated for the reconstruction in the design notes):
+
+* EMA state v' and, for fp32 outputs, r, a, b: |x - ref| <= 1e-7 + 1e-5 |ref|.
+* bf16 r: equals the round-to-nearest-even bf16 of the oracle's fp64 value,
+  unless that value lies within 1e-7 + 1e-5 |ref| of a bf16 rounding midpoint
+  (then either neighbour is accepted).
+* Codes and the chosen candidate index are bit-exact, except in groups where
+  the oracle's margin to a rounding boundary (code margin relative to the
+  clipping range; E2M1/E4M3 margins relative to the boundary) or its
+  candidate-error tie margin is below 1e-6.  An exempt group passes if
+  (i) its codes differ from the oracle's codes for the GPU's candidate only at
+  elements whose margin is below 1e-6, (ii) the fp64 error of the GPU's
+  reconstruction is within 1e-6 (relative) of the oracle's best, and
+  (iii) its a, b (or E4M3 scale) and r match the fp64 fit of its own codes.
+"""
+from __future__ import annotations
+
+import numpy as np
+
+TOL_ABS = 1e-7
+TOL_REL = 1e-5
+MARGIN = 1e-6
+
+
+def close(x, ref, abs_=TOL_ABS, rel=TOL_REL):
+    x = np.asarray(x, np.float64)
+    ref = np.asarray(ref, np.float64)
+    return np.abs(x - ref) <= abs_ + rel * np.abs(ref)
+
+
+def _bf16_rne(x):
+    """Round-to-nearest-even of fp64 values to bf16 (through fp32), as floats."""
+    x32 = np.asarray(x, np.float64).astype(np.float32)
+    bits = x32.view(np.uint32).astype(np.uint64)
+    bits = (bits + np.uint64(0x7FFF) + ((bits >> np.uint64(16)) & np.uint64(1))) & np.uint64(0xFFFF0000)
+    return bits.astype(np.uint32).view(np.float32).astype(np.float64)
+
+
+def bf16_ok(r_ref, r_gpu):
+    """Elementwise acceptance of bf16 outputs (given as floats): the GPU value
+    must be the bf16 rounding of some value within the fp32 tolerance band
+    around the oracle's value.  Away from zero the band is far narrower than
+    a bf16 step, so this is the nearest-even bf16 of the oracle's value unless
+    that value sits within the tolerance of a rounding midpoint."""
+    r_ref = np.asarray(r_ref, np.float64)
+    g = np.asarray(r_gpu, np.float64)
+    tol = TOL_ABS + TOL_REL * np.abs(r_ref)
+    lo = _bf16_rne(r_ref - tol)
+    hi = _bf16_rne(r_ref + tol)
+    return (g >= lo) & (g <= hi)
+
+
+def r_ok(r_ref, r_gpu, r_is_bf16):
+    return bf16_ok(r_ref, r_gpu) if r_is_bf16 else close(r_gpu, r_ref)
+
+
+def _report(kind, n, exempt, fails, examples=None):
+    rep = {"kind": kind, "units": int(n), "exempt": int(exempt)}
+    rep.update({k: int(v) for k, v in fails.items()})
+    rep["ok"] = all(v == 0 for v in fails.values())
+    if examples:
+        rep["examples"] = examples[:8]
+    return rep
+
+
+def _example(examples, **kw):
+    if len(examples) < 8:
+        examples.append({k: (v.tolist() if hasattr(v, "tolist") else v) for k, v in kw.items()})
+
+
+def check_ema(v_ref, v_gpu):
+    bad = ~close(v_gpu, v_ref)
+    return _report("ema", np.asarray(v_ref).size, 0, {"fail_v": np.count_nonzero(bad)})
+
+
+def _codes_from_r(r, a, b, qmax):
+    with np.errstate(divide="ignore", invalid="ignore"):
+        q = np.rint((np.asarray(r, np.float64) - b) / a)
+    return np.clip(np.nan_to_num(q), 0, qmax).astype(np.uint8)
+
+
+def _flips(q, margin, t, qmax, limit=4):
+    """Code vectors reachable by rounding the elements within MARGIN of a
+    decision boundary j + 1/2 to its other side (at most 2^limit of them)."""
+    idx = np.flatnonzero(margin < MARGIN)[:limit]
+    out = []
+    for mask in range(1, 1 << len(idx)):
+        qq = q.astype(np.int64).copy()
+        for b, i in enumerate(idx):
+            if mask >> b & 1:
+                j = int(min(max(np.floor(t[i]), 0), qmax - 1))
+                qq[i] = 2 * j + 1 - qq[i]
+        out.append(qq.astype(np.uint8))
+    return out
+
+
+def _alt_best_int(oracle, wg, hg, bits, clip, O, g):
+    """Largest error the kept candidate of the oracle can show when its
+    boundary elements are rounded the other way: a GPU that picked another
+    candidate is accepted if it is no worse than that."""
+    qmax = (1 << bits) - 1
+    k = int(O["idx"][g])
+    q, margin, t = oracle.codes_int(wg, bits, float(clip[k]), with_t=True)
+    worst = float(O["err"][g])
+    for qq in _flips(q, margin, t, qmax):
+        worst = max(worst, oracle.refit_int(wg, hg, qq, bits, float(clip[k]))[2])
+    return worst
+
+
+def check_int(oracle, w, h, bits, clip, O, gpu, group_size, r_is_bf16):
+    """w, h: fp32 flat host arrays (h = the oracle's saliency).  O: output of
+    oracle.recon_int.  gpu: dict with r (float array), a, b, and optionally
+    codes and idx (host numpy)."""
+    G = group_size
+    qmax = (1 << bits) - 1
+    n = w.size // G
+    exempt = (O["m_round"] < MARGIN) | (O["m_tie"] < MARGIN)
+    ne = ~exempt
+    fails = {"fail_idx": 0, "fail_codes": 0, "fail_a": 0, "fail_b": 0, "fail_r": 0,
+             "fail_exempt": 0}
+
+    r_ref = O["r"].reshape(n, G)
+    r_gpu = np.asarray(gpu["r"], np.float64).reshape(n, G)
+    a_gpu = np.asarray(gpu["a"], np.float64)
+    b_gpu = np.asarray(gpu["b"], np.float64)
+    if gpu.get("idx") is not None:
+        fails["fail_idx"] = np.count_nonzero((gpu["idx"].astype(np.int64) != O["idx"]) & ne)
+    if gpu.get("codes") is not None:
+        cg = gpu["codes"].reshape(n, G)
+        fails["fail_codes"] = np.count_nonzero(np.any(cg != O["codes"].reshape(n, G), axis=1) & ne)
+    fails["fail_a"] = np.count_nonzero(~close(a_gpu, O["a"]) & ne)
+    fails["fail_b"] = np.count_nonzero(~close(b_gpu, O["b"]) & ne)
+    rok = r_ok(r_ref, r_gpu, r_is_bf16).all(axis=1)
+    fails["fail_r"] = np.count_nonzero(~rok & ne)
+
+    wg = w.reshape(n, G)
+    hg = h.reshape(n, G)
+    ex = []
+    bad = ~close(a_gpu, O["a"]) | ~close(b_gpu, O["b"]) | ~rok
+    if gpu.get("idx") is not None:
+        bad |= gpu["idx"].astype(np.int64) != O["idx"]
+    for g in np.flatnonzero(bad & ne)[:8]:
+        _example(ex, group=int(g), idx_ref=int(O["idx"][g]),
+                 idx_gpu=None if gpu.get("idx") is None else int(gpu["idx"][g]),
+                 a_ref=float(O["a"][g]), a_gpu=float(a_gpu[g]), b_ref=float(O["b"][g]),
+                 b_gpu=float(b_gpu[g]), r_bad=int(np.count_nonzero(~r_ok(r_ref[g], r_gpu[g], r_is_bf16))),
+                 m_round=float(O["m_round"][g]), m_tie=float(O["m_tie"][g]),
+                 cand_err=O["cand_err"][g], err=float(O["err"][g]))
+    for g in np.flatnonzero(exempt):
+        if gpu.get("idx") is not None:
+            k = int(gpu["idx"][g])
+        else:
+            k = int(O["idx"][g])
+        if not 0 <= k < len(clip):
+            fails["fail_exempt"] += 1
+            continue
+        f = float(clip[k])
+        if gpu.get("codes") is not None:
+            cg = gpu["codes"].reshape(n, G)[g]
+        else:
+            cg = _codes_from_r(r_gpu[g], a_gpu[g], b_gpu[g], qmax)
+        q_ref, margin = oracle.codes_int(wg[g], bits, f)
+        diff = cg != q_ref
+        ok = bool(np.all(margin[diff] < MARGIN))
+        s, z, e = oracle.refit_int(wg[g], hg[g], cg, bits, f)
+        if k != int(O["idx"][g]):
+            ok &= e <= _alt_best_int(oracle, wg[g], hg[g], bits, clip, O, g) * (1 + MARGIN) + 1e-300
+        ok &= bool(close(a_gpu[g], s)) and bool(close(b_gpu[g], z))
+        ok &= bool(r_ok(s * cg.astype(np.float64) + z, r_gpu[g], r_is_bf16).all())
+        if not ok:
+            fails["fail_exempt"] += 1
+            _example(ex, exempt_group=int(g), k=k, idx_ref=int(O["idx"][g]),
+                     n_diff=int(diff.sum()), max_margin_diff=float(margin[diff].max()) if diff.any() else 0.0,
+                     refit_err=e, err_ref=float(O["err"][g]), a_gpu=float(a_gpu[g]), a_fit=s,
+                     b_gpu=float(b_gpu[g]), b_fit=z, m_round=float(O["m_round"][g]),
+                     m_tie=float(O["m_tie"][g]))
+    return _report("int", n, np.count_nonzero(exempt), fails, ex)
+
+
+def _nibble_value(c):
+    mags = np.array([0.0, 0.5, 1.0, 1.5, 2.0, 3.0, 4.0, 6.0])
+    c = np.asarray(c, np.int64)
+    v = mags[c & 7]
+    return np.where(c & 8, -v, v)
+
+
+def _nibbles_from_r(r, alpha):
+    mags = np.array([0.0, 0.5, 1.0, 1.5, 2.0, 3.0, 4.0, 6.0])
+    if alpha == 0:
+        return np.zeros(np.asarray(r).shape, np.uint8)
+    y = np.asarray(r, np.float64) / alpha
+    m = np.argmin(np.abs(np.abs(y)[:, None] - mags[None, :]), axis=1)
+    neg = (y < 0) & (m != 0)
+    return ((neg.astype(np.int64) << 3) | m).astype(np.uint8)
+
+
+_E2M1 = np.array([0.0, 0.5, 1.0, 1.5, 2.0, 3.0, 4.0, 6.0])
+
+
+def _alt_best_nvfp4(oracle, wb, hb, s_T, clip, O, blk, limit=4):
+    """As _alt_best_int for NVFP4: the oracle's kept candidate with its
+    elements near an E2M1 boundary rounded to the other side, scale refitted."""
+    k = int(O["idx"][blk])
+    f = float(clip[k])
+    q, margin, y = oracle.codes_nvfp4(wb, f, with_y=True)
+    worst = float(O["err"][blk])
+    idx = np.flatnonzero(margin < MARGIN)[:limit]
+    mids = 0.5 * (_E2M1[:-1] + _E2M1[1:])
+    for mask in range(1, 1 << len(idx)):
+        qq = q.astype(np.int64).copy()
+        for b, i in enumerate(idx):
+            if mask >> b & 1:
+                j = int(np.argmin(np.abs(mids - min(y[i], 6.0))))
+                mag = 2 * j + 1 - (qq[i] & 7)
+                neg = (wb[i] < 0) and mag != 0
+                qq[i] = (int(neg) << 3) | mag
+        qq = qq.astype(np.uint8)
+        e, _ = oracle.fit_nvfp4_scale(wb, hb, float(s_T), f, qq)
+        worst = max(worst, oracle.eval_nvfp4(wb, hb, float(s_T), qq, e))
+    return worst
+
+
+def check_nvfp4(oracle, w, h, clip, s_T, O, gpu, r_is_bf16):
+    """NVFP4 blocks.  gpu: r, scale, tensor_scale and optionally codes, idx."""
+    n = w.size // 16
+    exempt = (O["m_round"] < MARGIN) | (O["m_scale"] < MARGIN) | (O["m_tie"] < MARGIN)
+    ne = ~exempt
+    fails = {"fail_tensor_scale": 0, "fail_idx": 0, "fail_codes": 0, "fail_scale": 0,
+             "fail_r": 0, "fail_exempt": 0}
+    fails["fail_tensor_scale"] = int(np.float32(gpu["tensor_scale"]) != np.float32(s_T))
+    if gpu.get("idx") is not None:
+        fails["fail_idx"] = np.count_nonzero((gpu["idx"].astype(np.int64) != O["idx"]) & ne)
+    if gpu.get("codes") is not None:
+        cg = gpu["codes"].reshape(n, 16)
+        fails["fail_codes"] = np.count_nonzero(np.any(cg != O["codes"].reshape(n, 16), axis=1) & ne)
+    fails["fail_scale"] = np.count_nonzero((gpu["scale"] != O["scale"]) & ne)
+    r_ref = O["r"].reshape(n, 16)
+    r_gpu = np.asarray(gpu["r"], np.float64).reshape(n, 16)
+    rok = r_ok(r_ref, r_gpu, r_is_bf16).all(axis=1)
+    fails["fail_r"] = np.count_nonzero(~rok & ne)
+
+    wb = w.reshape(n, 16)
+    hb = h.reshape(n, 16)
+    ex = []
+    bad = (gpu["scale"] != O["scale"]) | ~rok
+    if gpu.get("idx") is not None:
+        bad |= gpu["idx"].astype(np.int64) != O["idx"]
+    if gpu.get("codes") is not None:
+        bad |= np.any(gpu["codes"].reshape(n, 16) != O["codes"].reshape(n, 16), axis=1)
+    for blk in np.flatnonzero(bad & ne)[:8]:
+        _example(ex, block=int(blk), idx_ref=int(O["idx"][blk]),
+                 idx_gpu=None if gpu.get("idx") is None else int(gpu["idx"][blk]),
+                 scale_ref=int(O["scale"][blk]), scale_gpu=int(gpu["scale"][blk]),
+                 codes_ref=O["codes"].reshape(n, 16)[blk],
+                 codes_gpu=None if gpu.get("codes") is None else gpu["codes"].reshape(n, 16)[blk],
+                 cand_err=O["cand_err"][blk], cand_scale=O["cand_scale"][blk],
+                 m_round=float(O["m_round"][blk]), m_scale=float(O["m_scale"][blk]),
+                 m_tie=float(O["m_tie"][blk]))
+    for blk in np.flatnonzero(exempt):
+        k = int(gpu["idx"][blk]) if gpu.get("idx") is not None else int(O["idx"][blk])
+        if not 0 <= k < len(clip):
+            fails["fail_exempt"] += 1
+            continue
+        f = float(clip[k])
+        e_gpu = int(gpu["scale"][blk])
+        alpha = float(s_T) * oracle.e4m3_value(e_gpu) if e_gpu < 0x7F else float("nan")
+        if gpu.get("codes") is not None:
+            cg = gpu["codes"].reshape(n, 16)[blk]
+        else:
+            cg = _nibbles_from_r(r_gpu[blk], alpha)
+        q_ref, margin = oracle.codes_nvfp4(wb[blk], f)
+        diff = cg != q_ref
+        ok = bool(np.all(margin[diff] < MARGIN))
+        fit, mscale = oracle.fit_nvfp4_scale(wb[blk], hb[blk], float(s_T), f, cg)
+        ok &= (fit == e_gpu) or (mscale < MARGIN)
+        err = oracle.eval_nvfp4(wb[blk], hb[blk], float(s_T), cg, e_gpu)
+        if k != int(O["idx"][blk]):
+            ok &= err <= _alt_best_nvfp4(oracle, wb[blk], hb[blk], s_T, clip, O, blk) * (1 + MARGIN) + 1e-300
+        ok &= bool(r_ok(alpha * _nibble_value(cg), r_gpu[blk], r_is_bf16).all())
+        if not ok:
+            fails["fail_exempt"] += 1
+            _example(ex, exempt_block=int(blk), k=k, idx_ref=int(O["idx"][blk]),
+                     scale_gpu=e_gpu, scale_fit=fit, mscale=mscale, err=err,
+                     err_ref=float(O["err"][blk]), n_diff=int(diff.sum()))
+    return _report("nvfp4", n, np.count_nonzero(exempt), fails, ex)

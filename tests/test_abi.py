@@ -1,0 +1,127 @@
+"""C-ABI checks that need no GPU: the library builds for sm_103a, loads,
+exports every function include/quasar.h declares, and rejects bad arguments
+on the host without launching anything."""
+import ctypes
+import os
+import re
+
+import pytest
+
+from paper_2608_13966_gb300 import build as qbuild
+from paper_2608_13966_gb300 import quasar as Q
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "quasar.h")
+
+# Fake, 16-byte aligned device addresses: validation must reject before use.
+A, B, C, D, E, F = (0x10000000 * (i + 1) for i in range(6))
+CLIP = [1.0, 0.9, 0.8]
+
+
+def declared_functions():
+    text = open(HEADER).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(quasar_\w+)\s*\(", text)))
+
+
+@pytest.fixture(scope="module")
+def lib():
+    qbuild.build()
+    return Q.load(build_if_missing=False)
+
+
+def test_header_and_binding_agree():
+    assert declared_functions() == sorted(Q.PROTOTYPES)
+
+
+def test_library_exports_every_declared_symbol(lib):
+    for name in declared_functions():
+        assert hasattr(lib, name), name
+    assert Q.quasar_version() >= 100
+
+
+def test_status_strings(lib):
+    for st in Q.QuasarStatus:
+        assert Q.quasar_status_string(st) == "QUASAR_" + st.name
+    assert Q.quasar_status_string(99) == "QUASAR_ERR_UNKNOWN"
+
+
+def _int(**kw):
+    args = dict(w=A, g=B, v=C, beta2=0.999, bits=3, group_size=128, clip=CLIP, rows=4,
+                cols=256, r=D, codes=None, a=E, b=F, cand_idx=None, stream=0,
+                g_dtype=Q.BF16, r_dtype=Q.BF16)
+    args.update(kw)
+    return Q.quasar_recon_int(**args)
+
+
+@pytest.mark.parametrize("kw,expect", [
+    (dict(bits=0), Q.QuasarStatus.ERR_INVALID_ARG),
+    (dict(bits=9), Q.QuasarStatus.ERR_INVALID_ARG),
+    (dict(group_size=100, cols=300), Q.QuasarStatus.ERR_UNSUPPORTED),
+    (dict(cols=200), Q.QuasarStatus.ERR_INVALID_ARG),          # cols % group_size
+    (dict(beta2=1.0), Q.QuasarStatus.ERR_INVALID_ARG),
+    (dict(beta2=-0.1), Q.QuasarStatus.ERR_INVALID_ARG),
+    (dict(clip=[]), Q.QuasarStatus.ERR_INVALID_ARG),
+    (dict(clip=[1.0] * 33), Q.QuasarStatus.ERR_INVALID_ARG),
+    (dict(clip=[1.0, 0.0]), Q.QuasarStatus.ERR_INVALID_ARG),
+    (dict(clip=[1.5]), Q.QuasarStatus.ERR_INVALID_ARG),
+    (dict(clip=[float("nan")]), Q.QuasarStatus.ERR_INVALID_ARG),
+    (dict(w=None), Q.QuasarStatus.ERR_INVALID_ARG),
+    (dict(v=None), Q.QuasarStatus.ERR_INVALID_ARG),
+    (dict(r=None), Q.QuasarStatus.ERR_INVALID_ARG),
+    (dict(a=None), Q.QuasarStatus.ERR_INVALID_ARG),
+    (dict(w=A + 4), Q.QuasarStatus.ERR_INVALID_ARG),           # misaligned
+    (dict(g=B + 8), Q.QuasarStatus.ERR_INVALID_ARG),
+    (dict(codes=D + 8), Q.QuasarStatus.ERR_INVALID_ARG),
+    (dict(rows=-1), Q.QuasarStatus.ERR_INVALID_ARG),
+    (dict(rows=1 << 40, cols=1 << 40), Q.QuasarStatus.ERR_INVALID_ARG),
+    (dict(r_dtype=7), Q.QuasarStatus.ERR_INVALID_ARG),
+    (dict(r=A + 512), Q.QuasarStatus.ERR_INVALID_ARG),         # r overlaps w
+    (dict(a=C + 64), Q.QuasarStatus.ERR_INVALID_ARG),          # a overlaps v
+    (dict(cand_idx=B + 16), Q.QuasarStatus.ERR_INVALID_ARG),   # idx overlaps g
+    (dict(rows=0), Q.QuasarStatus.OK),                         # empty: no-op
+])
+def test_int_argument_validation(lib, kw, expect):
+    assert _int(**kw) == expect
+
+
+def _nv(**kw):
+    args = dict(w=A, g=B, v=C, beta2=0.999, clip=CLIP, rows=4, cols=256, tensor_amax=None,
+                r=D, codes=None, block_scale=E, tensor_scale=F, cand_idx=None, stream=0,
+                g_dtype=Q.BF16, r_dtype=Q.BF16)
+    args.update(kw)
+    return Q.quasar_recon_nvfp4(**args)
+
+
+@pytest.mark.parametrize("kw,expect", [
+    (dict(cols=250), Q.QuasarStatus.ERR_INVALID_ARG),
+    (dict(block_scale=None), Q.QuasarStatus.ERR_INVALID_ARG),
+    (dict(tensor_scale=None), Q.QuasarStatus.ERR_INVALID_ARG),
+    (dict(tensor_scale=F + 2), Q.QuasarStatus.ERR_INVALID_ARG),
+    (dict(tensor_amax=F), Q.QuasarStatus.ERR_INVALID_ARG),     # amax aliases tensor_scale
+    (dict(block_scale=A + 16), Q.QuasarStatus.ERR_INVALID_ARG),
+    (dict(beta2=2.0), Q.QuasarStatus.ERR_INVALID_ARG),
+    (dict(clip=[0.5] * 40), Q.QuasarStatus.ERR_INVALID_ARG),
+    (dict(w=A + 4), Q.QuasarStatus.ERR_INVALID_ARG),
+])
+def test_nvfp4_argument_validation(lib, kw, expect):
+    assert _nv(**kw) == expect
+
+
+def test_amax_argument_validation(lib):
+    assert Q.quasar_tensor_amax(A, -1, B, stream=0) == Q.QuasarStatus.ERR_INVALID_ARG
+    assert Q.quasar_tensor_amax(A, 16, None, stream=0) == Q.QuasarStatus.ERR_INVALID_ARG
+    assert Q.quasar_tensor_amax(A + 4, 16, B, stream=0) == Q.QuasarStatus.ERR_INVALID_ARG
+
+
+def test_product_path_has_no_oracle_dependency():
+    """The CUDA library and its binding never reference the oracle."""
+    pkg = os.path.join(ROOT, "paper_2608_13966_gb300")
+    for dirpath, _, files in os.walk(pkg):
+        if "_build" in dirpath:
+            continue
+        for fn in files:
+            if fn.endswith((".py", ".cu", ".cuh", ".h")):
+                text = open(os.path.join(dirpath, fn)).read()
+                assert not re.search(r"^\s*(import|from)\s+oracle\b", text, re.M), fn
+                assert "quasar_oracle" not in text and "qo_" not in text, fn

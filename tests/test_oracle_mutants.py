@@ -43,7 +43,7 @@ MUTANTS = {
     "E4M3 subnormal exponent": ("ldexp((double)m / 8.0, -6)", "ldexp((double)m / 8.0, -7)"),
     "NVFP4 search scale": ("(double)clip[k] * amax_b / 6.0", "(double)clip[k] * amax_b / 4.0"),
     "NVFP4 error at unrounded scale": (
-        "const double alpha = sT * qo_e4m3_value(sk[k]);",
+        "const double alpha = sT * e4m3_tab[sk[k]];",
         "const double alpha = (s2 == 0.0) ? sigma : s3 / s2;"),
     "degenerate step dropped": ("s = step;", "s = 0.0;"),
     "code margin not normalised": ("margin[i] = fabs(t - (j + 0.5)) / (double)qmax;",

@@ -1,0 +1,158 @@
+"""GPU parity: the CUDA library (through the C ABI) against the fp64 oracle.
+
+Small cases span several units per warp, several warps per CTA and ragged
+tails; the named workloads are the paper-shaped layers at full size.
+"""
+import json
+
+import numpy as np
+import pytest
+import torch
+
+from paper_2608_13966_gb300 import workloads as wl
+from tests import gpu_harness as H
+
+pytestmark = pytest.mark.gpu
+
+CLIP8 = list(wl.CLIP_8)
+CLIP16 = list(wl.CLIP_16)
+
+
+def _inputs(rows, cols, seed, dist="t4", g_dtype=torch.bfloat16):
+    d = wl.random_groups(1, rows * cols, seed=seed, dist=dist, g_dtype=g_dtype, device="cuda")
+    return (d["w"].reshape(rows, cols), d["g"].reshape(rows, cols), d["v"].reshape(rows, cols))
+
+
+def _assert(rep, ema):
+    assert ema["ok"], json.dumps(ema)
+    assert rep["ok"], json.dumps(rep)
+
+
+def test_single_matrix_int4(oracle):
+    """256x1024 fp32 matrix, INT4, group 128, 8 candidates, fp32 g and r."""
+    w_ = wl.workload("single_int4")
+    d = wl.make_tensor(w_, w_.tensors[0], device="cuda")
+    rep, ema = H.run_int(oracle, d["w"], d["g"], d["v"], bits=4, group_size=128,
+                         clip=list(w_.clip), beta2=w_.beta2, r_dtype=torch.float32)
+    _assert(rep, ema)
+
+
+@pytest.mark.parametrize("bits", [2, 3, 4, 8])
+@pytest.mark.parametrize("G", [32, 64, 128, 256])
+def test_int_bits_groups_ragged(oracle, bits, G):
+    # 37 rows x 3 groups: the unit count is not a multiple of the warps
+    w, g, v = _inputs(37, 3 * G, seed=bits * 1000 + G)
+    rep, ema = H.run_int(oracle, w, g, v, bits=bits, group_size=G, clip=CLIP8)
+    _assert(rep, ema)
+
+
+@pytest.mark.parametrize("K", [1, 5, 8, 13, 16, 32])
+def test_int_candidate_counts(oracle, K):
+    clip = [round(1.0 - 0.7 * i / max(K - 1, 1), 4) for i in range(K)]
+    w, g, v = _inputs(64, 1024, seed=K)
+    rep, ema = H.run_int(oracle, w, g, v, bits=3, group_size=128, clip=clip)
+    _assert(rep, ema)
+
+
+def test_int_fp32_gradient_and_output(oracle):
+    w, g, v = _inputs(128, 512, seed=77, g_dtype=torch.float32)
+    rep, ema = H.run_int(oracle, w, g, v, bits=4, group_size=128, clip=CLIP8,
+                         r_dtype=torch.float32)
+    _assert(rep, ema)
+
+
+def test_int_without_gradient_and_optional_outputs(oracle):
+    w, _, v = _inputs(64, 512, seed=78)
+    v0 = v.clone()
+    rep, ema = H.run_int(oracle, w, None, v, bits=3, group_size=128, clip=CLIP8,
+                         codes=False, idx=False)
+    _assert(rep, ema)
+    assert torch.equal(v, v0)
+
+
+def test_int_degenerate_groups(oracle):
+    """Constant groups, all-zero saliency, one salient element, clipped heavy
+    tails, exact zeros -- each in its own group of the same launch."""
+    G = 128
+    w, g, v = _inputs(16, G, seed=79)
+    w[0] = 0.0123                       # zero range
+    w[1] = -0.5                         # zero range, negative
+    v[2] = 0.0; g[2] = 0.0              # all saliency zero
+    v[3] = 0.0; g[3] = 0.0; v[3, 17] = 1e-6   # one salient element
+    v[4] = 0.0; g[4] = 0.0; v[4, :2] = 1e-6   # two salient elements
+    w[5, ::2] = 0.0                     # many exact zeros
+    w[6, 5] = 3.0                       # one outlier
+    w[7] = torch.linspace(-1, 1, G, device="cuda")  # codes on grid boundaries
+    rep, ema = H.run_int(oracle, w, g, v, bits=3, group_size=G, clip=CLIP8)
+    _assert(rep, ema)
+
+
+def test_int_nonfinite_inputs_do_not_fault(oracle):
+    w, g, v = _inputs(8, 256, seed=80)
+    w[0, 3] = float("nan")
+    w[1, 5] = float("inf")
+    v[2, 7] = float("nan")
+    from paper_2608_13966_gb300 import api
+    api.recon_int(w, g, v, bits=3, group_size=128, clip=CLIP8)
+    torch.cuda.synchronize()
+
+
+def test_nvfp4_small_and_degenerate(oracle):
+    w, g, v = _inputs(48, 256, seed=81)
+    w[0, :16] = 0.0                      # zero block
+    v[1, :16] = 0.0; g[1, :16] = 0.0     # zero saliency block
+    v[2, :16] = 0.0; g[2, :16] = 0.0; v[2, 3] = 1e-6
+    rep, ema = H.run_nvfp4(oracle, w, g, v, clip=CLIP8)
+    _assert(rep, ema)
+
+
+@pytest.mark.parametrize("K", [1, 8, 13, 16, 32])
+def test_nvfp4_candidate_counts_supplied_amax(oracle, K):
+    clip = [round(1.0 - 0.7 * i / max(K - 1, 1), 4) for i in range(K)]
+    w, g, v = _inputs(40, 528, seed=100 + K)     # 1320 blocks: ragged unit count
+    rep, ema = H.run_nvfp4(oracle, w, g, v, clip=clip, supply_amax=True,
+                           r_dtype=torch.float32)
+    _assert(rep, ema)
+
+
+def _layer(name):
+    w_ = wl.workload(name)
+    for spec in w_.tensors:
+        yield w_, spec, wl.make_tensor(w_, spec, device="cuda")
+
+
+@pytest.mark.parametrize("name", ["llama_layer_int3", "qwen_layer_int2"])
+def test_paper_shaped_layer_int(oracle, name):
+    for w_, spec, d in _layer(name):
+        rep, ema = H.run_int(oracle, d["w"], d["g"], d["v"], bits=w_.bits,
+                             group_size=w_.group, clip=list(w_.clip), beta2=w_.beta2)
+        _assert(rep, ema)
+        del d
+        torch.cuda.empty_cache()
+
+
+def test_paper_shaped_layer_nvfp4(oracle):
+    for w_, spec, d in _layer("llama_layer_nvfp4"):
+        rep, ema = H.run_nvfp4(oracle, d["w"], d["g"], d["v"], clip=list(w_.clip),
+                               beta2=w_.beta2)
+        _assert(rep, ema)
+        del d
+        torch.cuda.empty_cache()
+
+
+def test_timeout_path_reports_and_recovers(oracle):
+    """A wait on a barrier that nothing signals runs out after 1 ms; the
+    kernel records the timeout and returns; the context stays usable."""
+    from paper_2608_13966_gb300 import api, quasar
+    w, g, v = _inputs(64, 512, seed=82)
+    assert quasar.quasar_get_device_status() == quasar.QuasarStatus.OK
+    quasar.quasar_debug_force_timeout(1_000_000)
+    try:
+        api.recon_int(w, g, v, bits=3, group_size=128, clip=CLIP8)
+    finally:
+        quasar.quasar_debug_force_timeout(0)
+    assert quasar.quasar_get_device_status() == quasar.QuasarStatus.ERR_TIMEOUT
+    assert quasar.quasar_get_device_status() == quasar.QuasarStatus.OK
+    rep, ema = H.run_int(oracle, *_inputs(64, 512, seed=83), bits=3, group_size=128,
+                         clip=CLIP8)
+    _assert(rep, ema)
