@@ -9,6 +9,9 @@ namespace quasar {
 constexpr unsigned kStatusTimeout = 1u;
 
 constexpr int kLanesPerGroup = 8;
+// Per-warp shared scratch of the integer kernel: 32 rows of 36 floats used to
+// transpose the per-candidate sums across the lanes of a group.
+constexpr uint32_t kIntScratchBytes = 32 * 36 * 4;
 constexpr int kGroupsPerUnit = 4;
 constexpr int kMaxClip = 32;
 

@@ -30,7 +30,9 @@ namespace {
 
 using namespace quasar;
 
-constexpr int kThreads = 256;
+// 7 warps per CTA: with two 5 KB tiles and the 4.5 KB transpose scratch
+// per warp, two CTAs fit in an SM's shared memory (14 resident warps).
+constexpr int kThreads = 224;
 constexpr int kWarps = kThreads / 32;
 constexpr uint64_t kDefaultTimeoutNs = 1000000000ull;  // 1 s per wait
 
@@ -120,20 +122,24 @@ struct Launch {
     size_t smem;
 };
 
-Launch plan(uint32_t unit_bytes)
+// Shared memory per CTA: for each warp, `stages` tiles of unit_bytes, a
+// scratch area, and stages + 1 mbarriers.
+Launch plan(uint32_t unit_bytes, uint32_t scratch_bytes)
 {
     const Tuning& t = tuning();
     Launch L;
     L.stage_bytes = (unit_bytes + 127u) & ~127u;
+    auto total = [&](int s) {
+        return (size_t)kWarps * s * L.stage_bytes + (size_t)kWarps * scratch_bytes +
+               (size_t)kWarps * (s + 1) * 8;
+    };
     int s = t.stages;
     if (s <= 0) {
         s = 2;
-        while (s < 4 && (size_t)kWarps * (s + 1) * L.stage_bytes + kWarps * (s + 2) * 8 <=
-                            (size_t)t.smem_budget)
-            ++s;
+        while (s < 4 && total(s + 1) <= (size_t)t.smem_budget) ++s;
     }
     L.stages = s;
-    L.smem = (size_t)kWarps * s * L.stage_bytes + (size_t)kWarps * (s + 1) * 8;
+    L.smem = total(s);
     return L;
 }
 
@@ -293,7 +299,7 @@ quasar_status quasar_recon_int(const float* w, const void* g, quasar_dtype g_dty
     if ((st = status_ptr(&p.status)) != QUASAR_OK) return st;
 
     const int gbytes = p.g_kind == 2 ? 2 : (p.g_kind == 1 ? 4 : 0);
-    const Launch L = plan((uint32_t)(kGroupsPerUnit * group_size * (8 + gbytes)));
+    const Launch L = plan((uint32_t)(kGroupsPerUnit * group_size * (8 + gbytes)), kIntScratchBytes);
     p.stages = L.stages;
     p.stage_bytes = L.stage_bytes;
 
@@ -393,7 +399,7 @@ quasar_status quasar_recon_nvfp4(const float* w, const void* g, quasar_dtype g_d
     }
 
     const int gbytes = p.g_kind == 2 ? 2 : (p.g_kind == 1 ? 4 : 0);
-    const Launch L = plan((uint32_t)(kBlocksPerUnit * 16 * (8 + gbytes)));
+    const Launch L = plan((uint32_t)(kBlocksPerUnit * 16 * (8 + gbytes)), 0);
     p.stages = L.stages;
     p.stage_bytes = L.stage_bytes;
     const void* fn = nvfp4_kernel(nch_for(n_clip));

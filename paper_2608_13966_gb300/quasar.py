@@ -52,17 +52,21 @@ PROTOTYPES = {
 
 
 def library_path() -> str:
-    return _build.LIB
+    return os.environ.get("QUASAR_LIBRARY") or _build.LIB
 
 
 def load(build_if_missing: bool = True):
-    """Load libquasar.so (building it first if asked and needed)."""
+    """Load libquasar.so (building it first if asked and needed).  The
+    environment variable QUASAR_LIBRARY names another build of the same
+    library to load instead (no build step then)."""
     global _lib
     with _lock:
         if _lib is not None:
             return _lib
         path = _build.LIB
-        if build_if_missing:
+        if os.environ.get("QUASAR_LIBRARY"):
+            path = os.environ["QUASAR_LIBRARY"]
+        elif build_if_missing:
             path = _build.build()
         if not os.path.exists(path):
             raise OSError(f"libquasar.so not found at {path}; run paper_2608_13966_gb300.build")
