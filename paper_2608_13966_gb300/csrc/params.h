@@ -32,7 +32,7 @@ struct IntParams {
     float beta2;
     float c1;  // 1 - beta2
     float tie_kappa;   // multiplier of the fp32 unit roundoff in the tie bound
-    float refit_cond;  // refit the kept candidate in two passes above this
+    float fit_ulps;    // error of the fp32 refit, in ulps of its scale (tier-2 trigger)
     int stages;
     uint32_t stage_bytes;
     uint64_t timeout_ns;

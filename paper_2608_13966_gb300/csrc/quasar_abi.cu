@@ -43,7 +43,7 @@ struct Tuning {
     int stages = 0;            // 0: chosen from the shared-memory budget
     int smem_budget = 100 * 1024;
     float tie_kappa = 16.0f;
-    float refit_cond = 8.0f;
+    float fit_ulps = 3.0f;
 };
 
 const Tuning& tuning()
@@ -53,7 +53,7 @@ const Tuning& tuning()
         if (const char* s = std::getenv("QUASAR_STAGES")) x.stages = std::atoi(s);
         if (const char* s = std::getenv("QUASAR_SMEM_BUDGET")) x.smem_budget = std::atoi(s);
         if (const char* s = std::getenv("QUASAR_TIE_KAPPA")) x.tie_kappa = (float)std::atof(s);
-        if (const char* s = std::getenv("QUASAR_REFIT_COND")) x.refit_cond = (float)std::atof(s);
+        if (const char* s = std::getenv("QUASAR_FIT_ULPS")) x.fit_ulps = (float)std::atof(s);
         return x;
     }();
     return t;
@@ -291,7 +291,7 @@ quasar_status quasar_recon_int(const float* w, const void* g, quasar_dtype g_dty
     p.beta2 = beta2;
     p.c1 = 1.0f - beta2;
     p.tie_kappa = tuning().tie_kappa;
-    p.refit_cond = tuning().refit_cond;
+    p.fit_ulps = tuning().fit_ulps;
     p.timeout_ns = kDefaultTimeoutNs;
     p.force_timeout_ns = (uint64_t)std::max<int64_t>(0, g_force_timeout_ns.load());
     p.stats = g_stats.load();

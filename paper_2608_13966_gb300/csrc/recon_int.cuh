@@ -20,9 +20,7 @@
 //   pass B  for 8 candidates at a time, codes q = clamp(rne(d*P_k + qmax/2))
 //           with d = w - c and P_k = qmax/(f_k*range) (the 1.5*2^23 rounding
 //           trick; codes are accumulated centred on Hc = floor(qmax/2)), and
-//           the sums S1 = sum h q, S2 = sum h q^2, S3 = sum h q d, plus the
-//           unweighted checksum U = sum q d (equal codes <=> equal (S, U),
-//           even where h is too small to move the weighted sums); packed
+//           the sums S1 = sum h q, S2 = sum h q^2, S3 = sum h q d; packed
 //           f32x2 arithmetic, two elements per instruction;
 //   reduce  the 8 lanes' partial sums are transposed through shared memory
 //           so that lane sl owns candidate sl of the chunk;
@@ -124,6 +122,22 @@ __device__ __forceinline__ float wsum32(float x)
 //
 // One group, evaluated by all 32 lanes (lane L takes elements L + 32m) from
 // the tile in shared memory: w at ws, saliency h at hs (or 1 if h_one).
+
+// True when candidates with scale factors Pa and Pb give the same codes on
+// every element of the group (whole warp).
+template <int G>
+__device__ bool coop_same_codes(const float* ws, float c, float Pa, float Pb, float H, float qmaxf)
+{
+    constexpr int M = G / 32;
+    const int lane = threadIdx.x & 31;
+    bool same = true;
+#pragma unroll
+    for (int m = 0; m < M; ++m) {
+        const float d = ws[lane + 32 * m] - c;
+        same &= int_code(d, Pa, H, qmaxf) == int_code(d, Pb, H, qmaxf);
+    }
+    return __all_sync(0xffffffffu, same);
+}
 
 // Exact evaluation of one candidate: codes, exact degenerate test (all
 // weighted elements on one code), two-pass centred fit, and the direct error
@@ -291,19 +305,6 @@ __device__ void coop_precise(const float* ws, const float* hs, bool h_one, float
     *B_lo = zl;
 }
 
-// fp32 error estimate of a fit taken on d = w - c with centred codes: b and
-// every level a*q + b err by a few ulp of |c| + range.  True when that could
-// exceed half the output tolerance 1e-7 + 1e-5|x| at the offset or at the
-// level closest to zero, or when the sums were badly conditioned.
-__device__ __forceinline__ bool needs_compensated_fit(float a, float B, float c, float range,
-                                                      float qmaxf, float cond, float cond_max)
-{
-    const float est = 2.3841858e-07f * (fabsf(c) + range);
-    const float q0 = fminf(fmaxf(rintf(-B / a), 0.0f), qmaxf);
-    const float rmin = fminf(fabsf(B), fabsf(fmaf(a, q0, B)));
-    return !(cond <= cond_max) || est > 0.5f * (1e-7f + 1e-5f * rmin);
-}
-
 // ------------------------------------------------------------------ kernel
 
 template <int EPL, int NCH>
@@ -389,6 +390,8 @@ __global__ void __launch_bounds__(256) k_recon_int(const IntParams p)
     const float2 magic2 = make_float2(kRoundMagic, kRoundMagic);
     const float2 nmagic_c2 = make_float2(-(kRoundMagic + Hc), -(kRoundMagic + Hc));
     const float ulp = 5.9604645e-8f * p.tie_kappa;
+    const float2 beta22 = make_float2(p.beta2, p.beta2);
+    const float2 c12 = make_float2(p.c1, p.c1);
     int s_cur = 0;
     uint32_t parity = 0;
 
@@ -424,10 +427,12 @@ __global__ void __launch_bounds__(256) k_recon_int(const IntParams p)
                     const float4 g4 = lds128(gsm + e * 4);
                     g0 = g4.x; g1 = g4.y; g2 = g4.z; g3 = g4.w;
                 }
-                h4.x = fmaf(p.beta2, h4.x, __fmul_rn(p.c1, __fmul_rn(g0, g0)));
-                h4.y = fmaf(p.beta2, h4.y, __fmul_rn(p.c1, __fmul_rn(g1, g1)));
-                h4.z = fmaf(p.beta2, h4.z, __fmul_rn(p.c1, __fmul_rn(g2, g2)));
-                h4.w = fmaf(p.beta2, h4.w, __fmul_rn(p.c1, __fmul_rn(g3, g3)));
+                const float2 gA = make_float2(g0, g1), gB = make_float2(g2, g3);
+                const float2 hA = __ffma2_rn(make_float2(h4.x, h4.y), beta22,
+                                             __fmul2_rn(c12, __fmul2_rn(gA, gA)));
+                const float2 hB = __ffma2_rn(make_float2(h4.z, h4.w), beta22,
+                                             __fmul2_rn(c12, __fmul2_rn(gB, gB)));
+                h4 = make_float4(hA.x, hA.y, hB.x, hB.y);
                 *reinterpret_cast<float4*>(hs + e) = h4;
                 if (valid) stg_cs(reinterpret_cast<float4*>(p.v + gbase + i * 32 + sl * 4), h4);
             }
@@ -446,13 +451,15 @@ __global__ void __launch_bounds__(256) k_recon_int(const IntParams p)
         const float range = mx - mn;
         const bool flat = !(range > 0.0f);
         const float c = 0.5f * (mn + mx);
-        const float R = flat ? 0.0f : qmaxf / range;
-        const float inv_ss = 1.0f / ss;
+        // approximate divisions (<= 2 ulp) are enough here: R scales the code
+        // positions (margins are measured against the clipping range), and
+        // the fit of the kept candidate is rechecked below
+        const float R = flat ? 0.0f : __fdividef(qmaxf, range);
+        const float inv_ss = __fdividef(1.0f, ss);
         const float2 nc2 = make_float2(-c, -c);
 
         // ---- pass B + reduction + fit, 8 candidates at a time
-        float Ek[NCH], dEk[NCH], ak[NCH], bk[NCH], condk[NCH], T1k[NCH], T2k[NCH], T3k[NCH],
-            Uk[NCH];
+        float Ek[NCH], dEk[NCH], ak[NCH], bk[NCH], T1k[NCH], T2k[NCH], T3k[NCH];
         bool suspk[NCH];
         float sd = 0.0f, sdd = 0.0f;
 #pragma unroll 1
@@ -463,10 +470,9 @@ __global__ void __launch_bounds__(256) k_recon_int(const IntParams p)
                 const float P = R * p.invf[ch * 8 + kk];
                 P2[kk] = make_float2(P, P);
             }
-            float2 A1[8], A2[8], A3[8], AU[8];
+            float2 A1[8], A2[8], A3[8];
 #pragma unroll
-            for (int kk = 0; kk < 8; ++kk)
-                A1[kk] = A2[kk] = A3[kk] = AU[kk] = make_float2(0.0f, 0.0f);
+            for (int kk = 0; kk < 8; ++kk) A1[kk] = A2[kk] = A3[kk] = make_float2(0.0f, 0.0f);
             float2 SD = make_float2(0.0f, 0.0f), SDD = make_float2(0.0f, 0.0f);
 #pragma unroll 1
             for (int i = 0; i < NCHK; ++i) {
@@ -495,7 +501,6 @@ __global__ void __launch_bounds__(256) k_recon_int(const IntParams p)
                         A1[kk] = __fadd2_rn(A1[kk], hq);
                         A2[kk] = __ffma2_rn(hq, q, A2[kk]);
                         A3[kk] = __ffma2_rn(q, hd[pr], A3[kk]);
-                        AU[kk] = __ffma2_rn(q, d[pr], AU[kk]);
                     }
             }
             // transpose through shared memory: lane L writes row L, lane
@@ -503,17 +508,15 @@ __global__ void __launch_bounds__(256) k_recon_int(const IntParams p)
 #pragma unroll
             for (int kk = 0; kk < 8; ++kk)
                 *reinterpret_cast<float4*>(red + lane * 36 + kk * 4) =
-                    make_float4(A1[kk].x + A1[kk].y, A2[kk].x + A2[kk].y, A3[kk].x + A3[kk].y,
-                                AU[kk].x + AU[kk].y);
+                    make_float4(A1[kk].x + A1[kk].y, A2[kk].x + A2[kk].y, A3[kk].x + A3[kk].y, 0.0f);
             __syncwarp();
-            float4 T = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
+            float3 T = make_float3(0.0f, 0.0f, 0.0f);
 #pragma unroll
             for (int j = 0; j < 8; ++j) {
                 const float4 x = *reinterpret_cast<const float4*>(red + (gs * 8 + j) * 36 + sl * 4);
                 T.x += x.x;
                 T.y += x.y;
                 T.z += x.z;
-                T.w += x.w;
             }
             __syncwarp();
             if (ch == 0) {
@@ -532,7 +535,7 @@ __global__ void __launch_bounds__(256) k_recon_int(const IntParams p)
             const float D = T.y - T.x * qbar;
             const float N = T.z - T.x * dbar;
             const bool susp = !(D > 1e-3f * T.y);
-            const float a = N / D;
+            const float a = __fdividef(N, D);
             const float E = susp ? 0.0f : N * a;
             const float dN = ulp * qmaxf * habsd;
             const float dD = ulp * T.y;
@@ -544,12 +547,10 @@ __global__ void __launch_bounds__(256) k_recon_int(const IntParams p)
                     dEk[cc] = 2.0f * fabsf(a) * dN + a * a * dD;
                     ak[cc] = a;
                     bk[cc] = dbar - a * (qbar + Hc);
-                    condk[cc] = T.y / D + (fabsf(T.z) + fabsf(T.x * dbar)) / fabsf(N);
                     suspk[cc] = real && susp;
                     T1k[cc] = T.x;
                     T2k[cc] = T.y;
                     T3k[cc] = T.z;
-                    Uk[cc] = T.w;
                 }
         }
         const float dbar = sd * inv_ss;
@@ -578,59 +579,57 @@ __global__ void __launch_bounds__(256) k_recon_int(const IntParams p)
         if (kb > 0x7ff) kb = 0;  // every candidate suspicious: the exact path picks
 
         // winner's fit and sums, from its owner lane
-        float a_sel = 0.0f, bc_sel = 0.0f, cond_sel = 0.0f, T1b = 0.0f, T2b = 0.0f, T3b = 0.0f,
-              Ub = 0.0f;
+        float a_sel = 0.0f, bc_sel = 0.0f, T1b = 0.0f, T2b = 0.0f, T3b = 0.0f;
         {
             const int owner = (gs * 8) | (kb & 7);
 #pragma unroll
             for (int ch = 0; ch < NCH; ++ch) {
                 const float av = __shfl_sync(0xffffffffu, ak[ch], owner);
                 const float bv = __shfl_sync(0xffffffffu, bk[ch], owner);
-                const float cv = __shfl_sync(0xffffffffu, condk[ch], owner);
                 const float t1 = __shfl_sync(0xffffffffu, T1k[ch], owner);
                 const float t2 = __shfl_sync(0xffffffffu, T2k[ch], owner);
                 const float t3 = __shfl_sync(0xffffffffu, T3k[ch], owner);
-                const float uu = __shfl_sync(0xffffffffu, Uk[ch], owner);
                 if ((kb >> 3) == ch) {
                     a_sel = av;
                     bc_sel = bv;
-                    cond_sel = cv;
                     T1b = t1;
                     T2b = t2;
                     T3b = t3;
-                    Ub = uu;
                 }
             }
         }
         // Candidates needing an exact comparison: within the fp32 error bound
-        // of the winner, unless their codes equal the winner's (same weighted
-        // sums and same unweighted checksum): equal codes give equal errors,
-        // and the lower index is kept, as Algorithm 1's argmin does.
-        unsigned my_set = 0;
+        // of the winner.  Those whose sums equal the winner's bit for bit
+        // ("twins") almost always have the winner's codes -- equal codes give
+        // equal errors, and the lower index is kept, as Algorithm 1's argmin
+        // does -- but an element of tiny saliency can differ without moving the
+        // sums, so twins are first checked code by code (cheaply, deferred).
+        unsigned my_set = 0, my_twin = 0;
 #pragma unroll
         for (int ch = 0; ch < NCH; ++ch) {
             const int k = ch * 8 + sl;
-            const bool same = T1k[ch] == T1b && T2k[ch] == T2b && T3k[ch] == T3b && Uk[ch] == Ub;
-            const bool contender = k != kb && Ek[ch] > -INFINITY && !same &&
-                                   Eb - Ek[ch] <= dEb + dEk[ch];
+            const bool twin = T1k[ch] == T1b && T2k[ch] == T2b && T3k[ch] == T3b;
+            const bool contender = k != kb && Ek[ch] > -INFINITY && Eb - Ek[ch] <= dEb + dEk[ch];
             if (contender || suspk[ch]) my_set |= 1u << ch;
+            if (contender && twin && !suspk[ch]) my_twin |= 1u << ch;
         }
-        unsigned set = 0;
+        unsigned set = 0, twins = 0;
 #pragma unroll
         for (int ch = 0; ch < NCH; ++ch) {
             const unsigned bal = __ballot_sync(0xffffffffu, (my_set >> ch) & 1u);
             set |= ((bal >> (gs * 8)) & 0xFFu) << (ch * 8);
+            const unsigned balt = __ballot_sync(0xffffffffu, (my_twin >> ch) & 1u);
+            twins |= ((balt >> (gs * 8)) & 0xFFu) << (ch * 8);
         }
         if (Eb == -INFINITY) set = (p.n_clip >= 32) ? 0xFFFFFFFFu : ((1u << p.n_clip) - 1u);
         else if (set) set |= 1u << kb;
 
         float Bsel = bc_sel + c, a_lo = 0.0f, B_lo = 0.0f;
-        const bool need_any =
-            valid && !flat &&
-            (set != 0 || needs_compensated_fit(a_sel, Bsel, c, range, qmaxf, cond_sel, p.refit_cond));
+        float qbar_sel = T1b * inv_ss + Hc;
+        bool deg_sel = false;
 
-        // ---- deferred rare work: the whole warp takes one group at a time
-        unsigned todo = __ballot_sync(0xffffffffu, need_any && sl == 0);
+        // ---- deferred exact comparisons: the whole warp takes one group at a time
+        unsigned todo = __ballot_sync(0xffffffffu, valid && !flat && set != 0 && sl == 0);
         if (todo) __syncwarp();  // h written by other lanes is read below
         while (todo) {
             const int g = (__ffs(todo) - 1) >> 3;
@@ -642,46 +641,186 @@ __global__ void __launch_bounds__(256) k_recon_int(const IntParams p)
             const float gss = __shfl_sync(0xffffffffu, ss, src);
             const float gdbar = __shfl_sync(0xffffffffu, dbar, src);
             const bool gh_one = __shfl_sync(0xffffffffu, (int)h_one, src) != 0;
-            const unsigned gset = __shfl_sync(0xffffffffu, set, src);
-            int gkb = __shfl_sync(0xffffffffu, kb, src);
-            float ga = __shfl_sync(0xffffffffu, a_sel, src);
-            float gB = __shfl_sync(0xffffffffu, Bsel, src);
-            float gcond = __shfl_sync(0xffffffffu, cond_sel, src);
-            bool gdeg = false;
+            unsigned gset = __shfl_sync(0xffffffffu, set, src);
+            const unsigned gtwins = __shfl_sync(0xffffffffu, twins, src);
+            const int gkb0 = __shfl_sync(0xffffffffu, kb, src);
             const float* gws = ws + g * G;
             const float* ghs = hs + g * G;
-            if (gset) {
-                if (p.stats && lane == 0) atomicAdd(&p.stats[0], 1u);
-                unsigned rem = gset;
-                float best_h = 0.0f, best_l = 0.0f;
-                int best_k = -1;
-                while (rem) {
-                    const int k = __ffs(rem) - 1;
-                    rem &= rem - 1;
-                    float eh, el, a_k, bc_k;
-                    bool deg_k;
-                    coop_exact<G>(gws, ghs, gh_one, gc, gR * p.invf[k], H, qmaxf, gss, gdbar,
-                                  p.f[k] * grange / qmaxf, &eh, &el, &a_k, &bc_k, &deg_k);
-                    if (best_k < 0 || ff_less(eh, el, best_h, best_l)) {
-                        best_h = eh;
-                        best_l = el;
-                        best_k = k;
-                        ga = a_k;
-                        gB = bc_k + gc;
-                        gdeg = deg_k;
-                    }
-                }
-                gkb = best_k;
-                gcond = 1.0f;
+            unsigned tw = gtwins;
+            while (tw) {
+                const int k = __ffs(tw) - 1;
+                tw &= tw - 1;
+                if (coop_same_codes<G>(gws, gc, gR * p.invf[k], gR * p.invf[gkb0], H, qmaxf))
+                    gset &= ~(1u << k);
             }
-            float ga_lo = 0.0f, gB_lo = 0.0f;
-            if (!gdeg && needs_compensated_fit(ga, gB, gc, grange, qmaxf, gcond, p.refit_cond)) {
-                if (p.stats && lane == 0) atomicAdd(&p.stats[1], 1u);
-                coop_precise<G>(gws, ghs, gh_one, gc, gR * p.invf[gkb], H, qmaxf, gss, gc + gdbar,
-                                &ga, &ga_lo, &gB, &gB_lo);
+            if (gset == (1u << gkb0)) continue;  // only the winner left
+            if (p.stats && lane == 0) atomicAdd(&p.stats[0], 1u);
+            float best_h = 0.0f, best_l = 0.0f, ga = 0.0f, gB = 0.0f;
+            int best_k = -1;
+            bool gdeg = false;
+            while (gset) {
+                const int k = __ffs(gset) - 1;
+                gset &= gset - 1;
+                float eh, el, a_k, bc_k;
+                bool deg_k;
+                coop_exact<G>(gws, ghs, gh_one, gc, gR * p.invf[k], H, qmaxf, gss, gdbar,
+                              p.f[k] * grange / qmaxf, &eh, &el, &a_k, &bc_k, &deg_k);
+                if (best_k < 0 || ff_less(eh, el, best_h, best_l)) {
+                    best_h = eh;
+                    best_l = el;
+                    best_k = k;
+                    ga = a_k;
+                    gB = bc_k + gc;
+                    gdeg = deg_k;
+                }
             }
             if (gs == g) {
-                kb = gkb;
+                kb = best_k;
+                a_sel = ga;
+                Bsel = gB;
+                deg_sel = gdeg;
+                qbar_sel = -1.0f;  // recomputed by the refit below
+            }
+        }
+
+        // ---- pass R: two-pass weighted least-squares fit (Eq. 4) of the kept
+        // candidate, centred on a short approximation m of its weighted mean
+        // code (q - m exact) and on the weighted mean weight; the offset is
+        // assembled in compensated arithmetic and kept as a float pair.
+        const float Pk = R * p.invf[kb];
+        const bool refit = !flat && !deg_sel;
+        float kap = 0.0f;
+        {
+            const float2 Pk2 = make_float2(Pk, Pk);
+            float qm = qbar_sel;
+            // winner changed in the exact pass: its mean code again (warp-uniform
+            // branch, the reduction below shuffles across all lanes)
+            if (__any_sync(0xffffffffu, qm < 0.0f)) {
+                float s1 = 0.0f;
+#pragma unroll 1
+                for (int i = 0; i < NCHK; ++i) {
+                    const int e = gs * G + i * 32 + sl * 4;
+                    const float4 w4 = lds128(ws + e);
+                    const float4 h4 = h_one ? make_float4(1.0f, 1.0f, 1.0f, 1.0f) : lds128(hs + e);
+                    s1 = fmaf(h4.x, int_code(w4.x - c, Pk, H, qmaxf), s1);
+                    s1 = fmaf(h4.y, int_code(w4.y - c, Pk, H, qmaxf), s1);
+                    s1 = fmaf(h4.z, int_code(w4.z - c, Pk, H, qmaxf), s1);
+                    s1 = fmaf(h4.w, int_code(w4.w - c, Pk, H, qmaxf), s1);
+                }
+#pragma unroll
+                for (int o = 4; o; o >>= 1) s1 += shx(s1, o);
+                if (qm < 0.0f) qm = s1 * inv_ss;
+            }
+            const float m = rintf(qm);  // integer: q - m is exact and magic + m too
+            const float2 nm2 = make_float2(-(kRoundMagic + m), -(kRoundMagic + m));
+            const float2 ndbar2 = make_float2(-dbar, -dbar);
+            float2 D2 = make_float2(0.0f, 0.0f), N2 = D2, A2 = D2, B2s = D2, W2 = D2;
+#pragma unroll 1
+            for (int i = 0; i < NCHK; ++i) {
+                const int e = gs * G + i * 32 + sl * 4;
+                const float4 w4 = lds128(ws + e);
+                const float4 h4 = h_one ? make_float4(1.0f, 1.0f, 1.0f, 1.0f) : lds128(hs + e);
+#pragma unroll
+                for (int pr = 0; pr < 2; ++pr) {
+                    const float2 wv = pr ? make_float2(w4.z, w4.w) : make_float2(w4.x, w4.y);
+                    const float2 hv = pr ? make_float2(h4.z, h4.w) : make_float2(h4.x, h4.y);
+                    const float2 d = __fadd2_rn(wv, nc2);
+                    float2 t = __ffma2_rn(d, Pk2, H2);
+                    t.x = fminf(fmaxf(t.x, 0.0f), qmaxf);
+                    t.y = fminf(fmaxf(t.y, 0.0f), qmaxf);
+                    const float2 dq = __fadd2_rn(__fadd2_rn(t, magic2), nm2);  // q - m, exact
+                    const float2 wd = __fadd2_rn(d, ndbar2);
+                    const float2 hdq = __fmul2_rn(hv, dq);
+                    D2 = __ffma2_rn(hdq, dq, D2);
+                    N2 = __ffma2_rn(hdq, wd, N2);
+                    A2 = __fadd2_rn(A2, hdq);
+                    B2s = __ffma2_rn(hv, wd, B2s);
+                    W2 = __ffma2_rn(__fmul2_rn(hv, wd), wd, W2);
+                }
+            }
+            float Dr = D2.x + D2.y, Nr = N2.x + N2.y, Ar = A2.x + A2.y, Br = B2s.x + B2s.y;
+            float Wr = W2.x + W2.y;
+#pragma unroll
+            for (int o = 4; o; o >>= 1) {
+                Dr += shx(Dr, o);
+                Nr += shx(Nr, o);
+                Ar += shx(Ar, o);
+                Br += shx(Br, o);
+                Wr += shx(Wr, o);
+            }
+            if (refit) {
+                const float Aq = Ar * inv_ss;  // mean of q - m
+                const float Bw = Br * inv_ss;  // mean of d - dbar
+                const float Nc = Nr - Ar * Bw, Dc = Dr - Ar * Aq;
+                const float an = Nc / Dc;
+                // b = (c + dbar + Bw) - a * (m + Aq), as a float pair
+                float mu_h, mu_l, p_h, p_l, bh, bl;
+                two_sum(c, dbar, mu_h, mu_l);
+                two_prod(an, m, p_h, p_l);
+                two_sum(mu_h, -p_h, bh, bl);
+                bl = __fadd_rn(bl, __fsub_rn(__fadd_rn(mu_l, Bw), fmaf(an, Aq, p_l)));
+                ff_norm(bh, bl);
+                a_sel = an;
+                Bsel = bh;
+                B_lo = bl;
+                // conditioning of the slope: rounding in the sums moves a by
+                // about ulp * (sum |h dq wd| / |Nc| + sum h dq^2 / Dc), and
+                // sum |h dq wd| <= sqrt(Dr Wr) (Cauchy-Schwarz)
+                kap = __fdividef(sqrtf(Dr * Wr), fabsf(Nc)) + __fdividef(Dr, Dc);
+            }
+        }
+
+        // ---- output accuracy check.  The refit's error at any level is at most
+        // about est = fit_ulps * ulp * (|a| qmax kap + |c| + range) (fit_ulps
+        // calibrated against the oracle with a margin).  The offset b (fp32)
+        // and a level written in fp32 must meet tol(x) = 1e-7 + 1e-5|x|.  A
+        // level written in bf16 is exact when no bf16 rounding midpoint lies
+        // within est of it, and within the tolerance band when est <= tol.
+        // Groups that could miss get the compensated (float-float) fit.
+        bool prec;
+        {
+            const float est = p.fit_ulps * 5.9604645e-8f * (fabsf(a_sel) * qmaxf * kap + fabsf(c) + range);
+            prec = est > 1e-7f + 1e-5f * fabsf(Bsel);
+            if (!p.r_bf16) {
+                const float q0 = fminf(fmaxf(rintf(__fdividef(-Bsel, a_sel)), 0.0f), qmaxf);
+                const float rmin = fminf(fabsf(Bsel), fabsf(fmaf(a_sel, q0, Bsel)));
+                prec |= est > 1e-7f + 1e-5f * rmin;
+            } else {
+                for (int q = sl; q <= p.qmax; q += kLanesPerGroup) {
+                    const float rq = fmaf(a_sel, (float)q, Bsel);
+                    if (est > 1e-7f + 1e-5f * fabsf(rq)) {
+                        const uint32_t bits = __float_as_uint(rq);
+                        const int dmid = abs((int)(bits & 0xFFFFu) - 0x8000);  // fp32 ulps to the midpoint
+                        const float ulp32 =
+                            __uint_as_float(max(bits & 0x7F800000u, 0x0C000000u) - 0x0B800000u);
+                        prec |= (float)dmid * ulp32 < 1.5f * est;
+                    }
+                }
+            }
+            prec = prec || est != est;  // NaN sums: take the careful path
+        }
+        {
+            // one decision per group: any lane of the segment that flagged
+            const unsigned flag = __ballot_sync(0xffffffffu, prec);
+            prec = ((flag >> (gs * kLanesPerGroup)) & 0xFFu) != 0;
+        }
+        todo = __ballot_sync(0xffffffffu, valid && refit && prec && sl == 0);
+        if (todo) __syncwarp();
+        while (todo) {
+            const int g = (__ffs(todo) - 1) >> 3;
+            todo &= todo - 1;
+            const int src = g * 8;
+            const float gc = __shfl_sync(0xffffffffu, c, src);
+            const float gR = __shfl_sync(0xffffffffu, R, src);
+            const float gss = __shfl_sync(0xffffffffu, ss, src);
+            const float gdbar = __shfl_sync(0xffffffffu, dbar, src);
+            const bool gh_one = __shfl_sync(0xffffffffu, (int)h_one, src) != 0;
+            const int gkb = __shfl_sync(0xffffffffu, kb, src);
+            if (p.stats && lane == 0) atomicAdd(&p.stats[1], 1u);
+            float ga, ga_lo, gB, gB_lo;
+            coop_precise<G>(ws + g * G, hs + g * G, gh_one, gc, gR * p.invf[gkb], H, qmaxf, gss,
+                            gc + gdbar, &ga, &ga_lo, &gB, &gB_lo);
+            if (gs == g) {
                 a_sel = ga;
                 a_lo = ga_lo;
                 Bsel = gB;
@@ -692,36 +831,42 @@ __global__ void __launch_bounds__(256) k_recon_int(const IntParams p)
         // ---- pass C: outputs of the kept candidate
         if (valid) {
             const float Pb = R * p.invf[kb];
+            const float2 Pb2 = make_float2(Pb, Pb);
+            const float2 a2 = make_float2(a_sel, a_sel), B2 = make_float2(Bsel, Bsel);
+            const float2 alo2 = make_float2(a_lo, a_lo), Blo2 = make_float2(B_lo, B_lo);
+            const bool comp = a_lo != 0.0f || B_lo != 0.0f;
+            const float2 nmagic2 = make_float2(-kRoundMagic, -kRoundMagic);
 #pragma unroll 1
             for (int i = 0; i < NCHK; ++i) {
                 const int e = gs * G + i * 32 + sl * 4;
                 const float4 w4 = lds128(ws + e);
-                const float wv[4] = {w4.x, w4.y, w4.z, w4.w};
-                float rv[4];
+                float2 rv[2];
                 uint32_t cw = 0;
 #pragma unroll
-                for (int jj = 0; jj < 4; ++jj) {
-                    if (flat) {
-                        rv[jj] = wv[jj];
-                    } else {
-                        float t = fmaf(wv[jj] - c, Pb, H);
-                        t = fminf(fmaxf(t, 0.0f), qmaxf);
-                        const float y = __fadd_rn(t, kRoundMagic);
-                        const float q = __fsub_rn(y, kRoundMagic);
-                        // a_lo, B_lo are zero unless the compensated fit ran
-                        rv[jj] = fmaf(a_sel, q, Bsel) + fmaf(a_lo, q, B_lo);
-                        cw |= (__float_as_uint(y) & 0xFFu) << (8 * jj);
-                    }
+                for (int pr = 0; pr < 2; ++pr) {
+                    const float2 wv = pr ? make_float2(w4.z, w4.w) : make_float2(w4.x, w4.y);
+                    float2 t = __ffma2_rn(__fadd2_rn(wv, nc2), Pb2, H2);
+                    t.x = fminf(fmaxf(t.x, 0.0f), qmaxf);
+                    t.y = fminf(fmaxf(t.y, 0.0f), qmaxf);
+                    const float2 y = __fadd2_rn(t, magic2);
+                    const float2 q = __fadd2_rn(y, nmagic2);
+                    rv[pr] = __ffma2_rn(a2, q, B2);
+                    // a_lo, B_lo are nonzero only where the compensated fit ran
+                    if (comp) rv[pr] = __fadd2_rn(rv[pr], __ffma2_rn(alo2, q, Blo2));
+                    if (flat) rv[pr] = wv;
+                    if (p.codes)
+                        cw |= ((__float_as_uint(y.x) & 0xFFu) | ((__float_as_uint(y.y) & 0xFFu) << 8))
+                              << (16 * pr);
                 }
                 const int64_t eo = gbase + i * 32 + sl * 4;
                 if (p.r_bf16) {
                     stg_cs(reinterpret_cast<uint2*>(static_cast<__nv_bfloat16*>(p.r) + eo),
-                           make_uint2(pack_bf16x2(rv[0], rv[1]), pack_bf16x2(rv[2], rv[3])));
+                           make_uint2(pack_bf16x2(rv[0].x, rv[0].y), pack_bf16x2(rv[1].x, rv[1].y)));
                 } else {
                     stg_cs(reinterpret_cast<float4*>(static_cast<float*>(p.r) + eo),
-                           make_float4(rv[0], rv[1], rv[2], rv[3]));
+                           make_float4(rv[0].x, rv[0].y, rv[1].x, rv[1].y));
                 }
-                if (p.codes) stg_cs(reinterpret_cast<uint32_t*>(p.codes + eo), cw);
+                if (p.codes) stg_cs(reinterpret_cast<uint32_t*>(p.codes + eo), flat ? 0u : cw);
             }
             if (sl == 0) {
                 p.a[grp] = flat ? 0.0f : a_sel;
