@@ -71,7 +71,8 @@ def barrier(world):
 def max_over_ranks(x, world):
     if world == 1:
         return x
-    t = torch.tensor([x], dtype=torch.float64, device="cuda")
+    dev = "cuda" if torch.distributed.get_backend() == "nccl" else "cpu"
+    t = torch.tensor([x], dtype=torch.float64, device=dev)
     torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
     return float(t.item())
 
@@ -89,11 +90,13 @@ def bytes_per_step(wlo, elements):
 class Model:
     """All tensors of a workload, resident on the device, with outputs."""
 
-    def __init__(self, wlo, device):
+    def __init__(self, wlo, device, shard=0):
+        """``shard``: the rank's shard of a weak-scaled job -- every rank holds
+        a full model's worth of distinct tensors (seed = shard)."""
         self.wlo = wlo
         self.tensors = []
         for spec in wlo.tensors:
-            d = WL.make_tensor(wlo, spec, device=device)
+            d = WL.make_tensor(wlo, spec, device=device, seed=shard)
             n = spec.numel
             d["r"] = torch.empty((spec.rows, spec.cols), dtype=torch.bfloat16, device=device)
             d["a"] = torch.empty(n // 128, dtype=torch.float32, device=device)
@@ -251,8 +254,10 @@ def kernel_source_hash():
 
 
 def profiled_traffic(kernel_tag):
-    """Per-launch DRAM bytes from the committed ncu summary, if it was taken
-    on the current kernel sources; else None."""
+    """DRAM bytes per weight (dram__bytes_read.sum + dram__bytes_write.sum of
+    one ncu capture, divided by the weights that launch processed) from the
+    committed summary, if it was taken on the current kernel sources; else
+    None."""
     path = os.path.join(ROOT, "profiles", "traffic.txt")
     if not os.path.exists(path):
         return None
@@ -382,7 +387,7 @@ def main():
     stream = torch.cuda.Stream()
     hbm_peak, peak_kind = peaks()
     wlo = WL.workload(args.workload)
-    model = Model(wlo, device)
+    model = Model(wlo, device, shard=rank)
     torch.cuda.synchronize()
     n_el = model.elements
 
@@ -428,7 +433,11 @@ def main():
 
     if rank != 0:
         return
-    traffic = profiled_traffic("k_recon_int_g128_k8" if wlo.fmt == "int" else "k_recon_nvfp4_k8")
+    # per-launch figures: the average launch of the step (the step's tensors
+    # differ in size; bytes and time both scale with the weights processed)
+    tag = "k_recon_int_g%d_k%d" % (wlo.group, len(wlo.clip)) if wlo.fmt == "int" else "k_recon_nvfp4_k%d" % len(wlo.clip)
+    tpw = profiled_traffic(tag)
+    traffic = None if tpw is None else tpw * n_el / len(step.calls)
     line = {
         "metric": METRIC, "value": value, "unit": "weights/s", "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_per_step,
@@ -445,7 +454,10 @@ def main():
                      "frac": achieved / hbm_peak, "traffic": traffic,
                      "peak_kind": peak_kind,
                      "kernel": "k_recon_int<16,1>" if wlo.fmt == "int" else "k_recon_nvfp4<1>",
-                     "bytes_per_weight": step_bytes / n_el},
+                     "bytes_per_weight": step_bytes / n_el,
+                     "launch_bytes": step_bytes / len(step.calls),
+                     "launch_ms": kernel_ms / args.steps / len(step.calls),
+                     "traffic_tag": tag},
         "cpu_baseline": cpu, "e2e": e2e,
         "gpu_launches": len(step.calls) * step.launches_per_call * args.steps,
         "clocks": clk, "sweep": sweep,
