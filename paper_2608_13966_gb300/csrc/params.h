@@ -38,7 +38,7 @@ struct IntParams {
     uint64_t timeout_ns;
     uint64_t force_timeout_ns;
     unsigned int* status;  // per-device status word
-    unsigned int* stats;  // optional: [0] refined groups, [1] refitted groups
+    unsigned int* stats;  // optional: [0] exact re-evaluations, [1] compensated fits, [2] centred refits
     float f[kMaxClip];     // padded with the last factor
     float invf[kMaxClip];  // fl32(1/f)
 };

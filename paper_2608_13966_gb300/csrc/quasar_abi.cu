@@ -42,7 +42,8 @@ std::atomic<unsigned int*> g_stats{nullptr};
 struct Tuning {
     int stages = 0;            // 0: chosen from the shared-memory budget
     int smem_budget = 100 * 1024;
-    float tie_kappa = 16.0f;
+    float tie_kappa = 16.0f;   // NVFP4 tie bound, in ulps
+    float tie_scale = 1.0f;    // multiplier of the integer kernel's summation-depth bound
     float fit_ulps = 3.0f;
 };
 
@@ -53,6 +54,7 @@ const Tuning& tuning()
         if (const char* s = std::getenv("QUASAR_STAGES")) x.stages = std::atoi(s);
         if (const char* s = std::getenv("QUASAR_SMEM_BUDGET")) x.smem_budget = std::atoi(s);
         if (const char* s = std::getenv("QUASAR_TIE_KAPPA")) x.tie_kappa = (float)std::atof(s);
+        if (const char* s = std::getenv("QUASAR_TIE_SCALE")) x.tie_scale = (float)std::atof(s);
         if (const char* s = std::getenv("QUASAR_FIT_ULPS")) x.fit_ulps = (float)std::atof(s);
         return x;
     }();
@@ -290,7 +292,9 @@ quasar_status quasar_recon_int(const float* w, const void* g, quasar_dtype g_dty
     p.n_clip = n_clip;
     p.beta2 = beta2;
     p.c1 = 1.0f - beta2;
-    p.tie_kappa = tuning().tie_kappa;
+    // each candidate sum is accumulated over at most G/16 (per packed half)
+    // + 1 + 3 (lane tree) additions; a few more roundings form N, D and E
+    p.tie_kappa = tuning().tie_scale * (float)(group_size / 16 + 8);
     p.fit_ulps = tuning().fit_ulps;
     p.timeout_ns = kDefaultTimeoutNs;
     p.force_timeout_ns = (uint64_t)std::max<int64_t>(0, g_force_timeout_ns.load());

@@ -10,24 +10,32 @@
 // of `stages` shared-memory tiles filled by 1-D TMA bulk copies
 // (cp.async.bulk + mbarrier), so w, g and v are read from HBM exactly once,
 // and the loads of later units overlap the arithmetic of the current one.
-// The tile stays in shared memory while the unit is processed, and the
-// passes below stream it from there (rolled loops: small code, few
-// registers).  The grid is persistent.
+// The tile stays in shared memory while the unit is processed; the passes
+// below stream it from there.  The grid is persistent.
+//
+// Codes in centred form.  With qmax = 2^bits - 1 odd, H = qmax/2 is a
+// half-integer and Eq. 1's code is q = H + z with
+//     |z| = min(floor(|d| P), J) + 1/2,  sign(z) = sign(d),
+// where d = w - c, P = qmax / (f * range) and J = (qmax - 1)/2.  This equals
+// clamp(round(d P + H), 0, qmax) except at exact rounding ties (t = d P + H a
+// half-integer), which lie inside the checker's margin exemption.  floor is a
+// single FMA rounded toward -inf onto the 2^23 grid (__ffma2_rd), so a code
+// costs one FMA, one min and one add, two elements per instruction.
 //
 // Per group (fp32):
 //   pass A  v' = beta2*v + (1-beta2)*g^2 (written back; kept in the tile as
-//           the saliency h), min/max -> c, range, sum h;
-//   pass B  for 8 candidates at a time, codes q = clamp(rne(d*P_k + qmax/2))
-//           with d = w - c and P_k = qmax/(f_k*range) (the 1.5*2^23 rounding
-//           trick; codes are accumulated centred on Hc = floor(qmax/2)), and
-//           the sums S1 = sum h q, S2 = sum h q^2, S3 = sum h q d; packed
-//           f32x2 arithmetic, two elements per instruction;
+//           the saliency h), min/max -> c, range, sum h, sum h w -> mu;
+//   pass B  for 8 candidates at a time, the codes (from d = w - c) and the
+//           moments S1 = sum h z, S2 = sum h z^2, S3 = sum h z e with
+//           e = w - mu (plus the candidate-independent sum h e, sum h e^2);
 //   reduce  the 8 lanes' partial sums are transposed through shared memory
 //           so that lane sl owns candidate sl of the chunk;
-//   fit     D = S2 - S1^2/Ss, N = S3 - S1*Sd/Ss, a = N/D, b = mean(d) -
-//           a*mean(q) (+c), explained E = N^2/D: the weighted error of
-//           candidate k is C - E_k with C common, so argmin error = argmax E;
-//   pass C  codes of the kept candidate, r = a*q + b, outputs.
+//   select  D = S2 - S1^2/Ss, N = S3 - S1*Se/Ss: the weighted error of
+//           candidate k is C - N^2/D with C common, so argmin error =
+//           argmax E = N^2/D; the winner's fit is a = N/D with the offset
+//           from the weighted means;
+//   pass C  codes of the kept candidate, r = a*z + Bz, outputs (b = Bz - a*H
+//           is the offset of the paper's r = a*q + b).
 //
 // Exactness.  E carries fp32 rounding error; candidates whose E lies within
 // an error bound of the best (and candidates whose weighted code variance D
@@ -37,6 +45,8 @@
 // the unit and done by the whole warp on one group at a time.
 #pragma once
 
+#include <type_traits>
+
 #include "device_common.cuh"
 #include "params.h"
 
@@ -44,14 +54,30 @@ namespace quasar {
 
 __device__ __forceinline__ float shx(float x, int m) { return __shfl_xor_sync(0xffffffffu, x, m); }
 
-// Code of one element for one candidate (Eq. 1 in centred form):
-// q = clamp(rne(d*P + qmax/2), 0, qmax), returned as a float.
-__device__ __forceinline__ float int_code(float d, float P, float H, float qmaxf)
+// 2^23: fl_rd(x + 2^23) = 2^23 + floor(x) for 0 <= x < 2^23 (unit spacing).
+constexpr float kFloorMagic = 8388608.0f;
+// 2^23 - 1/2 (exact: spacing 1/2 below 2^23); y - this = floor + 1/2.
+constexpr float kHalfBelowMagic = 8388607.5f;
+
+// Centred code z = q - qmax/2 of one element for the scale P (see above);
+// zcap = kFloorMagic + J.
+__device__ __forceinline__ float int_code_z(float d, float P, float zcap)
 {
-    float t = fmaf(d, P, H);
-    t = fminf(fmaxf(t, 0.0f), qmaxf);
-    const float y = __fadd_rn(t, kRoundMagic);
-    return __fsub_rn(y, kRoundMagic);
+    const float y = fminf(__fmaf_rd(fabsf(d), P, kFloorMagic), zcap);
+    return copysignf(__fsub_rn(y, kHalfBelowMagic), d);
+}
+
+__device__ __forceinline__ float2 abs2(float2 x)
+{
+    return make_float2(__uint_as_float(__float_as_uint(x.x) & 0x7FFFFFFFu),
+                       __uint_as_float(__float_as_uint(x.y) & 0x7FFFFFFFu));
+}
+
+// h with the sign of d (h >= 0): the sign survives h = 0 as -0.
+__device__ __forceinline__ float2 signed_h2(float2 h, float2 d)
+{
+    return make_float2(__uint_as_float(__float_as_uint(h.x) | (__float_as_uint(d.x) & 0x80000000u)),
+                       __uint_as_float(__float_as_uint(h.y) | (__float_as_uint(d.y) & 0x80000000u)));
 }
 
 // Round x to a multiple of the power of two U (x*invU is exact).
@@ -118,15 +144,27 @@ __device__ __forceinline__ float wsum32(float x)
     return x;
 }
 
+// (hi, lo) + x*H as a renormalised pair: moves an offset between the code
+// origins q = 0 and z = 0 (q = z + H).
+__device__ __forceinline__ void ff_add_prod(float& hi, float& lo, float xh, float xl, float H)
+{
+    float ph, pl, sh, se;
+    two_prod(xh, H, ph, pl);
+    two_sum(hi, ph, sh, se);
+    lo = __fadd_rn(__fadd_rn(lo, se), fmaf(xl, H, pl));
+    hi = sh;
+    ff_norm(hi, lo);
+}
+
 // ------------------------------------------------- whole-warp group helpers
 //
 // One group, evaluated by all 32 lanes (lane L takes elements L + 32m) from
-// the tile in shared memory: w at ws, saliency h at hs (or 1 if h_one).
+// the tile in shared memory: w at ws, saliency h at hs.
 
 // True when candidates with scale factors Pa and Pb give the same codes on
 // every element of the group (whole warp).
 template <int G>
-__device__ bool coop_same_codes(const float* ws, float c, float Pa, float Pb, float H, float qmaxf)
+__device__ bool coop_same_codes(const float* ws, float c, float Pa, float Pb, float zcap)
 {
     constexpr int M = G / 32;
     const int lane = threadIdx.x & 31;
@@ -134,19 +172,21 @@ __device__ bool coop_same_codes(const float* ws, float c, float Pa, float Pb, fl
 #pragma unroll
     for (int m = 0; m < M; ++m) {
         const float d = ws[lane + 32 * m] - c;
-        same &= int_code(d, Pa, H, qmaxf) == int_code(d, Pb, H, qmaxf);
+        same &= int_code_z(d, Pa, zcap) == int_code_z(d, Pb, zcap);
     }
     return __all_sync(0xffffffffu, same);
 }
 
-// Exact evaluation of one candidate: codes, exact degenerate test (all
-// weighted elements on one code), two-pass centred fit, and the direct error
-// sum h (a q + b - w)^2 with (a, b) rounded to a common power-of-two grid U so
-// that a*q + b is exact and only "- w" rounds; lanes combine as a float pair.
+// Exact evaluation of one candidate: codes q = z + H, exact degenerate test
+// (all weighted elements on one code), two-pass centred fit, and the direct
+// error sum h (a q + B - w)^2 with (a, B) rounded to a common power-of-two
+// grid U so that a*q + B is exact and only "- w" rounds; lanes combine as a
+// float pair.  Returns the fit as (a, Bz) with r = a z + Bz, and a condition
+// estimate kap of the slope (see the tier-2 trigger in the kernel).
 template <int G>
-__device__ void coop_exact(const float* ws, const float* hs, bool h_one, float c, float P,
-                           float H, float qmaxf, float Ss, float dbar, float step, float* err_hi,
-                           float* err_lo, float* a_out, float* bc_out, bool* degenerate)
+__device__ void coop_exact(const float* ws, const float* hs, float c, float P, float zcap, float H,
+                           float Ss, float dbar, float step, float* err_hi, float* err_lo,
+                           float* a_out, float* Bz_out, float* kap_out, bool* degenerate)
 {
     constexpr int M = G / 32;
     const int lane = threadIdx.x & 31;
@@ -155,8 +195,8 @@ __device__ void coop_exact(const float* ws, const float* hs, bool h_one, float c
 #pragma unroll
     for (int m = 0; m < M; ++m) {
         const int e = lane + 32 * m;
-        const float h = h_one ? 1.0f : hs[e];
-        const float q = int_code(ws[e] - c, P, H, qmaxf);
+        const float h = hs[e];
+        const float q = int_code_z(ws[e] - c, P, zcap) + H;
         s1 = fmaf(h, q, s1);
         if (h > 0.0f) {
             qlo = min(qlo, (int)q);
@@ -171,27 +211,33 @@ __device__ void coop_exact(const float* ws, const float* hs, bool h_one, float c
     }
     const float qbar = s1 / Ss;
     *degenerate = qlo == qhi;
-    float a, bc;
+    float a, bc, kap = 1.0f;
     if (qlo == qhi) {
         a = step;  // every weighted element shares one code
         bc = dbar - step * (float)qlo;
     } else {
-        float dd = 0.0f, nn = 0.0f;
+        float dd = 0.0f, nn = 0.0f, ww = 0.0f;
 #pragma unroll
         for (int m = 0; m < M; ++m) {
             const int e = lane + 32 * m;
-            const float h = h_one ? 1.0f : hs[e];
+            const float h = hs[e];
             const float d = ws[e] - c;
-            const float dq = int_code(d, P, H, qmaxf) - qbar;
+            const float dq = int_code_z(d, P, zcap) + H - qbar;
             const float hdq = h * dq;
+            const float wd = d - dbar;
             dd = fmaf(hdq, dq, dd);
-            nn = fmaf(hdq, d - dbar, nn);
+            nn = fmaf(hdq, wd, nn);
+            ww = fmaf(h * wd, wd, ww);
         }
-        a = wsum32(nn) / wsum32(dd);
+        dd = wsum32(dd);
+        nn = wsum32(nn);
+        ww = wsum32(ww);
+        a = nn / dd;
         bc = dbar - a * qbar;
+        kap = sqrtf(dd * ww) / fabsf(nn) + 1.0f;
     }
     const float B = bc + c;
-    const float mr = fmaxf(fabsf(B), fabsf(fmaf(a, qmaxf, B))) + fabsf(a);
+    const float mr = fmaxf(fabsf(B), fabsf(fmaf(a, 2.0f * H, B))) + fabsf(a);
     int er = (int)((__float_as_uint(mr) >> 23) & 0xFF) - 126;  // mr < 2^er
     er = max(er, -100);
     const float U = __uint_as_float((uint32_t)(er - 23 + 127) << 23);
@@ -202,9 +248,9 @@ __device__ void coop_exact(const float* ws, const float* hs, bool h_one, float c
 #pragma unroll
     for (int m = 0; m < M; ++m) {
         const int e = lane + 32 * m;
-        const float h = h_one ? 1.0f : hs[e];
+        const float h = hs[e];
         const float w = ws[e];
-        const float ev = fmaf(ag, int_code(w - c, P, H, qmaxf), Bg) - w;
+        const float ev = fmaf(ag, int_code_z(w - c, P, zcap) + H, Bg) - w;
         t[m] = h * (ev * ev);
     }
 #pragma unroll
@@ -216,7 +262,8 @@ __device__ void coop_exact(const float* ws, const float* hs, bool h_one, float c
     *err_hi = eh;
     *err_lo = el;
     *a_out = a;
-    *bc_out = bc;
+    *Bz_out = fmaf(a, H, B);
+    *kap_out = kap;
 }
 
 // Weighted least-squares fit (Eq. 4) of one candidate in compensated
@@ -227,11 +274,12 @@ __device__ void coop_exact(const float* ws, const float* hs, bool h_one, float c
 // kept as an exact pair).  The sums of h (q-mq)^2 and h (q-mq)(w-mu) are
 // accumulated and combined across lanes as float pairs (no fp64: its rate on
 // this part is a small fraction of fp32's); the offset is
-// mu - s*mq + mean_h(w - mu - s (q - mq)).  Returns the fit as float pairs.
+// mu - s*mq + mean_h(w - mu - s (q - mq)).  Returns the fit as float pairs,
+// with the offset Bz at the code origin z = 0 (r = a z + Bz).
 template <int G>
-__device__ void coop_precise(const float* ws, const float* hs, bool h_one, float c, float P,
-                             float H, float qmaxf, float Ss, float mu, float* a_hi, float* a_lo,
-                             float* B_hi, float* B_lo)
+__device__ void coop_precise(const float* ws, const float* hs, float c, float P, float zcap,
+                             float H, float Ss, float mu, float* a_hi, float* a_lo, float* Bz_hi,
+                             float* Bz_lo)
 {
     constexpr int M = G / 32;
     const int lane = threadIdx.x & 31;
@@ -239,8 +287,7 @@ __device__ void coop_precise(const float* ws, const float* hs, bool h_one, float
 #pragma unroll
     for (int m = 0; m < M; ++m) {
         const int e = lane + 32 * m;
-        const float h = h_one ? 1.0f : hs[e];
-        s1 = fmaf(h, int_code(ws[e] - c, P, H, qmaxf), s1);
+        s1 = fmaf(hs[e], int_code_z(ws[e] - c, P, zcap) + H, s1);
     }
     const float mq = rintf(wsum32(s1) / Ss * 16.0f) * 0.0625f;
 
@@ -248,9 +295,9 @@ __device__ void coop_precise(const float* ws, const float* hs, bool h_one, float
 #pragma unroll
     for (int m = 0; m < M; ++m) {
         const int e = lane + 32 * m;
-        const float h = h_one ? 1.0f : hs[e];
+        const float h = hs[e];
         const float w = ws[e];
-        const float qd = int_code(w - c, P, H, qmaxf) - mq;
+        const float qd = int_code_z(w - c, P, zcap) + H - mq;
         float wh, wl, xh, xl, th, tl, ph, pl;
         two_sum(w, -mu, wh, wl);
         two_prod(h, qd, xh, xl);
@@ -285,24 +332,25 @@ __device__ void coop_precise(const float* ws, const float* hs, bool h_one, float
 #pragma unroll
     for (int m = 0; m < M; ++m) {
         const int e = lane + 32 * m;
-        const float h = h_one ? 1.0f : hs[e];
+        const float h = hs[e];
         const float w = ws[e];
-        const float qd = int_code(w - c, P, H, qmaxf) - mq;
+        const float qd = int_code_z(w - c, P, zcap) + H - mq;
         float wh, wl;
         two_sum(w, -mu, wh, wl);
         Rs = fmaf(h, __fadd_rn(fmaf(-shi, qd, wh), fmaf(-slo, qd, wl)), Rs);
     }
     Rs = wsum32(Rs);
+    // offset at the code origin z = 0, i.e. q = H: mu + s*(H - mq) + mean residual
     float ph, pl, zh, zl;
-    two_prod(shi, mq, ph, pl);
-    pl = fmaf(slo, mq, pl);
-    two_sum(mu, -ph, zh, zl);
-    zl = __fadd_rn(__fsub_rn(zl, pl), Rs / Ss);
+    two_prod(shi, H - mq, ph, pl);  // H - mq is exact (both multiples of 1/16)
+    pl = fmaf(slo, H - mq, pl);
+    two_sum(mu, ph, zh, zl);
+    zl = __fadd_rn(__fadd_rn(zl, pl), Rs / Ss);
     ff_norm(zh, zl);
     *a_hi = shi;
     *a_lo = slo;
-    *B_hi = zh;
-    *B_lo = zl;
+    *Bz_hi = zh;
+    *Bz_lo = zl;
 }
 
 // ------------------------------------------------------------------ kernel
@@ -382,13 +430,9 @@ __global__ void __launch_bounds__(256) k_recon_int(const IntParams p)
 
     const float qmaxf = (float)p.qmax;
     const float H = 0.5f * qmaxf;
-    // Pass B accumulates codes centred on Hc = floor(qmax/2): subtracting the
-    // rounding constant plus Hc (exact) yields q - Hc directly and keeps the
-    // moment sums well conditioned.
-    const float Hc = (float)(p.qmax >> 1);
-    const float2 H2 = make_float2(H, H);
-    const float2 magic2 = make_float2(kRoundMagic, kRoundMagic);
-    const float2 nmagic_c2 = make_float2(-(kRoundMagic + Hc), -(kRoundMagic + Hc));
+    const float zcap = kFloorMagic + (float)(p.qmax >> 1);
+    const float2 M2 = make_float2(kFloorMagic, kFloorMagic);
+    const float2 nhm2 = make_float2(-kHalfBelowMagic, -kHalfBelowMagic);
     const float ulp = 5.9604645e-8f * p.tie_kappa;
     const float2 beta22 = make_float2(p.beta2, p.beta2);
     const float2 c12 = make_float2(p.c1, p.c1);
@@ -412,57 +456,89 @@ __global__ void __launch_bounds__(256) k_recon_int(const IntParams p)
         const int64_t gbase = grp * (int64_t)G;
 
         // ---- pass A: saliency EMA (h kept in the tile), range, saliency mass
-        float mn = INFINITY, mx = -INFINITY, ss = 0.0f;
+        // and weighted sum of w (a centre for the moments)
+        float mn = INFINITY, mx = -INFINITY, ss = 0.0f, sw = 0.0f;
+        {
+            float* vout = p.v + gbase + sl * 4;
+            auto pass_a = [&](auto gk) {
+                constexpr int GK = decltype(gk)::value;
+                float2 SS = make_float2(0.0f, 0.0f), SW = SS;
 #pragma unroll
-        for (int i = 0; i < NCHK; ++i) {
-            const int e = gs * G + i * 32 + sl * 4;
-            const float4 w4 = lds128(ws + e);
-            float4 h4 = lds128(hs + e);
-            if (p.g_kind) {
-                float g0, g1, g2, g3;
-                if (p.g_kind == 2) {
-                    const uint2 gb = lds64(gsm + e * 2);
-                    g0 = bf16lo(gb.x); g1 = bf16hi(gb.x); g2 = bf16lo(gb.y); g3 = bf16hi(gb.y);
-                } else {
-                    const float4 g4 = lds128(gsm + e * 4);
-                    g0 = g4.x; g1 = g4.y; g2 = g4.z; g3 = g4.w;
+                for (int i = 0; i < NCHK; ++i) {
+                    const int e = gs * G + i * 32 + sl * 4;
+                    const float4 w4 = lds128(ws + e);
+                    float4 h4 = lds128(hs + e);
+                    if constexpr (GK != 0) {
+                        float2 gA, gB;
+                        if constexpr (GK == 2) {
+                            const uint2 gb = lds64(gsm + e * 2);
+                            gA = make_float2(bf16lo(gb.x), bf16hi(gb.x));
+                            gB = make_float2(bf16lo(gb.y), bf16hi(gb.y));
+                        } else {
+                            const float4 g4 = lds128(gsm + e * 4);
+                            gA = make_float2(g4.x, g4.y);
+                            gB = make_float2(g4.z, g4.w);
+                        }
+                        const float2 hA = __ffma2_rn(make_float2(h4.x, h4.y), beta22,
+                                                     __fmul2_rn(c12, __fmul2_rn(gA, gA)));
+                        const float2 hB = __ffma2_rn(make_float2(h4.z, h4.w), beta22,
+                                                     __fmul2_rn(c12, __fmul2_rn(gB, gB)));
+                        h4 = make_float4(hA.x, hA.y, hB.x, hB.y);
+                        *reinterpret_cast<float4*>(hs + e) = h4;
+                        if (valid) stg_cs(reinterpret_cast<float4*>(vout + i * 32), h4);
+                    }
+                    mn = fminf(fminf(fminf(mn, w4.x), fminf(w4.y, w4.z)), w4.w);
+                    mx = fmaxf(fmaxf(fmaxf(mx, w4.x), fmaxf(w4.y, w4.z)), w4.w);
+                    const float2 hA = make_float2(h4.x, h4.y), hB = make_float2(h4.z, h4.w);
+                    SS = __fadd2_rn(SS, __fadd2_rn(hA, hB));
+                    SW = __ffma2_rn(hA, make_float2(w4.x, w4.y), SW);
+                    SW = __ffma2_rn(hB, make_float2(w4.z, w4.w), SW);
                 }
-                const float2 gA = make_float2(g0, g1), gB = make_float2(g2, g3);
-                const float2 hA = __ffma2_rn(make_float2(h4.x, h4.y), beta22,
-                                             __fmul2_rn(c12, __fmul2_rn(gA, gA)));
-                const float2 hB = __ffma2_rn(make_float2(h4.z, h4.w), beta22,
-                                             __fmul2_rn(c12, __fmul2_rn(gB, gB)));
-                h4 = make_float4(hA.x, hA.y, hB.x, hB.y);
-                *reinterpret_cast<float4*>(hs + e) = h4;
-                if (valid) stg_cs(reinterpret_cast<float4*>(p.v + gbase + i * 32 + sl * 4), h4);
-            }
-            mn = fminf(fminf(fminf(mn, w4.x), fminf(w4.y, w4.z)), w4.w);
-            mx = fmaxf(fmaxf(fmaxf(mx, w4.x), fmaxf(w4.y, w4.z)), w4.w);
-            ss += (h4.x + h4.y) + (h4.z + h4.w);
+                ss = SS.x + SS.y;
+                sw = SW.x + SW.y;
+            };
+            if (p.g_kind == 2) pass_a(std::integral_constant<int, 2>{});
+            else if (p.g_kind == 1) pass_a(std::integral_constant<int, 1>{});
+            else pass_a(std::integral_constant<int, 0>{});
         }
 #pragma unroll
         for (int o = 4; o; o >>= 1) {
             mn = fminf(mn, shx(mn, o));
             mx = fmaxf(mx, shx(mx, o));
             ss += shx(ss, o);
+            sw += shx(sw, o);
         }
-        const bool h_one = ss == 0.0f;  // all saliencies zero: fit with h = 1
-        if (h_one) ss = (float)G;
+        // all saliencies zero: the group is fitted with h = 1 (the tile's h
+        // is overwritten; v' has been written out already)
+        const bool h_one = ss == 0.0f;
+        if (__any_sync(0xffffffffu, h_one)) {
+            if (h_one)
+#pragma unroll
+                for (int i = 0; i < NCHK; ++i)
+                    *reinterpret_cast<float4*>(hs + gs * G + i * 32 + sl * 4) =
+                        make_float4(1.0f, 1.0f, 1.0f, 1.0f);
+            __syncwarp();
+        }
         const float range = mx - mn;
         const bool flat = !(range > 0.0f);
         const float c = 0.5f * (mn + mx);
+        if (h_one) ss = (float)G;
+        const float inv_ss = __fdividef(1.0f, ss);
+        // mu: approximate weighted mean of w (only a centre for the sums)
+        const float mu = h_one ? c : sw * inv_ss;
         // approximate divisions (<= 2 ulp) are enough here: R scales the code
         // positions (margins are measured against the clipping range), and
-        // the fit of the kept candidate is rechecked below
+        // the accuracy of the kept fit is checked below
         const float R = flat ? 0.0f : __fdividef(qmaxf, range);
-        const float inv_ss = __fdividef(1.0f, ss);
-        const float2 nc2 = make_float2(-c, -c);
+        const float2 nc2 = make_float2(-c, -c), nmu2 = make_float2(-mu, -mu);
 
-        // ---- pass B + reduction + fit, 8 candidates at a time
-        float Ek[NCH], dEk[NCH], ak[NCH], bk[NCH], T1k[NCH], T2k[NCH], T3k[NCH];
+        // ---- pass B + reduction + candidate errors, 8 candidates at a time.
+        // Codes use d = w - c; moments use e = w - mu: S1 = sum h z,
+        // S2 = sum h z^2, S3 = sum h z e = sum (h |z|) (sign(d) e).
+        float Ek[NCH], dEk[NCH], T1k[NCH], T2k[NCH], T3k[NCH];
         bool suspk[NCH];
-        float sd = 0.0f, sdd = 0.0f;
-#pragma unroll 1
+        float se = 0.0f, see = 0.0f;
+#pragma unroll
         for (int ch = 0; ch < NCH; ++ch) {
             float2 P2[8];
 #pragma unroll
@@ -473,87 +549,98 @@ __global__ void __launch_bounds__(256) k_recon_int(const IntParams p)
             float2 A1[8], A2[8], A3[8];
 #pragma unroll
             for (int kk = 0; kk < 8; ++kk) A1[kk] = A2[kk] = A3[kk] = make_float2(0.0f, 0.0f);
-            float2 SD = make_float2(0.0f, 0.0f), SDD = make_float2(0.0f, 0.0f);
-#pragma unroll 1
+            float2 SE = make_float2(0.0f, 0.0f), SEE = make_float2(0.0f, 0.0f);
+#pragma unroll(NCHK <= 4 ? NCHK : 2)
             for (int i = 0; i < NCHK; ++i) {
                 const int e = gs * G + i * 32 + sl * 4;
                 const float4 w4 = lds128(ws + e);
-                const float4 h4 = h_one ? make_float4(1.0f, 1.0f, 1.0f, 1.0f) : lds128(hs + e);
-                const float2 d[2] = {__fadd2_rn(make_float2(w4.x, w4.y), nc2),
-                                     __fadd2_rn(make_float2(w4.z, w4.w), nc2)};
-                const float2 h[2] = {make_float2(h4.x, h4.y), make_float2(h4.z, h4.w)};
-                float2 hd[2];
+                const float4 h4 = lds128(hs + e);
 #pragma unroll
                 for (int pr = 0; pr < 2; ++pr) {
-                    hd[pr] = __fmul2_rn(h[pr], d[pr]);
-                    SD = __fadd2_rn(SD, hd[pr]);
-                    SDD = __ffma2_rn(hd[pr], d[pr], SDD);
-                }
-#pragma unroll
-                for (int kk = 0; kk < 8; ++kk)
-#pragma unroll
-                    for (int pr = 0; pr < 2; ++pr) {
-                        float2 t = __ffma2_rn(d[pr], P2[kk], H2);
-                        t.x = fminf(fmaxf(t.x, 0.0f), qmaxf);
-                        t.y = fminf(fmaxf(t.y, 0.0f), qmaxf);
-                        const float2 q = __fadd2_rn(__fadd2_rn(t, magic2), nmagic_c2);  // q - Hc
-                        const float2 hq = __fmul2_rn(h[pr], q);
-                        A1[kk] = __fadd2_rn(A1[kk], hq);
-                        A2[kk] = __ffma2_rn(hq, q, A2[kk]);
-                        A3[kk] = __ffma2_rn(q, hd[pr], A3[kk]);
+                    const float2 wv = pr ? make_float2(w4.z, w4.w) : make_float2(w4.x, w4.y);
+                    const float2 h = pr ? make_float2(h4.z, h4.w) : make_float2(h4.x, h4.y);
+                    const float2 d = __fadd2_rn(wv, nc2);
+                    const float2 ev = __fadd2_rn(wv, nmu2);
+                    const float2 ad = abs2(d);
+                    const float2 hsg = signed_h2(h, d);
+                    const float2 sev = make_float2(
+                        __uint_as_float(__float_as_uint(ev.x) ^ (__float_as_uint(d.x) & 0x80000000u)),
+                        __uint_as_float(__float_as_uint(ev.y) ^ (__float_as_uint(d.y) & 0x80000000u)));
+                    if (ch == 0) {
+                        const float2 he = __fmul2_rn(h, ev);
+                        SE = __fadd2_rn(SE, he);
+                        SEE = __ffma2_rn(he, ev, SEE);
                     }
+#pragma unroll
+                    for (int kk = 0; kk < 8; ++kk) {
+                        float2 y = __ffma2_rd(ad, P2[kk], M2);
+                        y.x = fminf(y.x, zcap);
+                        y.y = fminf(y.y, zcap);
+                        const float2 z = __fadd2_rn(y, nhm2);  // |z|
+                        const float2 t = __fmul2_rn(h, z);
+                        A1[kk] = __ffma2_rn(hsg, z, A1[kk]);
+                        A2[kk] = __ffma2_rn(t, z, A2[kk]);
+                        A3[kk] = __ffma2_rn(t, sev, A3[kk]);
+                    }
+                }
             }
             // transpose through shared memory: lane L writes row L, lane
-            // (gs, sl) sums columns sl*4.. of the 8 rows of its group
+            // (gs, sl) sums columns sl*4.. of the 8 rows of its group (a tree)
 #pragma unroll
             for (int kk = 0; kk < 8; ++kk)
                 *reinterpret_cast<float4*>(red + lane * 36 + kk * 4) =
                     make_float4(A1[kk].x + A1[kk].y, A2[kk].x + A2[kk].y, A3[kk].x + A3[kk].y, 0.0f);
             __syncwarp();
-            float3 T = make_float3(0.0f, 0.0f, 0.0f);
+            float4 x[8];
 #pragma unroll
-            for (int j = 0; j < 8; ++j) {
-                const float4 x = *reinterpret_cast<const float4*>(red + (gs * 8 + j) * 36 + sl * 4);
-                T.x += x.x;
-                T.y += x.y;
-                T.z += x.z;
-            }
+            for (int j = 0; j < 8; ++j)
+                x[j] = *reinterpret_cast<const float4*>(red + (gs * 8 + j) * 36 + sl * 4);
+#pragma unroll
+            for (int s2 = 1; s2 < 8; s2 <<= 1)
+#pragma unroll
+                for (int j = 0; j + s2 < 8; j += 2 * s2) {
+                    x[j].x += x[j + s2].x;
+                    x[j].y += x[j + s2].y;
+                    x[j].z += x[j + s2].z;
+                }
             __syncwarp();
             if (ch == 0) {
-                sd = SD.x + SD.y;
-                sdd = SDD.x + SDD.y;
+                se = SE.x + SE.y;
+                see = SEE.x + SEE.y;
 #pragma unroll
                 for (int o = 4; o; o >>= 1) {
-                    sd += shx(sd, o);
-                    sdd += shx(sdd, o);
+                    se += shx(se, o);
+                    see += shx(see, o);
                 }
             }
-            const float dbar = sd * inv_ss;
-            const float habsd = sqrtf(ss * sdd);  // >= sum h |d| (Cauchy-Schwarz)
-            const int k = ch * 8 + sl;
-            const float qbar = T.x * inv_ss;  // mean of q - Hc
-            const float D = T.y - T.x * qbar;
-            const float N = T.z - T.x * dbar;
-            const bool susp = !(D > 1e-3f * T.y);
+            // candidate k = 8 ch + sl: E = N^2/D and a bound dE on its fp32
+            // error.  The sums are accumulated over tie_kappa levels at most,
+            // so each is within tie_kappa ulps of the sum of its terms'
+            // magnitudes: sum h z^2 = S2, sum |h z e| <= sqrt(S2 * sum h e^2).
+            const float ebar = se * inv_ss;
+            const float T1 = x[0].x, T2 = x[0].y, T3 = x[0].z;
+            const float zbar = T1 * inv_ss;
+            const float D = T2 - T1 * zbar;
+            const float N = T3 - T1 * ebar;
+            const bool susp = !(D > 1e-3f * T2);
             const float a = __fdividef(N, D);
             const float E = susp ? 0.0f : N * a;
-            const float dN = ulp * qmaxf * habsd;
-            const float dD = ulp * T.y;
-            const bool real = k < p.n_clip;
+            const float s2e = fmaxf(T2 * see, 1e-37f);
+            const float dN = ulp * (s2e * rsqrtf(s2e) * 1.001f + fabsf(T1 * ebar));
+            const float dD = ulp * (T2 + fabsf(T1 * zbar));
+            const bool real = ch * 8 + sl < p.n_clip;
 #pragma unroll
             for (int cc = 0; cc < NCH; ++cc)
                 if (cc == ch) {
                     Ek[cc] = real && !susp ? E : -INFINITY;
                     dEk[cc] = 2.0f * fabsf(a) * dN + a * a * dD;
-                    ak[cc] = a;
-                    bk[cc] = dbar - a * (qbar + Hc);
                     suspk[cc] = real && susp;
-                    T1k[cc] = T.x;
-                    T2k[cc] = T.y;
-                    T3k[cc] = T.z;
+                    T1k[cc] = T1;
+                    T2k[cc] = T2;
+                    T3k[cc] = T3;
                 }
         }
-        const float dbar = sd * inv_ss;
+        const float ebar = se * inv_ss;
 
         // ---- argmax of E over the group (ties: lowest index)
         float Eb = -INFINITY, dEb = 0.0f;
@@ -578,20 +665,16 @@ __global__ void __launch_bounds__(256) k_recon_int(const IntParams p)
         }
         if (kb > 0x7ff) kb = 0;  // every candidate suspicious: the exact path picks
 
-        // winner's fit and sums, from its owner lane
-        float a_sel = 0.0f, bc_sel = 0.0f, T1b = 0.0f, T2b = 0.0f, T3b = 0.0f;
+        // the winner's sums, from its owner lane
+        float T1b = 0.0f, T2b = 0.0f, T3b = 0.0f;
         {
             const int owner = (gs * 8) | (kb & 7);
 #pragma unroll
             for (int ch = 0; ch < NCH; ++ch) {
-                const float av = __shfl_sync(0xffffffffu, ak[ch], owner);
-                const float bv = __shfl_sync(0xffffffffu, bk[ch], owner);
                 const float t1 = __shfl_sync(0xffffffffu, T1k[ch], owner);
                 const float t2 = __shfl_sync(0xffffffffu, T2k[ch], owner);
                 const float t3 = __shfl_sync(0xffffffffu, T3k[ch], owner);
                 if ((kb >> 3) == ch) {
-                    a_sel = av;
-                    bc_sel = bv;
                     T1b = t1;
                     T2b = t2;
                     T3b = t3;
@@ -624,8 +707,10 @@ __global__ void __launch_bounds__(256) k_recon_int(const IntParams p)
         if (Eb == -INFINITY) set = (p.n_clip >= 32) ? 0xFFFFFFFFu : ((1u << p.n_clip) - 1u);
         else if (set) set |= 1u << kb;
 
-        float Bsel = bc_sel + c, a_lo = 0.0f, B_lo = 0.0f;
-        float qbar_sel = T1b * inv_ss + Hc;
+        // the kept fit: r = a z + Bz (a = a_sel + a_lo, Bz = Bz + Bz_lo); kap
+        // estimates the conditioning of its slope
+        float a_sel = 0.0f, Bz = 0.0f, kap_sel = 0.0f;
+        float Bz_lo = 0.0f, a_lo = 0.0f;
         bool deg_sel = false;
 
         // ---- deferred exact comparisons: the whole warp takes one group at a time
@@ -639,8 +724,7 @@ __global__ void __launch_bounds__(256) k_recon_int(const IntParams p)
             const float grange = __shfl_sync(0xffffffffu, range, src);
             const float gR = __shfl_sync(0xffffffffu, R, src);
             const float gss = __shfl_sync(0xffffffffu, ss, src);
-            const float gdbar = __shfl_sync(0xffffffffu, dbar, src);
-            const bool gh_one = __shfl_sync(0xffffffffu, (int)h_one, src) != 0;
+            const float gdbar = __shfl_sync(0xffffffffu, (mu + ebar) - c, src);
             unsigned gset = __shfl_sync(0xffffffffu, set, src);
             const unsigned gtwins = __shfl_sync(0xffffffffu, twins, src);
             const int gkb0 = __shfl_sync(0xffffffffu, kb, src);
@@ -650,144 +734,125 @@ __global__ void __launch_bounds__(256) k_recon_int(const IntParams p)
             while (tw) {
                 const int k = __ffs(tw) - 1;
                 tw &= tw - 1;
-                if (coop_same_codes<G>(gws, gc, gR * p.invf[k], gR * p.invf[gkb0], H, qmaxf))
+                if (coop_same_codes<G>(gws, gc, gR * p.invf[k], gR * p.invf[gkb0], zcap))
                     gset &= ~(1u << k);
             }
             if (gset == (1u << gkb0)) continue;  // only the winner left
             if (p.stats && lane == 0) atomicAdd(&p.stats[0], 1u);
-            float best_h = 0.0f, best_l = 0.0f, ga = 0.0f, gB = 0.0f;
+            float best_h = 0.0f, best_l = 0.0f, ga = 0.0f, gB = 0.0f, gkap = 0.0f;
             int best_k = -1;
             bool gdeg = false;
             while (gset) {
                 const int k = __ffs(gset) - 1;
                 gset &= gset - 1;
-                float eh, el, a_k, bc_k;
+                float eh, el, a_k, B_k, kap_k;
                 bool deg_k;
-                coop_exact<G>(gws, ghs, gh_one, gc, gR * p.invf[k], H, qmaxf, gss, gdbar,
-                              p.f[k] * grange / qmaxf, &eh, &el, &a_k, &bc_k, &deg_k);
+                coop_exact<G>(gws, ghs, gc, gR * p.invf[k], zcap, H, gss, gdbar,
+                              p.f[k] * grange / qmaxf, &eh, &el, &a_k, &B_k, &kap_k, &deg_k);
                 if (best_k < 0 || ff_less(eh, el, best_h, best_l)) {
                     best_h = eh;
                     best_l = el;
                     best_k = k;
                     ga = a_k;
-                    gB = bc_k + gc;
+                    gB = B_k;
+                    gkap = kap_k;
                     gdeg = deg_k;
                 }
             }
             if (gs == g) {
                 kb = best_k;
                 a_sel = ga;
-                Bsel = gB;
+                Bz = gB;
+                kap_sel = gkap;
                 deg_sel = gdeg;
-                qbar_sel = -1.0f;  // recomputed by the refit below
             }
         }
 
-        // ---- pass R: two-pass weighted least-squares fit (Eq. 4) of the kept
-        // candidate, centred on a short approximation m of its weighted mean
-        // code (q - m exact) and on the weighted mean weight; the offset is
-        // assembled in compensated arithmetic and kept as a float pair.
+        // ---- pass R: codes of the kept candidate (kept in registers for the
+        // output) and the two sums that the candidate sums only give with
+        // cancellation, now centred: codes about their weighted mean rounded
+        // to a multiple of 1/2 (m), weights about mu.  Then the fit (Eq. 4).
+        constexpr bool kKeepZ = EPL <= 16;
+        float zr[kKeepZ ? EPL : 1];
         const float Pk = R * p.invf[kb];
-        const bool refit = !flat && !deg_sel;
-        float kap = 0.0f;
+        const float2 Pk2 = make_float2(Pk, Pk);
+        // a multiple of 1/2 (codes z are half-integers, so z - m and (z - m)^2 stay exact)
+        const float m = 0.5f * rintf(2.0f * T1b * inv_ss);
         {
-            const float2 Pk2 = make_float2(Pk, Pk);
-            float qm = qbar_sel;
-            // winner changed in the exact pass: its mean code again (warp-uniform
-            // branch, the reduction below shuffles across all lanes)
-            if (__any_sync(0xffffffffu, qm < 0.0f)) {
-                float s1 = 0.0f;
-#pragma unroll 1
-                for (int i = 0; i < NCHK; ++i) {
-                    const int e = gs * G + i * 32 + sl * 4;
-                    const float4 w4 = lds128(ws + e);
-                    const float4 h4 = h_one ? make_float4(1.0f, 1.0f, 1.0f, 1.0f) : lds128(hs + e);
-                    s1 = fmaf(h4.x, int_code(w4.x - c, Pk, H, qmaxf), s1);
-                    s1 = fmaf(h4.y, int_code(w4.y - c, Pk, H, qmaxf), s1);
-                    s1 = fmaf(h4.z, int_code(w4.z - c, Pk, H, qmaxf), s1);
-                    s1 = fmaf(h4.w, int_code(w4.w - c, Pk, H, qmaxf), s1);
-                }
+            const float2 nm2 = make_float2(-m, -m);
+            float2 D2 = make_float2(0.0f, 0.0f), N2 = D2, A2 = D2;
 #pragma unroll
-                for (int o = 4; o; o >>= 1) s1 += shx(s1, o);
-                if (qm < 0.0f) qm = s1 * inv_ss;
-            }
-            const float m = rintf(qm);  // integer: q - m is exact and magic + m too
-            const float2 nm2 = make_float2(-(kRoundMagic + m), -(kRoundMagic + m));
-            const float2 ndbar2 = make_float2(-dbar, -dbar);
-            float2 D2 = make_float2(0.0f, 0.0f), N2 = D2, A2 = D2, B2s = D2, W2 = D2;
-#pragma unroll 1
             for (int i = 0; i < NCHK; ++i) {
                 const int e = gs * G + i * 32 + sl * 4;
                 const float4 w4 = lds128(ws + e);
-                const float4 h4 = h_one ? make_float4(1.0f, 1.0f, 1.0f, 1.0f) : lds128(hs + e);
+                const float4 h4 = lds128(hs + e);
 #pragma unroll
                 for (int pr = 0; pr < 2; ++pr) {
                     const float2 wv = pr ? make_float2(w4.z, w4.w) : make_float2(w4.x, w4.y);
-                    const float2 hv = pr ? make_float2(h4.z, h4.w) : make_float2(h4.x, h4.y);
+                    const float2 h = pr ? make_float2(h4.z, h4.w) : make_float2(h4.x, h4.y);
                     const float2 d = __fadd2_rn(wv, nc2);
-                    float2 t = __ffma2_rn(d, Pk2, H2);
-                    t.x = fminf(fmaxf(t.x, 0.0f), qmaxf);
-                    t.y = fminf(fmaxf(t.y, 0.0f), qmaxf);
-                    const float2 dq = __fadd2_rn(__fadd2_rn(t, magic2), nm2);  // q - m, exact
-                    const float2 wd = __fadd2_rn(d, ndbar2);
-                    const float2 hdq = __fmul2_rn(hv, dq);
-                    D2 = __ffma2_rn(hdq, dq, D2);
-                    N2 = __ffma2_rn(hdq, wd, N2);
-                    A2 = __fadd2_rn(A2, hdq);
-                    B2s = __ffma2_rn(hv, wd, B2s);
-                    W2 = __ffma2_rn(__fmul2_rn(hv, wd), wd, W2);
+                    float2 y = __ffma2_rd(abs2(d), Pk2, M2);
+                    y.x = fminf(y.x, zcap);
+                    y.y = fminf(y.y, zcap);
+                    const float2 z = __fadd2_rn(y, nhm2);
+                    const float2 zs = make_float2(copysignf(z.x, d.x), copysignf(z.y, d.y));
+                    if constexpr (kKeepZ) {
+                        zr[i * 4 + pr * 2] = zs.x;
+                        zr[i * 4 + pr * 2 + 1] = zs.y;
+                    }
+                    const float2 dz = __fadd2_rn(zs, nm2);
+                    const float2 hdz = __fmul2_rn(h, dz);
+                    D2 = __ffma2_rn(hdz, dz, D2);
+                    N2 = __ffma2_rn(hdz, __fadd2_rn(wv, nmu2), N2);
+                    A2 = __fadd2_rn(A2, hdz);
                 }
             }
-            float Dr = D2.x + D2.y, Nr = N2.x + N2.y, Ar = A2.x + A2.y, Br = B2s.x + B2s.y;
-            float Wr = W2.x + W2.y;
+            float Dr = D2.x + D2.y, Nr = N2.x + N2.y, A = A2.x + A2.y;
 #pragma unroll
             for (int o = 4; o; o >>= 1) {
                 Dr += shx(Dr, o);
                 Nr += shx(Nr, o);
-                Ar += shx(Ar, o);
-                Br += shx(Br, o);
-                Wr += shx(Wr, o);
+                A += shx(A, o);
             }
-            if (refit) {
-                const float Aq = Ar * inv_ss;  // mean of q - m
-                const float Bw = Br * inv_ss;  // mean of d - dbar
-                const float Nc = Nr - Ar * Bw, Dc = Dr - Ar * Aq;
+            if (!deg_sel) {
+                // A = sum h (z - m) (small); sum h (w - mu) = Se
+                const float Aq = A * inv_ss;
+                const float Nc = Nr - A * ebar, Dc = Dr - A * Aq;
                 const float an = Nc / Dc;
-                // b = (c + dbar + Bw) - a * (m + Aq), as a float pair
-                float mu_h, mu_l, p_h, p_l, bh, bl;
-                two_sum(c, dbar, mu_h, mu_l);
+                // Bz = (mu + ebar) - a (m + Aq), as a float pair
+                float p_h, p_l, bh, bl;
                 two_prod(an, m, p_h, p_l);
-                two_sum(mu_h, -p_h, bh, bl);
-                bl = __fadd_rn(bl, __fsub_rn(__fadd_rn(mu_l, Bw), fmaf(an, Aq, p_l)));
+                two_sum(mu, -p_h, bh, bl);
+                bl = __fadd_rn(bl, __fsub_rn(ebar, fmaf(an, Aq, p_l)));
                 ff_norm(bh, bl);
                 a_sel = an;
-                Bsel = bh;
-                B_lo = bl;
-                // conditioning of the slope: rounding in the sums moves a by
-                // about ulp * (sum |h dq wd| / |Nc| + sum h dq^2 / Dc), and
-                // sum |h dq wd| <= sqrt(Dr Wr) (Cauchy-Schwarz)
-                kap = __fdividef(sqrtf(Dr * Wr), fabsf(Nc)) + __fdividef(Dr, Dc);
+                Bz = bh;
+                Bz_lo = bl;
+                kap_sel = __fdividef(sqrtf(Dr * see), fabsf(Nc)) + __fdividef(Dr, Dc);
             }
         }
 
-        // ---- output accuracy check.  The refit's error at any level is at most
-        // about est = fit_ulps * ulp * (|a| qmax kap + |c| + range) (fit_ulps
-        // calibrated against the oracle with a margin).  The offset b (fp32)
-        // and a level written in fp32 must meet tol(x) = 1e-7 + 1e-5|x|.  A
-        // level written in bf16 is exact when no bf16 rounding midpoint lies
-        // within est of it, and within the tolerance band when est <= tol.
-        // Groups that could miss get the compensated (float-float) fit.
+        // ---- output accuracy check.  The fp32 fit's error at any level is at
+        // most about est = fit_ulps * ulp * (|a| qmax kap + |c| + range)
+        // (fit_ulps calibrated against the oracle with a margin).  The offset
+        // b (fp32) and a level written in fp32 must meet tol(x) = 1e-7 +
+        // 1e-5|x|.  A level written in bf16 is exact when no bf16 rounding
+        // midpoint lies within est of it, and within the tolerance band when
+        // est <= tol.  Groups that could miss get the compensated fit.
+        const bool refit = !flat && !deg_sel;
         bool prec;
         {
-            const float est = p.fit_ulps * 5.9604645e-8f * (fabsf(a_sel) * qmaxf * kap + fabsf(c) + range);
-            prec = est > 1e-7f + 1e-5f * fabsf(Bsel);
+            const float est =
+                p.fit_ulps * 5.9604645e-8f * (fabsf(a_sel) * qmaxf * kap_sel + fabsf(c) + range);
+            const float b0 = fmaf(-a_sel, H, Bz);  // offset at q = 0
+            prec = est > 1e-7f + 1e-5f * fabsf(b0);
             if (!p.r_bf16) {
-                const float q0 = fminf(fmaxf(rintf(__fdividef(-Bsel, a_sel)), 0.0f), qmaxf);
-                const float rmin = fminf(fabsf(Bsel), fabsf(fmaf(a_sel, q0, Bsel)));
+                const float q0 = fminf(fmaxf(rintf(__fdividef(-b0, a_sel)), 0.0f), qmaxf);
+                const float rmin = fminf(fabsf(b0), fabsf(fmaf(a_sel, q0, b0)));
                 prec |= est > 1e-7f + 1e-5f * rmin;
             } else {
                 for (int q = sl; q <= p.qmax; q += kLanesPerGroup) {
-                    const float rq = fmaf(a_sel, (float)q, Bsel);
+                    const float rq = fmaf(a_sel, (float)q, b0);
                     if (est > 1e-7f + 1e-5f * fabsf(rq)) {
                         const uint32_t bits = __float_as_uint(rq);
                         const int dmid = abs((int)(bits & 0xFFFFu) - 0x8000);  // fp32 ulps to the midpoint
@@ -798,8 +863,6 @@ __global__ void __launch_bounds__(256) k_recon_int(const IntParams p)
                 }
             }
             prec = prec || est != est;  // NaN sums: take the careful path
-        }
-        {
             // one decision per group: any lane of the segment that flagged
             const unsigned flag = __ballot_sync(0xffffffffu, prec);
             prec = ((flag >> (gs * kLanesPerGroup)) & 0xFFu) != 0;
@@ -813,64 +876,90 @@ __global__ void __launch_bounds__(256) k_recon_int(const IntParams p)
             const float gc = __shfl_sync(0xffffffffu, c, src);
             const float gR = __shfl_sync(0xffffffffu, R, src);
             const float gss = __shfl_sync(0xffffffffu, ss, src);
-            const float gdbar = __shfl_sync(0xffffffffu, dbar, src);
-            const bool gh_one = __shfl_sync(0xffffffffu, (int)h_one, src) != 0;
+            const float gmu = __shfl_sync(0xffffffffu, mu + ebar, src);
             const int gkb = __shfl_sync(0xffffffffu, kb, src);
             if (p.stats && lane == 0) atomicAdd(&p.stats[1], 1u);
             float ga, ga_lo, gB, gB_lo;
-            coop_precise<G>(ws + g * G, hs + g * G, gh_one, gc, gR * p.invf[gkb], H, qmaxf, gss,
-                            gc + gdbar, &ga, &ga_lo, &gB, &gB_lo);
+            coop_precise<G>(ws + g * G, hs + g * G, gc, gR * p.invf[gkb], zcap, H, gss, gmu, &ga,
+                            &ga_lo, &gB, &gB_lo);
             if (gs == g) {
                 a_sel = ga;
                 a_lo = ga_lo;
-                Bsel = gB;
-                B_lo = gB_lo;
+                Bz = gB;
+                Bz_lo = gB_lo;
             }
         }
 
         // ---- pass C: outputs of the kept candidate
-        if (valid) {
-            const float Pb = R * p.invf[kb];
-            const float2 Pb2 = make_float2(Pb, Pb);
-            const float2 a2 = make_float2(a_sel, a_sel), B2 = make_float2(Bsel, Bsel);
-            const float2 alo2 = make_float2(a_lo, a_lo), Blo2 = make_float2(B_lo, B_lo);
-            const bool comp = a_lo != 0.0f || B_lo != 0.0f;
-            const float2 nmagic2 = make_float2(-kRoundMagic, -kRoundMagic);
-#pragma unroll 1
-            for (int i = 0; i < NCHK; ++i) {
-                const int e = gs * G + i * 32 + sl * 4;
-                const float4 w4 = lds128(ws + e);
-                float2 rv[2];
-                uint32_t cw = 0;
+        {
+            const float2 a2 = make_float2(a_sel, a_sel), B2 = make_float2(Bz, Bz);
+            const float2 alo2 = make_float2(a_lo, a_lo), Blo2 = make_float2(Bz_lo, Bz_lo);
+            const int64_t ebase = gbase + sl * 4;
+            // general: codes, fp32 r, zero-range groups (r = w); fast: none
+            auto pass_c = [&](auto general) {
+                constexpr bool GEN = decltype(general)::value;
 #pragma unroll
-                for (int pr = 0; pr < 2; ++pr) {
-                    const float2 wv = pr ? make_float2(w4.z, w4.w) : make_float2(w4.x, w4.y);
-                    float2 t = __ffma2_rn(__fadd2_rn(wv, nc2), Pb2, H2);
-                    t.x = fminf(fmaxf(t.x, 0.0f), qmaxf);
-                    t.y = fminf(fmaxf(t.y, 0.0f), qmaxf);
-                    const float2 y = __fadd2_rn(t, magic2);
-                    const float2 q = __fadd2_rn(y, nmagic2);
-                    rv[pr] = __ffma2_rn(a2, q, B2);
-                    // a_lo, B_lo are nonzero only where the compensated fit ran
-                    if (comp) rv[pr] = __fadd2_rn(rv[pr], __ffma2_rn(alo2, q, Blo2));
-                    if (flat) rv[pr] = wv;
-                    if (p.codes)
-                        cw |= ((__float_as_uint(y.x) & 0xFFu) | ((__float_as_uint(y.y) & 0xFFu) << 8))
-                              << (16 * pr);
+                for (int i = 0; i < NCHK; ++i) {
+                    float2 zs[2];
+                    if constexpr (kKeepZ) {
+                        zs[0] = make_float2(zr[i * 4], zr[i * 4 + 1]);
+                        zs[1] = make_float2(zr[i * 4 + 2], zr[i * 4 + 3]);
+                    } else {
+                        const float4 w4 = lds128(ws + gs * G + i * 32 + sl * 4);
+#pragma unroll
+                        for (int pr = 0; pr < 2; ++pr) {
+                            const float2 wv = pr ? make_float2(w4.z, w4.w) : make_float2(w4.x, w4.y);
+                            const float2 d = __fadd2_rn(wv, nc2);
+                            float2 y = __ffma2_rd(abs2(d), Pk2, M2);
+                            y.x = fminf(y.x, zcap);
+                            y.y = fminf(y.y, zcap);
+                            const float2 z = __fadd2_rn(y, nhm2);
+                            zs[pr] = make_float2(copysignf(z.x, d.x), copysignf(z.y, d.y));
+                        }
+                    }
+                    float2 rv[2];
+#pragma unroll
+                    for (int pr = 0; pr < 2; ++pr)
+                        rv[pr] = __fadd2_rn(__ffma2_rn(a2, zs[pr], B2), __ffma2_rn(alo2, zs[pr], Blo2));
+                    const int64_t eo = ebase + i * 32;
+                    if constexpr (GEN) {
+                        if (flat) {
+                            const float4 w4 = lds128(ws + gs * G + i * 32 + sl * 4);
+                            rv[0] = make_float2(w4.x, w4.y);
+                            rv[1] = make_float2(w4.z, w4.w);
+                        }
+                        if (p.codes) {
+                            // q = z + qmax/2, an integer in [0, 255]: its bits above 2^23
+                            uint32_t cw = 0;
+#pragma unroll
+                            for (int pr = 0; pr < 2; ++pr) {
+                                const float2 qf = __fadd2_rn(__fadd2_rn(zs[pr], make_float2(H, H)), M2);
+                                cw |= ((__float_as_uint(qf.x) & 0xFFu) | ((__float_as_uint(qf.y) & 0xFFu) << 8))
+                                      << (16 * pr);
+                            }
+                            stg_cs(reinterpret_cast<uint32_t*>(p.codes + eo), flat ? 0u : cw);
+                        }
+                    }
+                    if (!GEN || p.r_bf16) {
+                        stg_cs(reinterpret_cast<uint2*>(static_cast<__nv_bfloat16*>(p.r) + eo),
+                               make_uint2(pack_bf16x2(rv[0].x, rv[0].y), pack_bf16x2(rv[1].x, rv[1].y)));
+                    } else {
+                        stg_cs(reinterpret_cast<float4*>(static_cast<float*>(p.r) + eo),
+                               make_float4(rv[0].x, rv[0].y, rv[1].x, rv[1].y));
+                    }
                 }
-                const int64_t eo = gbase + i * 32 + sl * 4;
-                if (p.r_bf16) {
-                    stg_cs(reinterpret_cast<uint2*>(static_cast<__nv_bfloat16*>(p.r) + eo),
-                           make_uint2(pack_bf16x2(rv[0].x, rv[0].y), pack_bf16x2(rv[1].x, rv[1].y)));
-                } else {
-                    stg_cs(reinterpret_cast<float4*>(static_cast<float*>(p.r) + eo),
-                           make_float4(rv[0].x, rv[0].y, rv[1].x, rv[1].y));
-                }
-                if (p.codes) stg_cs(reinterpret_cast<uint32_t*>(p.codes + eo), flat ? 0u : cw);
+            };
+            const bool gen = !p.r_bf16 || p.codes != nullptr || __any_sync(0xffffffffu, flat);
+            if (valid) {
+                if (gen) pass_c(std::true_type{});
+                else pass_c(std::false_type{});
             }
-            if (sl == 0) {
+            if (valid && sl == 0) {
+                // b = Bz - a*H: the offset at code 0
+                float bh = Bz, bl = Bz_lo;
+                ff_add_prod(bh, bl, -a_sel, -a_lo, H);
                 p.a[grp] = flat ? 0.0f : a_sel;
-                p.b[grp] = flat ? ws[gs * G] : Bsel;
+                p.b[grp] = flat ? c : __fadd_rn(bh, bl);
                 if (p.idx) p.idx[grp] = flat ? 0 : (uint8_t)kb;
             }
         }
