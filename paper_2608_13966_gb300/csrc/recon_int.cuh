@@ -550,7 +550,9 @@ __global__ void __launch_bounds__(256) k_recon_int(const IntParams p)
 #pragma unroll
             for (int kk = 0; kk < 8; ++kk) A1[kk] = A2[kk] = A3[kk] = make_float2(0.0f, 0.0f);
             float2 SE = make_float2(0.0f, 0.0f), SEE = make_float2(0.0f, 0.0f);
-#pragma unroll(NCHK <= 4 ? NCHK : 2)
+// rolled: a compact unit loop keeps the careful paths' code from evicting it
+// from the instruction cache when they run
+#pragma unroll 1
             for (int i = 0; i < NCHK; ++i) {
                 const int e = gs * G + i * 32 + sl * 4;
                 const float4 w4 = lds128(ws + e);
