@@ -11,12 +11,15 @@
 // a time, staged through its own ring of shared-memory buffers filled by 1-D
 // TMA bulk copies, exactly as the integer kernel.  A lane reads its block's
 // four 16-byte chunks in a lane-rotated order so that each shared-memory
-// access of the warp is bank-conflict free.
+// access of the warp is bank-conflict free.  Arithmetic is packed f32x2, two
+// elements per instruction.
 //
-// Exactness: the candidate error is evaluated from moments,
-// S_ww - 2*alpha*S3 + alpha^2*S2; candidates within an error bound of the
-// best are re-evaluated directly as sum h (alpha*q - |w|)^2, where
-// fma(alpha, q, -|w|) rounds once.
+// Per candidate the codes stay in registers: moments -> a* -> E4M3 scale,
+// then the error summed directly, sum h (alpha*q - |w|)^2 (no cancellation,
+// so its fp32 error is a few ulps of itself).  Candidates within that bound
+// of the best, unless their codes and scale equal the best's (the sum of
+// codes never decreases with the scale factor, so equal sums mean equal
+// codes), are re-evaluated exactly in float-float arithmetic.
 #pragma once
 
 #include "device_common.cuh"
@@ -27,16 +30,6 @@ namespace quasar {
 __device__ __forceinline__ float tensor_scale_of(float amax)
 {
     return amax > 0.0f ? __fdiv_rn(amax, 2688.0f) : 1.0f;
-}
-
-// E2M1 magnitude nearest to y in [0, 6] (ties to even): rounds y on the grid
-// spacing of its binade (0.5 below 2, 1 in [2,4), 2 in [4,6]) with a magic
-// constant whose ulp is that spacing.
-__device__ __forceinline__ float e2m1_mag(float y)
-{
-    const uint32_t eb = max(__float_as_uint(y), 0x3F800000u) & 0x7F800000u;
-    const float M = __uint_as_float(eb + 0x0B400000u);
-    return __fsub_rn(__fadd_rn(y, M), M);
 }
 
 // E4M3 (e4m3fn) round-to-nearest-even with saturation, and its value.
@@ -64,11 +57,27 @@ __device__ __forceinline__ uint32_t e2m1_nibble(float qs)
     return (uint32_t)(r & 0xFu);
 }
 
+// Error-free transformations for the exact comparison (Knuth TwoSum,
+// FMA-based TwoProd).
+__device__ __forceinline__ void two_sum_f(float a, float b, float& s, float& e)
+{
+    s = __fadd_rn(a, b);
+    const float bb = __fsub_rn(s, a);
+    e = __fadd_rn(__fsub_rn(a, __fsub_rn(s, bb)), __fsub_rn(b, bb));
+}
+
+__device__ __forceinline__ void two_prod_f(float a, float b, float& p, float& e)
+{
+    p = __fmul_rn(a, b);
+    e = fmaf(a, b, -p);
+}
+
 template <int NCH>
 __global__ void __launch_bounds__(256) k_recon_nvfp4(const Nvfp4Params p)
 {
     constexpr int KM = NCH * 8;
     constexpr int UNIT = kBlocksPerUnit * 16;
+    constexpr int SCS = 2 * KM + 1;  // per-lane scratch stride (odd: no bank conflicts)
     extern __shared__ __align__(128) unsigned char smem[];
 
     const int lane = threadIdx.x & 31;
@@ -76,7 +85,11 @@ __global__ void __launch_bounds__(256) k_recon_nvfp4(const Nvfp4Params p)
     const int nwarps = blockDim.x >> 5;
     const int S = p.stages;
     unsigned char* ring = smem + (size_t)warp * S * p.stage_bytes;
-    uint64_t* bars = reinterpret_cast<uint64_t*>(smem + (size_t)nwarps * S * p.stage_bytes) + warp * (S + 1);
+    uint32_t* scr = reinterpret_cast<uint32_t*>(smem + (size_t)nwarps * S * p.stage_bytes) +
+                    (size_t)warp * 32 * SCS + lane * SCS;
+    uint64_t* bars = reinterpret_cast<uint64_t*>(smem + (size_t)nwarps * S * p.stage_bytes +
+                                                 (size_t)nwarps * 32 * SCS * 4) +
+                     warp * (S + 1);
 
     const int gbytes = p.g_kind == 2 ? 2 : (p.g_kind == 1 ? 4 : 0);
     constexpr uint32_t kVOff = UNIT * 4;
@@ -132,8 +145,21 @@ __global__ void __launch_bounds__(256) k_recon_nvfp4(const Nvfp4Params p)
 
     const int rot = (lane >> 1) & 3;
     const float ulp = 5.9604645e-8f * p.tie_kappa;
+    const float2 beta22 = make_float2(p.beta2, p.beta2);
+    const float2 c12 = make_float2(p.c1, p.c1);
+    const float2 six2 = make_float2(6.0f, 6.0f), neg12 = make_float2(-1.0f, -1.0f);
     int s_cur = 0;
     uint32_t parity = 0;
+
+    // E2M1 magnitudes of two values y in [0, 6] (ties to even): each is
+    // rounded on the grid spacing of its binade (0.5 below 2, 1 in [2, 4), 2
+    // in [4, 6]) by adding and removing a constant whose ulp is that spacing.
+    auto e2m1_2 = [](float2 y) -> float2 {
+        const float2 M = make_float2(
+            __uint_as_float((__float_as_uint(fmaxf(y.x, 1.0f)) & 0x7F800000u) + 0x0B400000u),
+            __uint_as_float((__float_as_uint(fmaxf(y.y, 1.0f)) & 0x7F800000u) + 0x0B400000u));
+        return __ffma2_rn(M, make_float2(-1.0f, -1.0f), __fadd2_rn(y, M));
+    };
 
     for (int64_t it = 0;; ++it) {
         const int64_t u = first + it * stride;
@@ -144,30 +170,34 @@ __global__ void __launch_bounds__(256) k_recon_nvfp4(const Nvfp4Params p)
         }
         const unsigned char* st = ring + (size_t)s_cur * p.stage_bytes;
 
-        // element 4*cidx[i] + jj of this lane's block is held at slot 4*i + jj
-        float w[16], h[16];
+        // element 4*cidx[i] + jj of this lane's block is held at slot 4*i + jj,
+        // pairs (slot 2t, 2t+1) in w2[t], h2[t]
+        float2 w2[8], h2[8];
 #pragma unroll
         for (int i = 0; i < 4; ++i) {
             const int cidx = (i + rot) & 3;
             const int e = lane * 16 + cidx * 4;
             const float4 w4 = lds128(st + e * 4);
             const float4 v4 = lds128(st + kVOff + e * 4);
-            w[4 * i + 0] = w4.x; w[4 * i + 1] = w4.y; w[4 * i + 2] = w4.z; w[4 * i + 3] = w4.w;
-            h[4 * i + 0] = v4.x; h[4 * i + 1] = v4.y; h[4 * i + 2] = v4.z; h[4 * i + 3] = v4.w;
+            w2[2 * i] = make_float2(w4.x, w4.y);
+            w2[2 * i + 1] = make_float2(w4.z, w4.w);
+            float2 hA = make_float2(v4.x, v4.y), hB = make_float2(v4.z, v4.w);
             if (p.g_kind) {
-                float g0, g1, g2, g3;
+                float2 gA, gB;
                 if (p.g_kind == 2) {
                     const uint2 gb = lds64(st + kGOff + e * 2);
-                    g0 = bf16lo(gb.x); g1 = bf16hi(gb.x); g2 = bf16lo(gb.y); g3 = bf16hi(gb.y);
+                    gA = make_float2(bf16lo(gb.x), bf16hi(gb.x));
+                    gB = make_float2(bf16lo(gb.y), bf16hi(gb.y));
                 } else {
                     const float4 g4 = lds128(st + kGOff + e * 4);
-                    g0 = g4.x; g1 = g4.y; g2 = g4.z; g3 = g4.w;
+                    gA = make_float2(g4.x, g4.y);
+                    gB = make_float2(g4.z, g4.w);
                 }
-                h[4 * i + 0] = fmaf(p.beta2, h[4 * i + 0], __fmul_rn(p.c1, __fmul_rn(g0, g0)));
-                h[4 * i + 1] = fmaf(p.beta2, h[4 * i + 1], __fmul_rn(p.c1, __fmul_rn(g1, g1)));
-                h[4 * i + 2] = fmaf(p.beta2, h[4 * i + 2], __fmul_rn(p.c1, __fmul_rn(g2, g2)));
-                h[4 * i + 3] = fmaf(p.beta2, h[4 * i + 3], __fmul_rn(p.c1, __fmul_rn(g3, g3)));
+                hA = __ffma2_rn(hA, beta22, __fmul2_rn(c12, __fmul2_rn(gA, gA)));
+                hB = __ffma2_rn(hB, beta22, __fmul2_rn(c12, __fmul2_rn(gB, gB)));
             }
+            h2[2 * i] = hA;
+            h2[2 * i + 1] = hB;
         }
         __syncwarp();
         if (lane == 0) {
@@ -188,98 +218,137 @@ __global__ void __launch_bounds__(256) k_recon_nvfp4(const Nvfp4Params p)
             for (int i = 0; i < 4; ++i) {
                 const int cidx = (i + rot) & 3;
                 stg_cs(reinterpret_cast<float4*>(p.v + ebase + cidx * 4),
-                       make_float4(h[4 * i], h[4 * i + 1], h[4 * i + 2], h[4 * i + 3]));
+                       make_float4(h2[2 * i].x, h2[2 * i].y, h2[2 * i + 1].x, h2[2 * i + 1].y));
             }
         }
 
-        float amax_b = 0.0f, ss = 0.0f;
-        float aw[16];
+        float2 aw2[8], naw2[8];
+        float amax_b = 0.0f;
+        float2 SS = make_float2(0.0f, 0.0f);
 #pragma unroll
-        for (int j = 0; j < 16; ++j) {
-            aw[j] = fabsf(w[j]);
-            amax_b = fmaxf(amax_b, aw[j]);
-            ss += h[j];
+        for (int t = 0; t < 8; ++t) {
+            aw2[t] = make_float2(fabsf(w2[t].x), fabsf(w2[t].y));
+            naw2[t] = make_float2(-aw2[t].x, -aw2[t].y);
+            amax_b = fmaxf(amax_b, fmaxf(aw2[t].x, aw2[t].y));
+            SS = __fadd2_rn(SS, h2[t]);
         }
-        if (ss == 0.0f) {
+        if (SS.x + SS.y == 0.0f) {  // all saliencies zero: h = 1
 #pragma unroll
-            for (int j = 0; j < 16; ++j) h[j] = 1.0f;
+            for (int t = 0; t < 8; ++t) h2[t] = make_float2(1.0f, 1.0f);
         }
-        float sww = 0.0f;
-#pragma unroll
-        for (int j = 0; j < 16; ++j) sww = fmaf(h[j] * aw[j], aw[j], sww);
-
         const bool zero = !(amax_b > 0.0f);
-        const float P1 = zero ? 0.0f : 6.0f / amax_b;  // 1/sigma at f = 1
+        const float P1 = zero ? 0.0f : __fdiv_rn(6.0f, amax_b);  // 1/sigma at f = 1
 
-        // Candidate k: moments, fitted E4M3 scale and error from moments.
-        auto candidate = [&](int k, float& alpha, uint32_t& e, float& s2, float& s3) {
+        // ---- candidates: codes in registers, moments, E4M3 scale, direct error
+        float Eb = INFINITY;
+        int kb = 0;
+        uint32_t keyb = 0, e_sel = 0;
+        float alpha_sel = 0.0f;
+#pragma unroll 1
+        for (int k = 0; k < KM; ++k) {
             const float P = P1 * p.invf[k];
-            s2 = 0.0f;
-            s3 = 0.0f;
+            const float2 P2 = make_float2(P, P);
+            float2 q2[8];
+            float2 S2 = make_float2(0.0f, 0.0f), S3 = S2, U = S2;
 #pragma unroll
-            for (int j = 0; j < 16; ++j) {
-                const float q = e2m1_mag(fminf(aw[j] * P, 6.0f));
-                const float hq = __fmul_rn(h[j], q);
-                s2 = fmaf(hq, q, s2);
-                s3 = fmaf(hq, aw[j], s3);
+            for (int t = 0; t < 8; ++t) {
+                float2 y = __fmul2_rn(aw2[t], P2);
+                y.x = fminf(y.x, 6.0f);
+                y.y = fminf(y.y, 6.0f);
+                q2[t] = e2m1_2(y);
+                const float2 hq = __fmul2_rn(h2[t], q2[t]);
+                S2 = __ffma2_rn(hq, q2[t], S2);
+                S3 = __ffma2_rn(hq, aw2[t], S3);
+                U = __fadd2_rn(U, q2[t]);
             }
+            const float s2 = S2.x + S2.y, s3 = S3.x + S3.y;
+            // degenerate (every weighted element coded 0): the search scale
             const float x = s2 > 0.0f ? __fdividef(s3, s2) * inv_sT
                                       : amax_b * p.f[k] * (1.0f / 6.0f) * inv_sT;
-            e = e4m3_rn_satfinite(x);
-            alpha = sT * e4m3_value(e);
-        };
-
-        // Per candidate: the error from moments and its fp32 error bound.
-        float Sk[KM], dSk[KM];
-        float Sb = INFINITY, dSb = 0.0f, alpha_sel = 0.0f;
-        uint32_t e_sel = 0;
-        int kb = 0;
+            const uint32_t e = e4m3_rn_satfinite(x);
+            const float alpha = sT * e4m3_value(e);
+            const float2 a2 = make_float2(alpha, alpha);
+            float2 E2 = make_float2(0.0f, 0.0f);
 #pragma unroll
-        for (int k = 0; k < KM; ++k) {
-            float alpha, s2, s3;
-            uint32_t e;
-            candidate(k, alpha, e, s2, s3);
-            const float Sv = k < p.n_clip ? fmaf(alpha, fmaf(alpha, s2, -2.0f * s3), sww) : INFINITY;
-            Sk[k] = Sv;
-            dSk[k] = ulp * (sww + 2.0f * alpha * s3 + alpha * alpha * s2);
-            if (Sv < Sb) {  // strict: ties keep the lower index
-                Sb = Sv;
-                dSb = dSk[k];
-                alpha_sel = alpha;
-                e_sel = e;
+            for (int t = 0; t < 8; ++t) {
+                const float2 ev = __ffma2_rn(a2, q2[t], naw2[t]);
+                E2 = __ffma2_rn(__fmul2_rn(h2[t], ev), ev, E2);
+            }
+            const float err = k < p.n_clip ? E2.x + E2.y : INFINITY;
+            // identical codes (equal sums of codes) and scale: identical error
+            const uint32_t key = ((uint32_t)(2.0f * (U.x + U.y)) << 8) | e;
+            scr[2 * k] = __float_as_uint(err);
+            scr[2 * k + 1] = key;
+            if (err < Eb) {  // strict: ties keep the lower index
+                Eb = err;
                 kb = k;
+                keyb = key;
+                e_sel = e;
+                alpha_sel = alpha;
             }
         }
+        // contenders: within the direct sums' fp32 error bound of the best
         unsigned set = 0;
-#pragma unroll
-        for (int k = 0; k < KM; ++k)
-            if (k != kb && Sk[k] - Sb <= dSb + dSk[k]) set |= 1u << k;
+#pragma unroll 1
+        for (int k = 0; k < KM; ++k) {
+            const float ek = __uint_as_float(scr[2 * k]);
+            if (k != kb && ek - Eb <= ulp * (ek + Eb) && scr[2 * k + 1] != keyb) set |= 1u << k;
+        }
 
         if (set != 0 && valid && !zero) {
+            // exact comparison: sum h (alpha q - |w|)^2 with alpha*q - |w| as an
+            // exact pair (TwoProd, TwoSum) and the squares and sum in float pairs
             if (p.stats) atomicAdd(&p.stats[0], 1u);
             set |= 1u << kb;
-            float best = INFINITY;
+            float best_h = INFINITY, best_l = 0.0f;
             int bk = -1;
             while (set) {
                 const int k = __ffs(set) - 1;
                 set &= set - 1;
-                float alpha, s2, s3;
-                uint32_t e;
-                candidate(k, alpha, e, s2, s3);
                 const float P = P1 * p.invf[k];
-                float t[16];
+                const float2 P2 = make_float2(P, P);
+                float2 S2 = make_float2(0.0f, 0.0f), S3 = S2;
+                float2 q2[8];
 #pragma unroll
-                for (int j = 0; j < 16; ++j) {
-                    const float q = e2m1_mag(fminf(aw[j] * P, 6.0f));
-                    const float ej = fmaf(alpha, q, -aw[j]);
-                    t[j] = h[j] * (ej * ej);
+                for (int t = 0; t < 8; ++t) {
+                    float2 y = __fmul2_rn(aw2[t], P2);
+                    y.x = fminf(y.x, 6.0f);
+                    y.y = fminf(y.y, 6.0f);
+                    q2[t] = e2m1_2(y);
+                    const float2 hq = __fmul2_rn(h2[t], q2[t]);
+                    S2 = __ffma2_rn(hq, q2[t], S2);
+                    S3 = __ffma2_rn(hq, aw2[t], S3);
                 }
+                const float s2 = S2.x + S2.y, s3 = S3.x + S3.y;
+                const float x = s2 > 0.0f ? __fdividef(s3, s2) * inv_sT
+                                          : amax_b * p.f[k] * (1.0f / 6.0f) * inv_sT;
+                const uint32_t e = e4m3_rn_satfinite(x);
+                const float alpha = sT * e4m3_value(e);
+                float eh = 0.0f, el = 0.0f;
 #pragma unroll
-                for (int s = 1; s < 16; s <<= 1)
+                for (int t = 0; t < 8; ++t) {
 #pragma unroll
-                    for (int j = 0; j + s < 16; j += 2 * s) t[j] += t[j + s];
-                if (bk < 0 || t[0] < best) {
-                    best = t[0];
+                    for (int c2 = 0; c2 < 2; ++c2) {
+                        const float q = c2 ? q2[t].y : q2[t].x;
+                        const float aw = c2 ? aw2[t].y : aw2[t].x;
+                        const float h = c2 ? h2[t].y : h2[t].x;
+                        float ph, pl, dh, dl, sh, sl;
+                        two_prod_f(alpha, q, ph, pl);
+                        two_sum_f(ph, -aw, dh, dl);
+                        dl = __fadd_rn(dl, pl);  // alpha q - |w| = dh + dl
+                        two_prod_f(dh, dh, sh, sl);
+                        sl = fmaf(2.0f * dh, dl, sl);
+                        two_prod_f(h, sh, ph, pl);
+                        pl = fmaf(h, sl, pl);
+                        float t1, t2;
+                        two_sum_f(eh, ph, t1, t2);
+                        eh = t1;
+                        el = __fadd_rn(el, __fadd_rn(t2, pl));
+                    }
+                }
+                if (bk < 0 || eh < best_h || (eh == best_h && el < best_l)) {
+                    best_h = eh;
+                    best_l = el;
                     bk = k;
                     alpha_sel = alpha;
                     e_sel = e;
@@ -294,27 +363,35 @@ __global__ void __launch_bounds__(256) k_recon_nvfp4(const Nvfp4Params p)
             alpha_sel = 0.0f;
         }
 
+        // ---- outputs of the kept candidate
         const float Pb = P1 * p.invf[kb];
+        const float2 Pb2 = make_float2(Pb, Pb);
+        const float2 as2 = make_float2(alpha_sel, alpha_sel);
 #pragma unroll
         for (int i = 0; i < 4; ++i) {
             const int cidx = (i + rot) & 3;
-            float rv[4];
+            float2 rv[2];
             uint32_t cw = 0;
 #pragma unroll
-            for (int jj = 0; jj < 4; ++jj) {
-                const int j = 4 * i + jj;
-                const float q = zero ? 0.0f : e2m1_mag(fminf(aw[j] * Pb, 6.0f));
-                const float qs = q > 0.0f ? copysignf(q, w[j]) : 0.0f;
-                rv[jj] = alpha_sel * qs;
-                cw |= e2m1_nibble(qs) << (8 * jj);
+            for (int hh = 0; hh < 2; ++hh) {
+                const int t = 2 * i + hh;
+                float2 y = __fmul2_rn(aw2[t], Pb2);
+                y.x = fminf(y.x, 6.0f);
+                y.y = fminf(y.y, 6.0f);
+                const float2 q = e2m1_2(y);
+                // the code carries the sign of w (magnitude 0 is stored as +0)
+                const float2 qs = make_float2(q.x > 0.0f ? copysignf(q.x, w2[t].x) : 0.0f,
+                                              q.y > 0.0f ? copysignf(q.y, w2[t].y) : 0.0f);
+                rv[hh] = __fmul2_rn(as2, qs);
+                if (p.codes) cw |= (e2m1_nibble(qs.x) | (e2m1_nibble(qs.y) << 8)) << (16 * hh);
             }
             const int64_t e = ebase + cidx * 4;
             if (p.r_bf16) {
                 stg_cs(reinterpret_cast<uint2*>(static_cast<__nv_bfloat16*>(p.r) + e),
-                       make_uint2(pack_bf16x2(rv[0], rv[1]), pack_bf16x2(rv[2], rv[3])));
+                       make_uint2(pack_bf16x2(rv[0].x, rv[0].y), pack_bf16x2(rv[1].x, rv[1].y)));
             } else {
                 stg_cs(reinterpret_cast<float4*>(static_cast<float*>(p.r) + e),
-                       make_float4(rv[0], rv[1], rv[2], rv[3]));
+                       make_float4(rv[0].x, rv[0].y, rv[1].x, rv[1].y));
             }
             if (p.codes) stg_cs(reinterpret_cast<uint32_t*>(p.codes + e), cw);
         }
