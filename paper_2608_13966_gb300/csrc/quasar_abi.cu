@@ -403,9 +403,8 @@ quasar_status quasar_recon_nvfp4(const float* w, const void* g, quasar_dtype g_d
     }
 
     const int gbytes = p.g_kind == 2 ? 2 : (p.g_kind == 1 ? 4 : 0);
-    // per-warp scratch: each lane's candidate errors and code keys
     const int nch = nch_for(n_clip);
-    const Launch L = plan((uint32_t)(kBlocksPerUnit * 16 * (8 + gbytes)), 32u * (16u * nch + 1u) * 4u);
+    const Launch L = plan((uint32_t)(kBlocksPerUnit * 16 * (8 + gbytes)), 0);
     p.stages = L.stages;
     p.stage_bytes = L.stage_bytes;
     const void* fn = nvfp4_kernel(nch);

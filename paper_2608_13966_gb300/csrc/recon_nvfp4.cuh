@@ -42,9 +42,10 @@ __device__ __forceinline__ uint32_t e4m3_rn_satfinite(float x)
 
 __device__ __forceinline__ float e4m3_value(uint32_t bits)
 {
-    const uint32_t e = (bits >> 3) & 0xFu, m = bits & 7u;
-    if (e == 0) return (float)m * 0.001953125f;  // m * 2^-9
-    return __uint_as_float(((e + 120u) << 23) | (m << 20));
+    // normal: exponent e - 7 + 127, mantissa m << 20; subnormal (e = 0): m * 2^-9
+    const uint32_t b = bits & 0x7Fu;
+    const float normal = __uint_as_float((b << 20) + (120u << 23));
+    return b < 8u ? (float)b * 0.001953125f : normal;
 }
 
 // E2M1 nibble of a value that lies on the signed E2M1 grid.
@@ -77,7 +78,6 @@ __global__ void __launch_bounds__(256) k_recon_nvfp4(const Nvfp4Params p)
 {
     constexpr int KM = NCH * 8;
     constexpr int UNIT = kBlocksPerUnit * 16;
-    constexpr int SCS = 2 * KM + 1;  // per-lane scratch stride (odd: no bank conflicts)
     extern __shared__ __align__(128) unsigned char smem[];
 
     const int lane = threadIdx.x & 31;
@@ -85,11 +85,7 @@ __global__ void __launch_bounds__(256) k_recon_nvfp4(const Nvfp4Params p)
     const int nwarps = blockDim.x >> 5;
     const int S = p.stages;
     unsigned char* ring = smem + (size_t)warp * S * p.stage_bytes;
-    uint32_t* scr = reinterpret_cast<uint32_t*>(smem + (size_t)nwarps * S * p.stage_bytes) +
-                    (size_t)warp * 32 * SCS + lane * SCS;
-    uint64_t* bars = reinterpret_cast<uint64_t*>(smem + (size_t)nwarps * S * p.stage_bytes +
-                                                 (size_t)nwarps * 32 * SCS * 4) +
-                     warp * (S + 1);
+    uint64_t* bars = reinterpret_cast<uint64_t*>(smem + (size_t)nwarps * S * p.stage_bytes) + warp * (S + 1);
 
     const int gbytes = p.g_kind == 2 ? 2 : (p.g_kind == 1 ? 4 : 0);
     constexpr uint32_t kVOff = UNIT * 4;
@@ -155,9 +151,10 @@ __global__ void __launch_bounds__(256) k_recon_nvfp4(const Nvfp4Params p)
     // rounded on the grid spacing of its binade (0.5 below 2, 1 in [2, 4), 2
     // in [4, 6]) by adding and removing a constant whose ulp is that spacing.
     auto e2m1_2 = [](float2 y) -> float2 {
-        const float2 M = make_float2(
-            __uint_as_float((__float_as_uint(fmaxf(y.x, 1.0f)) & 0x7F800000u) + 0x0B400000u),
-            __uint_as_float((__float_as_uint(fmaxf(y.y, 1.0f)) & 0x7F800000u) + 0x0B400000u));
+        // binade of max(y, 1) (a power of two), times 1.5 * 2^22
+        const float2 B = make_float2(__uint_as_float(__float_as_uint(fmaxf(y.x, 1.0f)) & 0x7F800000u),
+                                     __uint_as_float(__float_as_uint(fmaxf(y.y, 1.0f)) & 0x7F800000u));
+        const float2 M = __fmul2_rn(B, make_float2(6291456.0f, 6291456.0f));
         return __ffma2_rn(M, make_float2(-1.0f, -1.0f), __fadd2_rn(y, M));
     };
 
@@ -240,16 +237,18 @@ __global__ void __launch_bounds__(256) k_recon_nvfp4(const Nvfp4Params p)
         const float P1 = zero ? 0.0f : __fdiv_rn(6.0f, amax_b);  // 1/sigma at f = 1
 
         // ---- candidates: codes in registers, moments, E4M3 scale, direct error
+        float Ek[KM];
+        uint32_t Kk[KM];
         float Eb = INFINITY;
         int kb = 0;
-        uint32_t keyb = 0, e_sel = 0;
+        uint32_t e_sel = 0;
         float alpha_sel = 0.0f;
-#pragma unroll 1
+#pragma unroll
         for (int k = 0; k < KM; ++k) {
             const float P = P1 * p.invf[k];
             const float2 P2 = make_float2(P, P);
             float2 q2[8];
-            float2 S2 = make_float2(0.0f, 0.0f), S3 = S2, U = S2;
+            float2 S2 = make_float2(0.0f, 0.0f), S3 = S2;
 #pragma unroll
             for (int t = 0; t < 8; ++t) {
                 float2 y = __fmul2_rn(aw2[t], P2);
@@ -259,7 +258,6 @@ __global__ void __launch_bounds__(256) k_recon_nvfp4(const Nvfp4Params p)
                 const float2 hq = __fmul2_rn(h2[t], q2[t]);
                 S2 = __ffma2_rn(hq, q2[t], S2);
                 S3 = __ffma2_rn(hq, aw2[t], S3);
-                U = __fadd2_rn(U, q2[t]);
             }
             const float s2 = S2.x + S2.y, s3 = S3.x + S3.y;
             // degenerate (every weighted element coded 0): the search scale
@@ -275,25 +273,26 @@ __global__ void __launch_bounds__(256) k_recon_nvfp4(const Nvfp4Params p)
                 E2 = __ffma2_rn(__fmul2_rn(h2[t], ev), ev, E2);
             }
             const float err = k < p.n_clip ? E2.x + E2.y : INFINITY;
-            // identical codes (equal sums of codes) and scale: identical error
-            const uint32_t key = ((uint32_t)(2.0f * (U.x + U.y)) << 8) | e;
-            scr[2 * k] = __float_as_uint(err);
-            scr[2 * k + 1] = key;
+            // candidates with equal moments and scale have, to within rounding
+            // below the tie margin, equal codes and errors: a key of the three
+            Ek[k] = err;
+            Kk[k] = (__float_as_uint(s2) * 0x9E3779B1u + __float_as_uint(s3)) ^ e;
             if (err < Eb) {  // strict: ties keep the lower index
                 Eb = err;
                 kb = k;
-                keyb = key;
                 e_sel = e;
                 alpha_sel = alpha;
             }
         }
         // contenders: within the direct sums' fp32 error bound of the best
+        uint32_t keyb = Kk[0];
+#pragma unroll
+        for (int k = 1; k < KM; ++k)
+            if (k == kb) keyb = Kk[k];
         unsigned set = 0;
-#pragma unroll 1
-        for (int k = 0; k < KM; ++k) {
-            const float ek = __uint_as_float(scr[2 * k]);
-            if (k != kb && ek - Eb <= ulp * (ek + Eb) && scr[2 * k + 1] != keyb) set |= 1u << k;
-        }
+#pragma unroll
+        for (int k = 0; k < KM; ++k)
+            if (k != kb && Ek[k] - Eb <= ulp * (Ek[k] + Eb) && Kk[k] != keyb) set |= 1u << k;
 
         if (set != 0 && valid && !zero) {
             // exact comparison: sum h (alpha q - |w|)^2 with alpha*q - |w| as an
