@@ -9,9 +9,10 @@ namespace quasar {
 constexpr unsigned kStatusTimeout = 1u;
 
 constexpr int kLanesPerGroup = 8;
-// Per-warp shared scratch of the integer kernel: 32 rows of 36 floats used to
-// transpose the per-candidate sums across the lanes of a group.
-constexpr uint32_t kIntScratchBytes = 32 * 36 * 4;
+// Per-warp shared scratch of the integer kernel: 32 rows of 32 floats used to
+// transpose the per-candidate sums across the lanes of a group (16-byte
+// columns XOR-swizzled by row, so neither side has bank conflicts).
+constexpr uint32_t kIntScratchBytes = 32 * 32 * 4;
 constexpr int kGroupsPerUnit = 4;
 constexpr int kMaxClip = 32;
 

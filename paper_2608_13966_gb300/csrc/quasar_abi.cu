@@ -30,9 +30,10 @@ namespace {
 
 using namespace quasar;
 
-// 7 warps per CTA: with two 5 KB tiles and the 4.5 KB transpose scratch
-// per warp, two CTAs fit in an SM's shared memory (14 resident warps).
-constexpr int kThreads = 224;
+// 8 warps per CTA: with two 5 KB tiles and the 4 KB transpose scratch per
+// warp, two CTAs fit in an SM's shared memory (16 resident warps, at 128
+// registers a thread the whole register file).
+constexpr int kThreads = 256;
 constexpr int kWarps = kThreads / 32;
 constexpr uint64_t kDefaultTimeoutNs = 1000000000ull;  // 1 s per wait
 

@@ -586,17 +586,18 @@ __global__ void __launch_bounds__(256) k_recon_int(const IntParams p)
                     }
                 }
             }
-            // transpose through shared memory: lane L writes row L, lane
-            // (gs, sl) sums columns sl*4.. of the 8 rows of its group (a tree)
+            // transpose through shared memory: lane L writes row L (its sums
+            // of candidate kk in 16-byte column kk ^ (L & 7)), lane (gs, sl)
+            // sums column sl of the 8 rows of its group (a tree)
 #pragma unroll
             for (int kk = 0; kk < 8; ++kk)
-                *reinterpret_cast<float4*>(red + lane * 36 + kk * 4) =
+                *reinterpret_cast<float4*>(red + lane * 32 + ((kk ^ (lane & 7)) << 2)) =
                     make_float4(A1[kk].x + A1[kk].y, A2[kk].x + A2[kk].y, A3[kk].x + A3[kk].y, 0.0f);
             __syncwarp();
             float4 x[8];
 #pragma unroll
             for (int j = 0; j < 8; ++j)
-                x[j] = *reinterpret_cast<const float4*>(red + (gs * 8 + j) * 36 + sl * 4);
+                x[j] = *reinterpret_cast<const float4*>(red + (gs * 8 + j) * 32 + ((sl ^ j) << 2));
 #pragma unroll
             for (int s2 = 1; s2 < 8; s2 <<= 1)
 #pragma unroll
