@@ -96,6 +96,41 @@ quasar_status quasar_recon_int(const float* w, const void* g, quasar_dtype g_dty
                                uint8_t* cand_idx, quasar_stream_t stream);
 
 /*
+ * quasar_int_tensor / quasar_recon_int_batch -- quasar_recon_int over many
+ * tensors in one launch (Algorithm 1 applied to every linear weight of a
+ * model at each step), with the same quantization settings for all of them.
+ * The units of work of all tensors are numbered consecutively and shared by
+ * one persistent grid, so small tensors cost no launch of their own and the
+ * step has a single tail.
+ *
+ * Each descriptor holds one tensor's arguments exactly as quasar_recon_int
+ * takes them (same meaning, layout and rules); either every non-empty tensor
+ * has a gradient g or none does.  The descriptor array is a HOST array read before
+ * the call returns; tensors may be listed in any order and may differ in
+ * shape.  More than 256 tensors are processed 256 per launch.
+ * Returns as quasar_recon_int; every tensor is validated before anything is
+ * launched.  The paper has no batched form: this entry point only removes
+ * per-tensor launches.
+ */
+typedef struct {
+    const float* w;
+    const void* g;
+    float* v;
+    void* r;
+    uint8_t* codes;
+    float* a;
+    float* b;
+    uint8_t* cand_idx;
+    int64_t rows;
+    int64_t cols;
+} quasar_int_tensor;
+
+quasar_status quasar_recon_int_batch(const quasar_int_tensor* tensors, int n_tensors,
+                                     quasar_dtype g_dtype, float beta2, int bits, int group_size,
+                                     const float* clip, int n_clip, quasar_dtype r_dtype,
+                                     quasar_stream_t stream);
+
+/*
  * quasar_recon_nvfp4 -- QUASAR for NVFP4 (Sec. 4.2): E2M1 codes, one FP8
  * (E4M3) scale per 16 consecutive elements, one FP32 scale per tensor.
  *

@@ -11,14 +11,19 @@
 
 namespace quasar {
 
-// Kernel entry for group size 8*epl, or nullptr if not built.
-const void* QUASAR_CAT(int_kernel_nch, QUASAR_NCH)(int epl)
+// Kernel entry for group size 8*epl, one tensor or a batch of up to
+// kMaxBatch tensors per launch, or nullptr if not built.
+const void* QUASAR_CAT(int_kernel_nch, QUASAR_NCH)(int epl, bool batch)
 {
     switch (epl) {
-    case 4: return reinterpret_cast<const void*>(&k_recon_int<4, QUASAR_NCH>);
-    case 8: return reinterpret_cast<const void*>(&k_recon_int<8, QUASAR_NCH>);
-    case 16: return reinterpret_cast<const void*>(&k_recon_int<16, QUASAR_NCH>);
-    case 32: return reinterpret_cast<const void*>(&k_recon_int<32, QUASAR_NCH>);
+    case 4: return batch ? reinterpret_cast<const void*>(&k_recon_int<4, QUASAR_NCH, kMaxBatch>)
+                         : reinterpret_cast<const void*>(&k_recon_int<4, QUASAR_NCH, 1>);
+    case 8: return batch ? reinterpret_cast<const void*>(&k_recon_int<8, QUASAR_NCH, kMaxBatch>)
+                         : reinterpret_cast<const void*>(&k_recon_int<8, QUASAR_NCH, 1>);
+    case 16: return batch ? reinterpret_cast<const void*>(&k_recon_int<16, QUASAR_NCH, kMaxBatch>)
+                          : reinterpret_cast<const void*>(&k_recon_int<16, QUASAR_NCH, 1>);
+    case 32: return batch ? reinterpret_cast<const void*>(&k_recon_int<32, QUASAR_NCH, kMaxBatch>)
+                          : reinterpret_cast<const void*>(&k_recon_int<32, QUASAR_NCH, 1>);
     default: return nullptr;
     }
 }

@@ -16,7 +16,9 @@ constexpr uint32_t kIntScratchBytes = 32 * 32 * 4;
 constexpr int kGroupsPerUnit = 4;
 constexpr int kMaxClip = 32;
 
-struct IntParams {
+// One tensor of an integer-code launch: its buffers, group count, and the
+// index of its first unit in the launch's sequence of units.
+struct IntTensor {
     const float* w;
     const void* g;
     float* v;
@@ -26,6 +28,14 @@ struct IntParams {
     float* b;
     uint8_t* idx;
     int64_t n_groups;
+    int64_t unit0;
+};
+
+// Tensors per launch of the batched entry point (the descriptors travel in
+// the kernel parameters: 256 x 80 bytes, within the 32 KB parameter limit).
+constexpr int kMaxBatch = 256;
+
+struct IntParams {
     int g_kind;  // 0 none, 1 fp32, 2 bf16
     int r_bf16;
     int qmax;
@@ -42,6 +52,16 @@ struct IntParams {
     unsigned int* stats;  // optional: [0] exact re-evaluations, [1] compensated fits, [2] centred refits
     float f[kMaxClip];     // padded with the last factor
     float invf[kMaxClip];  // fl32(1/f)
+};
+
+// Kernel parameters of an integer-code launch over MAXT tensors at most
+// (units numbered consecutively across the tensors).
+template <int MAXT>
+struct IntLaunch {
+    IntParams p;
+    int n_t;
+    int64_t n_units;
+    IntTensor t[MAXT];
 };
 
 constexpr int kBlocksPerUnit = 32;

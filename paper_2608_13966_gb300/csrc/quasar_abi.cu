@@ -15,9 +15,9 @@
 #include "quasar.h"
 
 namespace quasar {
-const void* int_kernel_nch1(int epl);
-const void* int_kernel_nch2(int epl);
-const void* int_kernel_nch4(int epl);
+const void* int_kernel_nch1(int epl, bool batch);
+const void* int_kernel_nch2(int epl, bool batch);
+const void* int_kernel_nch4(int epl, bool batch);
 const void* nvfp4_kernel(int nch);
 const void* amax_kernel();
 const void* amax_to_scale_kernel();
@@ -248,6 +248,94 @@ quasar_status launch_persistent(const void* fn, void* params, size_t smem, int64
 
 int g_kind_of(const void* g, quasar_dtype d) { return !g ? 0 : (d == QUASAR_BF16 ? 2 : 1); }
 
+
+// Validation of one tensor of an integer-code call; fills its descriptor
+// (unit0 is set by the caller).
+quasar_status int_tensor(const float* w, const void* g, quasar_dtype g_dtype, float* v,
+                         float beta2, const float* clip, int n_clip, int64_t rows, int64_t cols,
+                         void* r, quasar_dtype r_dtype, uint8_t* codes, float* a, float* b,
+                         uint8_t* cand_idx, int group_size, IntTensor* T)
+{
+    int64_t n = 0;
+    quasar_status st = check_common(w, g, g_dtype, v, beta2, clip, n_clip, rows, cols, r, r_dtype, &n);
+    if (st != QUASAR_OK) return st;
+    if (group_size <= 0 || cols % group_size != 0) return QUASAR_ERR_INVALID_ARG;
+    const int64_t n_groups = n / group_size;
+    if (n > 0) {
+        if (!a || !b) return QUASAR_ERR_INVALID_ARG;
+        if (codes && !aligned16(codes)) return QUASAR_ERR_INVALID_ARG;
+        const void* outs[] = {r, codes, a, b, cand_idx};
+        const size_t bytes[] = {(size_t)n * dtype_size(r_dtype), codes ? (size_t)n : 0,
+                                (size_t)n_groups * 4, (size_t)n_groups * 4,
+                                cand_idx ? (size_t)n_groups : 0};
+        if (outputs_alias_inputs(w, g, g_dtype, v, n, outs, bytes, 5)) return QUASAR_ERR_INVALID_ARG;
+    }
+    *T = IntTensor{w, g, v, r, codes, a, b, cand_idx, n_groups, 0};
+    return QUASAR_OK;
+}
+
+// Settings shared by the tensors of an integer-code call (no CUDA calls).
+quasar_status int_check(int bits, int group_size)
+{
+    if (bits < 1 || bits > 8) return QUASAR_ERR_INVALID_ARG;
+    if (group_size <= 0) return QUASAR_ERR_INVALID_ARG;
+    if (group_size != 32 && group_size != 64 && group_size != 128 && group_size != 256)
+        return QUASAR_ERR_UNSUPPORTED;
+    return QUASAR_OK;
+}
+
+// Parameters shared by the tensors of an integer-code call.
+quasar_status int_params(quasar_dtype g_dtype, bool has_g, float beta2, int bits, int group_size,
+                         const float* clip, int n_clip, quasar_dtype r_dtype, IntParams* p)
+{
+    quasar_status st0 = int_check(bits, group_size);
+    if (st0 != QUASAR_OK) return st0;
+    *p = IntParams{};
+    p->g_kind = has_g ? (g_dtype == QUASAR_BF16 ? 2 : 1) : 0;
+    p->r_bf16 = r_dtype == QUASAR_BF16;
+    p->qmax = (1 << bits) - 1;
+    p->n_clip = n_clip;
+    p->beta2 = beta2;
+    p->c1 = 1.0f - beta2;
+    // each candidate sum is accumulated over at most G/16 (per packed half)
+    // + 1 + 3 (lane tree) additions; a few more roundings form N, D and E
+    p->tie_kappa = tuning().tie_scale * (float)(group_size / 16 + 8);
+    p->fit_ulps = tuning().fit_ulps;
+    p->timeout_ns = kDefaultTimeoutNs;
+    p->force_timeout_ns = (uint64_t)std::max<int64_t>(0, g_force_timeout_ns.load());
+    p->stats = g_stats.load();
+    fill_clip(clip, n_clip, p->f, p->invf);
+    quasar_status st;
+    if ((st = status_ptr(&p->status)) != QUASAR_OK) return st;
+    const int gbytes = p->g_kind == 2 ? 2 : (p->g_kind == 1 ? 4 : 0);
+    const Launch L = plan((uint32_t)(kGroupsPerUnit * group_size * (8 + gbytes)), kIntScratchBytes);
+    p->stages = L.stages;
+    p->stage_bytes = L.stage_bytes;
+    return QUASAR_OK;
+}
+
+// Number the tensors' units consecutively and launch over all of them.
+template <int MAXT>
+quasar_status int_launch(IntLaunch<MAXT>& Lp, int group_size, int n_clip, cudaStream_t stream)
+{
+    int64_t units = 0;
+    for (int i = 0; i < Lp.n_t; ++i) {
+        Lp.t[i].unit0 = units;
+        units += (Lp.t[i].n_groups + kGroupsPerUnit - 1) / kGroupsPerUnit;
+    }
+    Lp.n_units = units;
+    if (units == 0) return QUASAR_OK;
+    const int gbytes = Lp.p.g_kind == 2 ? 2 : (Lp.p.g_kind == 1 ? 4 : 0);
+    const Launch L = plan((uint32_t)(kGroupsPerUnit * group_size * (8 + gbytes)), kIntScratchBytes);
+    const int epl = group_size / kLanesPerGroup;
+    const int nch = nch_for(n_clip);
+    const bool batch = MAXT > 1;
+    const void* fn = nch == 1 ? int_kernel_nch1(epl, batch)
+                              : (nch == 2 ? int_kernel_nch2(epl, batch) : int_kernel_nch4(epl, batch));
+    if (!fn) return QUASAR_ERR_UNSUPPORTED;
+    return launch_persistent(fn, &Lp, L.smem, units, stream);
+}
+
 }  // namespace
 
 extern "C" {
@@ -258,62 +346,63 @@ quasar_status quasar_recon_int(const float* w, const void* g, quasar_dtype g_dty
                                quasar_dtype r_dtype, uint8_t* codes, float* a, float* b,
                                uint8_t* cand_idx, quasar_stream_t stream)
 {
-    int64_t n = 0;
-    quasar_status st = check_common(w, g, g_dtype, v, beta2, clip, n_clip, rows, cols, r, r_dtype, &n);
+    IntLaunch<1> Lp;
+    quasar_status st = int_tensor(w, g, g_dtype, v, beta2, clip, n_clip, rows, cols, r, r_dtype,
+                                  codes, a, b, cand_idx, group_size > 0 ? group_size : 1, &Lp.t[0]);
     if (st != QUASAR_OK) return st;
-    if (bits < 1 || bits > 8) return QUASAR_ERR_INVALID_ARG;
-    if (group_size <= 0 || cols % group_size != 0) return QUASAR_ERR_INVALID_ARG;
-    if (group_size != 32 && group_size != 64 && group_size != 128 && group_size != 256)
-        return QUASAR_ERR_UNSUPPORTED;
-    if (n == 0) return QUASAR_OK;
-    if (!a || !b) return QUASAR_ERR_INVALID_ARG;
-    if (codes && !aligned16(codes)) return QUASAR_ERR_INVALID_ARG;
-    const int64_t n_groups = n / group_size;
-    {
-        const void* outs[] = {r, codes, a, b, cand_idx};
-        const size_t bytes[] = {(size_t)n * dtype_size(r_dtype), codes ? (size_t)n : 0,
-                                (size_t)n_groups * 4, (size_t)n_groups * 4,
-                                cand_idx ? (size_t)n_groups : 0};
-        if (outputs_alias_inputs(w, g, g_dtype, v, n, outs, bytes, 5)) return QUASAR_ERR_INVALID_ARG;
+    if ((st = int_check(bits, group_size)) != QUASAR_OK) return st;
+    if (Lp.t[0].n_groups == 0) return QUASAR_OK;  // empty: no-op
+    if ((st = int_params(g_dtype, g != nullptr, beta2, bits, group_size, clip, n_clip, r_dtype,
+                         &Lp.p)) != QUASAR_OK)
+        return st;
+    Lp.n_t = 1;
+    return int_launch(Lp, group_size, n_clip, reinterpret_cast<cudaStream_t>(stream));
+}
+
+quasar_status quasar_recon_int_batch(const quasar_int_tensor* tensors, int n_tensors,
+                                     quasar_dtype g_dtype, float beta2, int bits, int group_size,
+                                     const float* clip, int n_clip, quasar_dtype r_dtype,
+                                     quasar_stream_t stream)
+{
+    if (n_tensors < 0 || (n_tensors > 0 && !tensors)) return QUASAR_ERR_INVALID_ARG;
+    if (n_tensors == 0) return QUASAR_OK;
+    // all non-empty tensors carry a gradient, or none does
+    int with_g = 0, non_empty = 0;
+    for (int i = 0; i < n_tensors; ++i)
+        if (tensors[i].rows != 0 && tensors[i].cols != 0) {
+            ++non_empty;
+            with_g += tensors[i].g != nullptr;
+        }
+    if (with_g != 0 && with_g != non_empty) return QUASAR_ERR_INVALID_ARG;
+    const bool has_g = with_g != 0;
+    static thread_local IntLaunch<kMaxBatch> Lp;  // 20 KB: kept off the stack
+    quasar_status st = int_check(bits, group_size);
+    if (st != QUASAR_OK) return st;
+    // validate every tensor before launching anything
+    int64_t total = 0;
+    for (int i = 0; i < n_tensors; ++i) {
+        const quasar_int_tensor& x = tensors[i];
+        IntTensor T;
+        if ((st = int_tensor(x.w, x.g, g_dtype, x.v, beta2, clip, n_clip, x.rows, x.cols, x.r,
+                             r_dtype, x.codes, x.a, x.b, x.cand_idx, group_size, &T)) != QUASAR_OK)
+            return st;
+        total += T.n_groups;
     }
-
-    IntParams p{};
-    p.w = w;
-    p.g = g;
-    p.v = v;
-    p.r = r;
-    p.codes = codes;
-    p.a = a;
-    p.b = b;
-    p.idx = cand_idx;
-    p.n_groups = n_groups;
-    p.g_kind = g_kind_of(g, g_dtype);
-    p.r_bf16 = r_dtype == QUASAR_BF16;
-    p.qmax = (1 << bits) - 1;
-    p.n_clip = n_clip;
-    p.beta2 = beta2;
-    p.c1 = 1.0f - beta2;
-    // each candidate sum is accumulated over at most G/16 (per packed half)
-    // + 1 + 3 (lane tree) additions; a few more roundings form N, D and E
-    p.tie_kappa = tuning().tie_scale * (float)(group_size / 16 + 8);
-    p.fit_ulps = tuning().fit_ulps;
-    p.timeout_ns = kDefaultTimeoutNs;
-    p.force_timeout_ns = (uint64_t)std::max<int64_t>(0, g_force_timeout_ns.load());
-    p.stats = g_stats.load();
-    fill_clip(clip, n_clip, p.f, p.invf);
-    if ((st = status_ptr(&p.status)) != QUASAR_OK) return st;
-
-    const int gbytes = p.g_kind == 2 ? 2 : (p.g_kind == 1 ? 4 : 0);
-    const Launch L = plan((uint32_t)(kGroupsPerUnit * group_size * (8 + gbytes)), kIntScratchBytes);
-    p.stages = L.stages;
-    p.stage_bytes = L.stage_bytes;
-
-    const int epl = group_size / kLanesPerGroup;
-    const int nch = nch_for(n_clip);
-    const void* fn = nch == 1 ? int_kernel_nch1(epl) : (nch == 2 ? int_kernel_nch2(epl) : int_kernel_nch4(epl));
-    if (!fn) return QUASAR_ERR_UNSUPPORTED;
-    const int64_t n_units = (n_groups + kGroupsPerUnit - 1) / kGroupsPerUnit;
-    return launch_persistent(fn, &p, L.smem, n_units, reinterpret_cast<cudaStream_t>(stream));
+    if (total == 0) return QUASAR_OK;
+    if ((st = int_params(g_dtype, has_g, beta2, bits, group_size, clip, n_clip, r_dtype, &Lp.p)) !=
+        QUASAR_OK)
+        return st;
+    const cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+    for (int i0 = 0; i0 < n_tensors; i0 += kMaxBatch) {
+        Lp.n_t = std::min(kMaxBatch, n_tensors - i0);
+        for (int i = 0; i < Lp.n_t; ++i) {
+            const quasar_int_tensor& x = tensors[i0 + i];
+            int_tensor(x.w, x.g, g_dtype, x.v, beta2, clip, n_clip, x.rows, x.cols, x.r, r_dtype,
+                       x.codes, x.a, x.b, x.cand_idx, group_size, &Lp.t[i]);
+        }
+        if ((st = int_launch(Lp, group_size, n_clip, s)) != QUASAR_OK) return st;
+    }
+    return QUASAR_OK;
 }
 
 quasar_status quasar_tensor_amax(const float* w, int64_t n, float* amax_out, quasar_stream_t stream)

@@ -355,9 +355,10 @@ __device__ void coop_precise(const float* ws, const float* hs, float c, float P,
 
 // ------------------------------------------------------------------ kernel
 
-template <int EPL, int NCH>
-__global__ void __launch_bounds__(256) k_recon_int(const IntParams p)
+template <int EPL, int NCH, int MAXT>
+__global__ void __launch_bounds__(256) k_recon_int(const __grid_constant__ IntLaunch<MAXT> Lp)
 {
+    const IntParams& p = Lp.p;
     constexpr int G = EPL * kLanesPerGroup;
     constexpr int UNIT = kGroupsPerUnit * G;
     constexpr int NCHK = EPL / 4;  // 16-byte chunks per lane and group
@@ -381,7 +382,13 @@ __global__ void __launch_bounds__(256) k_recon_int(const IntParams p)
     constexpr uint32_t kVOff = UNIT * 4;
     constexpr uint32_t kGOff = UNIT * 8;
 
-    const int64_t n_units = (p.n_groups + kGroupsPerUnit - 1) / kGroupsPerUnit;
+    const int64_t n_units = Lp.n_units;
+    // the tensor of a unit: units are numbered consecutively across the
+    // launch's tensors, and each warp meets them in increasing order
+    auto tensor_of = [&](int64_t u, int& ti) {
+        while (ti + 1 < Lp.n_t && u >= Lp.t[ti + 1].unit0) ++ti;
+    };
+    int ti_issue = 0, ti = 0;
     const int64_t first = (int64_t)blockIdx.x * nwarps + warp;
     const int64_t stride = (int64_t)gridDim.x * nwarps;
 
@@ -392,15 +399,17 @@ __global__ void __launch_bounds__(256) k_recon_int(const IntParams p)
     __syncwarp();
 
     auto issue = [&](int64_t u, int s) {
-        const int64_t g0 = u * kGroupsPerUnit;
-        const int64_t ng = min((int64_t)kGroupsPerUnit, p.n_groups - g0);
+        tensor_of(u, ti_issue);
+        const IntTensor& T = Lp.t[ti_issue];
+        const int64_t g0 = (u - T.unit0) * kGroupsPerUnit;
+        const int64_t ng = min((int64_t)kGroupsPerUnit, T.n_groups - g0);
         const uint32_t elems = (uint32_t)(ng * G);
         unsigned char* st = ring + (size_t)s * p.stage_bytes;
         mbar_arrive_expect_tx(&bars[s], elems * (8u + (uint32_t)gbytes));
-        bulk_g2s(st, p.w + g0 * G, elems * 4u, &bars[s]);
-        bulk_g2s(st + kVOff, p.v + g0 * G, elems * 4u, &bars[s]);
+        bulk_g2s(st, T.w + g0 * G, elems * 4u, &bars[s]);
+        bulk_g2s(st + kVOff, T.v + g0 * G, elems * 4u, &bars[s]);
         if (gbytes)
-            bulk_g2s(st + kGOff, static_cast<const unsigned char*>(p.g) + g0 * G * gbytes,
+            bulk_g2s(st + kGOff, static_cast<const unsigned char*>(T.g) + g0 * G * gbytes,
                      elems * (uint32_t)gbytes, &bars[s]);
     };
 
@@ -451,15 +460,17 @@ __global__ void __launch_bounds__(256) k_recon_int(const IntParams p)
         float* hs = reinterpret_cast<float*>(st + kVOff);
         const unsigned char* gsm = st + kGOff;
 
-        const int64_t grp = u * kGroupsPerUnit + gs;
-        const bool valid = grp < p.n_groups;
+        tensor_of(u, ti);
+        const IntTensor& T = Lp.t[ti];
+        const int64_t grp = (u - T.unit0) * kGroupsPerUnit + gs;
+        const bool valid = grp < T.n_groups;
         const int64_t gbase = grp * (int64_t)G;
 
         // ---- pass A: saliency EMA (h kept in the tile), range, saliency mass
         // and weighted sum of w (a centre for the moments)
         float mn = INFINITY, mx = -INFINITY, ss = 0.0f, sw = 0.0f;
         {
-            float* vout = p.v + gbase + sl * 4;
+            float* vout = T.v + gbase + sl * 4;
             auto pass_a = [&](auto gk) {
                 constexpr int GK = decltype(gk)::value;
                 float2 SS = make_float2(0.0f, 0.0f), SW = SS;
@@ -931,7 +942,7 @@ __global__ void __launch_bounds__(256) k_recon_int(const IntParams p)
                             rv[0] = make_float2(w4.x, w4.y);
                             rv[1] = make_float2(w4.z, w4.w);
                         }
-                        if (p.codes) {
+                        if (T.codes) {
                             // q = z + qmax/2, an integer in [0, 255]: its bits above 2^23
                             uint32_t cw = 0;
 #pragma unroll
@@ -940,19 +951,19 @@ __global__ void __launch_bounds__(256) k_recon_int(const IntParams p)
                                 cw |= ((__float_as_uint(qf.x) & 0xFFu) | ((__float_as_uint(qf.y) & 0xFFu) << 8))
                                       << (16 * pr);
                             }
-                            stg_cs(reinterpret_cast<uint32_t*>(p.codes + eo), flat ? 0u : cw);
+                            stg_cs(reinterpret_cast<uint32_t*>(T.codes + eo), flat ? 0u : cw);
                         }
                     }
                     if (!GEN || p.r_bf16) {
-                        stg_cs(reinterpret_cast<uint2*>(static_cast<__nv_bfloat16*>(p.r) + eo),
+                        stg_cs(reinterpret_cast<uint2*>(static_cast<__nv_bfloat16*>(T.r) + eo),
                                make_uint2(pack_bf16x2(rv[0].x, rv[0].y), pack_bf16x2(rv[1].x, rv[1].y)));
                     } else {
-                        stg_cs(reinterpret_cast<float4*>(static_cast<float*>(p.r) + eo),
+                        stg_cs(reinterpret_cast<float4*>(static_cast<float*>(T.r) + eo),
                                make_float4(rv[0].x, rv[0].y, rv[1].x, rv[1].y));
                     }
                 }
             };
-            const bool gen = !p.r_bf16 || p.codes != nullptr || __any_sync(0xffffffffu, flat);
+            const bool gen = !p.r_bf16 || T.codes != nullptr || __any_sync(0xffffffffu, flat);
             if (valid) {
                 if (gen) pass_c(std::true_type{});
                 else pass_c(std::false_type{});
@@ -961,9 +972,9 @@ __global__ void __launch_bounds__(256) k_recon_int(const IntParams p)
                 // b = Bz - a*H: the offset at code 0
                 float bh = Bz, bl = Bz_lo;
                 ff_add_prod(bh, bl, -a_sel, -a_lo, H);
-                p.a[grp] = flat ? 0.0f : a_sel;
-                p.b[grp] = flat ? c : __fadd_rn(bh, bl);
-                if (p.idx) p.idx[grp] = flat ? 0 : (uint8_t)kb;
+                T.a[grp] = flat ? 0.0f : a_sel;
+                T.b[grp] = flat ? c : __fadd_rn(bh, bl);
+                if (T.idx) T.idx[grp] = flat ? 0 : (uint8_t)kb;
             }
         }
 

@@ -42,6 +42,7 @@ PROTOTYPES = {
                               _P, _P]),
     "quasar_recon_nvfp4": (_I, [_P, _P, _I, _P, _F, _P, _I, _I64, _I64, _P, _P, _I, _P, _P, _P,
                                 _P, _P]),
+    "quasar_recon_int_batch": (_I, [_P, _I, _I, _F, _I, _I, _P, _I, _I, _P]),
     "quasar_tensor_amax": (_I, [_P, _I64, _P, _P]),
     "quasar_get_device_status": (_I, [_P]),
     "quasar_debug_force_timeout": (None, [_I64]),
@@ -124,6 +125,37 @@ def quasar_recon_int(w, g, v, beta2, bits, group_size, clip, rows, cols, r, code
     st = lib.quasar_recon_int(_ptr(w), _ptr(g), gd, _ptr(v), beta2, bits, group_size, carr, nclip,
                               rows, cols, _ptr(r), rd, _ptr(codes), _ptr(a), _ptr(b),
                               _ptr(cand_idx), _stream(stream))
+    return QuasarStatus(st)
+
+
+class QuasarIntTensor(ctypes.Structure):
+    """quasar_int_tensor: one tensor's buffers (device pointers) and shape."""
+    _fields_ = [("w", ctypes.c_void_p), ("g", ctypes.c_void_p), ("v", ctypes.c_void_p),
+                ("r", ctypes.c_void_p), ("codes", ctypes.c_void_p), ("a", ctypes.c_void_p),
+                ("b", ctypes.c_void_p), ("cand_idx", ctypes.c_void_p), ("rows", ctypes.c_int64),
+                ("cols", ctypes.c_int64)]
+
+
+def int_tensor_array(items):
+    """A ctypes array of QuasarIntTensor from dicts with keys w, g, v, r,
+    codes, a, b, cand_idx (tensors, pointers or None), rows, cols."""
+    arr = (QuasarIntTensor * len(items))()
+    for i, d in enumerate(items):
+        arr[i] = QuasarIntTensor(_ptr(d["w"]), _ptr(d.get("g")), _ptr(d["v"]), _ptr(d["r"]),
+                                 _ptr(d.get("codes")), _ptr(d["a"]), _ptr(d["b"]),
+                                 _ptr(d.get("cand_idx")), int(d["rows"]), int(d["cols"]))
+    return arr
+
+
+def quasar_recon_int_batch(tensors, beta2, bits, group_size, clip, g_dtype=BF16, r_dtype=BF16,
+                           stream=None) -> QuasarStatus:
+    """tensors: a ctypes array from int_tensor_array (or a list of dicts)."""
+    lib = load()
+    if not isinstance(tensors, ctypes.Array):
+        tensors = int_tensor_array(tensors)
+    carr, nclip = _clip_array(clip)
+    st = lib.quasar_recon_int_batch(ctypes.cast(tensors, ctypes.c_void_p), len(tensors), g_dtype,
+                                    beta2, bits, group_size, carr, nclip, r_dtype, _stream(stream))
     return QuasarStatus(st)
 
 

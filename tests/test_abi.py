@@ -125,3 +125,25 @@ def test_product_path_has_no_oracle_dependency():
                 text = open(os.path.join(dirpath, fn)).read()
                 assert not re.search(r"^\s*(import|from)\s+oracle\b", text, re.M), fn
                 assert "quasar_oracle" not in text and "qo_" not in text, fn
+
+
+def _desc(**kw):
+    d = dict(w=A, g=B, v=C, r=D, codes=None, a=E, b=F, cand_idx=None, rows=4, cols=256)
+    d.update(kw)
+    return d
+
+
+def test_int_batch_argument_validation(lib):
+    st = Q.QuasarStatus
+    call = lambda items, **kw: Q.quasar_recon_int_batch(
+        items, kw.get("beta2", 0.999), kw.get("bits", 3), kw.get("group_size", 128), CLIP, stream=0)
+    assert Q.quasar_recon_int_batch([], 0.999, 3, 128, CLIP, stream=0) == st.OK  # nothing to do
+    assert call([_desc(rows=0), _desc(cols=0)]) == st.OK                         # all empty
+    assert call([_desc(), _desc(g=None)]) == st.ERR_INVALID_ARG                  # mixed gradients
+    assert call([_desc(), _desc(a=None)]) == st.ERR_INVALID_ARG                  # bad second tensor
+    assert call([_desc(), _desc(cols=200)]) == st.ERR_INVALID_ARG                # cols % group_size
+    assert call([_desc(), _desc(r=A)]) == st.ERR_INVALID_ARG                     # output aliases w
+    assert call([_desc()], bits=9) == st.ERR_INVALID_ARG
+    assert call([_desc()], group_size=48) == st.ERR_UNSUPPORTED
+    n = ctypes.c_void_p(None)
+    assert Q.load().quasar_recon_int_batch(n, 2, Q.BF16, 0.999, 3, 128, None, 0, Q.BF16, None) == st.ERR_INVALID_ARG

@@ -10,6 +10,7 @@ import pytest
 import torch
 
 from paper_2608_13966_gb300 import workloads as wl
+from tests import checker
 from tests import gpu_harness as H
 
 pytestmark = pytest.mark.gpu
@@ -156,3 +157,38 @@ def test_timeout_path_reports_and_recovers(oracle):
     rep, ema = H.run_int(oracle, *_inputs(64, 512, seed=83), bits=3, group_size=128,
                          clip=CLIP8)
     _assert(rep, ema)
+
+
+def test_int_batch_matches_oracle_and_single_calls(oracle):
+    """One launch over tensors of different shapes (group counts that leave
+    a partial last unit, a tiny tensor, an empty one) gives, tensor by
+    tensor, the oracle's result and bit-for-bit the single-call result."""
+    from paper_2608_13966_gb300 import api
+    shapes = [(64, 1024), (3, 384), (1, 128), (0, 256), (37, 640), (128, 512)]
+    items, copies = [], []
+    for i, (rows, cols) in enumerate(shapes):
+        w, g, v = _inputs(max(rows, 1), cols, seed=300 + i)
+        w, g, v = w[:rows].contiguous(), g[:rows].contiguous(), v[:rows].contiguous()
+        items.append((w, g, v))
+        copies.append((w.clone(), g.clone(), v.clone()))
+    clip = list(wl.CLIP_8)
+    w_h = [H._host(w) for w, _, _ in items]
+    g_h = [H._host(g) for _, g, _ in items]
+    v_h = [H._host(v) for _, _, v in items]
+    outs = api.recon_int_batch(items, bits=3, group_size=128, clip=clip, codes=True)
+    singles = [api.recon_int(w, g, v, bits=3, group_size=128, clip=clip, codes=True)
+               for (w, g, v) in copies]
+    torch.cuda.synchronize()
+    for i, (o, s1) in enumerate(zip(outs, singles)):
+        for key in ("r", "a", "b", "codes", "cand_idx"):
+            assert torch.equal(o[key], s1[key]), (shapes[i], key)
+        assert torch.equal(items[i][2], copies[i][2])  # v' identical
+        if w_h[i].size == 0:
+            continue
+        h = oracle.ema(v_h[i], g_h[i], 0.999)
+        O = oracle.recon_int(w_h[i], h, 128, 3, clip)
+        gpu = {"r": H._host(o["r"]), "a": o["a"].cpu().numpy(), "b": o["b"].cpu().numpy(),
+               "codes": o["codes"].cpu().numpy().ravel(), "idx": o["cand_idx"].cpu().numpy()}
+        rep = checker.check_int(oracle, w_h[i], h, 3, clip, O, gpu, 128, True)
+        ema = checker.check_ema(h, H._host(items[i][2]))
+        _assert(rep, ema)
