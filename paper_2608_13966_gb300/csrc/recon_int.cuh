@@ -388,7 +388,7 @@ __global__ void __launch_bounds__(256) k_recon_int(const __grid_constant__ IntLa
     auto tensor_of = [&](int64_t u, int& ti) {
         while (ti + 1 < Lp.n_t && u >= Lp.t[ti + 1].unit0) ++ti;
     };
-    int ti_issue = 0, ti = 0;
+    int ti = 0;
     const int64_t first = (int64_t)blockIdx.x * nwarps + warp;
     const int64_t stride = (int64_t)gridDim.x * nwarps;
 
@@ -398,9 +398,12 @@ __global__ void __launch_bounds__(256) k_recon_int(const __grid_constant__ IntLa
     }
     __syncwarp();
 
+    // (the unit issued is at or after the one being processed: its tensor
+    // index is found from ti onwards)
     auto issue = [&](int64_t u, int s) {
-        tensor_of(u, ti_issue);
-        const IntTensor& T = Lp.t[ti_issue];
+        int tj = ti;
+        tensor_of(u, tj);
+        const IntTensor& T = Lp.t[tj];
         const int64_t g0 = (u - T.unit0) * kGroupsPerUnit;
         const int64_t ng = min((int64_t)kGroupsPerUnit, T.n_groups - g0);
         const uint32_t elems = (uint32_t)(ng * G);
