@@ -129,13 +129,18 @@ class Step:
                     wlo.bits, wlo.group, self.clip, len(wlo.clip), Q.BF16, self.stream)
             self.calls.append((self.lib.quasar_recon_int_batch, args, model.elements))
         else:
-            for d in model.tensors:
-                s = d["spec"]
-                args = (d["w"].data_ptr(), d["g"].data_ptr(), Q.BF16, d["v"].data_ptr(), wlo.beta2,
-                        self.clip, len(wlo.clip), s.rows, s.cols, None, d["r"].data_ptr(), Q.BF16,
-                        None, d["scale"].data_ptr(), d["ts"].data_ptr(), d["idx"].data_ptr(),
-                        self.stream)
-                self.calls.append((self.lib.quasar_recon_nvfp4, args, s.numel))
+            # every tensor in one call (quasar_recon_nvfp4_batch): absmax of
+            # every tensor, their scales, one reconstruction launch
+            self.descs = Q.nvfp4_tensor_array([
+                {"w": d["w"], "g": d["g"], "v": d["v"], "tensor_amax": None, "r": d["r"],
+                 "codes": None, "block_scale": d["scale"], "tensor_scale": d["ts"],
+                 "cand_idx": d["idx"], "rows": d["spec"].rows, "cols": d["spec"].cols}
+                for d in model.tensors])
+            args = (ctypes.cast(self.descs, ctypes.c_void_p), len(self.descs), Q.BF16, wlo.beta2,
+                    self.clip, len(wlo.clip), Q.BF16, self.stream)
+            self.calls.append((self.lib.quasar_recon_nvfp4_batch, args, model.elements))
+        # INT: one launch; NVFP4: absmax, scale and reconstruction launches
+        # (plus one small memset of the scale slot per tensor)
         self.launches_per_call = 1 if wlo.fmt == "int" else 3
 
     def run(self, events=None):
@@ -456,7 +461,7 @@ def main():
         "roofline": {"bound": "hbm", "achieved": achieved, "peak": hbm_peak, "unit": "GB/s",
                      "frac": achieved / hbm_peak, "traffic": traffic,
                      "peak_kind": peak_kind,
-                     "kernel": "k_recon_int<16,1,256> (one launch per step)" if wlo.fmt == "int" else "k_recon_nvfp4<1>",
+                     "kernel": "k_recon_int<16,1,256> (one launch per step)" if wlo.fmt == "int" else "k_recon_nvfp4<1,256> (one launch per step)",
                      "bytes_per_weight": step_bytes / n_el,
                      "launch_bytes": step_bytes / len(step.calls),
                      "launch_ms": kernel_ms / args.steps / len(step.calls),

@@ -162,6 +162,36 @@ quasar_status quasar_recon_nvfp4(const float* w, const void* g, quasar_dtype g_d
                                  quasar_stream_t stream);
 
 /*
+ * quasar_nvfp4_tensor / quasar_recon_nvfp4_batch -- quasar_recon_nvfp4 over
+ * many tensors with the same settings: one absmax pass over the tensors
+ * whose amax is not supplied, one scale pass, and one persistent
+ * reconstruction launch whose units are numbered across the tensors.
+ * Each descriptor holds one tensor's arguments as quasar_recon_nvfp4 takes
+ * them (same meaning and rules; each tensor has its own tensor_scale slot and
+ * optional tensor_amax); either every non-empty tensor has a gradient or none
+ * does.  HOST array, read before the call returns; more than 256 tensors are
+ * processed 256 per launch.  Returns as quasar_recon_nvfp4; every tensor is
+ * validated before anything is launched.  The paper has no batched form.
+ */
+typedef struct {
+    const float* w;
+    const void* g;
+    float* v;
+    const float* tensor_amax;
+    void* r;
+    uint8_t* codes;
+    uint8_t* block_scale;
+    float* tensor_scale;
+    uint8_t* cand_idx;
+    int64_t rows;
+    int64_t cols;
+} quasar_nvfp4_tensor;
+
+quasar_status quasar_recon_nvfp4_batch(const quasar_nvfp4_tensor* tensors, int n_tensors,
+                                       quasar_dtype g_dtype, float beta2, const float* clip,
+                                       int n_clip, quasar_dtype r_dtype, quasar_stream_t stream);
+
+/*
  * quasar_tensor_amax -- amax_out[0] = max |w[i]| over n fp32 elements (the
  * NVFP4 tensor statistic of Sec. 4.2).  amax_out is a device pointer; it is
  * overwritten.  n == 0 writes 0.

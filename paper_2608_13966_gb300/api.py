@@ -5,8 +5,9 @@ from __future__ import annotations
 
 import torch
 
-from .quasar import (BF16, F32, QuasarError, QuasarStatus, int_tensor_array, quasar_recon_int,
-                     quasar_recon_int_batch, quasar_recon_nvfp4, quasar_tensor_amax)
+from .quasar import (BF16, F32, QuasarError, QuasarStatus, int_tensor_array, nvfp4_tensor_array,
+                     quasar_recon_int, quasar_recon_int_batch, quasar_recon_nvfp4,
+                     quasar_recon_nvfp4_batch, quasar_tensor_amax)
 
 
 def _check(st):
@@ -108,6 +109,40 @@ def recon_nvfp4(w, g, v, *, clip, beta2=0.999, tensor_amax=None, r_dtype=torch.b
     if k is not None:
         res["cand_idx"] = k
     return res
+
+
+def recon_nvfp4_batch(items, *, clip, beta2=0.999, r_dtype=torch.bfloat16, codes=False,
+                      cand_idx=True, stream=None):
+    """QUASAR NVFP4 reconstruction of several tensors (one absmax pass, one
+    scale pass, one reconstruction launch).  items: list of (w, g, v) or
+    (w, g, v, tensor_amax) CUDA tensors; each v is updated in place."""
+    descs, results = [], []
+    g_dtype = F32
+    for it in items:
+        w, g, v = it[:3]
+        amax = it[3] if len(it) > 3 else None
+        _check_2d(w)
+        rows, cols = w.shape
+        dev = w.device
+        n_blocks = rows * cols // 16
+        res = {"r": torch.empty((rows, cols), dtype=r_dtype, device=dev),
+               "block_scale": torch.empty(n_blocks, dtype=torch.uint8, device=dev),
+               "tensor_scale": torch.empty(1, dtype=torch.float32, device=dev)}
+        if codes:
+            res["codes"] = torch.empty((rows, cols), dtype=torch.uint8, device=dev)
+        if cand_idx:
+            res["cand_idx"] = torch.empty(n_blocks, dtype=torch.uint8, device=dev)
+        if g is not None and g.dtype == torch.bfloat16:
+            g_dtype = BF16
+        descs.append({"w": w, "g": g, "v": v, "tensor_amax": amax, "r": res["r"],
+                      "codes": res.get("codes"), "block_scale": res["block_scale"],
+                      "tensor_scale": res["tensor_scale"], "cand_idx": res.get("cand_idx"),
+                      "rows": rows, "cols": cols})
+        results.append(res)
+    rd = BF16 if r_dtype == torch.bfloat16 else F32
+    _check(quasar_recon_nvfp4_batch(nvfp4_tensor_array(descs), beta2, clip, g_dtype=g_dtype,
+                                    r_dtype=rd, stream=stream))
+    return results
 
 
 def tensor_amax(w, stream=None):

@@ -4,17 +4,29 @@
 
 namespace quasar {
 
-const void* nvfp4_kernel(int nch)
+const void* nvfp4_kernel(int nch, bool batch)
 {
     switch (nch) {
-    case 1: return reinterpret_cast<const void*>(&k_recon_nvfp4<1>);
-    case 2: return reinterpret_cast<const void*>(&k_recon_nvfp4<2>);
-    case 4: return reinterpret_cast<const void*>(&k_recon_nvfp4<4>);
+    case 1: return batch ? reinterpret_cast<const void*>(&k_recon_nvfp4<1, kMaxBatch>)
+                         : reinterpret_cast<const void*>(&k_recon_nvfp4<1, 1>);
+    case 2: return batch ? reinterpret_cast<const void*>(&k_recon_nvfp4<2, kMaxBatch>)
+                         : reinterpret_cast<const void*>(&k_recon_nvfp4<2, 1>);
+    case 4: return batch ? reinterpret_cast<const void*>(&k_recon_nvfp4<4, kMaxBatch>)
+                         : reinterpret_cast<const void*>(&k_recon_nvfp4<4, 1>);
     default: return nullptr;
     }
 }
 
-const void* amax_kernel() { return reinterpret_cast<const void*>(&k_amax); }
-const void* amax_to_scale_kernel() { return reinterpret_cast<const void*>(&k_amax_to_scale); }
+const void* amax_kernel(bool batch)
+{
+    return batch ? reinterpret_cast<const void*>(&k_amax<kMaxBatch>)
+                 : reinterpret_cast<const void*>(&k_amax<1>);
+}
+
+const void* amax_to_scale_kernel(bool batch)
+{
+    return batch ? reinterpret_cast<const void*>(&k_amax_to_scale<kMaxBatch>)
+                 : reinterpret_cast<const void*>(&k_amax_to_scale<1>);
+}
 
 }  // namespace quasar

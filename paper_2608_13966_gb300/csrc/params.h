@@ -66,7 +66,9 @@ struct IntLaunch {
 
 constexpr int kBlocksPerUnit = 32;
 
-struct Nvfp4Params {
+// One tensor of an NVFP4 launch.  tensor_scale holds s_T (written before
+// the reconstruction kernel runs); unit0 as for IntTensor.
+struct Nvfp4Tensor {
     const float* w;
     const void* g;
     float* v;
@@ -74,10 +76,12 @@ struct Nvfp4Params {
     uint8_t* codes;
     uint8_t* scale;
     uint8_t* idx;
-    const float* amax;     // device scalar (caller's, or the tensor_scale slot)
-    float* tensor_scale;   // written by block 0 when write_scale != 0
-    int write_scale;
+    const float* tensor_scale;
     int64_t n_blocks;
+    int64_t unit0;
+};
+
+struct Nvfp4Params {
     int g_kind;
     int r_bf16;
     int n_clip;
@@ -92,6 +96,30 @@ struct Nvfp4Params {
     unsigned int* stats;
     float f[kMaxClip];
     float invf[kMaxClip];
+};
+
+template <int MAXT>
+struct Nvfp4Launch {
+    Nvfp4Params p;
+    int n_t;
+    int64_t n_units;
+    Nvfp4Tensor t[MAXT];
+};
+
+// Per-tensor absmax and scale passes of a batched NVFP4 call (kernel
+// parameters): amax of w (n elements) into *slot unless amax_in is given;
+// then *slot := s_T of amax_in (or of the slot).
+struct AmaxItem {
+    const float* w;
+    int64_t n;
+    float* slot;
+    const float* amax_in;
+};
+
+template <int MAXT>
+struct AmaxBatch {
+    int n_t;
+    AmaxItem t[MAXT];
 };
 
 }  // namespace quasar

@@ -18,9 +18,9 @@ namespace quasar {
 const void* int_kernel_nch1(int epl, bool batch);
 const void* int_kernel_nch2(int epl, bool batch);
 const void* int_kernel_nch4(int epl, bool batch);
-const void* nvfp4_kernel(int nch);
-const void* amax_kernel();
-const void* amax_to_scale_kernel();
+const void* nvfp4_kernel(int nch, bool batch);
+const void* amax_kernel(bool batch);
+const void* amax_to_scale_kernel(bool batch);
 }  // namespace quasar
 
 // Per-device status word (bit 0: a kernel timed out on a wait).
@@ -336,6 +336,109 @@ quasar_status int_launch(IntLaunch<MAXT>& Lp, int group_size, int n_clip, cudaSt
     return launch_persistent(fn, &Lp, L.smem, units, stream);
 }
 
+// Validation of one tensor of an NVFP4 call; fills its descriptor and its
+// absmax/scale item (unit0 is set later).
+quasar_status nvfp4_tensor(const float* w, const void* g, quasar_dtype g_dtype, float* v,
+                           float beta2, const float* clip, int n_clip, int64_t rows, int64_t cols,
+                           const float* tensor_amax, void* r, quasar_dtype r_dtype, uint8_t* codes,
+                           uint8_t* block_scale, float* tensor_scale, uint8_t* cand_idx,
+                           Nvfp4Tensor* T, AmaxItem* A)
+{
+    int64_t n = 0;
+    quasar_status st = check_common(w, g, g_dtype, v, beta2, clip, n_clip, rows, cols, r, r_dtype, &n);
+    if (st != QUASAR_OK) return st;
+    if (cols % 16 != 0) return QUASAR_ERR_INVALID_ARG;
+    if (!tensor_scale || (reinterpret_cast<uintptr_t>(tensor_scale) & 3u) != 0)
+        return QUASAR_ERR_INVALID_ARG;
+    if (tensor_amax && (reinterpret_cast<uintptr_t>(tensor_amax) & 3u) != 0)
+        return QUASAR_ERR_INVALID_ARG;
+    const int64_t n_blocks = n / 16;
+    if (n > 0) {
+        if (!block_scale) return QUASAR_ERR_INVALID_ARG;
+        if (codes && !aligned16(codes)) return QUASAR_ERR_INVALID_ARG;
+        const void* outs[] = {r, codes, block_scale, tensor_scale, cand_idx};
+        const size_t bytes[] = {(size_t)n * dtype_size(r_dtype), codes ? (size_t)n : 0,
+                                (size_t)n_blocks, 4, cand_idx ? (size_t)n_blocks : 0};
+        if (outputs_alias_inputs(w, g, g_dtype, v, n, outs, bytes, 5)) return QUASAR_ERR_INVALID_ARG;
+        if (tensor_amax && overlaps(tensor_amax, 4, tensor_scale, 4)) return QUASAR_ERR_INVALID_ARG;
+    }
+    *T = Nvfp4Tensor{w, g, v, r, codes, block_scale, cand_idx, tensor_scale, n_blocks, 0};
+    *A = AmaxItem{w, n, tensor_scale, tensor_amax};
+    return QUASAR_OK;
+}
+
+quasar_status nvfp4_params(bool has_g, quasar_dtype g_dtype, float beta2, const float* clip,
+                           int n_clip, quasar_dtype r_dtype, Nvfp4Params* p)
+{
+    *p = Nvfp4Params{};
+    p->g_kind = has_g ? (g_dtype == QUASAR_BF16 ? 2 : 1) : 0;
+    p->r_bf16 = r_dtype == QUASAR_BF16;
+    p->n_clip = n_clip;
+    p->beta2 = beta2;
+    p->c1 = 1.0f - beta2;
+    p->tie_kappa = tuning().tie_kappa;
+    p->timeout_ns = kDefaultTimeoutNs;
+    p->force_timeout_ns = (uint64_t)std::max<int64_t>(0, g_force_timeout_ns.load());
+    p->stats = g_stats.load();
+    fill_clip(clip, n_clip, p->f, p->invf);
+    return status_ptr(&p->status);
+}
+
+// Absmax of the tensors whose amax is not supplied, into their scale slots
+// (zeroed first by the caller of each slot), then every slot := s_T.
+template <int MAXT>
+quasar_status launch_amax(const AmaxBatch<MAXT>& B, cudaStream_t s)
+{
+    int dev = 0;
+    const DeviceInfo* info = nullptr;
+    const quasar_status st = device_info(&dev, &info);
+    if (st != QUASAR_OK) return st;
+    int64_t nmax = 0;
+    for (int i = 0; i < B.n_t; ++i)
+        if (!B.t[i].amax_in) nmax = std::max(nmax, B.t[i].n);
+    if (nmax == 0) return QUASAR_OK;
+    const int64_t want = (nmax / 4 + kThreads - 1) / kThreads;
+    const int64_t per_sm = std::max<int64_t>(1, (int64_t)info->nsm * 8 / B.n_t);
+    const int gx = (int)std::max<int64_t>(1, std::min<int64_t>(per_sm, want));
+    void* args[] = {(void*)&B};
+    if (cudaLaunchKernel(amax_kernel(MAXT > 1), dim3(gx, B.n_t), dim3(kThreads), args, 0, s) !=
+        cudaSuccess)
+        return QUASAR_ERR_CUDA;
+    return QUASAR_OK;
+}
+
+template <int MAXT>
+quasar_status nvfp4_run(Nvfp4Launch<MAXT>& Lp, AmaxBatch<MAXT>& B, int n_clip, cudaStream_t s)
+{
+    // scale slots of tensors whose amax is computed start at 0
+    for (int i = 0; i < B.n_t; ++i)
+        if (!B.t[i].amax_in &&
+            cudaMemsetAsync(B.t[i].slot, 0, sizeof(float), s) != cudaSuccess)
+            return QUASAR_ERR_CUDA;
+    quasar_status st = launch_amax(B, s);
+    if (st != QUASAR_OK) return st;
+    {
+        void* args[] = {(void*)&B};
+        if (cudaLaunchKernel(amax_to_scale_kernel(MAXT > 1), dim3(1), dim3(256), args, 0, s) !=
+            cudaSuccess)
+            return QUASAR_ERR_CUDA;
+    }
+    int64_t units = 0;
+    for (int i = 0; i < Lp.n_t; ++i) {
+        Lp.t[i].unit0 = units;
+        units += (Lp.t[i].n_blocks + kBlocksPerUnit - 1) / kBlocksPerUnit;
+    }
+    Lp.n_units = units;
+    if (units == 0) return QUASAR_OK;
+    const int gbytes = Lp.p.g_kind == 2 ? 2 : (Lp.p.g_kind == 1 ? 4 : 0);
+    const Launch L = plan((uint32_t)(kBlocksPerUnit * 16 * (8 + gbytes)), 0);
+    Lp.p.stages = L.stages;
+    Lp.p.stage_bytes = L.stage_bytes;
+    const void* fn = nvfp4_kernel(nch_for(n_clip), MAXT > 1);
+    if (!fn) return QUASAR_ERR_UNSUPPORTED;
+    return launch_persistent(fn, &Lp, L.smem, units, s);
+}
+
 }  // namespace
 
 extern "C" {
@@ -413,17 +516,10 @@ quasar_status quasar_tensor_amax(const float* w, int64_t n, float* amax_out, qua
     cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
     if (cudaMemsetAsync(amax_out, 0, sizeof(float), s) != cudaSuccess) return QUASAR_ERR_CUDA;
     if (n == 0) return QUASAR_OK;
-    int dev = 0;
-    const DeviceInfo* info = nullptr;
-    const quasar_status st = device_info(&dev, &info);
-    if (st != QUASAR_OK) return st;
-    const int64_t want = (n / 4 + kThreads - 1) / kThreads;
-    const int grid = (int)std::max<int64_t>(1, std::min<int64_t>((int64_t)info->nsm * 8, want));
-    unsigned int* out = reinterpret_cast<unsigned int*>(amax_out);
-    void* args[] = {(void*)&w, (void*)&n, (void*)&out};
-    if (cudaLaunchKernel(amax_kernel(), dim3(grid), dim3(kThreads), args, 0, s) != cudaSuccess)
-        return QUASAR_ERR_CUDA;
-    return QUASAR_OK;
+    AmaxBatch<1> B;
+    B.n_t = 1;
+    B.t[0] = AmaxItem{w, n, amax_out, nullptr};
+    return launch_amax(B, s);
 }
 
 quasar_status quasar_recon_nvfp4(const float* w, const void* g, quasar_dtype g_dtype, float* v,
@@ -432,79 +528,56 @@ quasar_status quasar_recon_nvfp4(const float* w, const void* g, quasar_dtype g_d
                                  quasar_dtype r_dtype, uint8_t* codes, uint8_t* block_scale,
                                  float* tensor_scale, uint8_t* cand_idx, quasar_stream_t stream)
 {
-    int64_t n = 0;
-    quasar_status st = check_common(w, g, g_dtype, v, beta2, clip, n_clip, rows, cols, r, r_dtype, &n);
+    Nvfp4Launch<1> Lp;
+    AmaxBatch<1> B;
+    quasar_status st = nvfp4_tensor(w, g, g_dtype, v, beta2, clip, n_clip, rows, cols, tensor_amax, r,
+                                    r_dtype, codes, block_scale, tensor_scale, cand_idx, &Lp.t[0],
+                                    &B.t[0]);
     if (st != QUASAR_OK) return st;
-    if (cols % 16 != 0) return QUASAR_ERR_INVALID_ARG;
-    if (!tensor_scale || (reinterpret_cast<uintptr_t>(tensor_scale) & 3u) != 0)
-        return QUASAR_ERR_INVALID_ARG;
-    if (tensor_amax && (reinterpret_cast<uintptr_t>(tensor_amax) & 3u) != 0)
-        return QUASAR_ERR_INVALID_ARG;
-    const int64_t n_blocks = n / 16;
-    if (n > 0) {
-        if (!block_scale) return QUASAR_ERR_INVALID_ARG;
-        if (codes && !aligned16(codes)) return QUASAR_ERR_INVALID_ARG;
-        const void* outs[] = {r, codes, block_scale, tensor_scale, cand_idx};
-        const size_t bytes[] = {(size_t)n * dtype_size(r_dtype), codes ? (size_t)n : 0,
-                                (size_t)n_blocks, 4, cand_idx ? (size_t)n_blocks : 0};
-        if (outputs_alias_inputs(w, g, g_dtype, v, n, outs, bytes, 5)) return QUASAR_ERR_INVALID_ARG;
-        if (tensor_amax && overlaps(tensor_amax, 4, tensor_scale, 4)) return QUASAR_ERR_INVALID_ARG;
-    }
-    cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
-    if (n == 0) {
-        // empty tensor: amax = 0, so s_T = 1
-        if (cudaMemsetAsync(tensor_scale, 0, sizeof(float), s) != cudaSuccess) return QUASAR_ERR_CUDA;
-        void* args[] = {(void*)&tensor_scale};
-        if (cudaLaunchKernel(amax_to_scale_kernel(), dim3(1), dim3(1), args, 0, s) != cudaSuccess)
-            return QUASAR_ERR_CUDA;
-        return QUASAR_OK;
-    }
+    Lp.n_t = B.n_t = 1;
+    if ((st = nvfp4_params(g != nullptr, g_dtype, beta2, clip, n_clip, r_dtype, &Lp.p)) != QUASAR_OK)
+        return st;
+    return nvfp4_run(Lp, B, n_clip, reinterpret_cast<cudaStream_t>(stream));
+}
 
-    Nvfp4Params p{};
-    p.w = w;
-    p.g = g;
-    p.v = v;
-    p.r = r;
-    p.codes = codes;
-    p.scale = block_scale;
-    p.idx = cand_idx;
-    p.tensor_scale = tensor_scale;
-    p.n_blocks = n_blocks;
-    p.g_kind = g_kind_of(g, g_dtype);
-    p.r_bf16 = r_dtype == QUASAR_BF16;
-    p.n_clip = n_clip;
-    p.beta2 = beta2;
-    p.c1 = 1.0f - beta2;
-    p.tie_kappa = tuning().tie_kappa;
-    p.timeout_ns = kDefaultTimeoutNs;
-    p.force_timeout_ns = (uint64_t)std::max<int64_t>(0, g_force_timeout_ns.load());
-    p.stats = g_stats.load();
-    fill_clip(clip, n_clip, p.f, p.invf);
-    if ((st = status_ptr(&p.status)) != QUASAR_OK) return st;
-
-    if (tensor_amax) {
-        p.amax = tensor_amax;
-        p.write_scale = 1;
-    } else {
-        // amax is accumulated in the tensor_scale slot, then converted.
-        if ((st = quasar_tensor_amax(w, n, tensor_scale, stream)) != QUASAR_OK) return st;
-        p.amax = tensor_scale;
-        p.write_scale = 0;
+quasar_status quasar_recon_nvfp4_batch(const quasar_nvfp4_tensor* tensors, int n_tensors,
+                                       quasar_dtype g_dtype, float beta2, const float* clip,
+                                       int n_clip, quasar_dtype r_dtype, quasar_stream_t stream)
+{
+    if (n_tensors < 0 || (n_tensors > 0 && !tensors)) return QUASAR_ERR_INVALID_ARG;
+    if (n_tensors == 0) return QUASAR_OK;
+    int with_g = 0, non_empty = 0;
+    for (int i = 0; i < n_tensors; ++i)
+        if (tensors[i].rows != 0 && tensors[i].cols != 0) {
+            ++non_empty;
+            with_g += tensors[i].g != nullptr;
+        }
+    if (with_g != 0 && with_g != non_empty) return QUASAR_ERR_INVALID_ARG;
+    const bool has_g = with_g != 0;
+    static thread_local Nvfp4Launch<kMaxBatch> Lp;  // kept off the stack
+    static thread_local AmaxBatch<kMaxBatch> B;
+    quasar_status st;
+    for (int i = 0; i < n_tensors; ++i) {  // validate everything first
+        const quasar_nvfp4_tensor& x = tensors[i];
+        Nvfp4Tensor T;
+        AmaxItem A;
+        if ((st = nvfp4_tensor(x.w, x.g, g_dtype, x.v, beta2, clip, n_clip, x.rows, x.cols,
+                               x.tensor_amax, x.r, r_dtype, x.codes, x.block_scale, x.tensor_scale,
+                               x.cand_idx, &T, &A)) != QUASAR_OK)
+            return st;
     }
-
-    const int gbytes = p.g_kind == 2 ? 2 : (p.g_kind == 1 ? 4 : 0);
-    const int nch = nch_for(n_clip);
-    const Launch L = plan((uint32_t)(kBlocksPerUnit * 16 * (8 + gbytes)), 0);
-    p.stages = L.stages;
-    p.stage_bytes = L.stage_bytes;
-    const void* fn = nvfp4_kernel(nch);
-    if (!fn) return QUASAR_ERR_UNSUPPORTED;
-    const int64_t n_units = (n_blocks + kBlocksPerUnit - 1) / kBlocksPerUnit;
-    if ((st = launch_persistent(fn, &p, L.smem, n_units, s)) != QUASAR_OK) return st;
-    if (!tensor_amax) {
-        void* args[] = {(void*)&tensor_scale};
-        if (cudaLaunchKernel(amax_to_scale_kernel(), dim3(1), dim3(1), args, 0, s) != cudaSuccess)
-            return QUASAR_ERR_CUDA;
+    if ((st = nvfp4_params(has_g, g_dtype, beta2, clip, n_clip, r_dtype, &Lp.p)) != QUASAR_OK)
+        return st;
+    const cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+    for (int i0 = 0; i0 < n_tensors; i0 += kMaxBatch) {
+        Lp.n_t = B.n_t = std::min(kMaxBatch, n_tensors - i0);
+        for (int i = 0; i < Lp.n_t; ++i) {
+            const quasar_nvfp4_tensor& x = tensors[i0 + i];
+            nvfp4_tensor(x.w, x.g, g_dtype, x.v, beta2, clip, n_clip, x.rows, x.cols, x.tensor_amax,
+                         x.r, r_dtype, x.codes, x.block_scale, x.tensor_scale, x.cand_idx, &Lp.t[i],
+                         &B.t[i]);
+        }
+        if ((st = nvfp4_run(Lp, B, n_clip, s)) != QUASAR_OK) return st;
     }
     return QUASAR_OK;
 }

@@ -73,9 +73,10 @@ __device__ __forceinline__ void two_prod_f(float a, float b, float& p, float& e)
     e = fmaf(a, b, -p);
 }
 
-template <int NCH>
-__global__ void __launch_bounds__(256) k_recon_nvfp4(const Nvfp4Params p)
+template <int NCH, int MAXT>
+__global__ void __launch_bounds__(256) k_recon_nvfp4(const __grid_constant__ Nvfp4Launch<MAXT> Lp)
 {
+    const Nvfp4Params& p = Lp.p;
     constexpr int KM = NCH * 8;
     constexpr int UNIT = kBlocksPerUnit * 16;
     extern __shared__ __align__(128) unsigned char smem[];
@@ -91,14 +92,17 @@ __global__ void __launch_bounds__(256) k_recon_nvfp4(const Nvfp4Params p)
     constexpr uint32_t kVOff = UNIT * 4;
     constexpr uint32_t kGOff = UNIT * 8;
 
-    const int64_t n_units = (p.n_blocks + kBlocksPerUnit - 1) / kBlocksPerUnit;
+    const int64_t n_units = Lp.n_units;
+    // the tensor of a unit (units numbered consecutively across tensors,
+    // met by each warp in increasing order)
+    auto tensor_of = [&](int64_t u, int& ti) {
+        while (ti + 1 < Lp.n_t && u >= Lp.t[ti + 1].unit0) ++ti;
+    };
+    int ti = 0, ti_s = -1;
+    float sT = 1.0f, inv_sT = 1.0f;
     const int64_t first = (int64_t)blockIdx.x * nwarps + warp;
     const int64_t stride = (int64_t)gridDim.x * nwarps;
 
-    const float amax_t = *p.amax;
-    const float sT = tensor_scale_of(amax_t);
-    const float inv_sT = 1.0f / sT;
-    if (p.write_scale && blockIdx.x == 0 && threadIdx.x == 0) *p.tensor_scale = sT;
 
     if (lane == 0) {
         for (int s = 0; s <= S; ++s) mbar_init(&bars[s], 1);
@@ -107,15 +111,18 @@ __global__ void __launch_bounds__(256) k_recon_nvfp4(const Nvfp4Params p)
     __syncwarp();
 
     auto issue = [&](int64_t u, int s) {
-        const int64_t b0 = u * kBlocksPerUnit;
-        const int64_t nb = min((int64_t)kBlocksPerUnit, p.n_blocks - b0);
+        int tj = ti;
+        tensor_of(u, tj);
+        const Nvfp4Tensor& T = Lp.t[tj];
+        const int64_t b0 = (u - T.unit0) * kBlocksPerUnit;
+        const int64_t nb = min((int64_t)kBlocksPerUnit, T.n_blocks - b0);
         const uint32_t elems = (uint32_t)(nb * 16);
         unsigned char* st = ring + (size_t)s * p.stage_bytes;
         mbar_arrive_expect_tx(&bars[s], elems * (8u + (uint32_t)gbytes));
-        bulk_g2s(st, p.w + b0 * 16, elems * 4u, &bars[s]);
-        bulk_g2s(st + kVOff, p.v + b0 * 16, elems * 4u, &bars[s]);
+        bulk_g2s(st, T.w + b0 * 16, elems * 4u, &bars[s]);
+        bulk_g2s(st + kVOff, T.v + b0 * 16, elems * 4u, &bars[s]);
         if (gbytes)
-            bulk_g2s(st + kGOff, static_cast<const unsigned char*>(p.g) + b0 * 16 * gbytes,
+            bulk_g2s(st + kGOff, static_cast<const unsigned char*>(T.g) + b0 * 16 * gbytes,
                      elems * (uint32_t)gbytes, &bars[s]);
     };
     auto fail = [&](int64_t it) {
@@ -206,15 +213,22 @@ __global__ void __launch_bounds__(256) k_recon_nvfp4(const Nvfp4Params p)
             parity ^= 1u;
         }
 
-        const int64_t blk = u * kBlocksPerUnit + lane;
-        const bool valid = blk < p.n_blocks;
+        tensor_of(u, ti);
+        const Nvfp4Tensor& T = Lp.t[ti];
+        if (ti != ti_s) {  // a new tensor: its scale s_T
+            ti_s = ti;
+            sT = *T.tensor_scale;
+            inv_sT = 1.0f / sT;
+        }
+        const int64_t blk = (u - T.unit0) * kBlocksPerUnit + lane;
+        const bool valid = blk < T.n_blocks;
         const int64_t ebase = blk * 16;
 
         if (valid && p.g_kind) {
 #pragma unroll
             for (int i = 0; i < 4; ++i) {
                 const int cidx = (i + rot) & 3;
-                stg_cs(reinterpret_cast<float4*>(p.v + ebase + cidx * 4),
+                stg_cs(reinterpret_cast<float4*>(T.v + ebase + cidx * 4),
                        make_float4(h2[2 * i].x, h2[2 * i].y, h2[2 * i + 1].x, h2[2 * i + 1].y));
             }
         }
@@ -382,27 +396,34 @@ __global__ void __launch_bounds__(256) k_recon_nvfp4(const Nvfp4Params p)
                 const float2 qs = make_float2(q.x > 0.0f ? copysignf(q.x, w2[t].x) : 0.0f,
                                               q.y > 0.0f ? copysignf(q.y, w2[t].y) : 0.0f);
                 rv[hh] = __fmul2_rn(as2, qs);
-                if (p.codes) cw |= (e2m1_nibble(qs.x) | (e2m1_nibble(qs.y) << 8)) << (16 * hh);
+                if (T.codes) cw |= (e2m1_nibble(qs.x) | (e2m1_nibble(qs.y) << 8)) << (16 * hh);
             }
             const int64_t e = ebase + cidx * 4;
             if (p.r_bf16) {
-                stg_cs(reinterpret_cast<uint2*>(static_cast<__nv_bfloat16*>(p.r) + e),
+                stg_cs(reinterpret_cast<uint2*>(static_cast<__nv_bfloat16*>(T.r) + e),
                        make_uint2(pack_bf16x2(rv[0].x, rv[0].y), pack_bf16x2(rv[1].x, rv[1].y)));
             } else {
-                stg_cs(reinterpret_cast<float4*>(static_cast<float*>(p.r) + e),
+                stg_cs(reinterpret_cast<float4*>(static_cast<float*>(T.r) + e),
                        make_float4(rv[0].x, rv[0].y, rv[1].x, rv[1].y));
             }
-            if (p.codes) stg_cs(reinterpret_cast<uint32_t*>(p.codes + e), cw);
+            if (T.codes) stg_cs(reinterpret_cast<uint32_t*>(T.codes + e), cw);
         }
-        p.scale[blk] = (uint8_t)e_sel;
-        if (p.idx) p.idx[blk] = (uint8_t)kb;
+        T.scale[blk] = (uint8_t)e_sel;
+        if (T.idx) T.idx[blk] = (uint8_t)kb;
     }
 }
 
-// max |w| over n elements, accumulated into *out (which must start at 0) as
-// the bit pattern of a non-negative float (such patterns order like uints).
-__global__ void __launch_bounds__(256) k_amax(const float* __restrict__ w, int64_t n, unsigned int* out)
+// Tensor absmax of a batch: blockIdx.y picks the tensor; max |w| over its n
+// elements is accumulated into *slot (which must start at 0) as the bit
+// pattern of a non-negative float (such patterns order like uints).
+// Tensors whose amax is supplied are skipped.
+template <int MAXT>
+__global__ void __launch_bounds__(256) k_amax(const __grid_constant__ AmaxBatch<MAXT> B)
 {
+    const AmaxItem& it = B.t[blockIdx.y];
+    if (it.amax_in || it.n == 0) return;
+    const float* w = it.w;
+    const int64_t n = it.n;
     float m = 0.0f;
     const int64_t n4 = n / 4;
     const float4* w4 = reinterpret_cast<const float4*>(w);
@@ -423,14 +444,20 @@ __global__ void __launch_bounds__(256) k_amax(const float* __restrict__ w, int64
         m = threadIdx.x < (blockDim.x >> 5) ? red[threadIdx.x] : 0.0f;
 #pragma unroll
         for (int o = 16; o; o >>= 1) m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, o));
-        if (threadIdx.x == 0) atomicMax(out, __float_as_uint(m));
+        if (threadIdx.x == 0 && m > 0.0f)
+            atomicMax(reinterpret_cast<unsigned int*>(it.slot), __float_as_uint(m));
     }
 }
 
-// tensor_scale[0] := s_T of the amax it holds.
-__global__ void k_amax_to_scale(float* tensor_scale)
+// *slot := s_T of the supplied amax, or of the amax the slot holds.
+template <int MAXT>
+__global__ void k_amax_to_scale(const __grid_constant__ AmaxBatch<MAXT> B)
 {
-    *tensor_scale = tensor_scale_of(*tensor_scale);
+    for (int i = threadIdx.x; i < B.n_t; i += blockDim.x) {
+        const AmaxItem& it = B.t[i];
+        const float amax = it.amax_in ? *it.amax_in : *it.slot;
+        *it.slot = tensor_scale_of(amax);
+    }
 }
 
 }  // namespace quasar

@@ -43,6 +43,7 @@ PROTOTYPES = {
     "quasar_recon_nvfp4": (_I, [_P, _P, _I, _P, _F, _P, _I, _I64, _I64, _P, _P, _I, _P, _P, _P,
                                 _P, _P]),
     "quasar_recon_int_batch": (_I, [_P, _I, _I, _F, _I, _I, _P, _I, _I, _P]),
+    "quasar_recon_nvfp4_batch": (_I, [_P, _I, _I, _F, _P, _I, _I, _P]),
     "quasar_tensor_amax": (_I, [_P, _I64, _P, _P]),
     "quasar_get_device_status": (_I, [_P]),
     "quasar_debug_force_timeout": (None, [_I64]),
@@ -156,6 +157,39 @@ def quasar_recon_int_batch(tensors, beta2, bits, group_size, clip, g_dtype=BF16,
     carr, nclip = _clip_array(clip)
     st = lib.quasar_recon_int_batch(ctypes.cast(tensors, ctypes.c_void_p), len(tensors), g_dtype,
                                     beta2, bits, group_size, carr, nclip, r_dtype, _stream(stream))
+    return QuasarStatus(st)
+
+
+class QuasarNvfp4Tensor(ctypes.Structure):
+    """quasar_nvfp4_tensor: one tensor's buffers (device pointers) and shape."""
+    _fields_ = [("w", ctypes.c_void_p), ("g", ctypes.c_void_p), ("v", ctypes.c_void_p),
+                ("tensor_amax", ctypes.c_void_p), ("r", ctypes.c_void_p),
+                ("codes", ctypes.c_void_p), ("block_scale", ctypes.c_void_p),
+                ("tensor_scale", ctypes.c_void_p), ("cand_idx", ctypes.c_void_p),
+                ("rows", ctypes.c_int64), ("cols", ctypes.c_int64)]
+
+
+def nvfp4_tensor_array(items):
+    """A ctypes array of QuasarNvfp4Tensor from dicts with keys w, g, v,
+    tensor_amax, r, codes, block_scale, tensor_scale, cand_idx, rows, cols."""
+    arr = (QuasarNvfp4Tensor * len(items))()
+    for i, d in enumerate(items):
+        arr[i] = QuasarNvfp4Tensor(_ptr(d["w"]), _ptr(d.get("g")), _ptr(d["v"]),
+                                   _ptr(d.get("tensor_amax")), _ptr(d["r"]), _ptr(d.get("codes")),
+                                   _ptr(d["block_scale"]), _ptr(d["tensor_scale"]),
+                                   _ptr(d.get("cand_idx")), int(d["rows"]), int(d["cols"]))
+    return arr
+
+
+def quasar_recon_nvfp4_batch(tensors, beta2, clip, g_dtype=BF16, r_dtype=BF16,
+                             stream=None) -> QuasarStatus:
+    """tensors: a ctypes array from nvfp4_tensor_array (or a list of dicts)."""
+    lib = load()
+    if not isinstance(tensors, ctypes.Array):
+        tensors = nvfp4_tensor_array(tensors)
+    carr, nclip = _clip_array(clip)
+    st = lib.quasar_recon_nvfp4_batch(ctypes.cast(tensors, ctypes.c_void_p), len(tensors), g_dtype,
+                                      beta2, carr, nclip, r_dtype, _stream(stream))
     return QuasarStatus(st)
 
 

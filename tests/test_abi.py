@@ -147,3 +147,21 @@ def test_int_batch_argument_validation(lib):
     assert call([_desc()], group_size=48) == st.ERR_UNSUPPORTED
     n = ctypes.c_void_p(None)
     assert Q.load().quasar_recon_int_batch(n, 2, Q.BF16, 0.999, 3, 128, None, 0, Q.BF16, None) == st.ERR_INVALID_ARG
+
+
+def _ndesc(**kw):
+    d = dict(w=A, g=B, v=C, tensor_amax=None, r=D, codes=None, block_scale=E, tensor_scale=F,
+             cand_idx=None, rows=4, cols=256)
+    d.update(kw)
+    return d
+
+
+def test_nvfp4_batch_argument_validation(lib):
+    st = Q.QuasarStatus
+    call = lambda items: Q.quasar_recon_nvfp4_batch(items, 0.999, CLIP, stream=0)
+    assert call([]) == st.OK
+    assert call([_ndesc(), _ndesc(g=None)]) == st.ERR_INVALID_ARG      # mixed gradients
+    assert call([_ndesc(), _ndesc(block_scale=None)]) == st.ERR_INVALID_ARG
+    assert call([_ndesc(), _ndesc(cols=40)]) == st.ERR_INVALID_ARG     # cols % 16
+    assert call([_ndesc(), _ndesc(tensor_scale=None)]) == st.ERR_INVALID_ARG
+    assert call([_ndesc(), _ndesc(r=C)]) == st.ERR_INVALID_ARG         # output aliases v

@@ -192,3 +192,42 @@ def test_int_batch_matches_oracle_and_single_calls(oracle):
         rep = checker.check_int(oracle, w_h[i], h, 3, clip, O, gpu, 128, True)
         ema = checker.check_ema(h, H._host(items[i][2]))
         _assert(rep, ema)
+
+
+def test_nvfp4_batch_matches_oracle_and_single_calls(oracle):
+    """One absmax pass, one scale pass and one reconstruction launch over
+    tensors of different shapes (one with its amax supplied, a tiny one, an
+    empty one) give, tensor by tensor, the oracle's result and bit-for-bit
+    the single-call result."""
+    from paper_2608_13966_gb300 import api
+    shapes = [(48, 512), (3, 48), (0, 64), (37, 528), (1, 16), (64, 1024)]
+    items, copies = [], []
+    for i, (rows, cols) in enumerate(shapes):
+        w, g, v = _inputs(max(rows, 1), cols, seed=400 + i)
+        w, g, v = w[:rows].contiguous(), g[:rows].contiguous(), v[:rows].contiguous()
+        amax = w.abs().max().reshape(1).float() if (i == 3 and rows) else None
+        items.append((w, g, v, amax))
+        copies.append((w.clone(), g.clone(), v.clone(), amax))
+    clip = list(wl.CLIP_8)
+    hosts = [(H._host(w), H._host(g), H._host(v)) for w, g, v, _ in items]
+    outs = api.recon_nvfp4_batch(items, clip=clip, codes=True)
+    singles = [api.recon_nvfp4(w, g, v, clip=clip, tensor_amax=amax, codes=True)
+               for (w, g, v, amax) in copies]
+    torch.cuda.synchronize()
+    for i, (o, s1) in enumerate(zip(outs, singles)):
+        for key in ("r", "block_scale", "tensor_scale", "codes", "cand_idx"):
+            assert torch.equal(o[key], s1[key]), (shapes[i], key)
+        assert torch.equal(items[i][2], copies[i][2])  # v' identical
+        w_h, g_h, v_h = hosts[i]
+        if w_h.size == 0:
+            assert float(o["tensor_scale"].cpu()[0]) == 1.0
+            continue
+        h = oracle.ema(v_h, g_h, 0.999)
+        _, s_T = oracle.tensor_scale(w_h)
+        O = oracle.recon_nvfp4(w_h, h, s_T, clip)
+        gpu = {"r": H._host(o["r"]), "scale": o["block_scale"].cpu().numpy(),
+               "tensor_scale": float(o["tensor_scale"].cpu()[0]),
+               "codes": o["codes"].cpu().numpy().ravel(), "idx": o["cand_idx"].cpu().numpy()}
+        rep = checker.check_nvfp4(oracle, w_h, h, clip, s_T, O, gpu, True)
+        ema = checker.check_ema(h, H._host(items[i][2]))
+        _assert(rep, ema)
