@@ -48,6 +48,8 @@ def _load():
         i64, i32, f32, f64 = ctypes.c_int64, ctypes.c_int, ctypes.c_float, ctypes.c_double
         lib.qo_ema.argtypes = [P, P, i64, f32, P]
         lib.qo_ema.restype = None
+        lib.qo_adamw.argtypes = [P, P, P, P, i64, f64, f64, f64, f64, f64, i64, P, P, P]
+        lib.qo_adamw.restype = None
         lib.qo_recon_int.argtypes = [P, P, i64, i32, i32, P, i32] + [P] * 11
         lib.qo_recon_int.restype = i32
         lib.qo_refit_int.argtypes = [P, P, P, i32, i32, f32, P, P]
@@ -101,6 +103,21 @@ def ema(v, g, beta2: float) -> np.ndarray:
     out = np.empty_like(v)
     _load().qo_ema(_ptr(v), _ptr(gg), v.size, ctypes.c_float(beta2), _ptr(out))
     return out
+
+
+def adamw(w, g, m, v, *, lr: float, beta1: float, beta2: float, eps: float, weight_decay: float,
+          step: int):
+    """One AdamW step in fp64 (stored state rounded to fp32): returns
+    (w', m', v') as fp32 arrays."""
+    w = _c(w, np.float32).ravel()
+    g = _c(g, np.float32).ravel()
+    m = _c(m, np.float32).ravel()
+    v = _c(v, np.float32).ravel()
+    wo, mo, vo = np.empty_like(w), np.empty_like(w), np.empty_like(w)
+    _load().qo_adamw(_ptr(w), _ptr(g), _ptr(m), _ptr(v), w.size, float(lr), float(beta1),
+                     float(beta2), float(eps), float(weight_decay), int(step), _ptr(wo), _ptr(mo),
+                     _ptr(vo))
+    return wo, mo, vo
 
 
 def recon_int(w, h, group_size: int, bits: int, clip) -> dict:

@@ -9,6 +9,8 @@
  * What it computes (paper: "QUASAR: Lowering the Loss Floor of
  * Quantization-Aware Training with Loss-Aware Reconstruction"):
  *
+ *   qo_adamw        one AdamW step whose second moment is the saliency
+ *                   (the step fused with the reconstruction on the GPU).
  *   qo_ema          saliency EMA of squared gradients (Sec. 4.1.1: the Adam
  *                   second moment as diagonal-Fisher saliency; App. A.2: an
  *                   explicitly kept EMA of squared gradients).
@@ -97,6 +99,30 @@ void qo_ema(const float* v, const float* g, int64_t n, float beta2, float* v_out
         } else {
             v_out[i] = v[i];
         }
+    }
+}
+
+/* One AdamW step (the optimizer whose second moment is the saliency, Sec.
+ * 4.1.1), decoupled weight decay, bias-corrected moments, t >= 1:
+ *   m' = beta1 m + (1-beta1) g,   v' = beta2 v + (1-beta2) g^2,
+ *   w' = w (1 - lr wd) - lr (m'/(1-beta1^t)) / (sqrt(v'/(1-beta2^t)) + eps).
+ * Evaluated in fp64 from the fp32 inputs; the stored m', v' are rounded to
+ * fp32 first, and w' is computed from those stored values (the state the next
+ * step reads).  Outputs may alias the inputs. */
+void qo_adamw(const float* w, const float* g, const float* m, const float* v, int64_t n,
+              double lr, double beta1, double beta2, double eps, double wd, int64_t step,
+              float* w_out, float* m_out, float* v_out)
+{
+    const double bc1 = 1.0 - pow(beta1, (double)step);
+    const double bc2 = 1.0 - pow(beta2, (double)step);
+    for (int64_t i = 0; i < n; ++i) {
+        const double gi = (double)g[i];
+        const float mi = (float)(beta1 * (double)m[i] + (1.0 - beta1) * gi);
+        const float vi = (float)(beta2 * (double)v[i] + (1.0 - beta2) * gi * gi);
+        const double denom = sqrt((double)vi / bc2) + eps;
+        w_out[i] = (float)((double)w[i] * (1.0 - lr * wd) - lr * ((double)mi / bc1) / denom);
+        m_out[i] = mi;
+        v_out[i] = vi;
     }
 }
 

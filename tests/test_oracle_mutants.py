@@ -50,6 +50,9 @@ MUTANTS = {
                                    "margin[i] = fabs(t - (j + 0.5));"),
     "E2M1 ties to odd": ("if (d < bd || (d == bd && (m % 2) == 0)) {",
                          "if (d < bd || (d == bd && (m % 2) == 1)) {"),
+    "AdamW without bias correction": ("lr * ((double)mi / bc1) / denom", "lr * (double)mi / denom"),
+    "AdamW coupled weight decay": ("(double)w[i] * (1.0 - lr * wd) - lr", "(double)w[i] - lr * wd - lr"),
+    "AdamW eps inside the root": ("sqrt((double)vi / bc2) + eps", "sqrt((double)vi / bc2 + eps)"),
 }
 
 PIN_TESTS = [
@@ -64,6 +67,8 @@ PIN_TESTS = [
     (pins.test_e4m3_values_match_torch, {}),
     (pins.test_e2m1_grid_from_format, {}),
     (pins.test_nvfp4_fit_and_scale_are_optimal, {}),
+    (pins.test_adamw_matches_torch_optimizer, {}),
+    (pins.test_adamw_first_step_closed_form, {}),
 ]
 
 
@@ -85,7 +90,7 @@ def test_pins_catch_planted_mistake(oracle, tmp_path, name):
     real = oracle_mod._load()
     lib = ctypes.CDLL(so)
     # give the mutant the same prototypes as the real library
-    for sym in ("qo_ema", "qo_recon_int", "qo_refit_int", "qo_codes_int", "qo_tensor_scale",
+    for sym in ("qo_ema", "qo_adamw", "qo_recon_int", "qo_refit_int", "qo_codes_int", "qo_tensor_scale",
                 "qo_recon_nvfp4", "qo_e2m1_round", "qo_e4m3_round", "qo_e4m3_value",
                 "qo_set_threads", "qo_get_threads"):
         f_real, f_mut = getattr(real, sym), getattr(lib, sym)

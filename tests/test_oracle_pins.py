@@ -485,3 +485,69 @@ def test_heavy_tailed_groups_mostly_clip(oracle):
     assert np.mean(o["idx"] > 0) > 0.6
     base = np.array([_minmax_error(w[g], h[g], 3) for g in range(512)])
     assert np.sum(o["err"]) < 0.9 * np.sum(base)
+
+
+# ---------------------------------------------------------------- AdamW step
+
+def test_adamw_matches_torch_optimizer(oracle):
+    """One AdamW step from a given state equals torch.optim.AdamW's (float64,
+    single-tensor implementation) up to the fp32 rounding of the stored
+    moments, over several step counts and hyperparameters."""
+    import torch
+    rng = np.random.default_rng(11)
+    for step, lr, b1, b2, eps, wd in [(1, 1e-3, 0.9, 0.999, 1e-8, 0.01), (7, 3e-4, 0.8, 0.99, 1e-6, 0.1),
+                                      (1000, 1e-2, 0.95, 0.999, 1e-8, 0.0)]:
+        n = 4096
+        w = (0.02 * rng.standard_normal(n)).astype(np.float32)
+        g = (1e-3 * rng.standard_normal(n)).astype(np.float32)
+        m = (1e-4 * rng.standard_normal(n)).astype(np.float32)
+        v = np.exp(-14.0 + 2.0 * rng.standard_normal(n)).astype(np.float32)
+        wo, mo, vo = oracle.adamw(w, g, m, v, lr=lr, beta1=b1, beta2=b2, eps=eps, weight_decay=wd,
+                                  step=step)
+        p = torch.nn.Parameter(torch.tensor(w, dtype=torch.float64))
+        opt = torch.optim.AdamW([p], lr=lr, betas=(b1, b2), eps=eps, weight_decay=wd,
+                                foreach=False, fused=False)
+        opt.state[p] = {"step": torch.tensor(float(step - 1)),
+                        "exp_avg": torch.tensor(m, dtype=torch.float64),
+                        "exp_avg_sq": torch.tensor(v, dtype=torch.float64)}
+        p.grad = torch.tensor(g, dtype=torch.float64)
+        opt.step()
+        st = opt.state[p]
+        np.testing.assert_allclose(mo, st["exp_avg"].numpy(), rtol=1e-6, atol=1e-12)
+        np.testing.assert_allclose(vo, st["exp_avg_sq"].numpy(), rtol=1e-6, atol=1e-20)
+        # w' to within one fp32 ulp of the fp64 result, plus the update's own
+        # relative change from the moments being stored in fp32 first
+        ref = p.detach().numpy()
+        tol = np.spacing(np.abs(ref).astype(np.float32)) * 1.01 + 2e-7 * np.abs(w - ref)
+        np.testing.assert_array_less(np.abs(wo - ref), tol)
+
+
+def test_adamw_first_step_closed_form(oracle):
+    """From zero moments at t = 1 the bias corrections give m^ = g and v^ = g^2:
+    w' = w (1 - lr wd) - lr g / (|g| + eps)."""
+    rng = np.random.default_rng(12)
+    n = 1000
+    w = rng.standard_normal(n).astype(np.float32)
+    g = rng.standard_normal(n).astype(np.float32)
+    z = np.zeros(n, np.float32)
+    lr, wd, eps = 1e-2, 0.05, 1e-8
+    wo, mo, vo = oracle.adamw(w, g, z, z, lr=lr, beta1=0.9, beta2=0.999, eps=eps, weight_decay=wd,
+                              step=1)
+    g64 = g.astype(np.float64)
+    expect = w * (1 - lr * wd) - lr * g64 / (np.abs(g64) + eps)
+    np.testing.assert_allclose(wo, expect, rtol=2e-7, atol=1e-9)
+    np.testing.assert_allclose(mo, 0.1 * g64, rtol=1e-6)
+    np.testing.assert_allclose(vo, 0.001 * g64 * g64, rtol=1e-6)
+
+
+def test_adamw_zero_learning_rate_keeps_weights(oracle):
+    rng = np.random.default_rng(13)
+    n = 256
+    w, g, m = (rng.standard_normal(n).astype(np.float32) for _ in range(3))
+    v = np.abs(rng.standard_normal(n)).astype(np.float32)
+    b2 = float(np.float32(0.999))  # the fp32 value the EMA uses
+    wo, mo, vo = oracle.adamw(w, g, m, v, lr=0.0, beta1=0.9, beta2=b2, eps=1e-8,
+                              weight_decay=0.1, step=5)
+    assert np.array_equal(wo, w)
+    # the second moment is the saliency EMA of the reconstruction
+    assert np.array_equal(vo, oracle.ema(v, g, 0.999))
