@@ -7,8 +7,9 @@ the kept candidate -- over every linear weight of a 32-layer
 Llama-3.1-8B-shaped model (224 tensors, 6.98e9 weights, ~84 GB resident:
 fp32 w and v, bf16 g and r), with inputs already resident in HBM.  The
 headline format is INT3 with group 128 and 8 clip candidates; the other
-formats of the sweep (INT2, INT4, NVFP4) are timed after it and reported in
-"sweep".  Each step streams ~70 GB of inputs, far more than the 129 MB L2.
+formats of the sweep (INT2, INT4, NVFP4, and one AdamW step fused with the
+INT3 reconstruction) are timed after it and reported in "sweep".  Each step
+streams ~70 GB of inputs, far more than the 129 MB L2.
 
 Usage: python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
 With N > 1 it runs under torchrun, one rank per GPU; every rank processes the
@@ -81,7 +82,10 @@ def bytes_per_step(wlo, elements):
     """Algorithmic HBM bytes of one step: read w (4) + g (2) + v (4), write
     v (4) + r (2) per weight; per group a, b (fp32) and the kept index (u8)
     for integer codes; per 16-block the E4M3 scale and index for NVFP4, plus
-    the tensor-absmax pre-pass (one more read of w)."""
+    the tensor-absmax pre-pass (one more read of w).  The fused AdamW step
+    also reads m and writes w' and m' (12 more bytes a weight)."""
+    if wlo.fmt == "int" and wlo.adamw:
+        return elements * 28 + (elements // wlo.group) * 9
     if wlo.fmt == "int":
         return elements * 16 + (elements // wlo.group) * 9
     return elements * 16 + (elements // 16) * 2 + elements * 4
@@ -94,6 +98,7 @@ class Model:
         """``shard``: the rank's shard of a weak-scaled job -- every rank holds
         a full model's worth of distinct tensors (seed = shard)."""
         self.wlo = wlo
+        self.seed = shard
         self.tensors = []
         for spec in wlo.tensors:
             d = WL.make_tensor(wlo, spec, device=device, seed=shard)
@@ -119,7 +124,26 @@ class Step:
         self.stream = stream.cuda_stream
         self.clip = (ctypes.c_float * len(wlo.clip))(*wlo.clip)
         self.calls = []
-        if wlo.fmt == "int":
+        if wlo.adamw:
+            # AdamW step + reconstruction of every tensor in one launch
+            # (quasar_adamw_recon_int_batch); m is drawn here if the model
+            # was built for a workload without an optimizer step
+            for d in model.tensors:
+                if "m" not in d:
+                    spec = d["spec"]
+                    d["m"] = WL.first_moment((spec.rows, spec.cols), model.seed * 1000 + spec.index,
+                                             d["w"].device)
+            hp = wlo.adamw
+            self.descs = Q.adamw_tensor_array([
+                {"w": d["w"], "g": d["g"], "m": d["m"], "v": d["v"], "r": d["r"], "codes": None,
+                 "a": d["a"], "b": d["b"], "cand_idx": d["idx"], "rows": d["spec"].rows,
+                 "cols": d["spec"].cols}
+                for d in model.tensors])
+            args = (ctypes.cast(self.descs, ctypes.c_void_p), len(self.descs), Q.BF16, hp["lr"],
+                    hp["beta1"], wlo.beta2, hp["eps"], hp["weight_decay"], hp["step"], wlo.bits,
+                    wlo.group, self.clip, len(wlo.clip), Q.BF16, self.stream)
+            self.calls.append((self.lib.quasar_adamw_recon_int_batch, args, model.elements))
+        elif wlo.fmt == "int":
             # every tensor of the model in one launch (quasar_recon_int_batch)
             self.descs = Q.int_tensor_array([
                 {"w": d["w"], "g": d["g"], "v": d["v"], "r": d["r"], "codes": None, "a": d["a"],
@@ -379,7 +403,7 @@ def main():
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--workload", default="llama_int3")
-    ap.add_argument("--sweep", default="llama_int2,llama_int4,llama_nvfp4")
+    ap.add_argument("--sweep", default="llama_int2,llama_int4,llama_nvfp4,llama_int3_adamw")
     ap.add_argument("--sweep-steps", type=int, default=10)
     ap.add_argument("--e2e-steps", type=int, default=2)
     ap.add_argument("--cpu-budget", type=float, default=12.0)

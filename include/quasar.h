@@ -131,6 +131,52 @@ quasar_status quasar_recon_int_batch(const quasar_int_tensor* tensors, int n_ten
                                      quasar_stream_t stream);
 
 /*
+ * quasar_adamw_tensor / quasar_adamw_recon_int_batch -- one AdamW step fused
+ * with the integer-code reconstruction of the updated weights.  The paper
+ * trains with AdamW and takes AdamW's second moment as the saliency h
+ * (Sec. 4.1.1; training setup in Sec. 5); the reconstruction of Algorithm 1
+ * follows every optimizer step.  Here both run in one pass over the weights:
+ * each element of w, g, m, v is read once and w', m', v', r written once.
+ *
+ * Per element (t = step, decoupled weight decay, bias-corrected moments):
+ *   m' = beta1*m + (1-beta1)*g           written back to m
+ *   v' = beta2*v + (1-beta2)*g^2         written back to v
+ *   w' = w*(1 - lr*wd) - (lr/(1-beta1^t)) * m' / (sqrt(v')/sqrt(1-beta2^t) + eps)
+ *                                        written back to w
+ * then quasar_recon_int of w' with saliency h = v' (steps 2-4 there).
+ * Arithmetic is fp32: m', v' within one rounding of each product, w' the
+ * fp32 sum w + (the decrement), sqrt and division correctly rounded.
+ *
+ * Descriptor fields as in quasar_int_tensor, plus m (fp32 first moment,
+ * [rows, cols], read and overwritten), and w is overwritten with w'.  g is
+ * required for every non-empty tensor.  w, m, v, g must not overlap one
+ * another; the outputs r, codes, a, b, cand_idx must not overlap any of
+ * them.  Hyper-parameters: lr >= 0, 0 <= beta1 < 1, 0 <= beta2 < 1,
+ * eps > 0, weight_decay >= 0 (all finite), step >= 1.
+ * Returns as quasar_recon_int_batch.
+ */
+typedef struct {
+    float* w;
+    const void* g;
+    float* m;
+    float* v;
+    void* r;
+    uint8_t* codes;
+    float* a;
+    float* b;
+    uint8_t* cand_idx;
+    int64_t rows;
+    int64_t cols;
+} quasar_adamw_tensor;
+
+quasar_status quasar_adamw_recon_int_batch(const quasar_adamw_tensor* tensors, int n_tensors,
+                                           quasar_dtype g_dtype, float lr, float beta1,
+                                           float beta2, float eps, float weight_decay,
+                                           int64_t step, int bits, int group_size,
+                                           const float* clip, int n_clip, quasar_dtype r_dtype,
+                                           quasar_stream_t stream);
+
+/*
  * quasar_recon_nvfp4 -- QUASAR for NVFP4 (Sec. 4.2): E2M1 codes, one FP8
  * (E4M3) scale per 16 consecutive elements, one FP32 scale per tensor.
  *

@@ -5,9 +5,10 @@ from __future__ import annotations
 
 import torch
 
-from .quasar import (BF16, F32, QuasarError, QuasarStatus, int_tensor_array, nvfp4_tensor_array,
-                     quasar_recon_int, quasar_recon_int_batch, quasar_recon_nvfp4,
-                     quasar_recon_nvfp4_batch, quasar_tensor_amax)
+from .quasar import (BF16, F32, QuasarError, QuasarStatus, adamw_tensor_array, int_tensor_array,
+                     nvfp4_tensor_array, quasar_adamw_recon_int_batch, quasar_recon_int,
+                     quasar_recon_int_batch, quasar_recon_nvfp4, quasar_recon_nvfp4_batch,
+                     quasar_tensor_amax)
 
 
 def _check(st):
@@ -81,6 +82,42 @@ def recon_int_batch(items, *, bits, group_size, clip, beta2=0.999, r_dtype=torch
     rd = BF16 if r_dtype == torch.bfloat16 else F32
     _check(quasar_recon_int_batch(int_tensor_array(descs), beta2, bits, group_size, clip,
                                   g_dtype=g_dtype, r_dtype=rd, stream=stream))
+    return results
+
+
+def adamw_recon_int_batch(items, *, lr, step, bits, group_size, clip, beta1=0.9, beta2=0.999,
+                          eps=1e-8, weight_decay=0.0, r_dtype=torch.bfloat16, codes=False,
+                          cand_idx=True, stream=None):
+    """One AdamW step fused with the integer reconstruction of the updated
+    weights, over several tensors in one launch.
+
+    items: list of (w, g, m, v) CUDA tensors; w, m and v are updated in
+    place (w', m', v').  Returns one result dict per tensor, as recon_int
+    does."""
+    descs, results = [], []
+    g_dtype = F32
+    for w, g, m, v in items:
+        _check_2d(w)
+        rows, cols = w.shape
+        dev = w.device
+        n_groups = rows * cols // group_size
+        res = {"r": torch.empty((rows, cols), dtype=r_dtype, device=dev),
+               "a": torch.empty(n_groups, dtype=torch.float32, device=dev),
+               "b": torch.empty(n_groups, dtype=torch.float32, device=dev)}
+        if codes:
+            res["codes"] = torch.empty((rows, cols), dtype=torch.uint8, device=dev)
+        if cand_idx:
+            res["cand_idx"] = torch.empty(n_groups, dtype=torch.uint8, device=dev)
+        if g is not None and g.dtype == torch.bfloat16:
+            g_dtype = BF16
+        descs.append({"w": w, "g": g, "m": m, "v": v, "r": res["r"], "codes": res.get("codes"),
+                      "a": res["a"], "b": res["b"], "cand_idx": res.get("cand_idx"),
+                      "rows": rows, "cols": cols})
+        results.append(res)
+    rd = BF16 if r_dtype == torch.bfloat16 else F32
+    _check(quasar_adamw_recon_int_batch(adamw_tensor_array(descs), lr, beta1, beta2, eps,
+                                        weight_decay, step, bits, group_size, clip,
+                                        g_dtype=g_dtype, r_dtype=rd, stream=stream))
     return results
 
 

@@ -12,18 +12,24 @@
 namespace quasar {
 
 // Kernel entry for group size 8*epl, one tensor or a batch of up to
-// kMaxBatch tensors per launch, or nullptr if not built.
-const void* QUASAR_CAT(int_kernel_nch, QUASAR_NCH)(int epl, bool batch)
+// kMaxBatch tensors per launch (the AdamW-fused variant: batches only), or
+// nullptr if not built.
+const void* QUASAR_CAT(int_kernel_nch, QUASAR_NCH)(int epl, bool batch, bool adam)
 {
+    constexpr int C = QUASAR_NCH;
+    constexpr int B = kMaxBatch;
+    if (adam && !batch) return nullptr;
     switch (epl) {
-    case 4: return batch ? reinterpret_cast<const void*>(&k_recon_int<4, QUASAR_NCH, kMaxBatch>)
-                         : reinterpret_cast<const void*>(&k_recon_int<4, QUASAR_NCH, 1>);
-    case 8: return batch ? reinterpret_cast<const void*>(&k_recon_int<8, QUASAR_NCH, kMaxBatch>)
-                         : reinterpret_cast<const void*>(&k_recon_int<8, QUASAR_NCH, 1>);
-    case 16: return batch ? reinterpret_cast<const void*>(&k_recon_int<16, QUASAR_NCH, kMaxBatch>)
-                          : reinterpret_cast<const void*>(&k_recon_int<16, QUASAR_NCH, 1>);
-    case 32: return batch ? reinterpret_cast<const void*>(&k_recon_int<32, QUASAR_NCH, kMaxBatch>)
-                          : reinterpret_cast<const void*>(&k_recon_int<32, QUASAR_NCH, 1>);
+#define QUASAR_EPL(E)                                                                  \
+    case E:                                                                            \
+        return adam    ? reinterpret_cast<const void*>(&k_recon_int<E, C, B, true>)    \
+               : batch ? reinterpret_cast<const void*>(&k_recon_int<E, C, B, false>)   \
+                       : reinterpret_cast<const void*>(&k_recon_int<E, C, 1, false>);
+    QUASAR_EPL(4)
+    QUASAR_EPL(8)
+    QUASAR_EPL(16)
+    QUASAR_EPL(32)
+#undef QUASAR_EPL
     default: return nullptr;
     }
 }

@@ -19,9 +19,10 @@ constexpr int kMaxClip = 32;
 // One tensor of an integer-code launch: its buffers, group count, and the
 // index of its first unit in the launch's sequence of units.
 struct IntTensor {
-    const float* w;
+    const float* w;  // w' is written back here by the fused AdamW variant
     const void* g;
     float* v;
+    float* m;        // AdamW first moment (fused variant only)
     void* r;
     uint8_t* codes;
     float* a;
@@ -52,6 +53,12 @@ struct IntParams {
     unsigned int* stats;  // optional: [0] exact re-evaluations, [1] compensated fits, [2] centred refits
     float f[kMaxClip];     // padded with the last factor
     float invf[kMaxClip];  // fl32(1/f)
+    // fused AdamW step: w' = w - (w*lr_wd + step_size * m' / (sqrt(v') * isbc2 + eps))
+    float beta1, c1b;      // beta1, 1 - beta1
+    float lr_wd;           // lr * weight_decay
+    float step_size;       // lr / (1 - beta1^t)
+    float isbc2;           // 1 / sqrt(1 - beta2^t)
+    float eps;
 };
 
 // Kernel parameters of an integer-code launch over MAXT tensors at most

@@ -15,9 +15,9 @@
 #include "quasar.h"
 
 namespace quasar {
-const void* int_kernel_nch1(int epl, bool batch);
-const void* int_kernel_nch2(int epl, bool batch);
-const void* int_kernel_nch4(int epl, bool batch);
+const void* int_kernel_nch1(int epl, bool batch, bool adam);
+const void* int_kernel_nch2(int epl, bool batch, bool adam);
+const void* int_kernel_nch4(int epl, bool batch, bool adam);
 const void* nvfp4_kernel(int nch, bool batch);
 const void* amax_kernel(bool batch);
 const void* amax_to_scale_kernel(bool batch);
@@ -35,6 +35,9 @@ using namespace quasar;
 // registers a thread the whole register file).
 constexpr int kThreads = 256;
 constexpr int kWarps = kThreads / 32;
+// The AdamW-fused integer kernel also stages m (14 instead of 10 bytes a
+// weight): 6 warps per CTA keep two CTAs in an SM's shared memory.
+constexpr int kAdamWarps = 6;
 constexpr uint64_t kDefaultTimeoutNs = 1000000000ull;  // 1 s per wait
 
 std::atomic<int64_t> g_force_timeout_ns{0};
@@ -125,16 +128,16 @@ struct Launch {
     size_t smem;
 };
 
-// Shared memory per CTA: for each warp, `stages` tiles of unit_bytes, a
-// scratch area, and stages + 1 mbarriers.
-Launch plan(uint32_t unit_bytes, uint32_t scratch_bytes)
+// Shared memory per CTA: for each of its warps, `stages` tiles of
+// unit_bytes, a scratch area, and stages + 1 mbarriers.
+Launch plan(uint32_t unit_bytes, uint32_t scratch_bytes, int warps = kWarps)
 {
     const Tuning& t = tuning();
     Launch L;
     L.stage_bytes = (unit_bytes + 127u) & ~127u;
     auto total = [&](int s) {
-        return (size_t)kWarps * s * L.stage_bytes + (size_t)kWarps * scratch_bytes +
-               (size_t)kWarps * (s + 1) * 8;
+        return (size_t)warps * s * L.stage_bytes + (size_t)warps * scratch_bytes +
+               (size_t)warps * (s + 1) * 8;
     };
     int s = t.stages;
     if (s <= 0) {
@@ -203,7 +206,7 @@ quasar_status status_ptr(unsigned int** p)
 // Resident CTAs per SM for (fn, smem) on device dev.  The kernel's dynamic
 // shared-memory limit only ever grows (to the largest size requested so far),
 // so a configuration cached earlier stays launchable.
-quasar_status occupancy(const void* fn, size_t smem, int dev, int* occ)
+quasar_status occupancy(const void* fn, size_t smem, int threads, int dev, int* occ)
 {
     std::lock_guard<std::mutex> lock(g_mu);
     size_t limit = 0;
@@ -220,28 +223,28 @@ quasar_status occupancy(const void* fn, size_t smem, int dev, int* occ)
             cudaSuccess)
         return QUASAR_ERR_CUDA;
     int o = 0;
-    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&o, fn, kThreads, smem) != cudaSuccess)
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&o, fn, threads, smem) != cudaSuccess)
         return QUASAR_ERR_CUDA;
     if (g_ncfg < kMaxConfigs) g_cfg[g_ncfg++] = KernelConfig{fn, smem, dev, o};
     *occ = o;
     return QUASAR_OK;
 }
 
-// Persistent launch: at most (#SMs x resident CTAs) CTAs of 8 warps, no more
-// than there are units of work for the warps.
+// Persistent launch: at most (#SMs x resident CTAs) CTAs of `warps` warps,
+// no more than there are units of work for the warps.
 quasar_status launch_persistent(const void* fn, void* params, size_t smem, int64_t n_units,
-                                cudaStream_t stream)
+                                cudaStream_t stream, int warps = kWarps)
 {
     int dev = 0, occ = 0;
     const DeviceInfo* info = nullptr;
     quasar_status st = device_info(&dev, &info);
     if (st != QUASAR_OK) return st;
-    if ((st = occupancy(fn, smem, dev, &occ)) != QUASAR_OK) return st;
+    if ((st = occupancy(fn, smem, warps * 32, dev, &occ)) != QUASAR_OK) return st;
     if (occ < 1) return QUASAR_ERR_UNSUPPORTED;
-    const int64_t want = (n_units + kWarps - 1) / kWarps;
+    const int64_t want = (n_units + warps - 1) / warps;
     const int grid = (int)std::max<int64_t>(1, std::min<int64_t>((int64_t)info->nsm * occ, want));
     void* args[] = {params};
-    if (cudaLaunchKernel(fn, dim3(grid), dim3(kThreads), args, smem, stream) != cudaSuccess)
+    if (cudaLaunchKernel(fn, dim3(grid), dim3(warps * 32), args, smem, stream) != cudaSuccess)
         return QUASAR_ERR_CUDA;
     return QUASAR_OK;
 }
@@ -270,7 +273,7 @@ quasar_status int_tensor(const float* w, const void* g, quasar_dtype g_dtype, fl
                                 cand_idx ? (size_t)n_groups : 0};
         if (outputs_alias_inputs(w, g, g_dtype, v, n, outs, bytes, 5)) return QUASAR_ERR_INVALID_ARG;
     }
-    *T = IntTensor{w, g, v, r, codes, a, b, cand_idx, n_groups, 0};
+    *T = IntTensor{w, g, v, nullptr, r, codes, a, b, cand_idx, n_groups, 0};
     return QUASAR_OK;
 }
 
@@ -284,9 +287,24 @@ quasar_status int_check(int bits, int group_size)
     return QUASAR_OK;
 }
 
-// Parameters shared by the tensors of an integer-code call.
+// Hyper-parameters of the fused AdamW step (validated by the caller).
+struct AdamHp {
+    float lr, beta1, eps, weight_decay;
+    int64_t step;
+};
+
+// Stage bytes of one unit of the integer kernel: w, v, (m,) g.
+uint32_t int_unit_bytes(int group_size, int g_kind, bool adam)
+{
+    const int gbytes = g_kind == 2 ? 2 : (g_kind == 1 ? 4 : 0);
+    return (uint32_t)(kGroupsPerUnit * group_size * ((adam ? 12 : 8) + gbytes));
+}
+
+// Parameters shared by the tensors of an integer-code call (adam: the
+// AdamW-fused variant's step, else nullptr).
 quasar_status int_params(quasar_dtype g_dtype, bool has_g, float beta2, int bits, int group_size,
-                         const float* clip, int n_clip, quasar_dtype r_dtype, IntParams* p)
+                         const float* clip, int n_clip, quasar_dtype r_dtype, IntParams* p,
+                         const AdamHp* adam = nullptr)
 {
     quasar_status st0 = int_check(bits, group_size);
     if (st0 != QUASAR_OK) return st0;
@@ -307,8 +325,20 @@ quasar_status int_params(quasar_dtype g_dtype, bool has_g, float beta2, int bits
     fill_clip(clip, n_clip, p->f, p->invf);
     quasar_status st;
     if ((st = status_ptr(&p->status)) != QUASAR_OK) return st;
-    const int gbytes = p->g_kind == 2 ? 2 : (p->g_kind == 1 ? 4 : 0);
-    const Launch L = plan((uint32_t)(kGroupsPerUnit * group_size * (8 + gbytes)), kIntScratchBytes);
+    if (adam) {
+        // fp32 constants of the step, formed in double from the fp32
+        // hyper-parameters: w' = w - (w*lr*wd + step_size * m' / den),
+        // den = sqrt(v') / sqrt(1 - beta2^t) + eps
+        const double t = (double)adam->step;
+        p->beta1 = adam->beta1;
+        p->c1b = 1.0f - adam->beta1;
+        p->lr_wd = (float)((double)adam->lr * (double)adam->weight_decay);
+        p->step_size = (float)((double)adam->lr / (1.0 - std::pow((double)adam->beta1, t)));
+        p->isbc2 = (float)(1.0 / std::sqrt(1.0 - std::pow((double)beta2, t)));
+        p->eps = adam->eps;
+    }
+    const Launch L = plan(int_unit_bytes(group_size, p->g_kind, adam != nullptr), kIntScratchBytes,
+                          adam ? kAdamWarps : kWarps);
     p->stages = L.stages;
     p->stage_bytes = L.stage_bytes;
     return QUASAR_OK;
@@ -316,7 +346,8 @@ quasar_status int_params(quasar_dtype g_dtype, bool has_g, float beta2, int bits
 
 // Number the tensors' units consecutively and launch over all of them.
 template <int MAXT>
-quasar_status int_launch(IntLaunch<MAXT>& Lp, int group_size, int n_clip, cudaStream_t stream)
+quasar_status int_launch(IntLaunch<MAXT>& Lp, int group_size, int n_clip, cudaStream_t stream,
+                         bool adam = false)
 {
     int64_t units = 0;
     for (int i = 0; i < Lp.n_t; ++i) {
@@ -325,15 +356,16 @@ quasar_status int_launch(IntLaunch<MAXT>& Lp, int group_size, int n_clip, cudaSt
     }
     Lp.n_units = units;
     if (units == 0) return QUASAR_OK;
-    const int gbytes = Lp.p.g_kind == 2 ? 2 : (Lp.p.g_kind == 1 ? 4 : 0);
-    const Launch L = plan((uint32_t)(kGroupsPerUnit * group_size * (8 + gbytes)), kIntScratchBytes);
+    const int warps = adam ? kAdamWarps : kWarps;
+    const Launch L = plan(int_unit_bytes(group_size, Lp.p.g_kind, adam), kIntScratchBytes, warps);
     const int epl = group_size / kLanesPerGroup;
     const int nch = nch_for(n_clip);
     const bool batch = MAXT > 1;
-    const void* fn = nch == 1 ? int_kernel_nch1(epl, batch)
-                              : (nch == 2 ? int_kernel_nch2(epl, batch) : int_kernel_nch4(epl, batch));
+    const void* fn = nch == 1   ? int_kernel_nch1(epl, batch, adam)
+                     : nch == 2 ? int_kernel_nch2(epl, batch, adam)
+                                : int_kernel_nch4(epl, batch, adam);
     if (!fn) return QUASAR_ERR_UNSUPPORTED;
-    return launch_persistent(fn, &Lp, L.smem, units, stream);
+    return launch_persistent(fn, &Lp, L.smem, units, stream, warps);
 }
 
 // Validation of one tensor of an NVFP4 call; fills its descriptor and its
@@ -504,6 +536,65 @@ quasar_status quasar_recon_int_batch(const quasar_int_tensor* tensors, int n_ten
                        x.codes, x.a, x.b, x.cand_idx, group_size, &Lp.t[i]);
         }
         if ((st = int_launch(Lp, group_size, n_clip, s)) != QUASAR_OK) return st;
+    }
+    return QUASAR_OK;
+}
+
+quasar_status quasar_adamw_recon_int_batch(const quasar_adamw_tensor* tensors, int n_tensors,
+                                           quasar_dtype g_dtype, float lr, float beta1,
+                                           float beta2, float eps, float weight_decay,
+                                           int64_t step, int bits, int group_size,
+                                           const float* clip, int n_clip, quasar_dtype r_dtype,
+                                           quasar_stream_t stream)
+{
+    if (n_tensors < 0 || (n_tensors > 0 && !tensors)) return QUASAR_ERR_INVALID_ARG;
+    if (!(std::isfinite(lr) && lr >= 0.0f) || !(beta1 >= 0.0f && beta1 < 1.0f) ||
+        !(std::isfinite(eps) && eps > 0.0f) ||
+        !(std::isfinite(weight_decay) && weight_decay >= 0.0f) || step < 1)
+        return QUASAR_ERR_INVALID_ARG;
+    if (n_tensors == 0) return QUASAR_OK;
+    static thread_local IntLaunch<kMaxBatch> Lp;
+    quasar_status st = int_check(bits, group_size);
+    if (st != QUASAR_OK) return st;
+    // one tensor's descriptor; checks beyond those of the reconstruction:
+    // g and m present, and w, g, m, v pairwise disjoint
+    auto describe = [&](const quasar_adamw_tensor& x, IntTensor* T) {
+        quasar_status s1 = int_tensor(x.w, x.g, g_dtype, x.v, beta2, clip, n_clip, x.rows, x.cols,
+                                      x.r, r_dtype, x.codes, x.a, x.b, x.cand_idx, group_size, T);
+        if (s1 != QUASAR_OK) return s1;
+        T->m = x.m;
+        if (T->n_groups == 0) return QUASAR_OK;
+        if (!x.g || !x.m || !aligned16(x.m)) return QUASAR_ERR_INVALID_ARG;
+        const size_t n = (size_t)(x.rows * x.cols);
+        const void* outs[] = {x.r, x.codes, x.a, x.b, x.cand_idx};
+        const size_t bytes[] = {n * dtype_size(r_dtype), x.codes ? n : 0,
+                                (size_t)T->n_groups * 4, (size_t)T->n_groups * 4,
+                                x.cand_idx ? (size_t)T->n_groups : 0};
+        for (int i = 0; i < 5; ++i)
+            if (overlaps(outs[i], bytes[i], x.m, n * 4)) return QUASAR_ERR_INVALID_ARG;
+        const void* state[] = {x.w, x.g, x.m, x.v};
+        const size_t sbytes[] = {n * 4, n * dtype_size(g_dtype), n * 4, n * 4};
+        for (int i = 0; i < 4; ++i)
+            for (int j = i + 1; j < 4; ++j)
+                if (overlaps(state[i], sbytes[i], state[j], sbytes[j])) return QUASAR_ERR_INVALID_ARG;
+        return QUASAR_OK;
+    };
+    int64_t total = 0;
+    for (int i = 0; i < n_tensors; ++i) {
+        IntTensor T;
+        if ((st = describe(tensors[i], &T)) != QUASAR_OK) return st;
+        total += T.n_groups;
+    }
+    if (total == 0) return QUASAR_OK;
+    const AdamHp hp{lr, beta1, eps, weight_decay, step};
+    if ((st = int_params(g_dtype, true, beta2, bits, group_size, clip, n_clip, r_dtype, &Lp.p,
+                         &hp)) != QUASAR_OK)
+        return st;
+    const cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+    for (int i0 = 0; i0 < n_tensors; i0 += kMaxBatch) {
+        Lp.n_t = std::min(kMaxBatch, n_tensors - i0);
+        for (int i = 0; i < Lp.n_t; ++i) describe(tensors[i0 + i], &Lp.t[i]);
+        if ((st = int_launch(Lp, group_size, n_clip, s, true)) != QUASAR_OK) return st;
     }
     return QUASAR_OK;
 }

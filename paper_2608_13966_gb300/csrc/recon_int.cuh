@@ -355,8 +355,10 @@ __device__ void coop_precise(const float* ws, const float* hs, float c, float P,
 
 // ------------------------------------------------------------------ kernel
 
-template <int EPL, int NCH, int MAXT>
-__global__ void __launch_bounds__(256) k_recon_int(const __grid_constant__ IntLaunch<MAXT> Lp)
+// Two CTAs per SM: 8-warp CTAs, 6-warp ones for the AdamW-fused variant.
+template <int EPL, int NCH, int MAXT, bool ADAM>
+__global__ void __launch_bounds__(ADAM ? 192 : 256, 2)
+    k_recon_int(const __grid_constant__ IntLaunch<MAXT> Lp)
 {
     const IntParams& p = Lp.p;
     constexpr int G = EPL * kLanesPerGroup;
@@ -379,8 +381,10 @@ __global__ void __launch_bounds__(256) k_recon_int(const __grid_constant__ IntLa
                      warp * (S + 1);
 
     const int gbytes = p.g_kind == 2 ? 2 : (p.g_kind == 1 ? 4 : 0);
+    // stage: w | v | m (fused AdamW only) | g
     constexpr uint32_t kVOff = UNIT * 4;
-    constexpr uint32_t kGOff = UNIT * 8;
+    constexpr uint32_t kMOff = UNIT * 8;
+    constexpr uint32_t kGOff = UNIT * (ADAM ? 12 : 8);
 
     const int64_t n_units = Lp.n_units;
     // the tensor of a unit: units are numbered consecutively across the
@@ -408,9 +412,10 @@ __global__ void __launch_bounds__(256) k_recon_int(const __grid_constant__ IntLa
         const int64_t ng = min((int64_t)kGroupsPerUnit, T.n_groups - g0);
         const uint32_t elems = (uint32_t)(ng * G);
         unsigned char* st = ring + (size_t)s * p.stage_bytes;
-        mbar_arrive_expect_tx(&bars[s], elems * (8u + (uint32_t)gbytes));
+        mbar_arrive_expect_tx(&bars[s], elems * ((ADAM ? 12u : 8u) + (uint32_t)gbytes));
         bulk_g2s(st, T.w + g0 * G, elems * 4u, &bars[s]);
         bulk_g2s(st + kVOff, T.v + g0 * G, elems * 4u, &bars[s]);
+        if constexpr (ADAM) bulk_g2s(st + kMOff, T.m + g0 * G, elems * 4u, &bars[s]);
         if (gbytes)
             bulk_g2s(st + kGOff, static_cast<const unsigned char*>(T.g) + g0 * G * gbytes,
                      elems * (uint32_t)gbytes, &bars[s]);
@@ -448,6 +453,10 @@ __global__ void __launch_bounds__(256) k_recon_int(const __grid_constant__ IntLa
     const float ulp = 5.9604645e-8f * p.tie_kappa;
     const float2 beta22 = make_float2(p.beta2, p.beta2);
     const float2 c12 = make_float2(p.c1, p.c1);
+    const float2 beta12 = make_float2(p.beta1, p.beta1), c1b2 = make_float2(p.c1b, p.c1b);
+    const float2 nlrwd2 = make_float2(-p.lr_wd, -p.lr_wd);
+    const float2 nstep2 = make_float2(-p.step_size, -p.step_size);
+    const float2 isbc22 = make_float2(p.isbc2, p.isbc2), eps2 = make_float2(p.eps, p.eps);
     int s_cur = 0;
     uint32_t parity = 0;
 
@@ -459,7 +468,7 @@ __global__ void __launch_bounds__(256) k_recon_int(const __grid_constant__ IntLa
             return;
         }
         unsigned char* st = ring + (size_t)s_cur * p.stage_bytes;
-        const float* ws = reinterpret_cast<const float*>(st);
+        float* ws = reinterpret_cast<float*>(st);
         float* hs = reinterpret_cast<float*>(st + kVOff);
         const unsigned char* gsm = st + kGOff;
 
@@ -470,19 +479,62 @@ __global__ void __launch_bounds__(256) k_recon_int(const __grid_constant__ IntLa
         const int64_t gbase = grp * (int64_t)G;
 
         // ---- pass A: saliency EMA (h kept in the tile), range, saliency mass
-        // and weighted sum of w (a centre for the moments)
+        // and weighted sum of w (a centre for the moments).  The fused variant
+        // first takes one AdamW step and keeps w' in the tile, so everything
+        // after this pass reconstructs the updated weights.
         float mn = INFINITY, mx = -INFINITY, ss = 0.0f, sw = 0.0f;
         {
             float* vout = T.v + gbase + sl * 4;
+            float* wout = const_cast<float*>(T.w) + gbase + sl * 4;
+            float* mout = T.m + gbase + sl * 4;
             auto pass_a = [&](auto gk) {
                 constexpr int GK = decltype(gk)::value;
                 float2 SS = make_float2(0.0f, 0.0f), SW = SS;
 #pragma unroll
                 for (int i = 0; i < NCHK; ++i) {
                     const int e = gs * G + i * 32 + sl * 4;
-                    const float4 w4 = lds128(ws + e);
+                    float4 w4 = lds128(ws + e);
                     float4 h4 = lds128(hs + e);
-                    if constexpr (GK != 0) {
+                    if constexpr (ADAM) {
+                        float2 gv[2];
+                        if constexpr (GK == 2) {
+                            const uint2 gb = lds64(gsm + e * 2);
+                            gv[0] = make_float2(bf16lo(gb.x), bf16hi(gb.x));
+                            gv[1] = make_float2(bf16lo(gb.y), bf16hi(gb.y));
+                        } else {
+                            const float4 g4 = lds128(gsm + e * 4);
+                            gv[0] = make_float2(g4.x, g4.y);
+                            gv[1] = make_float2(g4.z, g4.w);
+                        }
+                        const float4 m4 = lds128(reinterpret_cast<const float*>(st + kMOff) + e);
+                        float2 wv[2] = {make_float2(w4.x, w4.y), make_float2(w4.z, w4.w)};
+                        float2 mv[2] = {make_float2(m4.x, m4.y), make_float2(m4.z, m4.w)};
+                        float2 hv[2] = {make_float2(h4.x, h4.y), make_float2(h4.z, h4.w)};
+#pragma unroll
+                        for (int pr = 0; pr < 2; ++pr) {
+                            mv[pr] = __ffma2_rn(mv[pr], beta12, __fmul2_rn(c1b2, gv[pr]));
+                            hv[pr] = __ffma2_rn(hv[pr], beta22,
+                                                __fmul2_rn(c12, __fmul2_rn(gv[pr], gv[pr])));
+                            const float2 den = __ffma2_rn(
+                                make_float2(__fsqrt_rn(hv[pr].x), __fsqrt_rn(hv[pr].y)), isbc22, eps2);
+                            const float2 upd = make_float2(__fdiv_rn(mv[pr].x, den.x),
+                                                           __fdiv_rn(mv[pr].y, den.y));
+                            // the decrement is formed first and added once, so
+                            // w' is w + t rounded a single time
+                            const float2 t = __ffma2_rn(wv[pr], nlrwd2, __fmul2_rn(nstep2, upd));
+                            wv[pr] = __fadd2_rn(wv[pr], t);
+                        }
+                        w4 = make_float4(wv[0].x, wv[0].y, wv[1].x, wv[1].y);
+                        h4 = make_float4(hv[0].x, hv[0].y, hv[1].x, hv[1].y);
+                        *reinterpret_cast<float4*>(ws + e) = w4;
+                        *reinterpret_cast<float4*>(hs + e) = h4;
+                        if (valid) {
+                            stg_cs(reinterpret_cast<float4*>(wout + i * 32), w4);
+                            stg_cs(reinterpret_cast<float4*>(mout + i * 32),
+                                   make_float4(mv[0].x, mv[0].y, mv[1].x, mv[1].y));
+                            stg_cs(reinterpret_cast<float4*>(vout + i * 32), h4);
+                        }
+                    } else if constexpr (GK != 0) {
                         float2 gA, gB;
                         if constexpr (GK == 2) {
                             const uint2 gb = lds64(gsm + e * 2);
@@ -512,7 +564,7 @@ __global__ void __launch_bounds__(256) k_recon_int(const __grid_constant__ IntLa
                 sw = SW.x + SW.y;
             };
             if (p.g_kind == 2) pass_a(std::integral_constant<int, 2>{});
-            else if (p.g_kind == 1) pass_a(std::integral_constant<int, 1>{});
+            else if (ADAM || p.g_kind == 1) pass_a(std::integral_constant<int, 1>{});
             else pass_a(std::integral_constant<int, 0>{});
         }
 #pragma unroll

@@ -43,6 +43,8 @@ PROTOTYPES = {
     "quasar_recon_nvfp4": (_I, [_P, _P, _I, _P, _F, _P, _I, _I64, _I64, _P, _P, _I, _P, _P, _P,
                                 _P, _P]),
     "quasar_recon_int_batch": (_I, [_P, _I, _I, _F, _I, _I, _P, _I, _I, _P]),
+    "quasar_adamw_recon_int_batch": (_I, [_P, _I, _I, _F, _F, _F, _F, _F, _I64, _I, _I, _P, _I,
+                                          _I, _P]),
     "quasar_recon_nvfp4_batch": (_I, [_P, _I, _I, _F, _P, _I, _I, _P]),
     "quasar_tensor_amax": (_I, [_P, _I64, _P, _P]),
     "quasar_get_device_status": (_I, [_P]),
@@ -157,6 +159,39 @@ def quasar_recon_int_batch(tensors, beta2, bits, group_size, clip, g_dtype=BF16,
     carr, nclip = _clip_array(clip)
     st = lib.quasar_recon_int_batch(ctypes.cast(tensors, ctypes.c_void_p), len(tensors), g_dtype,
                                     beta2, bits, group_size, carr, nclip, r_dtype, _stream(stream))
+    return QuasarStatus(st)
+
+
+class QuasarAdamwTensor(ctypes.Structure):
+    """quasar_adamw_tensor: one tensor's buffers (device pointers) and shape."""
+    _fields_ = [("w", ctypes.c_void_p), ("g", ctypes.c_void_p), ("m", ctypes.c_void_p),
+                ("v", ctypes.c_void_p), ("r", ctypes.c_void_p), ("codes", ctypes.c_void_p),
+                ("a", ctypes.c_void_p), ("b", ctypes.c_void_p), ("cand_idx", ctypes.c_void_p),
+                ("rows", ctypes.c_int64), ("cols", ctypes.c_int64)]
+
+
+def adamw_tensor_array(items):
+    """A ctypes array of QuasarAdamwTensor from dicts with keys w, g, m, v,
+    r, codes, a, b, cand_idx (tensors, pointers or None), rows, cols."""
+    arr = (QuasarAdamwTensor * len(items))()
+    for i, d in enumerate(items):
+        arr[i] = QuasarAdamwTensor(_ptr(d["w"]), _ptr(d.get("g")), _ptr(d.get("m")), _ptr(d["v"]),
+                                   _ptr(d["r"]), _ptr(d.get("codes")), _ptr(d["a"]), _ptr(d["b"]),
+                                   _ptr(d.get("cand_idx")), int(d["rows"]), int(d["cols"]))
+    return arr
+
+
+def quasar_adamw_recon_int_batch(tensors, lr, beta1, beta2, eps, weight_decay, step, bits,
+                                 group_size, clip, g_dtype=BF16, r_dtype=BF16,
+                                 stream=None) -> QuasarStatus:
+    """tensors: a ctypes array from adamw_tensor_array (or a list of dicts)."""
+    lib = load()
+    if not isinstance(tensors, ctypes.Array):
+        tensors = adamw_tensor_array(tensors)
+    carr, nclip = _clip_array(clip)
+    st = lib.quasar_adamw_recon_int_batch(ctypes.cast(tensors, ctypes.c_void_p), len(tensors),
+                                          g_dtype, lr, beta1, beta2, eps, weight_decay, step,
+                                          bits, group_size, carr, nclip, r_dtype, _stream(stream))
     return QuasarStatus(st)
 
 

@@ -24,7 +24,15 @@ Z / sqrt(chi2_nu / nu) with chi2_nu the sum of nu squared standard normals.
 
 Every tensor has its own generator seeded with ``seed*1000 + index`` where
 ``index = 7*layer + j`` (j over q, k, v, o, gate, up, down), and the draws are
-taken in the order w, warm-up gradient (first workload only), g, v.
+taken in the order w, warm-up gradient (first workload only), g, v.  Adam's
+first moment m, for the workloads that take an AdamW step, comes from a
+generator of its own (seed ``seed*1000 + index + 500000``): N(0, (3e-4)^2),
+a smoothed gradient of the gradient's scale.
+
+AdamW workloads use the paper's Llama-3.1-8B INT3 learning rate 2e-5
+(Sec. 5 setup) and, where the paper gives none, PyTorch's AdamW defaults
+(beta1 0.9, eps 1e-8, weight decay 0.01); the step counter is 100, a point
+where both bias corrections still differ from 1.
 """
 from __future__ import annotations
 
@@ -55,6 +63,9 @@ QWEN3_8B_LAYER = (
 CLIP_8 = tuple(round(1.00 - 0.05 * i, 2) for i in range(8))    # 1.00 ... 0.65
 CLIP_16 = tuple(round(1.00 - 0.05 * i, 2) for i in range(16))  # 1.00 ... 0.25
 CLIP_PAPER = tuple(round(0.30 + 0.05 * i, 2) for i in range(15))  # 0.30 ... 1.00
+
+# AdamW hyper-parameters of the fused-step workloads
+ADAMW_LLAMA_INT3 = {"lr": 2e-5, "beta1": 0.9, "eps": 1e-8, "weight_decay": 0.01, "step": 100}
 
 
 @dataclass(frozen=True)
@@ -88,6 +99,7 @@ class Workload:
     v_dist: str               # "warm_g2" or "lognormal"
     notes: str = ""
     extra: dict = field(default_factory=dict, compare=False)
+    adamw: dict = field(default_factory=dict, compare=False)  # AdamW step, if any
 
     @property
     def numel(self) -> int:
@@ -128,6 +140,17 @@ def workload(name: str) -> Workload:
                             _layer_tensors(LLAMA31_8B_LAYER, 32), "t4", "lognormal",
                             f"all linear weights of a 32-layer Llama-3.1-8B-shaped model, "
                             f"INT{bits} group 128")
+    if name == "llama_layer_int3_adamw":
+        return Workload(name, "int", 3, 128, CLIP_8, 0.999, bf16, bf16, True,
+                        _layer_tensors(LLAMA31_8B_LAYER, 1), "t4", "lognormal",
+                        "one Llama-3.1-8B-shaped layer, AdamW step + INT3 group 128",
+                        adamw=dict(ADAMW_LLAMA_INT3))
+    if name == "llama_int3_adamw":
+        return Workload(name, "int", 3, 128, CLIP_8, 0.999, bf16, bf16, False,
+                        _layer_tensors(LLAMA31_8B_LAYER, 32), "t4", "lognormal",
+                        "AdamW step fused with INT3 group-128 reconstruction of all linear "
+                        "weights of a 32-layer Llama-3.1-8B-shaped model",
+                        adamw=dict(ADAMW_LLAMA_INT3))
     if name == "llama_nvfp4":
         return Workload(name, "nvfp4", 4, 16, CLIP_8, 0.999, bf16, bf16, False,
                         _layer_tensors(LLAMA31_8B_LAYER, 32), "t4", "lognormal",
@@ -136,7 +159,8 @@ def workload(name: str) -> Workload:
 
 
 WORKLOADS = ("single_int4", "llama_layer_int3", "qwen_layer_int2", "llama_layer_nvfp4",
-             "llama_int2", "llama_int3", "llama_int4", "llama_nvfp4")
+             "llama_layer_int3_adamw", "llama_int2", "llama_int3", "llama_int4", "llama_nvfp4",
+             "llama_int3_adamw")
 
 
 def _student_t(gen, shape, nu: int, device) -> torch.Tensor:
@@ -146,6 +170,14 @@ def _student_t(gen, shape, nu: int, device) -> torch.Tensor:
         x = torch.randn(shape, generator=gen, device=device, dtype=torch.float32)
         chi2.addcmul_(x, x)
     return z / torch.sqrt(chi2 / nu)
+
+
+def first_moment(shape, seed: int, device="cpu") -> torch.Tensor:
+    """Adam's first moment m ~ N(0, (3e-4)^2), fp32, from its own generator."""
+    device = torch.device(device)
+    gen = torch.Generator(device=device)
+    gen.manual_seed(seed + 500000)
+    return (3e-4 * torch.randn(shape, generator=gen, device=device, dtype=torch.float32)).contiguous()
 
 
 def make_tensor(wl: Workload, spec: TensorSpec, device="cpu", seed: int = 0) -> dict:
@@ -177,7 +209,10 @@ def make_tensor(wl: Workload, spec: TensorSpec, device="cpu", seed: int = 0) -> 
     else:
         raise ValueError(wl.v_dist)
 
-    return {"w": w.contiguous(), "g": g.to(wl.g_dtype).contiguous(), "v": v.contiguous()}
+    out = {"w": w.contiguous(), "g": g.to(wl.g_dtype).contiguous(), "v": v.contiguous()}
+    if wl.adamw:
+        out["m"] = first_moment(shape, seed * 1000 + spec.index, device)
+    return out
 
 
 def random_groups(n_groups: int, group: int, *, seed: int = 0, dist: str = "t4",

@@ -75,6 +75,33 @@ def check_ema(v_ref, v_gpu):
     return _report("ema", np.asarray(v_ref).size, 0, {"fail_v": np.count_nonzero(bad)})
 
 
+def check_adamw(w_in, g_in, m_in, hp, w_ref, m_ref, v_ref, w_gpu, m_gpu, v_gpu):
+    """AdamW state after the fused step (hp: lr, beta1, beta2, eps,
+    weight_decay, step as the kernel received them).  m', v' within the EMA
+    tolerance.  w' within one fp32 ulp of the oracle's w' plus 2^-20 of the
+    magnitude the decrement is formed from, |w| lr wd + lr/(1-beta1^t) *
+    (beta1 |m| + (1-beta1) |g|) / den: fp32 arithmetic forms the decrement
+    with an error of a few ulps of that magnitude (m' may cancel, so its
+    error is relative to the terms, not to m'), and adds it to w once."""
+    w_in = np.asarray(w_in, np.float64)
+    w_ref64 = np.asarray(w_ref, np.float64)
+    lr, b1, b2 = float(hp["lr"]), float(hp["beta1"]), float(hp["beta2"])
+    t = int(hp["step"])
+    den = np.sqrt(np.asarray(v_ref, np.float64) / (1.0 - b2 ** t)) + float(hp["eps"])
+    mag = (np.abs(w_in) * lr * float(hp["weight_decay"]) +
+           lr / (1.0 - b1 ** t) * (b1 * np.abs(np.asarray(m_in, np.float64)) +
+                                   (1.0 - b1) * np.abs(np.asarray(g_in, np.float64))) / den)
+    ulp = np.spacing(np.abs(np.asarray(w_ref, np.float32))).astype(np.float64)
+    bad_w = np.abs(np.asarray(w_gpu, np.float64) - w_ref64) > ulp + 2.0 ** -20 * mag
+    fails = {"fail_w": np.count_nonzero(bad_w),
+             "fail_m": np.count_nonzero(~close(m_gpu, m_ref)),
+             "fail_v": np.count_nonzero(~close(v_gpu, v_ref))}
+    rep = _report("adamw", w_in.size, 0, fails)
+    rep["w_exact_frac"] = (float(np.mean(np.asarray(w_gpu, np.float32) ==
+                                         np.asarray(w_ref, np.float32))) if w_in.size else 1.0)
+    return rep
+
+
 def _codes_from_r(r, a, b, qmax):
     with np.errstate(divide="ignore", invalid="ignore"):
         q = np.rint((np.asarray(r, np.float64) - b) / a)

@@ -165,3 +165,42 @@ def test_nvfp4_batch_argument_validation(lib):
     assert call([_ndesc(), _ndesc(cols=40)]) == st.ERR_INVALID_ARG     # cols % 16
     assert call([_ndesc(), _ndesc(tensor_scale=None)]) == st.ERR_INVALID_ARG
     assert call([_ndesc(), _ndesc(r=C)]) == st.ERR_INVALID_ARG         # output aliases v
+
+
+M_ADDR = 0x70000000
+
+
+def _adesc(**kw):
+    d = dict(w=A, g=B, m=M_ADDR, v=C, r=D, codes=None, a=E, b=F, cand_idx=None, rows=4, cols=256)
+    d.update(kw)
+    return d
+
+
+@pytest.mark.parametrize("kw,expect", [
+    (dict(items=[]), Q.QuasarStatus.OK),
+    (dict(items=[_adesc(rows=0, g=None, m=None)]), Q.QuasarStatus.OK),       # empty: no-op
+    (dict(items=[_adesc(g=None)]), Q.QuasarStatus.ERR_INVALID_ARG),         # gradient required
+    (dict(items=[_adesc(m=None)]), Q.QuasarStatus.ERR_INVALID_ARG),         # m required
+    (dict(items=[_adesc(m=M_ADDR + 4)]), Q.QuasarStatus.ERR_INVALID_ARG),   # misaligned m
+    (dict(items=[_adesc(m=A + 1024)]), Q.QuasarStatus.ERR_INVALID_ARG),     # m overlaps w
+    (dict(items=[_adesc(m=C)]), Q.QuasarStatus.ERR_INVALID_ARG),            # m is v
+    (dict(items=[_adesc(g=C + 16)]), Q.QuasarStatus.ERR_INVALID_ARG),       # g overlaps v
+    (dict(items=[_adesc(r=M_ADDR + 64)]), Q.QuasarStatus.ERR_INVALID_ARG),  # r overlaps m
+    (dict(items=[_adesc(a=M_ADDR)]), Q.QuasarStatus.ERR_INVALID_ARG),       # a overlaps m
+    (dict(items=[_adesc(), _adesc(cols=200)]), Q.QuasarStatus.ERR_INVALID_ARG),
+    (dict(lr=-1.0), Q.QuasarStatus.ERR_INVALID_ARG),
+    (dict(lr=float("inf")), Q.QuasarStatus.ERR_INVALID_ARG),
+    (dict(beta1=1.0), Q.QuasarStatus.ERR_INVALID_ARG),
+    (dict(beta2=1.0), Q.QuasarStatus.ERR_INVALID_ARG),
+    (dict(eps=0.0), Q.QuasarStatus.ERR_INVALID_ARG),
+    (dict(weight_decay=-0.1), Q.QuasarStatus.ERR_INVALID_ARG),
+    (dict(step=0), Q.QuasarStatus.ERR_INVALID_ARG),
+    (dict(bits=0), Q.QuasarStatus.ERR_INVALID_ARG),
+    (dict(group_size=48), Q.QuasarStatus.ERR_UNSUPPORTED),
+])
+def test_adamw_batch_argument_validation(lib, kw, expect):
+    args = dict(items=[_adesc()], lr=1e-5, beta1=0.9, beta2=0.999, eps=1e-8, weight_decay=0.0,
+                step=1, bits=3, group_size=128)
+    args.update(kw)
+    items = args.pop("items")
+    assert Q.quasar_adamw_recon_int_batch(items, clip=CLIP, stream=0, **args) == expect

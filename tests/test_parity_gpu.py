@@ -231,3 +231,97 @@ def test_nvfp4_batch_matches_oracle_and_single_calls(oracle):
         rep = checker.check_nvfp4(oracle, w_h, h, clip, s_T, O, gpu, True)
         ema = checker.check_ema(h, H._host(items[i][2]))
         _assert(rep, ema)
+
+
+def _hp32(hp, beta2):
+    """The hyper-parameters as the kernel receives them (fp32 values)."""
+    f32 = lambda x: float(np.float32(x))
+    return dict(lr=f32(hp["lr"]), beta1=f32(hp["beta1"]), beta2=f32(beta2), eps=f32(hp["eps"]),
+                weight_decay=f32(hp["weight_decay"]), step=int(hp["step"]))
+
+
+def _adamw_case(oracle, shapes, seed0, hp, bits=3, G=128, clip=CLIP8, g_dtype=torch.bfloat16,
+                r_dtype=torch.bfloat16):
+    """Fused AdamW step + reconstruction over tensors of the given shapes,
+    checked tensor by tensor: the AdamW state against the oracle's step, the
+    reconstruction against the oracle's Algorithm 1 on the oracle's w', v'."""
+    from paper_2608_13966_gb300 import api
+    items, hosts = [], []
+    for i, (rows, cols) in enumerate(shapes):
+        w, g, v = _inputs(max(rows, 1), cols, seed=seed0 + i, g_dtype=g_dtype)
+        m = wl.first_moment((max(rows, 1), cols), seed0 + i, device="cuda")
+        w, g, m, v = (t[:rows].contiguous() for t in (w, g, m, v))
+        items.append((w, g, m, v))
+        hosts.append(tuple(H._host(t) for t in (w, g, m, v)))
+    outs = api.adamw_recon_int_batch(items, lr=hp["lr"], beta1=hp["beta1"], beta2=0.999,
+                                     eps=hp["eps"], weight_decay=hp["weight_decay"],
+                                     step=hp["step"], bits=bits, group_size=G, clip=clip,
+                                     r_dtype=r_dtype, codes=True)
+    torch.cuda.synchronize()
+    for i, (o, (w_h, g_h, m_h, v_h)) in enumerate(zip(outs, hosts)):
+        if w_h.size == 0:
+            continue
+        hp32 = _hp32(hp, 0.999)
+        w1, m1, v1 = oracle.adamw(w_h, g_h, m_h, v_h, **hp32)
+        w_gpu, _, m_gpu, v_gpu = (H._host(t) for t in items[i])
+        st = checker.check_adamw(w_h, g_h, m_h, hp32, w1, m1, v1, w_gpu, m_gpu, v_gpu)
+        assert st["ok"], (shapes[i], json.dumps(st))
+        O = oracle.recon_int(w1, v1, G, bits, clip)
+        gpu = {"r": H._host(o["r"]), "a": o["a"].cpu().numpy(), "b": o["b"].cpu().numpy(),
+               "codes": o["codes"].cpu().numpy().ravel(), "idx": o["cand_idx"].cpu().numpy()}
+        rep = checker.check_int(oracle, w1, v1, bits, clip, O, gpu, G,
+                                r_dtype == torch.bfloat16)
+        assert rep["ok"], (shapes[i], json.dumps(rep))
+
+
+ADAMW_PAPER = dict(wl.ADAMW_LLAMA_INT3)
+
+
+def test_adamw_recon_int_batch_matches_oracle(oracle):
+    """Tensors of different shapes (a partial last unit, a tiny tensor, an
+    empty one) at the paper's Llama INT3 learning rate."""
+    _adamw_case(oracle, [(64, 1024), (3, 384), (0, 256), (37, 640), (128, 512)], 500,
+                ADAMW_PAPER)
+
+
+@pytest.mark.parametrize("hp", [
+    dict(lr=1e-3, beta1=0.9, eps=1e-8, weight_decay=0.1, step=1),    # first step, large lr
+    dict(lr=3e-5, beta1=0.0, eps=1e-6, weight_decay=0.0, step=7),    # no momentum, no decay
+    dict(lr=0.0, beta1=0.9, eps=1e-8, weight_decay=0.01, step=100),  # w unchanged
+])
+def test_adamw_recon_int_hyperparameters(oracle, hp):
+    _adamw_case(oracle, [(48, 512)], 600, hp)
+
+
+@pytest.mark.parametrize("bits,G,K", [(2, 64, 16), (4, 256, 8), (8, 32, 5)])
+def test_adamw_recon_int_settings(oracle, bits, G, K):
+    clip = [round(1.0 - 0.7 * i / max(K - 1, 1), 4) for i in range(K)]
+    _adamw_case(oracle, [(40, 4 * G), (7, 2 * G)], 700 + bits, ADAMW_PAPER, bits=bits, G=G,
+                clip=clip, g_dtype=torch.float32, r_dtype=torch.float32)
+
+
+def test_adamw_layer_matches_oracle(oracle):
+    """A full Llama-3.1-8B-shaped layer (all seven linear weights) in one
+    fused launch, as the training step runs it."""
+    from paper_2608_13966_gb300 import api
+    w_ = wl.workload("llama_layer_int3_adamw")
+    hp = w_.adamw
+    ds = [wl.make_tensor(w_, spec, device="cuda") for spec in w_.tensors]
+    hosts = [tuple(H._host(d[k]) for k in ("w", "g", "m", "v")) for d in ds]
+    outs = api.adamw_recon_int_batch([(d["w"], d["g"], d["m"], d["v"]) for d in ds],
+                                     lr=hp["lr"], beta1=hp["beta1"], beta2=w_.beta2,
+                                     eps=hp["eps"], weight_decay=hp["weight_decay"],
+                                     step=hp["step"], bits=w_.bits, group_size=w_.group,
+                                     clip=list(w_.clip), codes=True)
+    torch.cuda.synchronize()
+    for spec, d, o, (w_h, g_h, m_h, v_h) in zip(w_.tensors, ds, outs, hosts):
+        hp32 = _hp32(hp, w_.beta2)
+        w1, m1, v1 = oracle.adamw(w_h, g_h, m_h, v_h, **hp32)
+        st = checker.check_adamw(w_h, g_h, m_h, hp32, w1, m1, v1, H._host(d["w"]),
+                                 H._host(d["m"]), H._host(d["v"]))
+        assert st["ok"], (spec.name, json.dumps(st))
+        O = oracle.recon_int(w1, v1, w_.group, w_.bits, list(w_.clip))
+        gpu = {"r": H._host(o["r"]), "a": o["a"].cpu().numpy(), "b": o["b"].cpu().numpy(),
+               "codes": o["codes"].cpu().numpy().ravel(), "idx": o["cand_idx"].cpu().numpy()}
+        rep = checker.check_int(oracle, w1, v1, w_.bits, list(w_.clip), O, gpu, w_.group, True)
+        assert rep["ok"], (spec.name, json.dumps(rep))
