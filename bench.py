@@ -467,7 +467,13 @@ def main():
         return
     # per-launch figures: the average launch of the step (the step's tensors
     # differ in size; bytes and time both scale with the weights processed)
-    tag = "k_recon_int_g%d_k%d" % (wlo.group, len(wlo.clip)) if wlo.fmt == "int" else "k_recon_nvfp4_k%d" % len(wlo.clip)
+    if wlo.fmt == "int":
+        tag = "k_recon_int_g%d_k%d%s" % (wlo.group, len(wlo.clip), "_adamw" if wlo.adamw else "")
+        kname = "k_recon_int<%d,1,256,%s> (one launch per step)" % (
+            wlo.group // 8, "true" if wlo.adamw else "false")
+    else:
+        tag = "k_recon_nvfp4_k%d" % len(wlo.clip)
+        kname = "k_recon_nvfp4<1,256> (one launch per step)"
     tpw = profiled_traffic(tag)
     traffic = None if tpw is None else tpw * n_el / len(step.calls)
     line = {
@@ -485,7 +491,7 @@ def main():
         "roofline": {"bound": "hbm", "achieved": achieved, "peak": hbm_peak, "unit": "GB/s",
                      "frac": achieved / hbm_peak, "traffic": traffic,
                      "peak_kind": peak_kind,
-                     "kernel": "k_recon_int<16,1,256> (one launch per step)" if wlo.fmt == "int" else "k_recon_nvfp4<1,256> (one launch per step)",
+                     "kernel": kname,
                      "bytes_per_weight": step_bytes / n_el,
                      "launch_bytes": step_bytes / len(step.calls),
                      "launch_ms": kernel_ms / args.steps / len(step.calls),

@@ -144,8 +144,11 @@ quasar_status quasar_recon_int_batch(const quasar_int_tensor* tensors, int n_ten
  *   w' = w*(1 - lr*wd) - (lr/(1-beta1^t)) * m' / (sqrt(v')/sqrt(1-beta2^t) + eps)
  *                                        written back to w
  * then quasar_recon_int of w' with saliency h = v' (steps 2-4 there).
- * Arithmetic is fp32: m', v' within one rounding of each product, w' the
- * fp32 sum w + (the decrement), sqrt and division correctly rounded.
+ * Arithmetic is fp32: m', v' within one rounding of each product; the
+ * decrement w*lr*wd + step_size*m'/den is formed to a few ulps (root and
+ * quotient by the fast reciprocal-square-root and reciprocal, 2 ulps each)
+ * and added to w once, so w' is the correctly rounded result up to those
+ * ulps of the decrement.
  *
  * Descriptor fields as in quasar_int_tensor, plus m (fp32 first moment,
  * [rows, cols], read and overwritten), and w is overwritten with w'.  g is

@@ -515,10 +515,16 @@ __global__ void __launch_bounds__(ADAM ? 192 : 256, 2)
                             mv[pr] = __ffma2_rn(mv[pr], beta12, __fmul2_rn(c1b2, gv[pr]));
                             hv[pr] = __ffma2_rn(hv[pr], beta22,
                                                 __fmul2_rn(c12, __fmul2_rn(gv[pr], gv[pr])));
-                            const float2 den = __ffma2_rn(
-                                make_float2(__fsqrt_rn(hv[pr].x), __fsqrt_rn(hv[pr].y)), isbc22, eps2);
-                            const float2 upd = make_float2(__fdiv_rn(mv[pr].x, den.x),
-                                                           __fdiv_rn(mv[pr].y, den.y));
+                            // sqrt(v') as v' * rsqrt(v') (v' = 0 gives 0) and the
+                            // quotient by the fast reciprocal: each within 2 ulps,
+                            // small beside the ulp of w that w' is rounded to
+                            float2 sq = __fmul2_rn(hv[pr], make_float2(rsqrtf(hv[pr].x),
+                                                                       rsqrtf(hv[pr].y)));
+                            sq.x = hv[pr].x > 0.0f ? sq.x : 0.0f;
+                            sq.y = hv[pr].y > 0.0f ? sq.y : 0.0f;
+                            const float2 den = __ffma2_rn(sq, isbc22, eps2);
+                            const float2 upd = make_float2(__fdividef(mv[pr].x, den.x),
+                                                           __fdividef(mv[pr].y, den.y));
                             // the decrement is formed first and added once, so
                             // w' is w + t rounded a single time
                             const float2 t = __ffma2_rn(wv[pr], nlrwd2, __fmul2_rn(nstep2, upd));
