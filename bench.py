@@ -104,8 +104,9 @@ class Model:
             d = WL.make_tensor(wlo, spec, device=device, seed=shard)
             n = spec.numel
             d["r"] = torch.empty((spec.rows, spec.cols), dtype=torch.bfloat16, device=device)
-            d["a"] = torch.empty(n // 128, dtype=torch.float32, device=device)
-            d["b"] = torch.empty(n // 128, dtype=torch.float32, device=device)
+            gsz = min(wlo.group, 128) if wlo.fmt == "int" else 128
+            d["a"] = torch.empty(n // gsz, dtype=torch.float32, device=device)
+            d["b"] = torch.empty(n // gsz, dtype=torch.float32, device=device)
             d["idx"] = torch.empty(n // 16, dtype=torch.uint8, device=device)
             d["scale"] = torch.empty(n // 16, dtype=torch.uint8, device=device)
             d["ts"] = torch.empty(1, dtype=torch.float32, device=device)
@@ -141,7 +142,7 @@ class Step:
                 for d in model.tensors])
             args = (ctypes.cast(self.descs, ctypes.c_void_p), len(self.descs), Q.BF16, hp["lr"],
                     hp["beta1"], wlo.beta2, hp["eps"], hp["weight_decay"], hp["step"], wlo.bits,
-                    wlo.group, self.clip, len(wlo.clip), Q.BF16, self.stream)
+                    wlo.group, self.clip, len(wlo.clip), Q.BF16, None, self.stream)
             self.calls.append((self.lib.quasar_adamw_recon_int_batch, args, model.elements))
         elif wlo.fmt == "int":
             # every tensor of the model in one launch (quasar_recon_int_batch)

@@ -53,6 +53,48 @@ typedef enum {
 typedef enum { QUASAR_F32 = 0, QUASAR_BF16 = 1 } quasar_dtype;
 
 /*
+ * quasar_options -- variants of the reconstruction, for the *_ex batch entry
+ * points and quasar_adamw_recon_int_batch (NULL = all defaults).
+ *
+ *   saliency      the weights h of the fit (Eq. 4) and the error (Eq. 3):
+ *     QUASAR_SALIENCY_EMA          h = v', the EMA of squared gradients
+ *                                  (Sec. 4.1.1; the default);
+ *     QUASAR_SALIENCY_EMA_SQUARED  h = v'^2 (fp32 square), the alternative
+ *                                  weighting the paper compares against
+ *                                  (App. A.3);
+ *     QUASAR_SALIENCY_UNIFORM      h = 1: scale search and least-squares fit
+ *                                  without saliency (the "scale search only"
+ *                                  ablation, Sec. 6.5).
+ *                 In every mode v is still updated to v' when g is given.
+ *   codes_layout  the codes output, when a codes pointer is given:
+ *     QUASAR_CODES_U8      one code per byte, [rows, cols] (the default);
+ *     QUASAR_CODES_PACKED  the deployment format.  Integer codes: each group
+ *                          is one little-endian bitstream of `bits` bits a
+ *                          code (code j of the group in bits [j*bits,
+ *                          (j+1)*bits) of the group's group_size*bits/8
+ *                          bytes), groups in order: rows*cols*bits/8 bytes.
+ *                          NVFP4: two E2M1 codes a byte, the even element in
+ *                          the low nibble: rows*cols/2 bytes.  (The paper
+ *                          deploys real NVFP4 checkpoints, Sec. 6.1, but
+ *                          prints no byte layout: these are the usual
+ *                          little-endian conventions.)
+ * The "Adam weighting only" ablation (no scale search) is F = {1}: clip =
+ * {1.0}, n_clip = 1.
+ */
+typedef enum {
+    QUASAR_SALIENCY_EMA = 0,
+    QUASAR_SALIENCY_EMA_SQUARED = 1,
+    QUASAR_SALIENCY_UNIFORM = 2
+} quasar_saliency;
+
+typedef enum { QUASAR_CODES_U8 = 0, QUASAR_CODES_PACKED = 1 } quasar_codes_layout;
+
+typedef struct {
+    quasar_saliency saliency;
+    quasar_codes_layout codes_layout;
+} quasar_options;
+
+/*
  * quasar_recon_int -- QUASAR reconstruction with asymmetric b-bit integer
  * codes (Algorithm 1; code assignment Eq. 1; dequantizer fit Eq. 4; error
  * Eq. 3; saliency EMA Sec. 4.1.1 / App. A.2).
@@ -130,11 +172,21 @@ quasar_status quasar_recon_int_batch(const quasar_int_tensor* tensors, int n_ten
                                      const float* clip, int n_clip, quasar_dtype r_dtype,
                                      quasar_stream_t stream);
 
+/* quasar_recon_int_batch with variant options (see quasar_options; NULL =
+ * defaults).  With packed codes, each descriptor's codes buffer holds
+ * rows*cols*bits/8 bytes (16-byte aligned).  An invalid option value gives
+ * QUASAR_ERR_INVALID_ARG. */
+quasar_status quasar_recon_int_batch_ex(const quasar_int_tensor* tensors, int n_tensors,
+                                        quasar_dtype g_dtype, float beta2, int bits,
+                                        int group_size, const float* clip, int n_clip,
+                                        quasar_dtype r_dtype, const quasar_options* options,
+                                        quasar_stream_t stream);
+
 /*
  * quasar_adamw_tensor / quasar_adamw_recon_int_batch -- one AdamW step fused
  * with the integer-code reconstruction of the updated weights.  The paper
  * trains with AdamW and takes AdamW's second moment as the saliency h
- * (Sec. 4.1.1; training setup in Sec. 5); the reconstruction of Algorithm 1
+ * (Sec. 4.1.1; training setup in Sec. 6.1); the reconstruction of Algorithm 1
  * follows every optimizer step.  Here both run in one pass over the weights:
  * each element of w, g, m, v is read once and w', m', v', r written once.
  *
@@ -155,7 +207,8 @@ quasar_status quasar_recon_int_batch(const quasar_int_tensor* tensors, int n_ten
  * required for every non-empty tensor.  w, m, v, g must not overlap one
  * another; the outputs r, codes, a, b, cand_idx must not overlap any of
  * them.  Hyper-parameters: lr >= 0, 0 <= beta1 < 1, 0 <= beta2 < 1,
- * eps > 0, weight_decay >= 0 (all finite), step >= 1.
+ * eps > 0, weight_decay >= 0 (all finite), step >= 1.  options as in
+ * quasar_recon_int_batch_ex (NULL = defaults).
  * Returns as quasar_recon_int_batch.
  */
 typedef struct {
@@ -177,7 +230,7 @@ quasar_status quasar_adamw_recon_int_batch(const quasar_adamw_tensor* tensors, i
                                            float beta2, float eps, float weight_decay,
                                            int64_t step, int bits, int group_size,
                                            const float* clip, int n_clip, quasar_dtype r_dtype,
-                                           quasar_stream_t stream);
+                                           const quasar_options* options, quasar_stream_t stream);
 
 /*
  * quasar_recon_nvfp4 -- QUASAR for NVFP4 (Sec. 4.2): E2M1 codes, one FP8
@@ -239,6 +292,15 @@ typedef struct {
 quasar_status quasar_recon_nvfp4_batch(const quasar_nvfp4_tensor* tensors, int n_tensors,
                                        quasar_dtype g_dtype, float beta2, const float* clip,
                                        int n_clip, quasar_dtype r_dtype, quasar_stream_t stream);
+
+/* quasar_recon_nvfp4_batch with variant options (see quasar_options; NULL =
+ * defaults).  With packed codes, each descriptor's codes buffer holds
+ * rows*cols/2 bytes (16-byte aligned).  An invalid option value gives
+ * QUASAR_ERR_INVALID_ARG. */
+quasar_status quasar_recon_nvfp4_batch_ex(const quasar_nvfp4_tensor* tensors, int n_tensors,
+                                          quasar_dtype g_dtype, float beta2, const float* clip,
+                                          int n_clip, quasar_dtype r_dtype,
+                                          const quasar_options* options, quasar_stream_t stream);
 
 /*
  * quasar_tensor_amax -- amax_out[0] = max |w[i]| over n fp32 elements (the

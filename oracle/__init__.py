@@ -105,6 +105,60 @@ def ema(v, g, beta2: float) -> np.ndarray:
     return out
 
 
+def saliency(v_prime, mode: str = "ema") -> np.ndarray:
+    """The weights h of the fit and the error from the EMA state v':
+    "ema" h = v' (Sec. 4.1.1), "ema_squared" h = v'^2 (App. A.3, the
+    alternative weighting; the square of an fp32 value is exact in fp64 and
+    rounded once where it is stored as fp32 saliency), "uniform" h = 1 (scale
+    search without saliency, the Sec. 6.5 ablation)."""
+    v = _c(v_prime, np.float32).ravel()
+    if mode == "ema":
+        return v.copy()
+    if mode == "ema_squared":
+        return (v.astype(np.float64) * v.astype(np.float64)).astype(np.float32)
+    if mode == "uniform":
+        return np.ones_like(v)
+    raise ValueError(mode)
+
+
+def pack_int_codes(codes, bits: int) -> np.ndarray:
+    """Deployment format of integer codes: one little-endian bitstream of
+    `bits` bits a code, element j in bits [j*bits, (j+1)*bits) (byte k holds
+    bits 8k .. 8k+7, least significant first).  Groups of group_size*bits/8
+    whole bytes follow one another, so the flat tensor is one stream."""
+    q = _c(codes, np.uint8).ravel().astype(np.int64)
+    assert q.size * bits % 8 == 0
+    stream = np.zeros(q.size * bits, np.uint8)
+    for b in range(bits):
+        stream[b::bits] = (q >> b) & 1
+    return np.packbits(stream, bitorder="little")
+
+
+def unpack_int_codes(packed, bits: int, n: int) -> np.ndarray:
+    """Inverse of pack_int_codes for n codes."""
+    stream = np.unpackbits(_c(packed, np.uint8).ravel(), bitorder="little")[: n * bits]
+    q = np.zeros(n, np.int64)
+    for b in range(bits):
+        q |= stream[b::bits].astype(np.int64) << b
+    return q.astype(np.uint8)
+
+
+def pack_nvfp4_codes(codes) -> np.ndarray:
+    """Two E2M1 codes (4-bit sign|magnitude nibbles) a byte, the even
+    element in the low nibble."""
+    q = _c(codes, np.uint8).ravel()
+    assert q.size % 2 == 0 and np.all(q < 16)
+    return (q[0::2] | (q[1::2] << 4)).astype(np.uint8)
+
+
+def unpack_nvfp4_codes(packed) -> np.ndarray:
+    p = _c(packed, np.uint8).ravel()
+    out = np.empty(p.size * 2, np.uint8)
+    out[0::2] = p & 0xF
+    out[1::2] = p >> 4
+    return out
+
+
 def adamw(w, g, m, v, *, lr: float, beta1: float, beta2: float, eps: float, weight_decay: float,
           step: int):
     """One AdamW step in fp64 (stored state rounded to fp32): returns

@@ -6,8 +6,8 @@ from __future__ import annotations
 import torch
 
 from .quasar import (BF16, F32, QuasarError, QuasarStatus, adamw_tensor_array, int_tensor_array,
-                     nvfp4_tensor_array, quasar_adamw_recon_int_batch, quasar_recon_int,
-                     quasar_recon_int_batch, quasar_recon_nvfp4, quasar_recon_nvfp4_batch,
+                     nvfp4_tensor_array, options, quasar_adamw_recon_int_batch, quasar_recon_int,
+                     quasar_recon_int_batch_ex, quasar_recon_nvfp4, quasar_recon_nvfp4_batch_ex,
                      quasar_tensor_amax)
 
 
@@ -52,13 +52,21 @@ def recon_int(w, g, v, *, bits, group_size, clip, beta2=0.999, r_dtype=torch.bfl
     return res
 
 
+def _int_codes(rows, cols, bits, packed, dev):
+    if packed:  # the group bitstreams: rows*cols*bits/8 bytes
+        return torch.empty(rows * cols * bits // 8, dtype=torch.uint8, device=dev)
+    return torch.empty((rows, cols), dtype=torch.uint8, device=dev)
+
+
 def recon_int_batch(items, *, bits, group_size, clip, beta2=0.999, r_dtype=torch.bfloat16,
-                    codes=False, cand_idx=True, stream=None):
+                    codes=False, cand_idx=True, saliency="ema", packed_codes=False, stream=None):
     """QUASAR integer reconstruction of several tensors in one launch.
 
     items: list of (w, g, v) CUDA tensors (g may be None for all of them);
-    each v is updated in place.  Returns one result dict per tensor, as
-    recon_int does."""
+    each v is updated in place.  saliency: "ema" (h = v'), "ema_squared"
+    (h = v'^2) or "uniform" (h = 1); packed_codes: codes as the packed
+    deployment format.  Returns one result dict per tensor, as recon_int
+    does."""
     descs, results = [], []
     g_dtype = F32
     for w, g, v in items:
@@ -70,7 +78,7 @@ def recon_int_batch(items, *, bits, group_size, clip, beta2=0.999, r_dtype=torch
                "a": torch.empty(n_groups, dtype=torch.float32, device=dev),
                "b": torch.empty(n_groups, dtype=torch.float32, device=dev)}
         if codes:
-            res["codes"] = torch.empty((rows, cols), dtype=torch.uint8, device=dev)
+            res["codes"] = _int_codes(rows, cols, bits, packed_codes, dev)
         if cand_idx:
             res["cand_idx"] = torch.empty(n_groups, dtype=torch.uint8, device=dev)
         if g is not None and g.dtype == torch.bfloat16:
@@ -80,14 +88,15 @@ def recon_int_batch(items, *, bits, group_size, clip, beta2=0.999, r_dtype=torch
                       "rows": rows, "cols": cols})
         results.append(res)
     rd = BF16 if r_dtype == torch.bfloat16 else F32
-    _check(quasar_recon_int_batch(int_tensor_array(descs), beta2, bits, group_size, clip,
-                                  g_dtype=g_dtype, r_dtype=rd, stream=stream))
+    _check(quasar_recon_int_batch_ex(int_tensor_array(descs), beta2, bits, group_size, clip,
+                                     options(saliency, packed_codes), g_dtype=g_dtype, r_dtype=rd,
+                                     stream=stream))
     return results
 
 
 def adamw_recon_int_batch(items, *, lr, step, bits, group_size, clip, beta1=0.9, beta2=0.999,
                           eps=1e-8, weight_decay=0.0, r_dtype=torch.bfloat16, codes=False,
-                          cand_idx=True, stream=None):
+                          cand_idx=True, saliency="ema", packed_codes=False, stream=None):
     """One AdamW step fused with the integer reconstruction of the updated
     weights, over several tensors in one launch.
 
@@ -105,7 +114,7 @@ def adamw_recon_int_batch(items, *, lr, step, bits, group_size, clip, beta1=0.9,
                "a": torch.empty(n_groups, dtype=torch.float32, device=dev),
                "b": torch.empty(n_groups, dtype=torch.float32, device=dev)}
         if codes:
-            res["codes"] = torch.empty((rows, cols), dtype=torch.uint8, device=dev)
+            res["codes"] = _int_codes(rows, cols, bits, packed_codes, dev)
         if cand_idx:
             res["cand_idx"] = torch.empty(n_groups, dtype=torch.uint8, device=dev)
         if g is not None and g.dtype == torch.bfloat16:
@@ -117,7 +126,8 @@ def adamw_recon_int_batch(items, *, lr, step, bits, group_size, clip, beta1=0.9,
     rd = BF16 if r_dtype == torch.bfloat16 else F32
     _check(quasar_adamw_recon_int_batch(adamw_tensor_array(descs), lr, beta1, beta2, eps,
                                         weight_decay, step, bits, group_size, clip,
-                                        g_dtype=g_dtype, r_dtype=rd, stream=stream))
+                                        g_dtype=g_dtype, r_dtype=rd,
+                                        options=options(saliency, packed_codes), stream=stream))
     return results
 
 
@@ -149,10 +159,12 @@ def recon_nvfp4(w, g, v, *, clip, beta2=0.999, tensor_amax=None, r_dtype=torch.b
 
 
 def recon_nvfp4_batch(items, *, clip, beta2=0.999, r_dtype=torch.bfloat16, codes=False,
-                      cand_idx=True, stream=None):
+                      cand_idx=True, saliency="ema", packed_codes=False, stream=None):
     """QUASAR NVFP4 reconstruction of several tensors (one absmax pass, one
     scale pass, one reconstruction launch).  items: list of (w, g, v) or
-    (w, g, v, tensor_amax) CUDA tensors; each v is updated in place."""
+    (w, g, v, tensor_amax) CUDA tensors; each v is updated in place.
+    saliency and packed_codes as in recon_int_batch (packed: two codes a
+    byte, rows*cols/2 bytes)."""
     descs, results = [], []
     g_dtype = F32
     for it in items:
@@ -166,7 +178,8 @@ def recon_nvfp4_batch(items, *, clip, beta2=0.999, r_dtype=torch.bfloat16, codes
                "block_scale": torch.empty(n_blocks, dtype=torch.uint8, device=dev),
                "tensor_scale": torch.empty(1, dtype=torch.float32, device=dev)}
         if codes:
-            res["codes"] = torch.empty((rows, cols), dtype=torch.uint8, device=dev)
+            res["codes"] = (torch.empty(rows * cols // 2, dtype=torch.uint8, device=dev) if packed_codes
+                            else torch.empty((rows, cols), dtype=torch.uint8, device=dev))
         if cand_idx:
             res["cand_idx"] = torch.empty(n_blocks, dtype=torch.uint8, device=dev)
         if g is not None and g.dtype == torch.bfloat16:
@@ -177,8 +190,9 @@ def recon_nvfp4_batch(items, *, clip, beta2=0.999, r_dtype=torch.bfloat16, codes
                       "rows": rows, "cols": cols})
         results.append(res)
     rd = BF16 if r_dtype == torch.bfloat16 else F32
-    _check(quasar_recon_nvfp4_batch(nvfp4_tensor_array(descs), beta2, clip, g_dtype=g_dtype,
-                                    r_dtype=rd, stream=stream))
+    _check(quasar_recon_nvfp4_batch_ex(nvfp4_tensor_array(descs), beta2, clip,
+                                       options(saliency, packed_codes), g_dtype=g_dtype,
+                                       r_dtype=rd, stream=stream))
     return results
 
 

@@ -11,20 +11,23 @@
 
 namespace quasar {
 
-// Kernel entry for group size 8*epl, one tensor or a batch of up to
-// kMaxBatch tensors per launch (the AdamW-fused variant: batches only), or
-// nullptr if not built.
-const void* QUASAR_CAT(int_kernel_nch, QUASAR_NCH)(int epl, bool batch, bool adam)
+// Kernel entry for group size 8*epl: one tensor or a batch of up to
+// kMaxBatch tensors per launch; the AdamW-fused variant and the option
+// variants (var) are built for batches only.  nullptr if not built.
+const void* QUASAR_CAT(int_kernel_nch, QUASAR_NCH)(int epl, bool batch, bool adam, bool var)
 {
     constexpr int C = QUASAR_NCH;
     constexpr int B = kMaxBatch;
-    if (adam && !batch) return nullptr;
+    if ((adam || var) && !batch) return nullptr;
     switch (epl) {
-#define QUASAR_EPL(E)                                                                  \
-    case E:                                                                            \
-        return adam    ? reinterpret_cast<const void*>(&k_recon_int<E, C, B, true>)    \
-               : batch ? reinterpret_cast<const void*>(&k_recon_int<E, C, B, false>)   \
-                       : reinterpret_cast<const void*>(&k_recon_int<E, C, 1, false>);
+#define QUASAR_EPL(E)                                                                          \
+    case E:                                                                                    \
+        if (!batch) return reinterpret_cast<const void*>(&k_recon_int<E, C, 1, false, false>); \
+        if (adam)                                                                              \
+            return var ? reinterpret_cast<const void*>(&k_recon_int<E, C, B, true, true>)      \
+                       : reinterpret_cast<const void*>(&k_recon_int<E, C, B, true, false>);    \
+        return var ? reinterpret_cast<const void*>(&k_recon_int<E, C, B, false, true>)         \
+                   : reinterpret_cast<const void*>(&k_recon_int<E, C, B, false, false>);
     QUASAR_EPL(4)
     QUASAR_EPL(8)
     QUASAR_EPL(16)

@@ -36,9 +36,16 @@ struct IntTensor {
 // the kernel parameters: 256 x 80 bytes, within the 32 KB parameter limit).
 constexpr int kMaxBatch = 256;
 
+// Saliency used by the fit and the search: h = v', h = v'^2, or h = 1
+// (v' is still the EMA state written back).
+enum : int { kSalEma = 0, kSalEmaSquared = 1, kSalUniform = 2 };
+
 struct IntParams {
     int g_kind;  // 0 none, 1 fp32, 2 bf16
     int r_bf16;
+    int h_mode;        // kSal*
+    int codes_packed;  // codes as a bits-per-code bitstream per group
+    int bits;
     int qmax;
     int n_clip;
     float beta2;
@@ -91,6 +98,8 @@ struct Nvfp4Tensor {
 struct Nvfp4Params {
     int g_kind;
     int r_bf16;
+    int h_mode;        // kSal*
+    int codes_packed;  // two E2M1 codes per byte, low nibble first
     int n_clip;
     float beta2;
     float c1;

@@ -15,9 +15,9 @@
 #include "quasar.h"
 
 namespace quasar {
-const void* int_kernel_nch1(int epl, bool batch, bool adam);
-const void* int_kernel_nch2(int epl, bool batch, bool adam);
-const void* int_kernel_nch4(int epl, bool batch, bool adam);
+const void* int_kernel_nch1(int epl, bool batch, bool adam, bool var);
+const void* int_kernel_nch2(int epl, bool batch, bool adam, bool var);
+const void* int_kernel_nch4(int epl, bool batch, bool adam, bool var);
 const void* nvfp4_kernel(int nch, bool batch);
 const void* amax_kernel(bool batch);
 const void* amax_to_scale_kernel(bool batch);
@@ -251,13 +251,36 @@ quasar_status launch_persistent(const void* fn, void* params, size_t smem, int64
 
 int g_kind_of(const void* g, quasar_dtype d) { return !g ? 0 : (d == QUASAR_BF16 ? 2 : 1); }
 
+// Variant options of a call (quasar_options; NULL means the defaults).
+struct Opts {
+    int h_mode = kSalEma;
+    bool packed = false;
+};
+
+quasar_status read_options(const quasar_options* o, Opts* out)
+{
+    *out = Opts{};
+    if (!o) return QUASAR_OK;
+    if (o->saliency != QUASAR_SALIENCY_EMA && o->saliency != QUASAR_SALIENCY_EMA_SQUARED &&
+        o->saliency != QUASAR_SALIENCY_UNIFORM)
+        return QUASAR_ERR_INVALID_ARG;
+    if (o->codes_layout != QUASAR_CODES_U8 && o->codes_layout != QUASAR_CODES_PACKED)
+        return QUASAR_ERR_INVALID_ARG;
+    out->h_mode = o->saliency == QUASAR_SALIENCY_EMA_SQUARED ? kSalEmaSquared
+                  : o->saliency == QUASAR_SALIENCY_UNIFORM   ? kSalUniform
+                                                             : kSalEma;
+    out->packed = o->codes_layout == QUASAR_CODES_PACKED;
+    return QUASAR_OK;
+}
+
 
 // Validation of one tensor of an integer-code call; fills its descriptor
 // (unit0 is set by the caller).
 quasar_status int_tensor(const float* w, const void* g, quasar_dtype g_dtype, float* v,
                          float beta2, const float* clip, int n_clip, int64_t rows, int64_t cols,
                          void* r, quasar_dtype r_dtype, uint8_t* codes, float* a, float* b,
-                         uint8_t* cand_idx, int group_size, IntTensor* T)
+                         uint8_t* cand_idx, int group_size, IntTensor* T, int bits = 8,
+                         bool packed = false)
 {
     int64_t n = 0;
     quasar_status st = check_common(w, g, g_dtype, v, beta2, clip, n_clip, rows, cols, r, r_dtype, &n);
@@ -268,7 +291,8 @@ quasar_status int_tensor(const float* w, const void* g, quasar_dtype g_dtype, fl
         if (!a || !b) return QUASAR_ERR_INVALID_ARG;
         if (codes && !aligned16(codes)) return QUASAR_ERR_INVALID_ARG;
         const void* outs[] = {r, codes, a, b, cand_idx};
-        const size_t bytes[] = {(size_t)n * dtype_size(r_dtype), codes ? (size_t)n : 0,
+        const size_t code_bytes = packed ? (size_t)n / 8 * (size_t)bits : (size_t)n;
+        const size_t bytes[] = {(size_t)n * dtype_size(r_dtype), codes ? code_bytes : 0,
                                 (size_t)n_groups * 4, (size_t)n_groups * 4,
                                 cand_idx ? (size_t)n_groups : 0};
         if (outputs_alias_inputs(w, g, g_dtype, v, n, outs, bytes, 5)) return QUASAR_ERR_INVALID_ARG;
@@ -304,13 +328,16 @@ uint32_t int_unit_bytes(int group_size, int g_kind, bool adam)
 // AdamW-fused variant's step, else nullptr).
 quasar_status int_params(quasar_dtype g_dtype, bool has_g, float beta2, int bits, int group_size,
                          const float* clip, int n_clip, quasar_dtype r_dtype, IntParams* p,
-                         const AdamHp* adam = nullptr)
+                         const AdamHp* adam = nullptr, const Opts& opt = Opts{})
 {
     quasar_status st0 = int_check(bits, group_size);
     if (st0 != QUASAR_OK) return st0;
     *p = IntParams{};
     p->g_kind = has_g ? (g_dtype == QUASAR_BF16 ? 2 : 1) : 0;
     p->r_bf16 = r_dtype == QUASAR_BF16;
+    p->h_mode = opt.h_mode;
+    p->codes_packed = opt.packed;
+    p->bits = bits;
     p->qmax = (1 << bits) - 1;
     p->n_clip = n_clip;
     p->beta2 = beta2;
@@ -361,9 +388,10 @@ quasar_status int_launch(IntLaunch<MAXT>& Lp, int group_size, int n_clip, cudaSt
     const int epl = group_size / kLanesPerGroup;
     const int nch = nch_for(n_clip);
     const bool batch = MAXT > 1;
-    const void* fn = nch == 1   ? int_kernel_nch1(epl, batch, adam)
-                     : nch == 2 ? int_kernel_nch2(epl, batch, adam)
-                                : int_kernel_nch4(epl, batch, adam);
+    const bool var = Lp.p.h_mode != kSalEma || Lp.p.codes_packed;
+    const void* fn = nch == 1   ? int_kernel_nch1(epl, batch, adam, var)
+                     : nch == 2 ? int_kernel_nch2(epl, batch, adam, var)
+                                : int_kernel_nch4(epl, batch, adam, var);
     if (!fn) return QUASAR_ERR_UNSUPPORTED;
     return launch_persistent(fn, &Lp, L.smem, units, stream, warps);
 }
@@ -374,7 +402,7 @@ quasar_status nvfp4_tensor(const float* w, const void* g, quasar_dtype g_dtype, 
                            float beta2, const float* clip, int n_clip, int64_t rows, int64_t cols,
                            const float* tensor_amax, void* r, quasar_dtype r_dtype, uint8_t* codes,
                            uint8_t* block_scale, float* tensor_scale, uint8_t* cand_idx,
-                           Nvfp4Tensor* T, AmaxItem* A)
+                           Nvfp4Tensor* T, AmaxItem* A, bool packed = false)
 {
     int64_t n = 0;
     quasar_status st = check_common(w, g, g_dtype, v, beta2, clip, n_clip, rows, cols, r, r_dtype, &n);
@@ -389,8 +417,9 @@ quasar_status nvfp4_tensor(const float* w, const void* g, quasar_dtype g_dtype, 
         if (!block_scale) return QUASAR_ERR_INVALID_ARG;
         if (codes && !aligned16(codes)) return QUASAR_ERR_INVALID_ARG;
         const void* outs[] = {r, codes, block_scale, tensor_scale, cand_idx};
-        const size_t bytes[] = {(size_t)n * dtype_size(r_dtype), codes ? (size_t)n : 0,
-                                (size_t)n_blocks, 4, cand_idx ? (size_t)n_blocks : 0};
+        const size_t bytes[] = {(size_t)n * dtype_size(r_dtype),
+                                codes ? (packed ? (size_t)n / 2 : (size_t)n) : 0, (size_t)n_blocks, 4,
+                                cand_idx ? (size_t)n_blocks : 0};
         if (outputs_alias_inputs(w, g, g_dtype, v, n, outs, bytes, 5)) return QUASAR_ERR_INVALID_ARG;
         if (tensor_amax && overlaps(tensor_amax, 4, tensor_scale, 4)) return QUASAR_ERR_INVALID_ARG;
     }
@@ -400,11 +429,14 @@ quasar_status nvfp4_tensor(const float* w, const void* g, quasar_dtype g_dtype, 
 }
 
 quasar_status nvfp4_params(bool has_g, quasar_dtype g_dtype, float beta2, const float* clip,
-                           int n_clip, quasar_dtype r_dtype, Nvfp4Params* p)
+                           int n_clip, quasar_dtype r_dtype, Nvfp4Params* p,
+                           const Opts& opt = Opts{})
 {
     *p = Nvfp4Params{};
     p->g_kind = has_g ? (g_dtype == QUASAR_BF16 ? 2 : 1) : 0;
     p->r_bf16 = r_dtype == QUASAR_BF16;
+    p->h_mode = opt.h_mode;
+    p->codes_packed = opt.packed;
     p->n_clip = n_clip;
     p->beta2 = beta2;
     p->c1 = 1.0f - beta2;
@@ -499,6 +531,18 @@ quasar_status quasar_recon_int_batch(const quasar_int_tensor* tensors, int n_ten
                                      const float* clip, int n_clip, quasar_dtype r_dtype,
                                      quasar_stream_t stream)
 {
+    return quasar_recon_int_batch_ex(tensors, n_tensors, g_dtype, beta2, bits, group_size, clip,
+                                     n_clip, r_dtype, nullptr, stream);
+}
+
+quasar_status quasar_recon_int_batch_ex(const quasar_int_tensor* tensors, int n_tensors,
+                                        quasar_dtype g_dtype, float beta2, int bits,
+                                        int group_size, const float* clip, int n_clip,
+                                        quasar_dtype r_dtype, const quasar_options* options,
+                                        quasar_stream_t stream)
+{
+    Opts opt;
+    if (read_options(options, &opt) != QUASAR_OK) return QUASAR_ERR_INVALID_ARG;
     if (n_tensors < 0 || (n_tensors > 0 && !tensors)) return QUASAR_ERR_INVALID_ARG;
     if (n_tensors == 0) return QUASAR_OK;
     // all non-empty tensors carry a gradient, or none does
@@ -519,13 +563,14 @@ quasar_status quasar_recon_int_batch(const quasar_int_tensor* tensors, int n_ten
         const quasar_int_tensor& x = tensors[i];
         IntTensor T;
         if ((st = int_tensor(x.w, x.g, g_dtype, x.v, beta2, clip, n_clip, x.rows, x.cols, x.r,
-                             r_dtype, x.codes, x.a, x.b, x.cand_idx, group_size, &T)) != QUASAR_OK)
+                             r_dtype, x.codes, x.a, x.b, x.cand_idx, group_size, &T, bits,
+                             opt.packed)) != QUASAR_OK)
             return st;
         total += T.n_groups;
     }
     if (total == 0) return QUASAR_OK;
-    if ((st = int_params(g_dtype, has_g, beta2, bits, group_size, clip, n_clip, r_dtype, &Lp.p)) !=
-        QUASAR_OK)
+    if ((st = int_params(g_dtype, has_g, beta2, bits, group_size, clip, n_clip, r_dtype, &Lp.p,
+                         nullptr, opt)) != QUASAR_OK)
         return st;
     const cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
     for (int i0 = 0; i0 < n_tensors; i0 += kMaxBatch) {
@@ -533,7 +578,7 @@ quasar_status quasar_recon_int_batch(const quasar_int_tensor* tensors, int n_ten
         for (int i = 0; i < Lp.n_t; ++i) {
             const quasar_int_tensor& x = tensors[i0 + i];
             int_tensor(x.w, x.g, g_dtype, x.v, beta2, clip, n_clip, x.rows, x.cols, x.r, r_dtype,
-                       x.codes, x.a, x.b, x.cand_idx, group_size, &Lp.t[i]);
+                       x.codes, x.a, x.b, x.cand_idx, group_size, &Lp.t[i], bits, opt.packed);
         }
         if ((st = int_launch(Lp, group_size, n_clip, s)) != QUASAR_OK) return st;
     }
@@ -545,8 +590,10 @@ quasar_status quasar_adamw_recon_int_batch(const quasar_adamw_tensor* tensors, i
                                            float beta2, float eps, float weight_decay,
                                            int64_t step, int bits, int group_size,
                                            const float* clip, int n_clip, quasar_dtype r_dtype,
-                                           quasar_stream_t stream)
+                                           const quasar_options* options, quasar_stream_t stream)
 {
+    Opts opt;
+    if (read_options(options, &opt) != QUASAR_OK) return QUASAR_ERR_INVALID_ARG;
     if (n_tensors < 0 || (n_tensors > 0 && !tensors)) return QUASAR_ERR_INVALID_ARG;
     if (!(std::isfinite(lr) && lr >= 0.0f) || !(beta1 >= 0.0f && beta1 < 1.0f) ||
         !(std::isfinite(eps) && eps > 0.0f) ||
@@ -560,14 +607,15 @@ quasar_status quasar_adamw_recon_int_batch(const quasar_adamw_tensor* tensors, i
     // g and m present, and w, g, m, v pairwise disjoint
     auto describe = [&](const quasar_adamw_tensor& x, IntTensor* T) {
         quasar_status s1 = int_tensor(x.w, x.g, g_dtype, x.v, beta2, clip, n_clip, x.rows, x.cols,
-                                      x.r, r_dtype, x.codes, x.a, x.b, x.cand_idx, group_size, T);
+                                      x.r, r_dtype, x.codes, x.a, x.b, x.cand_idx, group_size, T,
+                                      bits, opt.packed);
         if (s1 != QUASAR_OK) return s1;
         T->m = x.m;
         if (T->n_groups == 0) return QUASAR_OK;
         if (!x.g || !x.m || !aligned16(x.m)) return QUASAR_ERR_INVALID_ARG;
         const size_t n = (size_t)(x.rows * x.cols);
         const void* outs[] = {x.r, x.codes, x.a, x.b, x.cand_idx};
-        const size_t bytes[] = {n * dtype_size(r_dtype), x.codes ? n : 0,
+        const size_t bytes[] = {n * dtype_size(r_dtype), x.codes ? (opt.packed ? n / 8 * bits : n) : 0,
                                 (size_t)T->n_groups * 4, (size_t)T->n_groups * 4,
                                 x.cand_idx ? (size_t)T->n_groups : 0};
         for (int i = 0; i < 5; ++i)
@@ -588,7 +636,7 @@ quasar_status quasar_adamw_recon_int_batch(const quasar_adamw_tensor* tensors, i
     if (total == 0) return QUASAR_OK;
     const AdamHp hp{lr, beta1, eps, weight_decay, step};
     if ((st = int_params(g_dtype, true, beta2, bits, group_size, clip, n_clip, r_dtype, &Lp.p,
-                         &hp)) != QUASAR_OK)
+                         &hp, opt)) != QUASAR_OK)
         return st;
     const cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
     for (int i0 = 0; i0 < n_tensors; i0 += kMaxBatch) {
@@ -635,6 +683,17 @@ quasar_status quasar_recon_nvfp4_batch(const quasar_nvfp4_tensor* tensors, int n
                                        quasar_dtype g_dtype, float beta2, const float* clip,
                                        int n_clip, quasar_dtype r_dtype, quasar_stream_t stream)
 {
+    return quasar_recon_nvfp4_batch_ex(tensors, n_tensors, g_dtype, beta2, clip, n_clip, r_dtype,
+                                       nullptr, stream);
+}
+
+quasar_status quasar_recon_nvfp4_batch_ex(const quasar_nvfp4_tensor* tensors, int n_tensors,
+                                          quasar_dtype g_dtype, float beta2, const float* clip,
+                                          int n_clip, quasar_dtype r_dtype,
+                                          const quasar_options* options, quasar_stream_t stream)
+{
+    Opts opt;
+    if (read_options(options, &opt) != QUASAR_OK) return QUASAR_ERR_INVALID_ARG;
     if (n_tensors < 0 || (n_tensors > 0 && !tensors)) return QUASAR_ERR_INVALID_ARG;
     if (n_tensors == 0) return QUASAR_OK;
     int with_g = 0, non_empty = 0;
@@ -654,10 +713,10 @@ quasar_status quasar_recon_nvfp4_batch(const quasar_nvfp4_tensor* tensors, int n
         AmaxItem A;
         if ((st = nvfp4_tensor(x.w, x.g, g_dtype, x.v, beta2, clip, n_clip, x.rows, x.cols,
                                x.tensor_amax, x.r, r_dtype, x.codes, x.block_scale, x.tensor_scale,
-                               x.cand_idx, &T, &A)) != QUASAR_OK)
+                               x.cand_idx, &T, &A, opt.packed)) != QUASAR_OK)
             return st;
     }
-    if ((st = nvfp4_params(has_g, g_dtype, beta2, clip, n_clip, r_dtype, &Lp.p)) != QUASAR_OK)
+    if ((st = nvfp4_params(has_g, g_dtype, beta2, clip, n_clip, r_dtype, &Lp.p, opt)) != QUASAR_OK)
         return st;
     const cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
     for (int i0 = 0; i0 < n_tensors; i0 += kMaxBatch) {
@@ -666,7 +725,7 @@ quasar_status quasar_recon_nvfp4_batch(const quasar_nvfp4_tensor* tensors, int n
             const quasar_nvfp4_tensor& x = tensors[i0 + i];
             nvfp4_tensor(x.w, x.g, g_dtype, x.v, beta2, clip, n_clip, x.rows, x.cols, x.tensor_amax,
                          x.r, r_dtype, x.codes, x.block_scale, x.tensor_scale, x.cand_idx, &Lp.t[i],
-                         &B.t[i]);
+                         &B.t[i], opt.packed);
         }
         if ((st = nvfp4_run(Lp, B, n_clip, s)) != QUASAR_OK) return st;
     }

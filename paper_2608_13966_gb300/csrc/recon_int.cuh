@@ -356,7 +356,9 @@ __device__ void coop_precise(const float* ws, const float* hs, float c, float P,
 // ------------------------------------------------------------------ kernel
 
 // Two CTAs per SM: 8-warp CTAs, 6-warp ones for the AdamW-fused variant.
-template <int EPL, int NCH, int MAXT, bool ADAM>
+// VAR: the variants of the options (a saliency other than v', packed codes);
+// without it they compile out of the common kernel.
+template <int EPL, int NCH, int MAXT, bool ADAM, bool VAR>
 __global__ void __launch_bounds__(ADAM ? 192 : 256, 2)
     k_recon_int(const __grid_constant__ IntLaunch<MAXT> Lp)
 {
@@ -572,6 +574,27 @@ __global__ void __launch_bounds__(ADAM ? 192 : 256, 2)
             if (p.g_kind == 2) pass_a(std::integral_constant<int, 2>{});
             else if (ADAM || p.g_kind == 1) pass_a(std::integral_constant<int, 1>{});
             else pass_a(std::integral_constant<int, 0>{});
+            if (VAR && p.h_mode != kSalEma) {
+                // the fit's saliency is v'^2 or 1: rewrite h in the tile (v'
+                // went out already) and take its sums again
+                float2 SS = make_float2(0.0f, 0.0f), SW = SS;
+#pragma unroll 1
+                for (int i = 0; i < NCHK; ++i) {
+                    const int e = gs * G + i * 32 + sl * 4;
+                    const float4 w4 = lds128(ws + e);
+                    float4 h4 = lds128(hs + e);
+                    h4 = p.h_mode == kSalEmaSquared
+                             ? make_float4(h4.x * h4.x, h4.y * h4.y, h4.z * h4.z, h4.w * h4.w)
+                             : make_float4(1.0f, 1.0f, 1.0f, 1.0f);
+                    *reinterpret_cast<float4*>(hs + e) = h4;
+                    const float2 hA = make_float2(h4.x, h4.y), hB = make_float2(h4.z, h4.w);
+                    SS = __fadd2_rn(SS, __fadd2_rn(hA, hB));
+                    SW = __ffma2_rn(hA, make_float2(w4.x, w4.y), SW);
+                    SW = __ffma2_rn(hB, make_float2(w4.z, w4.w), SW);
+                }
+                ss = SS.x + SS.y;
+                sw = SW.x + SW.y;
+            }
         }
 #pragma unroll
         for (int o = 4; o; o >>= 1) {
@@ -1012,10 +1035,13 @@ __global__ void __launch_bounds__(ADAM ? 192 : 256, 2)
                                 cw |= ((__float_as_uint(qf.x) & 0xFFu) | ((__float_as_uint(qf.y) & 0xFFu) << 8))
                                       << (16 * pr);
                             }
-                            stg_cs(reinterpret_cast<uint32_t*>(T.codes + eo), flat ? 0u : cw);
+                            if (flat) cw = 0;
+                            if (!(VAR && p.codes_packed) && valid)
+                                stg_cs(reinterpret_cast<uint32_t*>(T.codes + eo), cw);
                         }
                     }
-                    if (!GEN || p.r_bf16) {
+                    if (!valid) {
+                    } else if (!GEN || p.r_bf16) {
                         stg_cs(reinterpret_cast<uint2*>(static_cast<__nv_bfloat16*>(T.r) + eo),
                                make_uint2(pack_bf16x2(rv[0].x, rv[0].y), pack_bf16x2(rv[1].x, rv[1].y)));
                     } else {
@@ -1024,10 +1050,43 @@ __global__ void __launch_bounds__(ADAM ? 192 : 256, 2)
                     }
                 }
             };
+            // lanes of a missing group store nothing (with VAR every lane runs
+            // pass C: the packed codes below synchronise the warp)
             const bool gen = !p.r_bf16 || T.codes != nullptr || __any_sync(0xffffffffu, flat);
-            if (valid) {
+            if (VAR || valid) {
                 if (gen) pass_c(std::true_type{});
                 else pass_c(std::false_type{});
+            }
+            if (VAR && T.codes && p.codes_packed) {
+                // the deployment format: the group's codes as one little-endian
+                // bitstream of `bits` bits a code.  Each 32-code chunk fills
+                // `bits` words; the 8 lanes' 4-code fields (4 bits wide) are
+                // OR-ed into them in the transpose scratch.
+                uint32_t* wsc = reinterpret_cast<uint32_t*>(red) + gs * 8;
+                const uint32_t o = (uint32_t)sl * 4u * (uint32_t)p.bits;
+// (codes recomputed from the tile, as pass R did: kept registers would
+// raise the pressure of the common path)
+#pragma unroll 1
+                for (int i = 0; i < NCHK; ++i) {
+                    uint32_t pk = 0;
+#pragma unroll
+                    for (int j = 0; j < 4; ++j) {
+                        const float z = int_code_z(ws[gs * G + i * 32 + sl * 4 + j] - c, Pk, zcap);
+                        const uint32_t q = flat ? 0u : (uint32_t)(int)(z + H);
+                        pk |= q << (j * p.bits);
+                    }
+                    const uint64_t f = (uint64_t)pk << (o & 31u);
+                    if (sl < p.bits) wsc[sl] = 0u;
+                    __syncwarp();
+                    atomicOr(&wsc[o >> 5], (uint32_t)f);
+                    if ((uint32_t)(f >> 32)) atomicOr(&wsc[(o >> 5) + 1], (uint32_t)(f >> 32));
+                    __syncwarp();
+                    if (valid && sl < p.bits)
+                        stg_cs(reinterpret_cast<uint32_t*>(T.codes) + grp * (int64_t)(G / 32) * p.bits +
+                                   i * p.bits + sl,
+                               wsc[sl]);
+                    __syncwarp();
+                }
             }
             if (valid && sl == 0) {
                 // b = Bz - a*H: the offset at code 0

@@ -233,6 +233,11 @@ __global__ void __launch_bounds__(256) k_recon_nvfp4(const __grid_constant__ Nvf
             }
         }
 
+        if (p.h_mode != kSalEma)  // the fit's saliency: v'^2 or 1
+#pragma unroll
+            for (int t = 0; t < 8; ++t)
+                h2[t] = p.h_mode == kSalEmaSquared ? __fmul2_rn(h2[t], h2[t]) : make_float2(1.0f, 1.0f);
+
         float2 aw2[8], naw2[8];
         float amax_b = 0.0f;
         float2 SS = make_float2(0.0f, 0.0f);
@@ -380,6 +385,7 @@ __global__ void __launch_bounds__(256) k_recon_nvfp4(const __grid_constant__ Nvf
         const float Pb = P1 * p.invf[kb];
         const float2 Pb2 = make_float2(Pb, Pb);
         const float2 as2 = make_float2(alpha_sel, alpha_sel);
+        uint64_t pk = 0;  // packed codes: element j's nibble at bit 4j
 #pragma unroll
         for (int i = 0; i < 4; ++i) {
             const int cidx = (i + rot) & 3;
@@ -406,8 +412,19 @@ __global__ void __launch_bounds__(256) k_recon_nvfp4(const __grid_constant__ Nvf
                 stg_cs(reinterpret_cast<float4*>(static_cast<float*>(T.r) + e),
                        make_float4(rv[0].x, rv[0].y, rv[1].x, rv[1].y));
             }
-            if (T.codes) stg_cs(reinterpret_cast<uint32_t*>(T.codes + e), cw);
+            if (T.codes) {
+                if (!p.codes_packed) {
+                    stg_cs(reinterpret_cast<uint32_t*>(T.codes + e), cw);
+                } else {
+                    // bytes q0 q1 q2 q3 -> nibbles q0 | q1 << 4 | q2 << 8 | q3 << 12
+                    const uint32_t nib = (cw & 0xFu) | ((cw >> 4) & 0xF0u) | ((cw >> 8) & 0xF00u) |
+                                         ((cw >> 12) & 0xF000u);
+                    pk |= (uint64_t)nib << (16 * cidx);
+                }
+            }
         }
+        if (T.codes && p.codes_packed) stg_cs(reinterpret_cast<uint2*>(T.codes + blk * 8),
+                                             make_uint2((uint32_t)pk, (uint32_t)(pk >> 32)));
         T.scale[blk] = (uint8_t)e_sel;
         if (T.idx) T.idx[blk] = (uint8_t)kb;
     }

@@ -43,9 +43,11 @@ PROTOTYPES = {
     "quasar_recon_nvfp4": (_I, [_P, _P, _I, _P, _F, _P, _I, _I64, _I64, _P, _P, _I, _P, _P, _P,
                                 _P, _P]),
     "quasar_recon_int_batch": (_I, [_P, _I, _I, _F, _I, _I, _P, _I, _I, _P]),
+    "quasar_recon_int_batch_ex": (_I, [_P, _I, _I, _F, _I, _I, _P, _I, _I, _P, _P]),
     "quasar_adamw_recon_int_batch": (_I, [_P, _I, _I, _F, _F, _F, _F, _F, _I64, _I, _I, _P, _I,
-                                          _I, _P]),
+                                          _I, _P, _P]),
     "quasar_recon_nvfp4_batch": (_I, [_P, _I, _I, _F, _P, _I, _I, _P]),
+    "quasar_recon_nvfp4_batch_ex": (_I, [_P, _I, _I, _F, _P, _I, _I, _P, _P]),
     "quasar_tensor_amax": (_I, [_P, _I64, _P, _P]),
     "quasar_get_device_status": (_I, [_P]),
     "quasar_debug_force_timeout": (None, [_I64]),
@@ -162,6 +164,42 @@ def quasar_recon_int_batch(tensors, beta2, bits, group_size, clip, g_dtype=BF16,
     return QuasarStatus(st)
 
 
+# quasar_saliency / quasar_codes_layout
+SALIENCY = {"ema": 0, "ema_squared": 1, "uniform": 2}
+CODES_U8, CODES_PACKED = 0, 1
+
+
+class QuasarOptions(ctypes.Structure):
+    """quasar_options: variant of the reconstruction (saliency, codes layout)."""
+    _fields_ = [("saliency", ctypes.c_int), ("codes_layout", ctypes.c_int)]
+
+
+def options(saliency="ema", packed_codes=False):
+    """A QuasarOptions; saliency is "ema", "ema_squared", "uniform" or a raw
+    integer (passed through unchecked, for the library's own validation)."""
+    sal = SALIENCY[saliency] if isinstance(saliency, str) else int(saliency)
+    lay = packed_codes if isinstance(packed_codes, int) and not isinstance(packed_codes, bool) \
+        else (CODES_PACKED if packed_codes else CODES_U8)
+    return QuasarOptions(sal, lay)
+
+
+def _opt_ptr(opt):
+    return None if opt is None else ctypes.cast(ctypes.pointer(opt), ctypes.c_void_p)
+
+
+def quasar_recon_int_batch_ex(tensors, beta2, bits, group_size, clip, options=None, g_dtype=BF16,
+                              r_dtype=BF16, stream=None) -> QuasarStatus:
+    """quasar_recon_int_batch with a QuasarOptions (None = defaults)."""
+    lib = load()
+    if not isinstance(tensors, ctypes.Array):
+        tensors = int_tensor_array(tensors)
+    carr, nclip = _clip_array(clip)
+    st = lib.quasar_recon_int_batch_ex(ctypes.cast(tensors, ctypes.c_void_p), len(tensors), g_dtype,
+                                       beta2, bits, group_size, carr, nclip, r_dtype,
+                                       _opt_ptr(options), _stream(stream))
+    return QuasarStatus(st)
+
+
 class QuasarAdamwTensor(ctypes.Structure):
     """quasar_adamw_tensor: one tensor's buffers (device pointers) and shape."""
     _fields_ = [("w", ctypes.c_void_p), ("g", ctypes.c_void_p), ("m", ctypes.c_void_p),
@@ -182,7 +220,7 @@ def adamw_tensor_array(items):
 
 
 def quasar_adamw_recon_int_batch(tensors, lr, beta1, beta2, eps, weight_decay, step, bits,
-                                 group_size, clip, g_dtype=BF16, r_dtype=BF16,
+                                 group_size, clip, g_dtype=BF16, r_dtype=BF16, options=None,
                                  stream=None) -> QuasarStatus:
     """tensors: a ctypes array from adamw_tensor_array (or a list of dicts)."""
     lib = load()
@@ -191,7 +229,8 @@ def quasar_adamw_recon_int_batch(tensors, lr, beta1, beta2, eps, weight_decay, s
     carr, nclip = _clip_array(clip)
     st = lib.quasar_adamw_recon_int_batch(ctypes.cast(tensors, ctypes.c_void_p), len(tensors),
                                           g_dtype, lr, beta1, beta2, eps, weight_decay, step,
-                                          bits, group_size, carr, nclip, r_dtype, _stream(stream))
+                                          bits, group_size, carr, nclip, r_dtype,
+                                          _opt_ptr(options), _stream(stream))
     return QuasarStatus(st)
 
 
@@ -225,6 +264,19 @@ def quasar_recon_nvfp4_batch(tensors, beta2, clip, g_dtype=BF16, r_dtype=BF16,
     carr, nclip = _clip_array(clip)
     st = lib.quasar_recon_nvfp4_batch(ctypes.cast(tensors, ctypes.c_void_p), len(tensors), g_dtype,
                                       beta2, carr, nclip, r_dtype, _stream(stream))
+    return QuasarStatus(st)
+
+
+def quasar_recon_nvfp4_batch_ex(tensors, beta2, clip, options=None, g_dtype=BF16, r_dtype=BF16,
+                                stream=None) -> QuasarStatus:
+    """quasar_recon_nvfp4_batch with a QuasarOptions (None = defaults)."""
+    lib = load()
+    if not isinstance(tensors, ctypes.Array):
+        tensors = nvfp4_tensor_array(tensors)
+    carr, nclip = _clip_array(clip)
+    st = lib.quasar_recon_nvfp4_batch_ex(ctypes.cast(tensors, ctypes.c_void_p), len(tensors),
+                                         g_dtype, beta2, carr, nclip, r_dtype, _opt_ptr(options),
+                                         _stream(stream))
     return QuasarStatus(st)
 
 

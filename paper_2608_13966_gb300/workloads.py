@@ -30,7 +30,7 @@ generator of its own (seed ``seed*1000 + index + 500000``): N(0, (3e-4)^2),
 a smoothed gradient of the gradient's scale.
 
 AdamW workloads use the paper's Llama-3.1-8B INT3 learning rate 2e-5
-(Sec. 5 setup) and, where the paper gives none, PyTorch's AdamW defaults
+(Sec. 6.1 setup) and, where the paper gives none, PyTorch's AdamW defaults
 (beta1 0.9, eps 1e-8, weight decay 0.01); the step counter is 100, a point
 where both bias corrections still differ from 1.
 """

@@ -204,3 +204,22 @@ def test_adamw_batch_argument_validation(lib, kw, expect):
     args.update(kw)
     items = args.pop("items")
     assert Q.quasar_adamw_recon_int_batch(items, clip=CLIP, stream=0, **args) == expect
+
+
+def test_options_validation(lib):
+    st = Q.QuasarStatus
+    ok_opt = Q.options("ema_squared", True)
+    call = lambda opt: Q.quasar_recon_int_batch_ex([_desc(rows=0)], 0.999, 3, 128, CLIP, opt, stream=0)
+    assert call(None) == st.OK
+    assert call(ok_opt) == st.OK
+    assert call(Q.options(7)) == st.ERR_INVALID_ARG                  # unknown saliency
+    assert call(Q.options("ema", 5)) == st.ERR_INVALID_ARG           # unknown codes layout
+    nd = [_ndesc(rows=0)]
+    assert Q.quasar_recon_nvfp4_batch_ex(nd, 0.999, CLIP, Q.options(3), stream=0) == st.ERR_INVALID_ARG
+    # packed INT3 codes of 4 x 256 weights take 384 bytes: a buffer whose
+    # last 16 of them overlap v is rejected (nothing here may pass
+    # validation: the addresses are fake)
+    assert Q.quasar_recon_int_batch_ex([_desc(codes=C - 368)], 0.999, 3, 128, CLIP,
+                                       Q.options("ema", True), stream=0) == st.ERR_INVALID_ARG
+    assert Q.quasar_recon_nvfp4_batch_ex([_ndesc(codes=C - 496)], 0.999, CLIP,
+                                         Q.options("ema", True), stream=0) == st.ERR_INVALID_ARG

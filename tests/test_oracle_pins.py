@@ -551,3 +551,61 @@ def test_adamw_zero_learning_rate_keeps_weights(oracle):
     assert np.array_equal(wo, w)
     # the second moment is the saliency EMA of the reconstruction
     assert np.array_equal(vo, oracle.ema(v, g, 0.999))
+
+
+# ---------------------------------------------------------------- variants
+
+def test_packed_codes_worked_examples(oracle):
+    """Hand-worked byte layouts of the deployment format (tests/golden)."""
+    import json, os
+    gold = json.load(open(os.path.join(os.path.dirname(__file__), "golden", "packed_codes.json")))
+    for case in gold["int"]:
+        got = oracle.pack_int_codes(np.array(case["codes"], np.uint8), case["bits"])
+        assert got.tolist() == case["packed"], case
+        back = oracle.unpack_int_codes(np.array(case["packed"], np.uint8), case["bits"],
+                                       len(case["codes"]))
+        assert back.tolist() == case["codes"]
+    for case in gold["nvfp4"]:
+        assert oracle.pack_nvfp4_codes(np.array(case["codes"], np.uint8)).tolist() == case["packed"]
+        assert oracle.unpack_nvfp4_codes(np.array(case["packed"], np.uint8)).tolist() == case["codes"]
+
+
+@pytest.mark.parametrize("bits", [1, 2, 3, 4, 5, 6, 7, 8])
+def test_packed_codes_roundtrip_and_size(oracle, bits):
+    rng = np.random.default_rng(bits)
+    q = rng.integers(0, 1 << bits, size=128 * 5, dtype=np.int64).astype(np.uint8)
+    p = oracle.pack_int_codes(q, bits)
+    assert p.size == q.size * bits // 8
+    assert np.array_equal(oracle.unpack_int_codes(p, bits, q.size), q)
+    # group g of 128 codes is bytes [16 g bits, 16 (g+1) bits): packing a
+    # group alone gives the same bytes
+    g = 3
+    assert np.array_equal(oracle.pack_int_codes(q[128 * g:128 * (g + 1)], bits),
+                          p[16 * bits * g:16 * bits * (g + 1)])
+
+
+def test_saliency_modes(oracle):
+    v = np.array([0.0, 1e-6, 3.0, 2.5e-3], np.float32)
+    assert np.array_equal(oracle.saliency(v, "ema"), v)
+    assert np.array_equal(oracle.saliency(v, "uniform"), np.ones(4, np.float32))
+    sq = oracle.saliency(v, "ema_squared")
+    assert sq.dtype == np.float32
+    assert np.array_equal(sq, (v.astype(np.float64) ** 2).astype(np.float32))
+    assert sq[2] == 9.0
+    with pytest.raises(ValueError):
+        oracle.saliency(v, "cubic")
+
+
+def test_uniform_saliency_is_ordinary_least_squares(oracle):
+    """h = 1 gives the unweighted fit: the kept candidate's (a, b) is the
+    ordinary least-squares line through (q, w) of its codes (lstsq)."""
+    rng = np.random.default_rng(5)
+    w = (0.02 * rng.standard_normal(128 * 4)).astype(np.float32)
+    h = oracle.saliency(np.zeros(w.size, np.float32), "uniform")
+    O = oracle.recon_int(w, h, 128, 3, [1.0, 0.9, 0.8])
+    for g in range(4):
+        q = O["codes"][128 * g:128 * (g + 1)].astype(np.float64)
+        A = np.stack([q, np.ones_like(q)], 1)
+        (a, b), *_ = np.linalg.lstsq(A, w[128 * g:128 * (g + 1)].astype(np.float64), rcond=None)
+        assert abs(O["a"][g] - a) <= 1e-12 * max(1.0, abs(a))
+        assert abs(O["b"][g] - b) <= 1e-12 * max(1.0, abs(b))

@@ -325,3 +325,127 @@ def test_adamw_layer_matches_oracle(oracle):
                "codes": o["codes"].cpu().numpy().ravel(), "idx": o["cand_idx"].cpu().numpy()}
         rep = checker.check_int(oracle, w1, v1, w_.bits, list(w_.clip), O, gpu, w_.group, True)
         assert rep["ok"], (spec.name, json.dumps(rep))
+
+
+# ------------------------------------------------ variants (quasar_options)
+
+@pytest.mark.parametrize("mode", ["ema_squared", "uniform"])
+def test_int_saliency_variants(oracle, mode):
+    """h = v'^2 (App. A.3) and h = 1 (the scale-search-only ablation): the
+    fit and the search use the variant's h while v is still updated to v'."""
+    from paper_2608_13966_gb300 import api
+    w, g, v = _inputs(64, 1024, seed=900 + len(mode))
+    w_h, g_h, v_h = H._host(w), H._host(g), H._host(v)
+    o = api.recon_int_batch([(w, g, v)], bits=3, group_size=128, clip=CLIP8, codes=True,
+                            saliency=mode)[0]
+    torch.cuda.synchronize()
+    v1 = oracle.ema(v_h, g_h, 0.999)
+    h = oracle.saliency(v1, mode)
+    O = oracle.recon_int(w_h, h, 128, 3, CLIP8)
+    gpu = {"r": H._host(o["r"]), "a": o["a"].cpu().numpy(), "b": o["b"].cpu().numpy(),
+           "codes": o["codes"].cpu().numpy().ravel(), "idx": o["cand_idx"].cpu().numpy()}
+    _assert(checker.check_int(oracle, w_h, h, 3, CLIP8, O, gpu, 128, True),
+            checker.check_ema(v1, H._host(v)))
+
+
+@pytest.mark.parametrize("mode", ["ema_squared", "uniform"])
+def test_nvfp4_saliency_variants(oracle, mode):
+    from paper_2608_13966_gb300 import api
+    w, g, v = _inputs(48, 512, seed=910 + len(mode))
+    w_h, g_h, v_h = H._host(w), H._host(g), H._host(v)
+    o = api.recon_nvfp4_batch([(w, g, v)], clip=CLIP8, codes=True, saliency=mode)[0]
+    torch.cuda.synchronize()
+    v1 = oracle.ema(v_h, g_h, 0.999)
+    h = oracle.saliency(v1, mode)
+    _, s_T = oracle.tensor_scale(w_h)
+    O = oracle.recon_nvfp4(w_h, h, s_T, CLIP8)
+    gpu = {"r": H._host(o["r"]), "scale": o["block_scale"].cpu().numpy(),
+           "tensor_scale": float(o["tensor_scale"].cpu()[0]),
+           "codes": o["codes"].cpu().numpy().ravel(), "idx": o["cand_idx"].cpu().numpy()}
+    _assert(checker.check_nvfp4(oracle, w_h, h, CLIP8, s_T, O, gpu, True),
+            checker.check_ema(v1, H._host(v)))
+
+
+@pytest.mark.parametrize("bits,G", [(1, 32), (2, 64), (3, 128), (3, 32), (4, 256), (5, 128),
+                                    (8, 64)])
+def test_int_packed_codes(oracle, bits, G):
+    """The packed deployment format: read back with the oracle's unpacking,
+    the codes pass the same parity check as one-byte codes, and equal the
+    one-byte codes of the same call bit for bit.  Tensors with a partial
+    last unit and a one-group tensor are included."""
+    from paper_2608_13966_gb300 import api
+    clip = CLIP8
+    shapes = [(37, 3 * G), (1, G), (16, 8 * G)]
+    items, copies, hosts = [], [], []
+    for i, (rows, cols) in enumerate(shapes):
+        w, g, v = _inputs(rows, cols, seed=950 + 10 * bits + i)
+        items.append((w, g, v))
+        copies.append((w.clone(), g.clone(), v.clone()))
+        hosts.append((H._host(w), H._host(g), H._host(v)))
+    packed = api.recon_int_batch(items, bits=bits, group_size=G, clip=clip, codes=True,
+                                 packed_codes=True)
+    plain = api.recon_int_batch(copies, bits=bits, group_size=G, clip=clip, codes=True)
+    torch.cuda.synchronize()
+    for (rows, cols), o, o1, (w_h, g_h, v_h) in zip(shapes, packed, plain, hosts):
+        n = rows * cols
+        assert o["codes"].numel() == n * bits // 8
+        q = oracle.unpack_int_codes(o["codes"].cpu().numpy(), bits, n)
+        assert np.array_equal(q, o1["codes"].cpu().numpy().ravel())
+        h = oracle.ema(v_h, g_h, 0.999)
+        O = oracle.recon_int(w_h, h, G, bits, clip)
+        gpu = {"r": H._host(o["r"]), "a": o["a"].cpu().numpy(), "b": o["b"].cpu().numpy(),
+               "codes": q, "idx": o["cand_idx"].cpu().numpy()}
+        _assert(checker.check_int(oracle, w_h, h, bits, clip, O, gpu, G, True),
+                checker.check_ema(h, H._host(items[shapes.index((rows, cols))][2])))
+
+
+def test_nvfp4_packed_codes(oracle):
+    from paper_2608_13966_gb300 import api
+    shapes = [(48, 512), (3, 48), (1, 16)]
+    items, copies, hosts = [], [], []
+    for i, (rows, cols) in enumerate(shapes):
+        w, g, v = _inputs(rows, cols, seed=990 + i)
+        items.append((w, g, v))
+        copies.append((w.clone(), g.clone(), v.clone()))
+        hosts.append((H._host(w), H._host(g), H._host(v)))
+    packed = api.recon_nvfp4_batch(items, clip=CLIP8, codes=True, packed_codes=True)
+    plain = api.recon_nvfp4_batch(copies, clip=CLIP8, codes=True)
+    torch.cuda.synchronize()
+    for (rows, cols), o, o1, (w_h, g_h, v_h) in zip(shapes, packed, plain, hosts):
+        n = rows * cols
+        assert o["codes"].numel() == n // 2
+        q = oracle.unpack_nvfp4_codes(o["codes"].cpu().numpy())
+        assert np.array_equal(q, o1["codes"].cpu().numpy().ravel())
+        h = oracle.ema(v_h, g_h, 0.999)
+        _, s_T = oracle.tensor_scale(w_h)
+        O = oracle.recon_nvfp4(w_h, h, s_T, CLIP8)
+        gpu = {"r": H._host(o["r"]), "scale": o["block_scale"].cpu().numpy(),
+               "tensor_scale": float(o["tensor_scale"].cpu()[0]), "codes": q,
+               "idx": o["cand_idx"].cpu().numpy()}
+        rep = checker.check_nvfp4(oracle, w_h, h, CLIP8, s_T, O, gpu, True)
+        assert rep["ok"], json.dumps(rep)
+
+
+def test_adamw_with_options(oracle):
+    """The fused AdamW step with h = v'^2 and packed codes."""
+    from paper_2608_13966_gb300 import api
+    hp = ADAMW_PAPER
+    w, g, v = _inputs(40, 512, seed=1001)
+    m = wl.first_moment((40, 512), 1001, device="cuda")
+    w_h, g_h, m_h, v_h = (H._host(t) for t in (w, g, m, v))
+    o = api.adamw_recon_int_batch([(w, g, m, v)], lr=hp["lr"], beta1=hp["beta1"], beta2=0.999,
+                                  eps=hp["eps"], weight_decay=hp["weight_decay"], step=hp["step"],
+                                  bits=3, group_size=128, clip=CLIP8, codes=True,
+                                  saliency="ema_squared", packed_codes=True)[0]
+    torch.cuda.synchronize()
+    hp32 = _hp32(hp, 0.999)
+    w1, m1, v1 = oracle.adamw(w_h, g_h, m_h, v_h, **hp32)
+    st = checker.check_adamw(w_h, g_h, m_h, hp32, w1, m1, v1, H._host(w), H._host(m), H._host(v))
+    assert st["ok"], json.dumps(st)
+    h = oracle.saliency(v1, "ema_squared")
+    O = oracle.recon_int(w1, h, 128, 3, CLIP8)
+    q = oracle.unpack_int_codes(o["codes"].cpu().numpy(), 3, w_h.size)
+    gpu = {"r": H._host(o["r"]), "a": o["a"].cpu().numpy(), "b": o["b"].cpu().numpy(),
+           "codes": q, "idx": o["cand_idx"].cpu().numpy()}
+    rep = checker.check_int(oracle, w1, h, 3, CLIP8, O, gpu, 128, True)
+    assert rep["ok"], json.dumps(rep)
