@@ -80,6 +80,8 @@ def _load():
         lib.qo_recon_lut.restype = i32
         lib.qo_lut_block.argtypes = [P, P, i32, f32, P, P, P, P]
         lib.qo_lut_block.restype = f64
+        lib.qo_lut_fit.argtypes = [P, P, i32, f32, P, P, P]
+        lib.qo_lut_fit.restype = None
         lib.qo_lut_eval.argtypes = [P, P, i32, P, P]
         lib.qo_lut_eval.restype = f64
         _lib = lib
@@ -367,6 +369,18 @@ def lut_block(w_block, h_block, f: float):
     e = _load().qo_lut_block(_ptr(w), _ptr(h), n, ctypes.c_float(f), _ptr(q), _ptr(book), _ptr(m),
                              _ptr(bm))
     return q, book, float(e), m, bm
+
+
+def lut_fit(w_block, h_block, f: float, codes):
+    """Table bits (Eq. rubin-fit) of given indices on one block for factor f,
+    with each entry's E4M3 boundary margin."""
+    w = _c(w_block, np.float32).ravel()
+    h = _c(h_block, np.float32).ravel()
+    q = _c(codes, np.uint8).ravel()
+    book = np.empty(8, np.uint8)
+    bm = np.empty(8)
+    _load().qo_lut_fit(_ptr(w), _ptr(h), w.size, ctypes.c_float(f), _ptr(q), _ptr(book), _ptr(bm))
+    return book, bm
 
 
 def lut_eval(w_block, h_block, codes, book) -> float:

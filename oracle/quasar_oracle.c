@@ -683,6 +683,22 @@ static double e4m3s_value(int bits)
  * weighted error by direct summation.  margin[i]: the index margin as in
  * int_codes; book_margin[k]: relative distance of the entry's unrounded
  * value to an E4M3 decision boundary.  rho > 0. */
+/* Eq. rubin-fit for fixed indices q on the grid lo + k*s (L3, L4). */
+static void lut_entries(const float* w, const double* hd, int n, double lo, double s,
+                        const uint8_t* q, int* book, double* book_margin)
+{
+    double H[8] = {0}, W[8] = {0};
+    for (int i = 0; i < n; ++i) {
+        H[q[i] & 7] += hd[i];
+        W[q[i] & 7] += hd[i] * (double)w[i];
+    }
+    for (int k = 0; k < 8; ++k) {
+        const double x = H[k] > 0.0 ? W[k] / H[k] : lo + (double)k * s;
+        book[k] = e4m3s_round(x);
+        if (book_margin) book_margin[k] = (x == 0.0) ? HUGE_VAL : e4m3_margin(fabs(x));
+    }
+}
+
 static double lut_candidate(const float* w, const double* hd, int n, double c, double rho,
                             double f, uint8_t* q, int* book, double* margin,
                             double* book_margin)
@@ -690,16 +706,7 @@ static double lut_candidate(const float* w, const double* hd, int n, double c, d
     int_codes(w, n, c, rho, f, 7, q, margin, NULL);
     const double lo = c - f * rho; /* the grid of Eq. 1: lo + k*s */
     const double s = 2.0 * f * rho / 7.0;
-    double H[8] = {0}, W[8] = {0};
-    for (int i = 0; i < n; ++i) {
-        H[q[i]] += hd[i];
-        W[q[i]] += hd[i] * (double)w[i];
-    }
-    for (int k = 0; k < 8; ++k) {
-        const double x = H[k] > 0.0 ? W[k] / H[k] : lo + (double)k * s;
-        book[k] = e4m3s_round(x);
-        if (book_margin) book_margin[k] = (x == 0.0) ? HUGE_VAL : e4m3_margin(fabs(x));
-    }
+    lut_entries(w, hd, n, lo, s, q, book, book_margin);
     double e = 0.0;
     for (int i = 0; i < n; ++i) {
         const double d = e4m3s_value(book[q[i]]) - (double)w[i];
@@ -752,6 +759,27 @@ double qo_lut_block(const float* w, const float* h, int n, float f, uint8_t* q, 
     for (int k = 0; k < 8; ++k) book[k] = (uint8_t)bk[k];
     free(hd);
     return e;
+}
+
+/* The table of given indices on one block for candidate f (the checker's
+ * refit of a GPU result): Eq. rubin-fit with rules D2, L3-L5. */
+void qo_lut_fit(const float* w, const float* h, int n, float f, const uint8_t* q, uint8_t* book,
+                double* book_margin)
+{
+    e4m3_init();
+    double* hd = (double*)malloc(sizeof(double) * (size_t)n);
+    double c, rho;
+    int bk[8];
+    if (!lut_block_setup(w, h, n, hd, &c, &rho)) {
+        for (int k = 0; k < 8; ++k) {
+            bk[k] = e4m3s_round(c);
+            if (book_margin) book_margin[k] = (c == 0.0) ? HUGE_VAL : e4m3_margin(fabs(c));
+        }
+    } else {
+        lut_entries(w, hd, n, c - (double)f * rho, 2.0 * (double)f * rho / 7.0, q, bk, book_margin);
+    }
+    for (int k = 0; k < 8; ++k) book[k] = (uint8_t)bk[k];
+    free(hd);
 }
 
 /* Weighted error of given indices and table on one block (rule D2). */

@@ -21,6 +21,7 @@ const void* int_kernel_nch4(int epl, bool batch, bool adam, bool var);
 const void* nvfp4_kernel(int nch, bool batch);
 const void* amax_kernel(bool batch);
 const void* amax_to_scale_kernel(bool batch);
+const void* lut_kernel();
 }  // namespace quasar
 
 // Per-device status word (bit 0: a kernel timed out on a wait).
@@ -728,6 +729,90 @@ quasar_status quasar_recon_nvfp4_batch_ex(const quasar_nvfp4_tensor* tensors, in
                          &B.t[i], opt.packed);
         }
         if ((st = nvfp4_run(Lp, B, n_clip, s)) != QUASAR_OK) return st;
+    }
+    return QUASAR_OK;
+}
+
+quasar_status quasar_recon_lut_batch(const quasar_lut_tensor* tensors, int n_tensors,
+                                     quasar_dtype g_dtype, float beta2, const float* clip,
+                                     int n_clip, quasar_dtype r_dtype, const quasar_options* options,
+                                     quasar_stream_t stream)
+{
+    Opts opt;
+    if (read_options(options, &opt) != QUASAR_OK) return QUASAR_ERR_INVALID_ARG;
+    if (n_tensors < 0 || (n_tensors > 0 && !tensors)) return QUASAR_ERR_INVALID_ARG;
+    if (n_tensors == 0) return QUASAR_OK;
+    int with_g = 0, non_empty = 0;
+    for (int i = 0; i < n_tensors; ++i)
+        if (tensors[i].rows != 0 && tensors[i].cols != 0) {
+            ++non_empty;
+            with_g += tensors[i].g != nullptr;
+        }
+    if (with_g != 0 && with_g != non_empty) return QUASAR_ERR_INVALID_ARG;
+    const bool has_g = with_g != 0;
+    // one tensor's checks; fills its descriptor (unit0 set later)
+    auto describe = [&](const quasar_lut_tensor& x, LutTensor* T) {
+        int64_t n = 0;
+        quasar_status s1 = check_common(x.w, x.g, g_dtype, x.v, beta2, clip, n_clip, x.rows, x.cols,
+                                        x.r, r_dtype, &n);
+        if (s1 != QUASAR_OK) return s1;
+        if (x.rows % kLutRows != 0 || x.cols % kLutCols != 0) return QUASAR_ERR_INVALID_ARG;
+        const int64_t n_blocks = n / kLutBlock;
+        if (n > 0) {
+            if (!x.book || !aligned16(x.book)) return QUASAR_ERR_INVALID_ARG;
+            if (x.codes && !aligned16(x.codes)) return QUASAR_ERR_INVALID_ARG;
+            const void* outs[] = {x.r, x.codes, x.book, x.cand_idx};
+            const size_t bytes[] = {(size_t)n * dtype_size(r_dtype),
+                                    x.codes ? (opt.packed ? (size_t)n / 8 * 3 : (size_t)n) : 0,
+                                    (size_t)n_blocks * 8, x.cand_idx ? (size_t)n_blocks : 0};
+            if (outputs_alias_inputs(x.w, x.g, g_dtype, x.v, n, outs, bytes, 4))
+                return QUASAR_ERR_INVALID_ARG;
+        }
+        *T = LutTensor{x.w, x.g, x.v, x.r, x.codes, x.book, x.cand_idx, x.cols, n_blocks, 0};
+        return QUASAR_OK;
+    };
+    static thread_local LutLaunch<kMaxBatch> Lp;
+    int64_t total = 0;
+    quasar_status st;
+    for (int i = 0; i < n_tensors; ++i) {
+        LutTensor T;
+        if ((st = describe(tensors[i], &T)) != QUASAR_OK) return st;
+        total += T.n_blocks;
+    }
+    if (total == 0) return QUASAR_OK;
+    LutParams& p = Lp.p;
+    p = LutParams{};
+    p.g_kind = has_g ? (g_dtype == QUASAR_BF16 ? 2 : 1) : 0;
+    p.r_bf16 = r_dtype == QUASAR_BF16;
+    p.h_mode = opt.h_mode;
+    p.codes_packed = opt.packed;
+    p.n_clip = n_clip;
+    p.beta2 = beta2;
+    p.c1 = 1.0f - beta2;
+    // summation depth of the per-index sums: 8 per packed half, the fold,
+    // 8 per reader accumulator and two combining levels, plus margin
+    p.tie_kappa = 24.0f * tuning().tie_scale;
+    p.timeout_ns = kDefaultTimeoutNs;
+    p.force_timeout_ns = (uint64_t)std::max<int64_t>(0, g_force_timeout_ns.load());
+    p.stats = g_stats.load();
+    fill_clip(clip, n_clip, p.f, p.invf);
+    if ((st = status_ptr(&p.status)) != QUASAR_OK) return st;
+    const int gbytes = p.g_kind == 2 ? 2 : (p.g_kind == 1 ? 4 : 0);
+    const Launch L = plan((uint32_t)(kLutBlock * (8 + gbytes)), kLutScratchBytes);
+    p.stages = L.stages;
+    p.stage_bytes = L.stage_bytes;
+    const cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+    for (int i0 = 0; i0 < n_tensors; i0 += kMaxBatch) {
+        Lp.n_t = std::min(kMaxBatch, n_tensors - i0);
+        int64_t units = 0;
+        for (int i = 0; i < Lp.n_t; ++i) {
+            describe(tensors[i0 + i], &Lp.t[i]);
+            Lp.t[i].unit0 = units;
+            units += Lp.t[i].n_blocks;
+        }
+        Lp.n_units = units;
+        if (units == 0) continue;
+        if ((st = launch_persistent(lut_kernel(), &Lp, L.smem, units, s)) != QUASAR_OK) return st;
     }
     return QUASAR_OK;
 }

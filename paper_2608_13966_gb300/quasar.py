@@ -48,6 +48,7 @@ PROTOTYPES = {
                                           _I, _P, _P]),
     "quasar_recon_nvfp4_batch": (_I, [_P, _I, _I, _F, _P, _I, _I, _P]),
     "quasar_recon_nvfp4_batch_ex": (_I, [_P, _I, _I, _F, _P, _I, _I, _P, _P]),
+    "quasar_recon_lut_batch": (_I, [_P, _I, _I, _F, _P, _I, _I, _P, _P]),
     "quasar_tensor_amax": (_I, [_P, _I64, _P, _P]),
     "quasar_get_device_status": (_I, [_P]),
     "quasar_debug_force_timeout": (None, [_I64]),
@@ -277,6 +278,36 @@ def quasar_recon_nvfp4_batch_ex(tensors, beta2, clip, options=None, g_dtype=BF16
     st = lib.quasar_recon_nvfp4_batch_ex(ctypes.cast(tensors, ctypes.c_void_p), len(tensors),
                                          g_dtype, beta2, carr, nclip, r_dtype, _opt_ptr(options),
                                          _stream(stream))
+    return QuasarStatus(st)
+
+
+class QuasarLutTensor(ctypes.Structure):
+    """quasar_lut_tensor: one tensor's buffers (device pointers) and shape."""
+    _fields_ = [("w", ctypes.c_void_p), ("g", ctypes.c_void_p), ("v", ctypes.c_void_p),
+                ("r", ctypes.c_void_p), ("codes", ctypes.c_void_p), ("book", ctypes.c_void_p),
+                ("cand_idx", ctypes.c_void_p), ("rows", ctypes.c_int64), ("cols", ctypes.c_int64)]
+
+
+def lut_tensor_array(items):
+    """A ctypes array of QuasarLutTensor from dicts with keys w, g, v, r,
+    codes, book, cand_idx (tensors, pointers or None), rows, cols."""
+    arr = (QuasarLutTensor * len(items))()
+    for i, d in enumerate(items):
+        arr[i] = QuasarLutTensor(_ptr(d["w"]), _ptr(d.get("g")), _ptr(d["v"]), _ptr(d["r"]),
+                                 _ptr(d.get("codes")), _ptr(d["book"]), _ptr(d.get("cand_idx")),
+                                 int(d["rows"]), int(d["cols"]))
+    return arr
+
+
+def quasar_recon_lut_batch(tensors, beta2, clip, options=None, g_dtype=BF16, r_dtype=BF16,
+                           stream=None) -> QuasarStatus:
+    """tensors: a ctypes array from lut_tensor_array (or a list of dicts)."""
+    lib = load()
+    if not isinstance(tensors, ctypes.Array):
+        tensors = lut_tensor_array(tensors)
+    carr, nclip = _clip_array(clip)
+    st = lib.quasar_recon_lut_batch(ctypes.cast(tensors, ctypes.c_void_p), len(tensors), g_dtype,
+                                    beta2, carr, nclip, r_dtype, _opt_ptr(options), _stream(stream))
     return QuasarStatus(st)
 
 

@@ -223,3 +223,28 @@ def test_options_validation(lib):
                                        Q.options("ema", True), stream=0) == st.ERR_INVALID_ARG
     assert Q.quasar_recon_nvfp4_batch_ex([_ndesc(codes=C - 496)], 0.999, CLIP,
                                          Q.options("ema", True), stream=0) == st.ERR_INVALID_ARG
+
+
+def _ldesc(**kw):
+    d = dict(w=A, g=B, v=C, r=D, codes=None, book=E, cand_idx=None, rows=8, cols=128)
+    d.update(kw)
+    return d
+
+
+@pytest.mark.parametrize("kw,expect", [
+    (dict(items=[]), Q.QuasarStatus.OK),
+    (dict(items=[_ldesc(rows=0)]), Q.QuasarStatus.OK),                      # empty: no-op
+    (dict(items=[_ldesc(rows=12)]), Q.QuasarStatus.ERR_INVALID_ARG),        # rows % 8
+    (dict(items=[_ldesc(cols=96)]), Q.QuasarStatus.ERR_INVALID_ARG),        # cols % 64
+    (dict(items=[_ldesc(book=None)]), Q.QuasarStatus.ERR_INVALID_ARG),
+    (dict(items=[_ldesc(book=E + 8)]), Q.QuasarStatus.ERR_INVALID_ARG),     # misaligned
+    (dict(items=[_ldesc(book=C + 64)]), Q.QuasarStatus.ERR_INVALID_ARG),    # book overlaps v
+    (dict(items=[_ldesc(r=A + 256)]), Q.QuasarStatus.ERR_INVALID_ARG),      # r overlaps w
+    (dict(items=[_ldesc(), _ldesc(g=None)]), Q.QuasarStatus.ERR_INVALID_ARG),
+    (dict(items=[_ldesc()], beta2=1.0), Q.QuasarStatus.ERR_INVALID_ARG),
+    (dict(items=[_ldesc()], opt=Q.options(9)), Q.QuasarStatus.ERR_INVALID_ARG),
+])
+def test_lut_argument_validation(lib, kw, expect):
+    items = kw.pop("items")
+    assert Q.quasar_recon_lut_batch(items, kw.get("beta2", 0.999), CLIP, kw.get("opt"),
+                                    stream=0) == expect

@@ -60,11 +60,11 @@ MUTANTS = {
     "AdamW without bias correction": ("lr * ((double)mi / bc1) / denom", "lr * (double)mi / denom"),
     "AdamW coupled weight decay": ("(double)w[i] * (1.0 - lr * wd) - lr", "(double)w[i] - lr * wd - lr"),
     "AdamW eps inside the root": ("sqrt((double)vi / bc2) + eps", "sqrt((double)vi / bc2 + eps)"),
-    "LUT entry unweighted mean": ("W[q[i]] += hd[i] * (double)w[i];", "W[q[i]] += (double)w[i];"),
+    "LUT entry unweighted mean": ("W[q[i] & 7] += hd[i] * (double)w[i];", "W[q[i] & 7] += (double)w[i];"),
     "LUT entry sign dropped": ("return (x < 0.0 && mag != 0) ? (0x80 | mag) : mag;", "return mag;"),
     "LUT empty index at grid offset": ("lo + (double)k * s;", "lo + (double)(k + 1) * s;"),
-    "LUT error at unrounded entry": ("const double d = e4m3s_value(book[q[i]]) - (double)w[i];\n        e += hd[i] * d * d;\n    }\n    return e;\n}\n\n/* Block range",
-                                     "const double d = (H[q[i]] > 0.0 ? W[q[i]] / H[q[i]] : 0.0) - (double)w[i];\n        e += hd[i] * d * d;\n    }\n    return e;\n}\n\n/* Block range"),
+    "LUT error at the grid point": ("const double d = e4m3s_value(book[q[i]]) - (double)w[i];\n        e += hd[i] * d * d;\n    }\n    return e;\n}\n\n/* Block range",
+                                    "const double d = (lo + (double)q[i] * s) - (double)w[i];\n        e += hd[i] * d * d;\n    }\n    return e;\n}\n\n/* Block range"),
 }
 
 PIN_TESTS = [
@@ -108,7 +108,7 @@ def test_pins_catch_planted_mistake(oracle, tmp_path, name):
     # give the mutant the same prototypes as the real library
     for sym in ("qo_ema", "qo_adamw", "qo_recon_int", "qo_refit_int", "qo_codes_int", "qo_tensor_scale",
                 "qo_recon_nvfp4", "qo_e2m1_round", "qo_e4m3_round", "qo_e4m3_value",
-                "qo_set_threads", "qo_get_threads", "qo_recon_lut", "qo_lut_block", "qo_lut_eval"):
+                "qo_set_threads", "qo_get_threads", "qo_recon_lut", "qo_lut_block", "qo_lut_eval", "qo_lut_fit"):
         f_real, f_mut = getattr(real, sym), getattr(lib, sym)
         f_mut.argtypes, f_mut.restype = f_real.argtypes, f_real.restype
     caught = []

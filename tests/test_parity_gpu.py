@@ -449,3 +449,97 @@ def test_adamw_with_options(oracle):
            "codes": q, "idx": o["cand_idx"].cpu().numpy()}
     rep = checker.check_int(oracle, w1, h, 3, CLIP8, O, gpu, 128, True)
     assert rep["ok"], json.dumps(rep)
+
+
+# ------------------------------------------------ Rubin INT3 LUT (App. B)
+
+def _lut_run(oracle, shapes, seed0, clip, saliency="ema", packed=False, g_dtype=torch.bfloat16,
+             r_dtype=torch.bfloat16, g_none=False):
+    from paper_2608_13966_gb300 import api
+    items, hosts = [], []
+    for i, (rows, cols) in enumerate(shapes):
+        w, g, v = _inputs(rows, cols, seed=seed0 + i, g_dtype=g_dtype)
+        if g_none:
+            g = None
+        items.append((w, g, v))
+        hosts.append((H._host(w), None if g is None else H._host(g), H._host(v)))
+    outs = api.recon_lut_batch(items, clip=clip, codes=True, saliency=saliency,
+                               packed_codes=packed, r_dtype=r_dtype)
+    torch.cuda.synchronize()
+    for (rows, cols), o, (w_h, g_h, v_h), it in zip(shapes, outs, hosts, items):
+        v1 = oracle.ema(v_h, g_h, 0.999) if g_h is not None else v_h
+        h = oracle.saliency(v1, saliency)
+        w2, h2 = w_h.reshape(rows, cols), h.reshape(rows, cols)
+        O = oracle.recon_lut(w2, h2, clip)
+        if packed:
+            nb = rows * cols // 512
+            qb = oracle.unpack_int_codes(o["codes"].cpu().numpy(), 3, nb * 512).reshape(nb, 512)
+            # block order -> tensor layout
+            codes = qb.reshape(rows // 8, cols // 64, 8, 64).transpose(0, 2, 1, 3).reshape(rows, cols)
+        else:
+            codes = o["codes"].cpu().numpy()
+        gpu = {"r": H._host(o["r"]), "book": o["book"].cpu().numpy(), "codes": codes,
+               "idx": o["cand_idx"].cpu().numpy()}
+        rep = checker.check_lut(oracle, w2, h2, clip, O, gpu)
+        assert rep["ok"], json.dumps(rep)
+        ema = checker.check_ema(v1, H._host(it[2]))
+        assert ema["ok"], json.dumps(ema)
+
+
+def test_lut_batch_shapes(oracle):
+    """Several tensors of different block counts, 8 candidates."""
+    _lut_run(oracle, [(64, 512), (8, 64), (16, 1024), (24, 192)], 1100, CLIP8)
+
+
+@pytest.mark.parametrize("K", [1, 5, 16, 32])
+def test_lut_candidate_counts(oracle, K):
+    clip = [round(1.0 - 0.7 * i / max(K - 1, 1), 4) for i in range(K)]
+    _lut_run(oracle, [(32, 512)], 1200 + K, clip)
+
+
+def test_lut_variants(oracle):
+    """fp32 gradient and output, no gradient, h = v'^2, uniform h, packed
+    indices."""
+    _lut_run(oracle, [(16, 256)], 1300, CLIP8, g_dtype=torch.float32, r_dtype=torch.float32)
+    _lut_run(oracle, [(16, 256)], 1301, CLIP8, g_none=True)
+    _lut_run(oracle, [(16, 256)], 1302, CLIP8, saliency="ema_squared")
+    _lut_run(oracle, [(16, 256)], 1303, CLIP8, saliency="uniform")
+    _lut_run(oracle, [(16, 256), (8, 64)], 1304, CLIP8, packed=True)
+
+
+def test_lut_degenerate_blocks(oracle):
+    from paper_2608_13966_gb300 import api
+    w, g, v = _inputs(16, 256, seed=1400)
+    w[:8, :64] = 0.0123                  # zero range
+    v[:8, 64:128] = 0.0
+    g[:8, 64:128] = 0.0                  # all saliency zero
+    w[8:, :64] = torch.linspace(-1, 1, 512, device="cuda").reshape(8, 64)  # on grid boundaries
+    w[8:, 64:128] = 0.0
+    w[8, 64] = 1.0                       # one outlier, everything else equal
+    w_h, g_h, v_h = H._host(w), H._host(g), H._host(v)
+    o = api.recon_lut_batch([(w, g, v)], clip=CLIP8, codes=True)[0]
+    torch.cuda.synchronize()
+    h = oracle.ema(v_h, g_h, 0.999).reshape(16, 256)
+    O = oracle.recon_lut(w_h.reshape(16, 256), h, CLIP8)
+    gpu = {"r": H._host(o["r"]), "book": o["book"].cpu().numpy(), "codes": o["codes"].cpu().numpy(),
+           "idx": o["cand_idx"].cpu().numpy()}
+    rep = checker.check_lut(oracle, w_h.reshape(16, 256), h, CLIP8, O, gpu)
+    assert rep["ok"], json.dumps(rep)
+
+
+def test_lut_paper_shaped_layer(oracle):
+    """A full Llama-3.1-8B-shaped layer (7 tensors, 426k blocks) in one launch."""
+    from paper_2608_13966_gb300 import api
+    w_ = wl.workload("llama_layer_int3")
+    ds = [wl.make_tensor(w_, spec, device="cuda") for spec in w_.tensors]
+    hosts = [tuple(H._host(d[k]) for k in ("w", "g", "v")) for d in ds]
+    outs = api.recon_lut_batch([(d["w"], d["g"], d["v"]) for d in ds], clip=list(w_.clip),
+                               codes=True)
+    torch.cuda.synchronize()
+    for spec, d, o, (w_h, g_h, v_h) in zip(w_.tensors, ds, outs, hosts):
+        h = oracle.ema(v_h, g_h, w_.beta2).reshape(spec.rows, spec.cols)
+        O = oracle.recon_lut(w_h.reshape(spec.rows, spec.cols), h, list(w_.clip))
+        gpu = {"r": H._host(o["r"]), "book": o["book"].cpu().numpy(),
+               "codes": o["codes"].cpu().numpy(), "idx": o["cand_idx"].cpu().numpy()}
+        rep = checker.check_lut(oracle, w_h.reshape(spec.rows, spec.cols), h, list(w_.clip), O, gpu)
+        assert rep["ok"], (spec.name, json.dumps(rep))
