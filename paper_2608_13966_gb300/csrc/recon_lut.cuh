@@ -9,11 +9,11 @@
 //
 // One warp owns one block: lane L holds block elements 16 L .. 16 L + 15
 // (row L / 4, columns 16 (L % 4) ..), read once from a per-warp TMA ring.
-// Per candidate each lane accumulates, for every index j, H_j = sum h,
-// W_j = sum h (w - g_j) and Q_j = sum h (w - g_j)^2 about the index's grid
-// point g_j (one-hot masks, packed f32x2); the 24 sums are transposed through
-// shared memory, and lane j forms entry j and its share of the error,
-//   S_j = H_j d_j^2 - 2 d_j W_j + Q_j,   d_j = C_j - g_j.
+// Per candidate each lane accumulates, for every index j, H_j = sum h and
+// W_j = sum h (w - g_j) about the index's grid point g_j (one-hot masks,
+// packed f32x2), and Q = sum h (w - g_q)^2 over all elements; the 17 sums are
+// transposed through shared memory, lane j forms entry j, and the error is
+//   sum_j (H_j d_j^2 - 2 d_j W_j) + Q,   d_j = C_j - g_j.
 // Both the entry's rounding and the error carry an fp32 bound.  Candidates
 // within the bound of the best, and undecided roundings, are settled exactly
 // (float-float sums, whole warp), so indices, tables and the kept candidate
@@ -182,7 +182,8 @@ __global__ void __launch_bounds__(256, 2) k_recon_lut(const __grid_constant__ Lu
     }
     __syncwarp();
 
-    // the 8 row segments of a block, each of w, v and g
+    // the 8 row segments of a block, each of w, v and g: lane 0 announces
+    // the bytes, lane r copies row r (every lane calls it)
     auto issue = [&](int64_t u, int s) {
         int tj = ti;
         tensor_of(u, tj);
@@ -191,8 +192,10 @@ __global__ void __launch_bounds__(256, 2) k_recon_lut(const __grid_constant__ Lu
         const int64_t nbc = T.cols / kLutCols;
         const int64_t base = (b / nbc) * kLutRows * T.cols + (b % nbc) * kLutCols;
         unsigned char* st = ring + (size_t)s * p.stage_bytes;
-        mbar_arrive_expect_tx(&bars[s], (uint32_t)kLutBlock * (8u + (uint32_t)gbytes));
-        for (int r = 0; r < kLutRows; ++r) {
+        if (lane == 0) mbar_arrive_expect_tx(&bars[s], (uint32_t)kLutBlock * (8u + (uint32_t)gbytes));
+        __syncwarp();
+        if (lane < kLutRows) {
+            const int r = lane;
             const int64_t off = base + r * T.cols;
             bulk_g2s(st + r * kLutCols * 4, T.w + off, kLutCols * 4, &bars[s]);
             bulk_g2s(st + kVOff + r * kLutCols * 4, T.v + off, kLutCols * 4, &bars[s]);
@@ -211,11 +214,10 @@ __global__ void __launch_bounds__(256, 2) k_recon_lut(const __grid_constant__ Lu
         }
     };
 
-    if (lane == 0)
-        for (int s = 0; s < S; ++s) {
-            const int64_t u = first + s * stride;
-            if (u < n_units) issue(u, s);
-        }
+    for (int s = 0; s < S; ++s) {
+        const int64_t u = first + s * stride;
+        if (u < n_units) issue(u, s);
+    }
     if (p.force_timeout_ns && blockIdx.x == 0 && warp == 0) {
         if (!mbar_wait_bounded(&bars[S], 0, p.force_timeout_ns)) {
             fail(0);
@@ -278,7 +280,7 @@ __global__ void __launch_bounds__(256, 2) k_recon_lut(const __grid_constant__ Lu
         }
         // the block is in registers: release the stage
         __syncwarp();
-        if (lane == 0) {
+        {
             const int64_t un = u + (int64_t)S * stride;
             if (un < n_units) issue(un, s_cur);
         }
@@ -324,9 +326,9 @@ __global__ void __launch_bounds__(256, 2) k_recon_lut(const __grid_constant__ Lu
                 const float P = R * p.invf[k];
                 const float sg = __fdividef(1.0f, P);  // the grid step
                 const float2 P2 = make_float2(P, P), nsg2 = make_float2(-sg, -sg);
-                float2 Hs[8], Ws[8], Qs[8];
+                float2 Hs[8], Ws[8], Qt = make_float2(0.0f, 0.0f);
 #pragma unroll
-                for (int j = 0; j < 8; ++j) Hs[j] = Ws[j] = Qs[j] = make_float2(0.0f, 0.0f);
+                for (int j = 0; j < 8; ++j) Hs[j] = Ws[j] = make_float2(0.0f, 0.0f);
 #pragma unroll
                 for (int t = 0; t < 8; ++t) {
                     const float2 d = __fadd2_rn(w2[t], nc2);
@@ -338,14 +340,13 @@ __global__ void __launch_bounds__(256, 2) k_recon_lut(const __grid_constant__ Lu
                     const float2 z = make_float2(copysignf(za.x, d.x), copysignf(za.y, d.y));
                     const float2 e = __ffma2_rn(z, nsg2, d);  // w - g_j, g_j = c + z sg
                     const float2 he = __fmul2_rn(h2[t], e);
-                    const float2 hee = __fmul2_rn(he, e);
+                    Qt = __ffma2_rn(he, e, Qt);
 #pragma unroll
                     for (int j = 0; j < 8; ++j) {
                         const float zj = (float)j - 3.5f;
                         const float2 m = make_float2(z.x == zj ? 1.0f : 0.0f, z.y == zj ? 1.0f : 0.0f);
                         Hs[j] = __ffma2_rn(m, h2[t], Hs[j]);
                         Ws[j] = __ffma2_rn(m, he, Ws[j]);
-                        Qs[j] = __ffma2_rn(m, hee, Qs[j]);
                     }
                 }
                 // transpose: row q of the scratch holds sum q of every lane
@@ -353,11 +354,11 @@ __global__ void __launch_bounds__(256, 2) k_recon_lut(const __grid_constant__ Lu
                 for (int j = 0; j < 8; ++j) {
                     sums[j * 33 + lane] = Hs[j].x + Hs[j].y;
                     sums[(8 + j) * 33 + lane] = Ws[j].x + Ws[j].y;
-                    sums[(16 + j) * 33 + lane] = Qs[j].x + Qs[j].y;
                 }
+                sums[16 * 33 + lane] = Qt.x + Qt.y;
                 __syncwarp();
                 float tot = 0.0f;
-                if (lane < 24) {
+                if (lane < 17) {
                     float a0 = 0.0f, a1 = 0.0f, a2 = 0.0f, a3 = 0.0f;
 #pragma unroll
                     for (int i = 0; i < 32; i += 4) {
@@ -373,9 +374,14 @@ __global__ void __launch_bounds__(256, 2) k_recon_lut(const __grid_constant__ Lu
                 const int j = lane & 7;
                 const float Hj = tot;
                 const float Wj = __shfl_sync(0xffffffffu, tot, j + 8);
-                const float Qj = __shfl_sync(0xffffffffu, tot, j + 16);
+                const float Qt1 = __shfl_sync(0xffffffffu, tot, 16);
                 const float gj = fmaf((float)j - 3.5f, sg, c);
-                const float A = sqrtf(fmaxf(Hj * Qj, 0.0f));  // >= sum h |w - g|
+                // A >= sum over index j of h |w - g_j|: |w - g_j| <= sg/2 inside
+                // the range, and up to (1 - f) rho + sg/2 for the clamped ends
+                const float emax = (j == 0 || j == 7)
+                                       ? fmaf(0.5f * range, fmaxf(1.0f - p.f[k], 0.0f), 0.5f * sg)
+                                       : 0.5f * sg;
+                const float A = Hj * (emax * (1.0f + 8.0f * kU) + eps_e);
                 float mean = gj, dm = 4.0f * kU * fabsf(gj);
                 if (Hj > 0.0f) {
                     const float q = __fdividef(Wj, Hj);
@@ -385,9 +391,9 @@ __global__ void __launch_bounds__(256, 2) k_recon_lut(const __grid_constant__ Lu
                 const uint32_t cb = e4m3_encode(mean);
                 const bool amb = e4m3_encode(mean - dm) != e4m3_encode(mean + dm);
                 const float dd = e4m3_decode(cb) - gj;
-                const float Sj = fmaf(Hj * dd, dd, fmaf(-2.0f * dd, Wj, Qj));
-                float bj = (gam + 4.0f * kU) * (Hj * dd * dd + 2.0f * fabsf(dd) * A + Qj) +
-                           2.0f * eps_e * (fabsf(dd) * Hj + A);
+                const float Sj = fmaf(Hj * dd, dd, -2.0f * dd * Wj);
+                float bj = (gam + 4.0f * kU) * (Hj * dd * dd + 2.0f * fabsf(dd) * A) +
+                           2.0f * eps_e * (fabsf(dd) * Hj + 2.0f * A);
                 if (amb)  // the other rounding differs by at most this much
                     bj += 2.0f * Hj * dm *
                           fabsf(e4m3_decode(e4m3_encode(mean + dm)) - e4m3_decode(e4m3_encode(mean - dm)));
@@ -398,6 +404,8 @@ __global__ void __launch_bounds__(256, 2) k_recon_lut(const __grid_constant__ Lu
                     E += __shfl_xor_sync(0xffffffffu, E, o);
                     dE += __shfl_xor_sync(0xffffffffu, dE, o);
                 }
+                E += Qt1;
+                dE += (gam + 4.0f * kU) * Qt1 + 4.0f * kU * fabsf(E);
 #pragma unroll
                 for (int o = 2; o; o >>= 1) wb |= __shfl_xor_sync(0xffffffffu, wb, o);
                 const uint32_t wb1 = __shfl_sync(0xffffffffu, wb, 4);
