@@ -87,6 +87,8 @@ def bytes_per_step(wlo, elements):
     also reads m and writes w' and m' (12 more bytes a weight)."""
     if wlo.fmt == "int" and wlo.adamw:
         return elements * 28 + (elements // wlo.group) * 9
+    if wlo.fmt == "nvfp4" and wlo.adamw:  # AdamW + absmax pass, then w', v' -> r
+        return elements * 26 + elements * 10 + (elements // 16) * 2
     if wlo.fmt == "lut":  # per 512-block: 8 table bytes and the kept index
         return elements * 16 + (elements // 512) * 9
     if wlo.fmt == "int":
@@ -128,7 +130,24 @@ class Step:
         self.stream = stream.cuda_stream
         self.clip = (ctypes.c_float * len(wlo.clip))(*wlo.clip)
         self.calls = []
-        if wlo.adamw:
+        if wlo.adamw and wlo.fmt == "nvfp4":
+            # AdamW step taking the absmax of w', then the NVFP4 batch
+            for d in model.tensors:
+                if "m" not in d:
+                    spec = d["spec"]
+                    d["m"] = WL.first_moment((spec.rows, spec.cols), model.seed * 1000 + spec.index,
+                                             d["w"].device)
+            hp = wlo.adamw
+            self.descs = Q.adamw_nvfp4_tensor_array([
+                {"w": d["w"], "g": d["g"], "m": d["m"], "v": d["v"], "r": d["r"], "codes": None,
+                 "block_scale": d["scale"], "tensor_scale": d["ts"], "cand_idx": d["idx"],
+                 "rows": d["spec"].rows, "cols": d["spec"].cols}
+                for d in model.tensors])
+            args = (ctypes.cast(self.descs, ctypes.c_void_p), len(self.descs), Q.BF16, hp["lr"],
+                    hp["beta1"], wlo.beta2, hp["eps"], hp["weight_decay"], hp["step"], self.clip,
+                    len(wlo.clip), Q.BF16, None, self.stream)
+            self.calls.append((self.lib.quasar_adamw_recon_nvfp4_batch, args, model.elements))
+        elif wlo.adamw:
             # AdamW step + reconstruction of every tensor in one launch
             # (quasar_adamw_recon_int_batch); m is drawn here if the model
             # was built for a workload without an optimizer step
@@ -422,7 +441,8 @@ def main():
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--workload", default="llama_int3")
-    ap.add_argument("--sweep", default="llama_int2,llama_int4,llama_nvfp4,llama_int3_adamw,llama_lut")
+    ap.add_argument("--sweep", default="llama_int2,llama_int4,llama_nvfp4,llama_int3_adamw,"
+                                       "llama_nvfp4_adamw,llama_lut")
     ap.add_argument("--sweep-steps", type=int, default=10)
     ap.add_argument("--e2e-steps", type=int, default=2)
     ap.add_argument("--cpu-budget", type=float, default=12.0)

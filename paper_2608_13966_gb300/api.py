@@ -5,8 +5,9 @@ from __future__ import annotations
 
 import torch
 
-from .quasar import (BF16, F32, QuasarError, QuasarStatus, adamw_tensor_array, int_tensor_array,
-                     lut_tensor_array, nvfp4_tensor_array, options, quasar_adamw_recon_int_batch,
+from .quasar import (BF16, F32, QuasarError, QuasarStatus, adamw_nvfp4_tensor_array,
+                     adamw_tensor_array, int_tensor_array, lut_tensor_array, nvfp4_tensor_array,
+                     options, quasar_adamw_recon_int_batch, quasar_adamw_recon_nvfp4_batch,
                      quasar_recon_int, quasar_recon_int_batch_ex, quasar_recon_lut_batch,
                      quasar_recon_nvfp4, quasar_recon_nvfp4_batch_ex, quasar_tensor_amax)
 
@@ -193,6 +194,41 @@ def recon_nvfp4_batch(items, *, clip, beta2=0.999, r_dtype=torch.bfloat16, codes
     _check(quasar_recon_nvfp4_batch_ex(nvfp4_tensor_array(descs), beta2, clip,
                                        options(saliency, packed_codes), g_dtype=g_dtype,
                                        r_dtype=rd, stream=stream))
+    return results
+
+
+def adamw_recon_nvfp4_batch(items, *, lr, step, clip, beta1=0.9, beta2=0.999, eps=1e-8,
+                            weight_decay=0.0, r_dtype=torch.bfloat16, codes=False, cand_idx=True,
+                            saliency="ema", packed_codes=False, stream=None):
+    """One AdamW step, then the NVFP4 reconstruction of the updated weights
+    (the step's pass also takes each tensor's absmax of w').  items: list of
+    (w, g, m, v) CUDA tensors; w, m and v are updated in place.  Returns one
+    result dict per tensor, as recon_nvfp4 does."""
+    descs, results = [], []
+    g_dtype = F32
+    for w, g, m, v in items:
+        _check_2d(w)
+        rows, cols = w.shape
+        dev = w.device
+        n_blocks = rows * cols // 16
+        res = {"r": torch.empty((rows, cols), dtype=r_dtype, device=dev),
+               "block_scale": torch.empty(n_blocks, dtype=torch.uint8, device=dev),
+               "tensor_scale": torch.empty(1, dtype=torch.float32, device=dev)}
+        if codes:
+            res["codes"] = (torch.empty(rows * cols // 2, dtype=torch.uint8, device=dev) if packed_codes
+                            else torch.empty((rows, cols), dtype=torch.uint8, device=dev))
+        if cand_idx:
+            res["cand_idx"] = torch.empty(n_blocks, dtype=torch.uint8, device=dev)
+        if g is not None and g.dtype == torch.bfloat16:
+            g_dtype = BF16
+        descs.append({"w": w, "g": g, "m": m, "v": v, "r": res["r"], "codes": res.get("codes"),
+                      "block_scale": res["block_scale"], "tensor_scale": res["tensor_scale"],
+                      "cand_idx": res.get("cand_idx"), "rows": rows, "cols": cols})
+        results.append(res)
+    rd = BF16 if r_dtype == torch.bfloat16 else F32
+    _check(quasar_adamw_recon_nvfp4_batch(adamw_nvfp4_tensor_array(descs), lr, beta1, beta2, eps,
+                                          weight_decay, step, clip, g_dtype=g_dtype, r_dtype=rd,
+                                          options=options(saliency, packed_codes), stream=stream))
     return results
 
 

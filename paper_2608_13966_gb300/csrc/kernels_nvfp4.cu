@@ -1,5 +1,6 @@
 // Instantiations of the NVFP4 kernel (1, 2 or 4 chunks of 8 candidates) and
 // of the tensor-absmax kernels.
+#include "recon_adamw.cuh"
 #include "recon_nvfp4.cuh"
 
 namespace quasar {
@@ -22,6 +23,8 @@ const void* amax_kernel(bool batch)
     return batch ? reinterpret_cast<const void*>(&k_amax<kMaxBatch>)
                  : reinterpret_cast<const void*>(&k_amax<1>);
 }
+
+const void* adamw_amax_kernel() { return reinterpret_cast<const void*>(&k_adamw_amax<kMaxBatch>); }
 
 const void* amax_to_scale_kernel(bool batch)
 {

@@ -191,4 +191,32 @@ struct AmaxBatch {
     AmaxItem t[MAXT];
 };
 
+// One tensor of the AdamW step that also takes the absmax of w' (the NVFP4
+// side of the fused step): w, m, v updated in place, max |w'| into *slot.
+struct AdamwItem {
+    float* w;
+    const void* g;
+    float* m;
+    float* v;
+    int64_t n;
+    float* slot;
+};
+
+struct AdamwHp {
+    int g_kind;            // 1 fp32, 2 bf16
+    float beta1, c1b;      // beta1, 1 - beta1
+    float beta2, c1;       // beta2, 1 - beta2
+    float lr_wd;           // lr * weight_decay
+    float step_size;       // lr / (1 - beta1^t)
+    float isbc2;           // 1 / sqrt(1 - beta2^t)
+    float eps;
+};
+
+template <int MAXT>
+struct AdamwBatch {
+    AdamwHp hp;
+    int n_t;
+    AdamwItem t[MAXT];
+};
+
 }  // namespace quasar

@@ -22,6 +22,7 @@ const void* nvfp4_kernel(int nch, bool batch);
 const void* amax_kernel(bool batch);
 const void* amax_to_scale_kernel(bool batch);
 const void* lut_kernel();
+const void* adamw_amax_kernel();
 }  // namespace quasar
 
 // Per-device status word (bit 0: a kernel timed out on a wait).
@@ -472,16 +473,21 @@ quasar_status launch_amax(const AmaxBatch<MAXT>& B, cudaStream_t s)
     return QUASAR_OK;
 }
 
+// amax_done: the slots already hold each tensor's absmax (the fused AdamW
+// step took it), so only the scale pass and the reconstruction remain.
 template <int MAXT>
-quasar_status nvfp4_run(Nvfp4Launch<MAXT>& Lp, AmaxBatch<MAXT>& B, int n_clip, cudaStream_t s)
+quasar_status nvfp4_run(Nvfp4Launch<MAXT>& Lp, AmaxBatch<MAXT>& B, int n_clip, cudaStream_t s,
+                        bool amax_done = false)
 {
-    // scale slots of tensors whose amax is computed start at 0
-    for (int i = 0; i < B.n_t; ++i)
-        if (!B.t[i].amax_in &&
-            cudaMemsetAsync(B.t[i].slot, 0, sizeof(float), s) != cudaSuccess)
-            return QUASAR_ERR_CUDA;
-    quasar_status st = launch_amax(B, s);
-    if (st != QUASAR_OK) return st;
+    quasar_status st;
+    if (!amax_done) {
+        // scale slots of tensors whose amax is computed start at 0
+        for (int i = 0; i < B.n_t; ++i)
+            if (!B.t[i].amax_in &&
+                cudaMemsetAsync(B.t[i].slot, 0, sizeof(float), s) != cudaSuccess)
+                return QUASAR_ERR_CUDA;
+        if ((st = launch_amax(B, s)) != QUASAR_OK) return st;
+    }
     {
         void* args[] = {(void*)&B};
         if (cudaLaunchKernel(amax_to_scale_kernel(MAXT > 1), dim3(1), dim3(256), args, 0, s) !=
@@ -813,6 +819,101 @@ quasar_status quasar_recon_lut_batch(const quasar_lut_tensor* tensors, int n_ten
         Lp.n_units = units;
         if (units == 0) continue;
         if ((st = launch_persistent(lut_kernel(), &Lp, L.smem, units, s)) != QUASAR_OK) return st;
+    }
+    return QUASAR_OK;
+}
+
+quasar_status quasar_adamw_recon_nvfp4_batch(const quasar_adamw_nvfp4_tensor* tensors,
+                                             int n_tensors, quasar_dtype g_dtype, float lr,
+                                             float beta1, float beta2, float eps,
+                                             float weight_decay, int64_t step, const float* clip,
+                                             int n_clip, quasar_dtype r_dtype,
+                                             const quasar_options* options, quasar_stream_t stream)
+{
+    Opts opt;
+    if (read_options(options, &opt) != QUASAR_OK) return QUASAR_ERR_INVALID_ARG;
+    if (n_tensors < 0 || (n_tensors > 0 && !tensors)) return QUASAR_ERR_INVALID_ARG;
+    if (!(std::isfinite(lr) && lr >= 0.0f) || !(beta1 >= 0.0f && beta1 < 1.0f) ||
+        !(std::isfinite(eps) && eps > 0.0f) ||
+        !(std::isfinite(weight_decay) && weight_decay >= 0.0f) || step < 1 || !valid_dtype(g_dtype))
+        return QUASAR_ERR_INVALID_ARG;
+    if (n_tensors == 0) return QUASAR_OK;
+    // one tensor: the reconstruction's checks (without a gradient: v is
+    // updated by the AdamW pass), plus g and m present and w, g, m, v
+    // pairwise disjoint
+    auto describe = [&](const quasar_adamw_nvfp4_tensor& x, Nvfp4Tensor* T, AmaxItem* A,
+                        AdamwItem* W) {
+        quasar_status s1 = nvfp4_tensor(x.w, nullptr, g_dtype, x.v, beta2, clip, n_clip, x.rows,
+                                        x.cols, nullptr, x.r, r_dtype, x.codes, x.block_scale,
+                                        x.tensor_scale, x.cand_idx, T, A, opt.packed);
+        if (s1 != QUASAR_OK) return s1;
+        const int64_t n = x.rows * x.cols;
+        *W = AdamwItem{x.w, x.g, x.m, x.v, n, x.tensor_scale};
+        if (n == 0) return QUASAR_OK;
+        if (!x.g || !x.m || !aligned16(x.g) || !aligned16(x.m)) return QUASAR_ERR_INVALID_ARG;
+        const size_t nb = (size_t)n;
+        const void* outs[] = {x.r, x.codes, x.block_scale, x.tensor_scale, x.cand_idx};
+        const size_t bytes[] = {nb * dtype_size(r_dtype), x.codes ? (opt.packed ? nb / 2 : nb) : 0,
+                                nb / 16, 4, x.cand_idx ? nb / 16 : 0};
+        for (int i = 0; i < 5; ++i)
+            if (overlaps(outs[i], bytes[i], x.m, nb * 4) ||
+                overlaps(outs[i], bytes[i], x.g, nb * dtype_size(g_dtype)))
+                return QUASAR_ERR_INVALID_ARG;
+        const void* state[] = {x.w, x.g, x.m, x.v};
+        const size_t sbytes[] = {nb * 4, nb * dtype_size(g_dtype), nb * 4, nb * 4};
+        for (int i = 0; i < 4; ++i)
+            for (int j = i + 1; j < 4; ++j)
+                if (overlaps(state[i], sbytes[i], state[j], sbytes[j])) return QUASAR_ERR_INVALID_ARG;
+        return QUASAR_OK;
+    };
+    static thread_local Nvfp4Launch<kMaxBatch> Lp;
+    static thread_local AmaxBatch<kMaxBatch> B;
+    static thread_local AdamwBatch<kMaxBatch> Ad;
+    quasar_status st;
+    for (int i = 0; i < n_tensors; ++i) {
+        Nvfp4Tensor T;
+        AmaxItem A;
+        AdamwItem W;
+        if ((st = describe(tensors[i], &T, &A, &W)) != QUASAR_OK) return st;
+    }
+    if ((st = nvfp4_params(false, g_dtype, beta2, clip, n_clip, r_dtype, &Lp.p, opt)) != QUASAR_OK)
+        return st;
+    {
+        const double t = (double)step;
+        AdamwHp& hp = Ad.hp;
+        hp.g_kind = g_dtype == QUASAR_BF16 ? 2 : 1;
+        hp.beta1 = beta1;
+        hp.c1b = 1.0f - beta1;
+        hp.beta2 = beta2;
+        hp.c1 = 1.0f - beta2;
+        hp.lr_wd = (float)((double)lr * (double)weight_decay);
+        hp.step_size = (float)((double)lr / (1.0 - std::pow((double)beta1, t)));
+        hp.isbc2 = (float)(1.0 / std::sqrt(1.0 - std::pow((double)beta2, t)));
+        hp.eps = eps;
+    }
+    int dev = 0;
+    const DeviceInfo* info = nullptr;
+    if ((st = device_info(&dev, &info)) != QUASAR_OK) return st;
+    const cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+    for (int i0 = 0; i0 < n_tensors; i0 += kMaxBatch) {
+        Lp.n_t = B.n_t = Ad.n_t = std::min(kMaxBatch, n_tensors - i0);
+        int64_t nmax = 0;
+        for (int i = 0; i < Lp.n_t; ++i) {
+            describe(tensors[i0 + i], &Lp.t[i], &B.t[i], &Ad.t[i]);
+            nmax = std::max(nmax, Ad.t[i].n);
+            if (cudaMemsetAsync(B.t[i].slot, 0, sizeof(float), s) != cudaSuccess)
+                return QUASAR_ERR_CUDA;
+        }
+        if (nmax > 0) {
+            const int64_t want = (nmax / 4 + kThreads - 1) / kThreads;
+            const int64_t per = std::max<int64_t>(1, (int64_t)info->nsm * 8 / Ad.n_t);
+            const int gx = (int)std::max<int64_t>(1, std::min<int64_t>(per, want));
+            void* args[] = {(void*)&Ad};
+            if (cudaLaunchKernel(adamw_amax_kernel(), dim3(gx, Ad.n_t), dim3(kThreads), args, 0, s) !=
+                cudaSuccess)
+                return QUASAR_ERR_CUDA;
+        }
+        if ((st = nvfp4_run(Lp, B, n_clip, s, true)) != QUASAR_OK) return st;
     }
     return QUASAR_OK;
 }

@@ -49,6 +49,8 @@ PROTOTYPES = {
     "quasar_recon_nvfp4_batch": (_I, [_P, _I, _I, _F, _P, _I, _I, _P]),
     "quasar_recon_nvfp4_batch_ex": (_I, [_P, _I, _I, _F, _P, _I, _I, _P, _P]),
     "quasar_recon_lut_batch": (_I, [_P, _I, _I, _F, _P, _I, _I, _P, _P]),
+    "quasar_adamw_recon_nvfp4_batch": (_I, [_P, _I, _I, _F, _F, _F, _F, _F, _I64, _P, _I, _I, _P,
+                                            _P]),
     "quasar_tensor_amax": (_I, [_P, _I64, _P, _P]),
     "quasar_get_device_status": (_I, [_P]),
     "quasar_debug_force_timeout": (None, [_I64]),
@@ -278,6 +280,41 @@ def quasar_recon_nvfp4_batch_ex(tensors, beta2, clip, options=None, g_dtype=BF16
     st = lib.quasar_recon_nvfp4_batch_ex(ctypes.cast(tensors, ctypes.c_void_p), len(tensors),
                                          g_dtype, beta2, carr, nclip, r_dtype, _opt_ptr(options),
                                          _stream(stream))
+    return QuasarStatus(st)
+
+
+class QuasarAdamwNvfp4Tensor(ctypes.Structure):
+    """quasar_adamw_nvfp4_tensor: one tensor's buffers (device pointers) and shape."""
+    _fields_ = [("w", ctypes.c_void_p), ("g", ctypes.c_void_p), ("m", ctypes.c_void_p),
+                ("v", ctypes.c_void_p), ("r", ctypes.c_void_p), ("codes", ctypes.c_void_p),
+                ("block_scale", ctypes.c_void_p), ("tensor_scale", ctypes.c_void_p),
+                ("cand_idx", ctypes.c_void_p), ("rows", ctypes.c_int64), ("cols", ctypes.c_int64)]
+
+
+def adamw_nvfp4_tensor_array(items):
+    """A ctypes array of QuasarAdamwNvfp4Tensor from dicts with keys w, g, m,
+    v, r, codes, block_scale, tensor_scale, cand_idx, rows, cols."""
+    arr = (QuasarAdamwNvfp4Tensor * len(items))()
+    for i, d in enumerate(items):
+        arr[i] = QuasarAdamwNvfp4Tensor(
+            _ptr(d["w"]), _ptr(d.get("g")), _ptr(d.get("m")), _ptr(d["v"]), _ptr(d["r"]),
+            _ptr(d.get("codes")), _ptr(d["block_scale"]), _ptr(d["tensor_scale"]),
+            _ptr(d.get("cand_idx")), int(d["rows"]), int(d["cols"]))
+    return arr
+
+
+def quasar_adamw_recon_nvfp4_batch(tensors, lr, beta1, beta2, eps, weight_decay, step, clip,
+                                   g_dtype=BF16, r_dtype=BF16, options=None,
+                                   stream=None) -> QuasarStatus:
+    """tensors: a ctypes array from adamw_nvfp4_tensor_array (or a list of dicts)."""
+    lib = load()
+    if not isinstance(tensors, ctypes.Array):
+        tensors = adamw_nvfp4_tensor_array(tensors)
+    carr, nclip = _clip_array(clip)
+    st = lib.quasar_adamw_recon_nvfp4_batch(ctypes.cast(tensors, ctypes.c_void_p), len(tensors),
+                                            g_dtype, lr, beta1, beta2, eps, weight_decay, step,
+                                            carr, nclip, r_dtype, _opt_ptr(options),
+                                            _stream(stream))
     return QuasarStatus(st)
 
 

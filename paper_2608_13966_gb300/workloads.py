@@ -66,6 +66,8 @@ CLIP_PAPER = tuple(round(0.30 + 0.05 * i, 2) for i in range(15))  # 0.30 ... 1.0
 
 # AdamW hyper-parameters of the fused-step workloads
 ADAMW_LLAMA_INT3 = {"lr": 2e-5, "beta1": 0.9, "eps": 1e-8, "weight_decay": 0.01, "step": 100}
+# the paper's NVFP4 QAD learning rate (Sec. 6.1)
+ADAMW_NVFP4 = {"lr": 1e-6, "beta1": 0.9, "eps": 1e-8, "weight_decay": 0.01, "step": 100}
 
 
 @dataclass(frozen=True)
@@ -151,6 +153,16 @@ def workload(name: str) -> Workload:
                         "AdamW step fused with INT3 group-128 reconstruction of all linear "
                         "weights of a 32-layer Llama-3.1-8B-shaped model",
                         adamw=dict(ADAMW_LLAMA_INT3))
+    if name == "llama_layer_nvfp4_adamw":
+        return Workload(name, "nvfp4", 4, 16, CLIP_8, 0.999, bf16, bf16, True,
+                        _layer_tensors(LLAMA31_8B_LAYER, 1), "t4", "lognormal",
+                        "one Llama-3.1-8B-shaped layer, AdamW step + NVFP4",
+                        adamw=dict(ADAMW_NVFP4))
+    if name == "llama_nvfp4_adamw":
+        return Workload(name, "nvfp4", 4, 16, CLIP_8, 0.999, bf16, bf16, False,
+                        _layer_tensors(LLAMA31_8B_LAYER, 32), "t4", "lognormal",
+                        "AdamW step then NVFP4 reconstruction of all linear weights of a 32-layer "
+                        "Llama-3.1-8B-shaped model", adamw=dict(ADAMW_NVFP4))
     if name == "llama_layer_lut":
         return Workload(name, "lut", 3, 512, CLIP_8, 0.999, bf16, bf16, True,
                         _layer_tensors(LLAMA31_8B_LAYER, 1), "t4", "lognormal",
@@ -168,8 +180,9 @@ def workload(name: str) -> Workload:
 
 
 WORKLOADS = ("single_int4", "llama_layer_int3", "qwen_layer_int2", "llama_layer_nvfp4",
-             "llama_layer_int3_adamw", "llama_layer_lut", "llama_int2", "llama_int3", "llama_int4",
-             "llama_nvfp4", "llama_int3_adamw", "llama_lut")
+             "llama_layer_int3_adamw", "llama_layer_nvfp4_adamw", "llama_layer_lut", "llama_int2",
+             "llama_int3", "llama_int4", "llama_nvfp4", "llama_int3_adamw", "llama_nvfp4_adamw",
+             "llama_lut")
 
 
 def _student_t(gen, shape, nu: int, device) -> torch.Tensor:

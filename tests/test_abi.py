@@ -248,3 +248,30 @@ def test_lut_argument_validation(lib, kw, expect):
     items = kw.pop("items")
     assert Q.quasar_recon_lut_batch(items, kw.get("beta2", 0.999), CLIP, kw.get("opt"),
                                     stream=0) == expect
+
+
+def _andesc(**kw):
+    d = dict(w=A, g=B, m=M_ADDR, v=C, r=D, codes=None, block_scale=E, tensor_scale=F,
+             cand_idx=None, rows=4, cols=256)
+    d.update(kw)
+    return d
+
+
+@pytest.mark.parametrize("kw,expect", [
+    (dict(items=[]), Q.QuasarStatus.OK),
+    (dict(items=[_andesc(g=None)]), Q.QuasarStatus.ERR_INVALID_ARG),       # gradient required
+    (dict(items=[_andesc(m=None)]), Q.QuasarStatus.ERR_INVALID_ARG),
+    (dict(items=[_andesc(m=A + 64)]), Q.QuasarStatus.ERR_INVALID_ARG),     # m overlaps w
+    (dict(items=[_andesc(r=M_ADDR + 64)]), Q.QuasarStatus.ERR_INVALID_ARG),  # r overlaps m
+    (dict(items=[_andesc(cols=40)]), Q.QuasarStatus.ERR_INVALID_ARG),      # cols % 16
+    (dict(items=[_andesc(tensor_scale=None)]), Q.QuasarStatus.ERR_INVALID_ARG),
+    (dict(lr=-1.0), Q.QuasarStatus.ERR_INVALID_ARG),
+    (dict(eps=0.0), Q.QuasarStatus.ERR_INVALID_ARG),
+    (dict(step=0), Q.QuasarStatus.ERR_INVALID_ARG),
+])
+def test_adamw_nvfp4_argument_validation(lib, kw, expect):
+    args = dict(items=[_andesc()], lr=1e-5, beta1=0.9, beta2=0.999, eps=1e-8, weight_decay=0.0,
+                step=1)
+    args.update(kw)
+    items = args.pop("items")
+    assert Q.quasar_adamw_recon_nvfp4_batch(items, clip=CLIP, stream=0, **args) == expect

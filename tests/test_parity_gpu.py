@@ -543,3 +543,40 @@ def test_lut_paper_shaped_layer(oracle):
                "codes": o["codes"].cpu().numpy(), "idx": o["cand_idx"].cpu().numpy()}
         rep = checker.check_lut(oracle, w_h.reshape(spec.rows, spec.cols), h, list(w_.clip), O, gpu)
         assert rep["ok"], (spec.name, json.dumps(rep))
+
+
+@pytest.mark.parametrize("hp", [ADAMW_PAPER, dict(lr=1e-3, beta1=0.9, eps=1e-8,
+                                                   weight_decay=0.1, step=1)])
+def test_adamw_recon_nvfp4_batch_matches_oracle(oracle, hp):
+    """AdamW step (w', m', v' and the absmax of w' in one pass), then NVFP4
+    reconstruction of w' with h = v': tensor by tensor against the oracle's
+    AdamW step followed by its Sec. 4.2 search on the oracle's w', v'."""
+    from paper_2608_13966_gb300 import api
+    shapes = [(48, 512), (3, 48), (0, 64), (37, 528)]
+    items, hosts = [], []
+    for i, (rows, cols) in enumerate(shapes):
+        w, g, v = _inputs(max(rows, 1), cols, seed=1500 + i)
+        m = wl.first_moment((max(rows, 1), cols), 1500 + i, device="cuda")
+        w, g, m, v = (t[:rows].contiguous() for t in (w, g, m, v))
+        items.append((w, g, m, v))
+        hosts.append(tuple(H._host(t) for t in (w, g, m, v)))
+    outs = api.adamw_recon_nvfp4_batch(items, lr=hp["lr"], beta1=hp["beta1"], beta2=0.999,
+                                       eps=hp["eps"], weight_decay=hp["weight_decay"],
+                                       step=hp["step"], clip=CLIP8, codes=True)
+    torch.cuda.synchronize()
+    hp32 = _hp32(hp, 0.999)
+    for (rows, cols), o, it, (w_h, g_h, m_h, v_h) in zip(shapes, outs, items, hosts):
+        if w_h.size == 0:
+            assert float(o["tensor_scale"].cpu()[0]) == 1.0
+            continue
+        w1, m1, v1 = oracle.adamw(w_h, g_h, m_h, v_h, **hp32)
+        st = checker.check_adamw(w_h, g_h, m_h, hp32, w1, m1, v1, H._host(it[0]), H._host(it[2]),
+                                 H._host(it[3]))
+        assert st["ok"], json.dumps(st)
+        _, s_T = oracle.tensor_scale(w1)
+        O = oracle.recon_nvfp4(w1, v1, s_T, CLIP8)
+        gpu = {"r": H._host(o["r"]), "scale": o["block_scale"].cpu().numpy(),
+               "tensor_scale": float(o["tensor_scale"].cpu()[0]),
+               "codes": o["codes"].cpu().numpy().ravel(), "idx": o["cand_idx"].cpu().numpy()}
+        rep = checker.check_nvfp4(oracle, w1, v1, CLIP8, s_T, O, gpu, True)
+        assert rep["ok"], json.dumps(rep)
