@@ -76,6 +76,12 @@ def _load():
         lib.qo_fit_nvfp4_scale.restype = i32
         lib.qo_eval_nvfp4.argtypes = [P, P, f32, P, i32]
         lib.qo_eval_nvfp4.restype = f64
+        lib.qo_recon_sym.argtypes = [P, P, i64, i32, i32, P, i32] + [P] * 8
+        lib.qo_recon_sym.restype = i32
+        lib.qo_codes_sym.argtypes = [P, i32, i32, f32, P, P]
+        lib.qo_codes_sym.restype = None
+        lib.qo_refit_sym.argtypes = [P, P, P, i32, i32, f32, P]
+        lib.qo_refit_sym.restype = f64
         lib.qo_recon_lut.argtypes = [P, P, i64, i64, i32, i32, P, i32] + [P] * 9
         lib.qo_recon_lut.restype = i32
         lib.qo_lut_block.argtypes = [P, P, i32, f32, P, P, P, P]
@@ -396,3 +402,47 @@ def e4m3s_value(bits: int) -> float:
     """Value of signed E4M3 bits (sign bit 0x80)."""
     v = e4m3_value(int(bits) & 0x7F)
     return -v if int(bits) & 0x80 else v
+
+
+# ------------------------------------------------------ symmetric integer codes
+
+def recon_sym(w, h, group_size: int, bits: int, clip) -> dict:
+    """Algorithm 1 with symmetric codes (readings S1, S2): per group and
+    candidate, q = clamp(rne(w / s_f), -Q, Q), s_f = f amax / Q, the fit
+    s* = sum h q w / sum h q^2, direct error, argmin.  codes are q + Q."""
+    w = _c(w, np.float32).ravel()
+    h = _c(h, np.float32).ravel()
+    clip = _c(clip, np.float32).ravel()
+    G, K = int(group_size), clip.size
+    assert w.size == h.size and w.size % G == 0
+    n = w.size // G
+    out = dict(idx=np.empty(n, np.int32), a=np.empty(n), codes=np.empty(w.size, np.uint8),
+               r=np.empty(w.size), err=np.empty(n), cand_err=np.empty(n * K), m_round=np.empty(n),
+               m_tie=np.empty(n))
+    rc = _load().qo_recon_sym(_ptr(w), _ptr(h), n, G, int(bits), _ptr(clip), K, _ptr(out["idx"]),
+                              _ptr(out["a"]), _ptr(out["codes"]), _ptr(out["r"]), _ptr(out["err"]),
+                              _ptr(out["cand_err"]), _ptr(out["m_round"]), _ptr(out["m_tie"]))
+    if rc != 0:
+        raise ValueError("qo_recon_sym: bad arguments")
+    out["cand_err"] = out["cand_err"].reshape(n, K)
+    return out
+
+
+def codes_sym(w_group, bits: int, f: float):
+    """Symmetric codes (q + Q) and boundary margins of one group for factor f."""
+    w = _c(w_group, np.float32).ravel()
+    q = np.empty(w.size, np.uint8)
+    m = np.empty(w.size)
+    _load().qo_codes_sym(_ptr(w), w.size, int(bits), ctypes.c_float(f), _ptr(q), _ptr(m))
+    return q, m
+
+
+def refit_sym(w_group, h_group, codes, bits: int, f: float):
+    """(s*, error) of given symmetric codes on one group."""
+    w = _c(w_group, np.float32).ravel()
+    h = _c(h_group, np.float32).ravel()
+    q = _c(codes, np.uint8).ravel()
+    s = ctypes.c_double()
+    e = _load().qo_refit_sym(_ptr(w), _ptr(h), _ptr(q), w.size, int(bits), ctypes.c_float(f),
+                             ctypes.byref(s))
+    return s.value, float(e)

@@ -27,6 +27,10 @@
  *                   Eq. 3, keep the candidate with the lowest error.
  *   qo_e4m3_round / qo_e2m1_round   the two codecs, by enumeration of the
  *                   representable values.
+ *   qo_recon_sym    Algorithm 1 with symmetric integer codes: the related
+ *                   closed form of Sec. 4.1.2 (no offset, s* = sum h q w /
+ *                   sum h q^2), codes on [-f amax, f amax], direct error,
+ *                   argmin over the clip grid.
  *   qo_recon_lut    App. B, the Rubin INT3 lookup-table instantiation: per
  *                   block, per candidate range, 3-bit indices on the range's
  *                   grid, each table entry the E4M3 rounding of its codes'
@@ -58,6 +62,12 @@
  *   N5  E2M1 rounding is nearest with ties to the even code; magnitude 0 is
  *       stored as +0;
  *   N6  the candidate error uses the E4M3-rounded scale.
+ *   S1  symmetric codes: q in {-Q..Q}, Q = 2^(bits-1) - 1, step
+ *       s_f = f*amax/Q with amax = max |w| of the group, q = clamp(
+ *       round_half_even(w / s_f), -Q, Q); stored as the unsigned code q + Q;
+ *   S2  symmetric fit: r = s* q with s* = sum h q w / sum h q^2; if every h > 0
+ *       element has q = 0, s* = s_f and the error is sum h w^2; amax = 0:
+ *       codes q = 0, s* = 0, r = 0, index 0;
  *   L1  a LUT block is 8 consecutive rows x 64 consecutive columns, its
  *       elements in row-major order (the oracle takes any block shape);
  *   L2  the indices of a candidate are the Eq. 1 codes with qmax = 7 on the
@@ -889,4 +899,150 @@ int qo_recon_lut(const float* w, const float* h, int64_t rows, int64_t cols, int
         free(qk);
     }
     return 0;
+}
+
+/* ------------------------------------------------------------------------ */
+/* Symmetric integer codes (Sec. 4.1.2: the closed form without offset).     */
+/* ------------------------------------------------------------------------ */
+
+/* Codes of one candidate of one group (S1): q in [-Q, Q] returned as q + Q;
+ * margin[i]: distance of t = w/s to the nearest decision boundary j + 1/2
+ * (|j| < Q), divided by 2Q (as a fraction of the clipping range). */
+static void sym_codes(const float* w, int G, double amax, double f, int Q, uint8_t* code,
+                      double* margin)
+{
+    const double s = f * amax / (double)Q;
+    for (int i = 0; i < G; ++i) {
+        const double t = (double)w[i] / s;
+        double k = nearbyint(t);
+        if (k < -(double)Q) k = -(double)Q;
+        if (k > (double)Q) k = (double)Q;
+        code[i] = (uint8_t)(int)(k + (double)Q);
+        if (margin) {
+            double j = floor(t);
+            if (j < -(double)Q) j = -(double)Q;
+            if (j > (double)(Q - 1)) j = (double)(Q - 1);
+            margin[i] = fabs(t - (j + 0.5)) / (2.0 * (double)Q);
+        }
+    }
+}
+
+/* S2 for fixed codes: returns the direct error, writes s*. */
+static double sym_fit(const float* w, const double* hd, const uint8_t* code, int G, int Q, double step,
+                      double* s_out)
+{
+    double s2 = 0.0, s3 = 0.0;
+    for (int i = 0; i < G; ++i) {
+        const double q = (double)code[i] - (double)Q;
+        s2 += hd[i] * q * q;
+        s3 += hd[i] * q * (double)w[i];
+    }
+    const double s = (s2 > 0.0) ? s3 / s2 : step;
+    double e = 0.0;
+    for (int i = 0; i < G; ++i) {
+        const double d = s * ((double)code[i] - (double)Q) - (double)w[i];
+        e += hd[i] * d * d;
+    }
+    *s_out = s;
+    return e;
+}
+
+int qo_recon_sym(const float* w, const float* h, int64_t n_groups, int G, int bits,
+                 const float* clip, int K, int32_t* idx, double* a, uint8_t* codes, double* r,
+                 double* err, double* cand_err, double* m_round, double* m_tie)
+{
+    if (G < 1 || bits < 2 || bits > 8 || K < 1 || K > QO_MAX_K || n_groups < 0) return -1;
+    const int Q = (1 << (bits - 1)) - 1;
+
+#pragma omp parallel for schedule(dynamic, 64)
+    for (int64_t grp = 0; grp < n_groups; ++grp) {
+        const float* wg = w + grp * G;
+        const float* hg = h + grp * G;
+        uint8_t* qk = (uint8_t*)malloc((size_t)K * (size_t)G);
+        double* hd = (double*)malloc(sizeof(double) * (size_t)G);
+        double* mg = (double*)malloc(sizeof(double) * (size_t)G);
+        double ek[QO_MAX_K], sk[QO_MAX_K];
+        double amax = 0.0;
+        for (int i = 0; i < G; ++i)
+            if (fabs((double)wg[i]) > amax) amax = fabs((double)wg[i]);
+        group_saliency(hg, G, hd);
+        int best = 0;
+        double mround = HUGE_VAL, mtie = HUGE_VAL;
+        if (amax == 0.0) {
+            memset(qk, Q, (size_t)K * (size_t)G);
+            for (int k = 0; k < K; ++k) {
+                ek[k] = 0.0;
+                sk[k] = 0.0;
+            }
+        } else {
+            for (int k = 0; k < K; ++k) {
+                const double f = (double)clip[k];
+                uint8_t* q = qk + (size_t)k * G;
+                sym_codes(wg, G, amax, f, Q, q, mg);
+                for (int i = 0; i < G; ++i)
+                    if (mg[i] < mround) mround = mg[i];
+                ek[k] = sym_fit(wg, hd, q, G, Q, f * amax / (double)Q, &sk[k]);
+            }
+            for (int k = 1; k < K; ++k)
+                best = (ek[k] < ek[best]) ? k : best; /* ties: the lowest index */
+            double second = HUGE_VAL;
+            for (int k = 0; k < K; ++k) {
+                if (k == best) continue;
+                if (memcmp(qk + (size_t)k * G, qk + (size_t)best * G, (size_t)G) == 0) continue;
+                if (ek[k] < second) second = ek[k];
+            }
+            if (second < HUGE_VAL) {
+                const double denom = ek[best] > 1e-300 ? ek[best] : 1e-300;
+                mtie = (second - ek[best]) / denom;
+            }
+        }
+        if (idx) idx[grp] = best;
+        if (a) a[grp] = sk[best];
+        if (err) err[grp] = ek[best];
+        if (m_round) m_round[grp] = mround;
+        if (m_tie) m_tie[grp] = mtie;
+        for (int k = 0; k < K; ++k)
+            if (cand_err) cand_err[grp * K + k] = ek[k];
+        const uint8_t* qb = qk + (size_t)best * G;
+        for (int i = 0; i < G; ++i) {
+            if (codes) codes[grp * G + i] = qb[i];
+            if (r) r[grp * G + i] = sk[best] * ((double)qb[i] - (double)Q);
+        }
+        free(qk);
+        free(hd);
+        free(mg);
+    }
+    return 0;
+}
+
+/* Symmetric codes and margins of one candidate of one group (checker). */
+void qo_codes_sym(const float* w, int G, int bits, float f, uint8_t* code, double* margin)
+{
+    const int Q = (1 << (bits - 1)) - 1;
+    double amax = 0.0;
+    for (int i = 0; i < G; ++i)
+        if (fabs((double)w[i]) > amax) amax = fabs((double)w[i]);
+    if (amax == 0.0) {
+        for (int i = 0; i < G; ++i) {
+            code[i] = (uint8_t)Q;
+            if (margin) margin[i] = HUGE_VAL;
+        }
+        return;
+    }
+    sym_codes(w, G, amax, (double)f, Q, code, margin);
+}
+
+/* S2 for given codes of one group (checker): returns the error, writes s*. */
+double qo_refit_sym(const float* w, const float* h, const uint8_t* code, int G, int bits, float f,
+                    double* s_out)
+{
+    const int Q = (1 << (bits - 1)) - 1;
+    double amax = 0.0;
+    for (int i = 0; i < G; ++i)
+        if (fabs((double)w[i]) > amax) amax = fabs((double)w[i]);
+    double* hd = (double*)malloc(sizeof(double) * (size_t)G);
+    group_saliency(h, G, hd);
+    const double e = sym_fit(w, hd, code, G, Q, (double)f * amax / (double)Q, s_out);
+    free(hd);
+    return e;
 }

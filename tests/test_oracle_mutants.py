@@ -60,6 +60,14 @@ MUTANTS = {
     "AdamW without bias correction": ("lr * ((double)mi / bc1) / denom", "lr * (double)mi / denom"),
     "AdamW coupled weight decay": ("(double)w[i] * (1.0 - lr * wd) - lr", "(double)w[i] - lr * wd - lr"),
     "AdamW eps inside the root": ("sqrt((double)vi / bc2) + eps", "sqrt((double)vi / bc2 + eps)"),
+    "symmetric argmin ties to last": ("best = (ek[k] < ek[best]) ? k : best;",
+                                      "best = (ek[k] <= ek[best]) ? k : best;"),
+    "symmetric fit with an offset": ("const double s = (s2 > 0.0) ? s3 / s2 : step;",
+                                     "const double s = (s2 > 0.0) ? (s3 + 1e-3 * s2) / s2 : step;"),
+    "symmetric grid on the full range": ("const double s = f * amax / (double)Q;",
+                                         "const double s = 2.0 * f * amax / (double)(2 * Q + 1);"),
+    "symmetric codes not clamped": ("if (k > (double)Q) k = (double)Q;\n        code[i]",
+                                    "if (k > (double)(Q + 1)) k = (double)(Q + 1);\n        code[i]"),
     "LUT entry unweighted mean": ("W[q[i] & 7] += hd[i] * (double)w[i];", "W[q[i] & 7] += (double)w[i];"),
     "LUT entry sign dropped": ("return (x < 0.0 && mag != 0) ? (0x80 | mag) : mag;", "return mag;"),
     "LUT empty index at grid offset": ("lo + (double)k * s;", "lo + (double)(k + 1) * s;"),
@@ -81,6 +89,9 @@ PIN_TESTS = [
     (pins.test_nvfp4_fit_and_scale_are_optimal, {}),
     (pins.test_adamw_matches_torch_optimizer, {}),
     (pins.test_adamw_first_step_closed_form, {}),
+    (pins.test_sym_worked_example, {}),
+    (pins.test_sym_codes_are_nearest_levels_and_fit_is_lstsq, {"bits": 3}),
+    (pins.test_sym_sign_symmetry_and_ties, {}),
     (pins.test_lut_worked_example, {}),
     (pins.test_lut_entries_are_the_best_e4m3_values, {}),
     (pins.test_lut_error_and_argmin, {}),
@@ -108,7 +119,8 @@ def test_pins_catch_planted_mistake(oracle, tmp_path, name):
     # give the mutant the same prototypes as the real library
     for sym in ("qo_ema", "qo_adamw", "qo_recon_int", "qo_refit_int", "qo_codes_int", "qo_tensor_scale",
                 "qo_recon_nvfp4", "qo_e2m1_round", "qo_e4m3_round", "qo_e4m3_value",
-                "qo_set_threads", "qo_get_threads", "qo_recon_lut", "qo_lut_block", "qo_lut_eval", "qo_lut_fit"):
+                "qo_set_threads", "qo_get_threads", "qo_recon_lut", "qo_lut_block", "qo_lut_eval", "qo_lut_fit",
+                "qo_recon_sym", "qo_codes_sym", "qo_refit_sym"):
         f_real, f_mut = getattr(real, sym), getattr(lib, sym)
         f_mut.argtypes, f_mut.restype = f_real.argtypes, f_real.restype
     caught = []

@@ -729,3 +729,79 @@ def test_lut_saliency_scale_invariance(oracle):
     for key in ("idx", "book", "codes"):
         assert np.array_equal(A[key], B[key])
     assert np.allclose(B["err"], 4.0 * A["err"], rtol=1e-13, atol=0)
+
+
+# ------------------------------------------------ symmetric integer codes
+
+def test_sym_worked_example(oracle):
+    import json, os
+    gold = json.load(open(os.path.join(os.path.dirname(__file__), "golden",
+                                       "sym_worked_example.json")))
+    O = oracle.recon_sym(np.array(gold["w"], np.float32), np.array(gold["h"], np.float32),
+                         gold["group"], gold["bits"], gold["clip"])
+    assert O["idx"][0] == gold["idx"]
+    assert O["codes"].tolist() == gold["codes"]
+    assert abs(O["a"][0] - gold["a"]) <= 1e-7
+    assert np.allclose(O["cand_err"][0], gold["cand_err"], rtol=0, atol=1e-6)
+
+
+def _sym_case(seed, n=128 * 6):
+    rng = np.random.default_rng(seed)
+    w = (0.02 * rng.standard_t(4, size=n)).astype(np.float32)
+    h = np.exp(-14.0 + 2.0 * rng.standard_normal(n)).astype(np.float32)
+    return w, h
+
+
+@pytest.mark.parametrize("bits", [2, 3, 4, 8])
+def test_sym_codes_are_nearest_levels_and_fit_is_lstsq(oracle, bits):
+    """Each code is the nearest level of the symmetric grid (enumerated), and
+    s* is the weighted least-squares slope through the origin (lstsq)."""
+    w, h = _sym_case(bits)
+    clip = [1.0, 0.9, 0.8, 0.7]
+    Q = (1 << (bits - 1)) - 1
+    O = oracle.recon_sym(w, h, 128, bits, clip)
+    for g in range(w.size // 128):
+        wg, hg = w[128 * g:128 * (g + 1)].astype(np.float64), h[128 * g:128 * (g + 1)].astype(np.float64)
+        f = clip[O["idx"][g]]
+        s = f * np.abs(wg).max() / Q
+        levels = np.arange(-Q, Q + 1) * s
+        near = np.argmin(np.abs(wg[:, None] - levels[None, :]), 1)
+        q = O["codes"][128 * g:128 * (g + 1)].astype(int)
+        _, m = oracle.codes_sym(w[128 * g:128 * (g + 1)], bits, f)
+        ok = (q == near) | (m < 1e-9)
+        assert np.all(ok)
+        qq = (q - Q).astype(np.float64)
+        sw = np.sqrt(hg)
+        (a,), *_ = np.linalg.lstsq((sw * qq)[:, None], sw * wg, rcond=None)
+        assert abs(O["a"][g] - a) <= 1e-10 * abs(a)
+        direct = (hg * (O["a"][g] * qq - wg) ** 2).sum()
+        assert abs(direct - O["err"][g]) <= 1e-12 * direct
+        assert O["err"][g] <= O["cand_err"][g].min()
+
+
+def test_sym_sign_symmetry_and_ties(oracle):
+    """Negating w negates the codes and keeps s*, the error and the index; a
+    repeated factor ties with itself and the lower index is kept."""
+    w, h = _sym_case(11)
+    A = oracle.recon_sym(w, h, 128, 3, [1.0, 0.85, 0.7])
+    B = oracle.recon_sym(-w, h, 128, 3, [1.0, 0.85, 0.7])
+    assert np.array_equal(A["idx"], B["idx"])
+    assert np.array_equal(A["codes"].astype(int) - 3, -(B["codes"].astype(int) - 3))
+    assert np.allclose(A["a"], B["a"], rtol=1e-14)
+    assert np.allclose(A["err"], B["err"], rtol=1e-14)
+    D = oracle.recon_sym(w, h, 128, 3, [0.9, 0.9])
+    assert np.all(D["idx"] == 0)
+
+
+def test_sym_degenerate_groups(oracle):
+    w, h = _sym_case(12, n=128 * 3)
+    w[:128] = 0.0                                    # amax = 0
+    h[128:256] = 0.0
+    h[128] = 1.0
+    w[128] = 1e-6                                    # the only salient element codes to 0
+    w[129] = 0.5
+    O = oracle.recon_sym(w, h, 128, 3, [1.0])
+    assert np.all(O["codes"][:128] == 3) and O["a"][0] == 0.0 and np.all(O["r"][:128] == 0.0)
+    step = 0.5 / 3.0
+    assert O["codes"][128] == 3 and abs(O["a"][1] - step) < 1e-12
+    assert abs(O["err"][1] - 1e-12) < 1e-18          # h w^2 of the one salient element
