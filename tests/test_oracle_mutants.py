@@ -18,7 +18,10 @@ SRC = os.path.join(os.path.dirname(os.path.dirname(os.path.abspath(__file__))),
                    "oracle", "quasar_oracle.c")
 
 MUTANTS = {
-    "round half up": ("nearbyint(t);", "floor(t + 0.5);"),
+    "round half up": ("double k = nearbyint(t); /* default rounding mode: half to even */",
+                      "double k = floor(t + 0.5);"),
+    "symmetric round half up": ("double k = nearbyint(t);\n        if (k < -(double)Q)",
+                                "double k = floor(t + 0.5);\n        if (k < -(double)Q)"),
     "offset sign": ("z = wbar - s * qbar;", "z = wbar + s * qbar;"),
     "error sign": ("const double d = s * (double)q[i] + z - (double)w[i];",
                    "const double d = s * (double)q[i] - z - (double)w[i];"),

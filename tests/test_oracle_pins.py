@@ -743,6 +743,10 @@ def test_sym_worked_example(oracle):
     assert O["codes"].tolist() == gold["codes"]
     assert abs(O["a"][0] - gold["a"]) <= 1e-7
     assert np.allclose(O["cand_err"][0], gold["cand_err"], rtol=0, atol=1e-6)
+    t = gold["ties"]                     # exact half-levels: round half to even
+    T = oracle.recon_sym(np.array(t["w"], np.float32), np.ones(t["group"], np.float32),
+                         t["group"], t["bits"], t["clip"])
+    assert T["codes"].tolist() == t["codes"]
 
 
 def _sym_case(seed, n=128 * 6):
