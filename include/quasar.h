@@ -78,6 +78,21 @@ typedef enum { QUASAR_F32 = 0, QUASAR_BF16 = 1 } quasar_dtype;
  *                          deploys real NVFP4 checkpoints, Sec. 6.1, but
  *                          prints no byte layout: these are the usual
  *                          little-endian conventions.)
+ *   grid          integer codes only (quasar_recon_int_batch_ex):
+ *     QUASAR_GRID_ASYMMETRIC  Eq. 1 and Eq. 4 (the default);
+ *     QUASAR_GRID_SYMMETRIC   the offset-free closed form of Sec. 4.1.2:
+ *                             Q = 2^(bits-1) - 1 (bits >= 2), step
+ *                             s_f = f * max|w| / Q per group, codes
+ *                             q = clamp(round_half_even(w / s_f), -Q, Q)
+ *                             stored as q + Q, fit s* = sum h q w / sum h q^2
+ *                             (s_f when every h > 0 element has q = 0), and
+ *                             r = s* q; a = s*, b = -s* Q, so r = a*code + b
+ *                             as for asymmetric codes.  A group with
+ *                             max|w| = 0 gives codes Q, a = b = 0, r = 0.
+ *                             Not available with the fused AdamW step
+ *                             (QUASAR_ERR_UNSUPPORTED); NVFP4 and the lookup
+ *                             table take only the default
+ *                             (QUASAR_ERR_INVALID_ARG).
  * The "Adam weighting only" ablation (no scale search) is F = {1}: clip =
  * {1.0}, n_clip = 1.
  */
@@ -89,9 +104,12 @@ typedef enum {
 
 typedef enum { QUASAR_CODES_U8 = 0, QUASAR_CODES_PACKED = 1 } quasar_codes_layout;
 
+typedef enum { QUASAR_GRID_ASYMMETRIC = 0, QUASAR_GRID_SYMMETRIC = 1 } quasar_int_grid;
+
 typedef struct {
     quasar_saliency saliency;
     quasar_codes_layout codes_layout;
+    quasar_int_grid grid;
 } quasar_options;
 
 /*

@@ -60,14 +60,16 @@ def _int_codes(rows, cols, bits, packed, dev):
 
 
 def recon_int_batch(items, *, bits, group_size, clip, beta2=0.999, r_dtype=torch.bfloat16,
-                    codes=False, cand_idx=True, saliency="ema", packed_codes=False, stream=None):
+                    codes=False, cand_idx=True, saliency="ema", packed_codes=False,
+                    symmetric=False, stream=None):
     """QUASAR integer reconstruction of several tensors in one launch.
 
     items: list of (w, g, v) CUDA tensors (g may be None for all of them);
     each v is updated in place.  saliency: "ema" (h = v'), "ema_squared"
     (h = v'^2) or "uniform" (h = 1); packed_codes: codes as the packed
-    deployment format.  Returns one result dict per tensor, as recon_int
-    does."""
+    deployment format; symmetric: symmetric codes (q + Q stored, r = a
+    code + b with b = -a Q).  Returns one result dict per tensor, as
+    recon_int does."""
     descs, results = [], []
     g_dtype = F32
     for w, g, v in items:
@@ -90,8 +92,8 @@ def recon_int_batch(items, *, bits, group_size, clip, beta2=0.999, r_dtype=torch
         results.append(res)
     rd = BF16 if r_dtype == torch.bfloat16 else F32
     _check(quasar_recon_int_batch_ex(int_tensor_array(descs), beta2, bits, group_size, clip,
-                                     options(saliency, packed_codes), g_dtype=g_dtype, r_dtype=rd,
-                                     stream=stream))
+                                     options(saliency, packed_codes, symmetric), g_dtype=g_dtype,
+                                     r_dtype=rd, stream=stream))
     return results
 
 

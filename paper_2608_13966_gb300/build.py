@@ -28,6 +28,7 @@ UNITS = [
     ("kernels_int.cu", ["-DQUASAR_NCH=4"], "kernels_int_nch4.o"),
     ("kernels_nvfp4.cu", [], "kernels_nvfp4.o"),
     ("kernels_lut.cu", [], "kernels_lut.o"),
+    ("kernels_sym.cu", [], "kernels_sym.o"),
 ]
 
 

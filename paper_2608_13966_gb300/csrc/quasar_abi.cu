@@ -23,6 +23,7 @@ const void* amax_kernel(bool batch);
 const void* amax_to_scale_kernel(bool batch);
 const void* lut_kernel();
 const void* adamw_amax_kernel();
+const void* sym_kernel(int epl);
 }  // namespace quasar
 
 // Per-device status word (bit 0: a kernel timed out on a wait).
@@ -257,6 +258,7 @@ int g_kind_of(const void* g, quasar_dtype d) { return !g ? 0 : (d == QUASAR_BF16
 struct Opts {
     int h_mode = kSalEma;
     bool packed = false;
+    bool symmetric = false;
 };
 
 quasar_status read_options(const quasar_options* o, Opts* out)
@@ -268,6 +270,9 @@ quasar_status read_options(const quasar_options* o, Opts* out)
         return QUASAR_ERR_INVALID_ARG;
     if (o->codes_layout != QUASAR_CODES_U8 && o->codes_layout != QUASAR_CODES_PACKED)
         return QUASAR_ERR_INVALID_ARG;
+    if (o->grid != QUASAR_GRID_ASYMMETRIC && o->grid != QUASAR_GRID_SYMMETRIC)
+        return QUASAR_ERR_INVALID_ARG;
+    out->symmetric = o->grid == QUASAR_GRID_SYMMETRIC;
     out->h_mode = o->saliency == QUASAR_SALIENCY_EMA_SQUARED ? kSalEmaSquared
                   : o->saliency == QUASAR_SALIENCY_UNIFORM   ? kSalUniform
                                                              : kSalEma;
@@ -376,7 +381,7 @@ quasar_status int_params(quasar_dtype g_dtype, bool has_g, float beta2, int bits
 // Number the tensors' units consecutively and launch over all of them.
 template <int MAXT>
 quasar_status int_launch(IntLaunch<MAXT>& Lp, int group_size, int n_clip, cudaStream_t stream,
-                         bool adam = false)
+                         bool adam = false, bool symmetric = false)
 {
     int64_t units = 0;
     for (int i = 0; i < Lp.n_t; ++i) {
@@ -391,7 +396,8 @@ quasar_status int_launch(IntLaunch<MAXT>& Lp, int group_size, int n_clip, cudaSt
     const int nch = nch_for(n_clip);
     const bool batch = MAXT > 1;
     const bool var = Lp.p.h_mode != kSalEma || Lp.p.codes_packed;
-    const void* fn = nch == 1   ? int_kernel_nch1(epl, batch, adam, var)
+    const void* fn = symmetric  ? (MAXT > 1 ? sym_kernel(epl) : nullptr)
+                     : nch == 1 ? int_kernel_nch1(epl, batch, adam, var)
                      : nch == 2 ? int_kernel_nch2(epl, batch, adam, var)
                                 : int_kernel_nch4(epl, batch, adam, var);
     if (!fn) return QUASAR_ERR_UNSUPPORTED;
@@ -551,6 +557,7 @@ quasar_status quasar_recon_int_batch_ex(const quasar_int_tensor* tensors, int n_
     Opts opt;
     if (read_options(options, &opt) != QUASAR_OK) return QUASAR_ERR_INVALID_ARG;
     if (n_tensors < 0 || (n_tensors > 0 && !tensors)) return QUASAR_ERR_INVALID_ARG;
+    if (opt.symmetric && bits < 2) return QUASAR_ERR_INVALID_ARG;  // Q = 2^(bits-1) - 1 >= 1
     if (n_tensors == 0) return QUASAR_OK;
     // all non-empty tensors carry a gradient, or none does
     int with_g = 0, non_empty = 0;
@@ -587,7 +594,7 @@ quasar_status quasar_recon_int_batch_ex(const quasar_int_tensor* tensors, int n_
             int_tensor(x.w, x.g, g_dtype, x.v, beta2, clip, n_clip, x.rows, x.cols, x.r, r_dtype,
                        x.codes, x.a, x.b, x.cand_idx, group_size, &Lp.t[i], bits, opt.packed);
         }
-        if ((st = int_launch(Lp, group_size, n_clip, s)) != QUASAR_OK) return st;
+        if ((st = int_launch(Lp, group_size, n_clip, s, false, opt.symmetric)) != QUASAR_OK) return st;
     }
     return QUASAR_OK;
 }
@@ -601,6 +608,7 @@ quasar_status quasar_adamw_recon_int_batch(const quasar_adamw_tensor* tensors, i
 {
     Opts opt;
     if (read_options(options, &opt) != QUASAR_OK) return QUASAR_ERR_INVALID_ARG;
+    if (opt.symmetric) return QUASAR_ERR_UNSUPPORTED;  // no fused AdamW kernel for symmetric codes
     if (n_tensors < 0 || (n_tensors > 0 && !tensors)) return QUASAR_ERR_INVALID_ARG;
     if (!(std::isfinite(lr) && lr >= 0.0f) || !(beta1 >= 0.0f && beta1 < 1.0f) ||
         !(std::isfinite(eps) && eps > 0.0f) ||
@@ -701,6 +709,7 @@ quasar_status quasar_recon_nvfp4_batch_ex(const quasar_nvfp4_tensor* tensors, in
 {
     Opts opt;
     if (read_options(options, &opt) != QUASAR_OK) return QUASAR_ERR_INVALID_ARG;
+    if (opt.symmetric) return QUASAR_ERR_INVALID_ARG;  // an integer-code option
     if (n_tensors < 0 || (n_tensors > 0 && !tensors)) return QUASAR_ERR_INVALID_ARG;
     if (n_tensors == 0) return QUASAR_OK;
     int with_g = 0, non_empty = 0;
@@ -746,6 +755,7 @@ quasar_status quasar_recon_lut_batch(const quasar_lut_tensor* tensors, int n_ten
 {
     Opts opt;
     if (read_options(options, &opt) != QUASAR_OK) return QUASAR_ERR_INVALID_ARG;
+    if (opt.symmetric) return QUASAR_ERR_INVALID_ARG;  // an integer-code option
     if (n_tensors < 0 || (n_tensors > 0 && !tensors)) return QUASAR_ERR_INVALID_ARG;
     if (n_tensors == 0) return QUASAR_OK;
     int with_g = 0, non_empty = 0;
@@ -832,6 +842,7 @@ quasar_status quasar_adamw_recon_nvfp4_batch(const quasar_adamw_nvfp4_tensor* te
 {
     Opts opt;
     if (read_options(options, &opt) != QUASAR_OK) return QUASAR_ERR_INVALID_ARG;
+    if (opt.symmetric) return QUASAR_ERR_INVALID_ARG;  // an integer-code option
     if (n_tensors < 0 || (n_tensors > 0 && !tensors)) return QUASAR_ERR_INVALID_ARG;
     if (!(std::isfinite(lr) && lr >= 0.0f) || !(beta1 >= 0.0f && beta1 < 1.0f) ||
         !(std::isfinite(eps) && eps > 0.0f) ||

@@ -173,17 +173,20 @@ CODES_U8, CODES_PACKED = 0, 1
 
 
 class QuasarOptions(ctypes.Structure):
-    """quasar_options: variant of the reconstruction (saliency, codes layout)."""
-    _fields_ = [("saliency", ctypes.c_int), ("codes_layout", ctypes.c_int)]
+    """quasar_options: variant of the reconstruction (saliency, codes layout,
+    integer grid)."""
+    _fields_ = [("saliency", ctypes.c_int), ("codes_layout", ctypes.c_int), ("grid", ctypes.c_int)]
 
 
-def options(saliency="ema", packed_codes=False):
+def options(saliency="ema", packed_codes=False, symmetric=False):
     """A QuasarOptions; saliency is "ema", "ema_squared", "uniform" or a raw
-    integer (passed through unchecked, for the library's own validation)."""
+    integer, packed_codes and symmetric booleans or raw integers (raw values
+    pass through unchecked, for the library's own validation)."""
+    raw = lambda x: isinstance(x, int) and not isinstance(x, bool)
     sal = SALIENCY[saliency] if isinstance(saliency, str) else int(saliency)
-    lay = packed_codes if isinstance(packed_codes, int) and not isinstance(packed_codes, bool) \
-        else (CODES_PACKED if packed_codes else CODES_U8)
-    return QuasarOptions(sal, lay)
+    lay = packed_codes if raw(packed_codes) else (CODES_PACKED if packed_codes else CODES_U8)
+    grid = symmetric if raw(symmetric) else (1 if symmetric else 0)
+    return QuasarOptions(sal, lay, grid)
 
 
 def _opt_ptr(opt):

@@ -363,3 +363,73 @@ def check_lut(oracle, w, h, clip, O, gpu, block=(8, 64)):
             _example(examples, block=int(b), idx=k, oracle_idx=int(O["idx"][b]), ok_k=ok_k,
                      ok_q=ok_q, ok_book=ok_book, n_diff=int(diff.sum()))
     return _report("lut", n, int(exempt.sum()), fails, examples)
+
+
+def _alt_best_sym(oracle, wg, hg, bits, clip, O, g):
+    """As _alt_best_int for symmetric codes: the largest error the oracle's
+    kept candidate shows with its boundary elements rounded the other way."""
+    k = int(O["idx"][g])
+    q, margin = oracle.codes_sym(wg, bits, float(clip[k]))
+    Q = (1 << (bits - 1)) - 1
+    s = float(clip[k]) * float(np.abs(wg.astype(np.float64)).max()) / Q
+    worst = float(O["err"][g])
+    idx = np.flatnonzero(margin < MARGIN)[:4]
+    for mask in range(1, 1 << len(idx)):
+        qq = q.astype(np.int64).copy()
+        for b, i in enumerate(idx):
+            if mask >> b & 1:
+                t = float(wg[i]) / s
+                j = int(min(max(np.floor(t), -Q), Q - 1))      # boundary j + 1/2
+                qq[i] = (2 * j + 1 + 2 * Q) - qq[i]           # the other side, in q + Q units
+        worst = max(worst, oracle.refit_sym(wg, hg, qq.astype(np.uint8), bits, float(clip[k]))[1])
+    return worst
+
+
+def check_sym(oracle, w, h, bits, clip, O, gpu, group_size, r_is_bf16):
+    """Symmetric codes against oracle.recon_sym, with the acceptance of
+    check_int: codes (q + Q) and the index bit-exact outside the margins; a
+    and r within the tolerance; b = -a Q; exempt groups accepted through the
+    oracle's refit of the GPU's own codes."""
+    G = group_size
+    Q = (1 << (bits - 1)) - 1
+    n = w.size // G
+    exempt = (O["m_round"] < MARGIN) | (O["m_tie"] < MARGIN)
+    ne = ~exempt
+    fails = {"fail_idx": 0, "fail_codes": 0, "fail_a": 0, "fail_b": 0, "fail_r": 0,
+             "fail_exempt": 0}
+    r_ref = O["r"].reshape(n, G)
+    r_gpu = np.asarray(gpu["r"], np.float64).reshape(n, G)
+    a_gpu = np.asarray(gpu["a"], np.float64)
+    b_gpu = np.asarray(gpu["b"], np.float64)
+    cg_all = gpu["codes"].reshape(n, G)
+    fails["fail_idx"] = np.count_nonzero((gpu["idx"].astype(np.int64) != O["idx"]) & ne)
+    fails["fail_codes"] = np.count_nonzero(np.any(cg_all != O["codes"].reshape(n, G), axis=1) & ne)
+    fails["fail_a"] = np.count_nonzero(~close(a_gpu, O["a"]) & ne)
+    fails["fail_b"] = np.count_nonzero(~close(b_gpu, -Q * a_gpu))
+    rok = r_ok(r_ref, r_gpu, r_is_bf16).all(axis=1)
+    fails["fail_r"] = np.count_nonzero(~rok & ne)
+    ex = []
+    for g in np.flatnonzero((~close(a_gpu, O["a"]) | ~rok | (gpu["idx"] != O["idx"])) & ne)[:8]:
+        _example(ex, group=int(g), idx_ref=int(O["idx"][g]), idx_gpu=int(gpu["idx"][g]),
+                 a_ref=float(O["a"][g]), a_gpu=float(a_gpu[g]), m_round=float(O["m_round"][g]),
+                 m_tie=float(O["m_tie"][g]), cand_err=O["cand_err"][g])
+    wg_all, hg_all = w.reshape(n, G), h.reshape(n, G)
+    for g in np.flatnonzero(exempt):
+        k = int(gpu["idx"][g])
+        if not 0 <= k < len(clip):
+            fails["fail_exempt"] += 1
+            continue
+        cg = cg_all[g]
+        q_ref, margin = oracle.codes_sym(wg_all[g], bits, float(clip[k]))
+        diff = cg != q_ref
+        ok = bool(np.all(margin[diff] < MARGIN))
+        s, e = oracle.refit_sym(wg_all[g], hg_all[g], cg, bits, float(clip[k]))
+        if k != int(O["idx"][g]):
+            ok &= e <= _alt_best_sym(oracle, wg_all[g], hg_all[g], bits, clip, O, g) * (1 + MARGIN) + 1e-300
+        ok &= bool(close(a_gpu[g], s))
+        ok &= bool(r_ok(s * (cg.astype(np.float64) - Q), r_gpu[g], r_is_bf16).all())
+        if not ok:
+            fails["fail_exempt"] += 1
+            _example(ex, exempt_group=int(g), k=k, idx_ref=int(O["idx"][g]), n_diff=int(diff.sum()),
+                     refit_err=e, err_ref=float(O["err"][g]), a_gpu=float(a_gpu[g]), a_fit=s)
+    return _report("sym", n, np.count_nonzero(exempt), fails, ex)

@@ -275,3 +275,16 @@ def test_adamw_nvfp4_argument_validation(lib, kw, expect):
     args.update(kw)
     items = args.pop("items")
     assert Q.quasar_adamw_recon_nvfp4_batch(items, clip=CLIP, stream=0, **args) == expect
+
+
+def test_symmetric_option_validation(lib):
+    st = Q.QuasarStatus
+    sym = Q.options(symmetric=True)
+    assert Q.quasar_recon_int_batch_ex([_desc(rows=0)], 0.999, 3, 128, CLIP, sym, stream=0) == st.OK
+    assert Q.quasar_recon_int_batch_ex([_desc()], 0.999, 1, 128, CLIP, sym, stream=0) == st.ERR_INVALID_ARG
+    assert Q.quasar_recon_int_batch_ex([_desc()], 0.999, 3, 128, CLIP, Q.options(symmetric=2),
+                                       stream=0) == st.ERR_INVALID_ARG
+    assert Q.quasar_adamw_recon_int_batch([_adesc()], 1e-5, 0.9, 0.999, 1e-8, 0.0, 1, 3, 128, CLIP,
+                                          options=sym, stream=0) == st.ERR_UNSUPPORTED
+    assert Q.quasar_recon_nvfp4_batch_ex([_ndesc()], 0.999, CLIP, sym, stream=0) == st.ERR_INVALID_ARG
+    assert Q.quasar_recon_lut_batch([_ldesc()], 0.999, CLIP, sym, stream=0) == st.ERR_INVALID_ARG

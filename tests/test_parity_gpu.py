@@ -580,3 +580,89 @@ def test_adamw_recon_nvfp4_batch_matches_oracle(oracle, hp):
                "codes": o["codes"].cpu().numpy().ravel(), "idx": o["cand_idx"].cpu().numpy()}
         rep = checker.check_nvfp4(oracle, w1, v1, CLIP8, s_T, O, gpu, True)
         assert rep["ok"], json.dumps(rep)
+
+
+# ------------------------------------------------ symmetric integer codes
+
+def _sym_case(oracle, shapes, seed0, bits, G, clip, saliency="ema", packed=False,
+              g_dtype=torch.bfloat16, r_dtype=torch.bfloat16, g_none=False):
+    from paper_2608_13966_gb300 import api
+    items, hosts = [], []
+    for i, (rows, cols) in enumerate(shapes):
+        w, g, v = _inputs(rows, cols, seed=seed0 + i, g_dtype=g_dtype)
+        if g_none:
+            g = None
+        items.append((w, g, v))
+        hosts.append((H._host(w), None if g is None else H._host(g), H._host(v)))
+    outs = api.recon_int_batch(items, bits=bits, group_size=G, clip=clip, codes=True,
+                               symmetric=True, saliency=saliency, packed_codes=packed,
+                               r_dtype=r_dtype)
+    torch.cuda.synchronize()
+    for (rows, cols), o, (w_h, g_h, v_h), it in zip(shapes, outs, hosts, items):
+        v1 = oracle.ema(v_h, g_h, 0.999) if g_h is not None else v_h
+        h = oracle.saliency(v1, saliency)
+        O = oracle.recon_sym(w_h, h, G, bits, clip)
+        codes = (oracle.unpack_int_codes(o["codes"].cpu().numpy(), bits, w_h.size) if packed
+                 else o["codes"].cpu().numpy().ravel())
+        gpu = {"r": H._host(o["r"]), "a": o["a"].cpu().numpy(), "b": o["b"].cpu().numpy(),
+               "codes": codes, "idx": o["cand_idx"].cpu().numpy()}
+        rep = checker.check_sym(oracle, w_h, h, bits, clip, O, gpu, G, r_dtype == torch.bfloat16)
+        assert rep["ok"], json.dumps(rep)
+        assert checker.check_ema(v1, H._host(it[2]))["ok"]
+
+
+@pytest.mark.parametrize("bits,G", [(2, 64), (3, 128), (4, 128), (4, 32), (8, 256)])
+def test_sym_bits_groups(oracle, bits, G):
+    _sym_case(oracle, [(37, 3 * G), (1, G), (64, 8 * G)], 1600 + bits * 10, bits, G, CLIP8)
+
+
+@pytest.mark.parametrize("K", [1, 13, 32])
+def test_sym_candidate_counts(oracle, K):
+    clip = [round(1.0 - 0.7 * i / max(K - 1, 1), 4) for i in range(K)]
+    _sym_case(oracle, [(64, 1024)], 1700 + K, 4, 128, clip)
+
+
+def test_sym_variants(oracle):
+    _sym_case(oracle, [(16, 512)], 1800, 4, 128, CLIP8, g_dtype=torch.float32, r_dtype=torch.float32)
+    _sym_case(oracle, [(16, 512)], 1801, 4, 128, CLIP8, g_none=True)
+    _sym_case(oracle, [(16, 512)], 1802, 3, 128, CLIP8, saliency="ema_squared")
+    _sym_case(oracle, [(16, 512)], 1803, 3, 128, CLIP8, saliency="uniform")
+    _sym_case(oracle, [(37, 384), (1, 128)], 1804, 3, 128, CLIP8, packed=True)
+
+
+def test_sym_degenerate_groups(oracle):
+    from paper_2608_13966_gb300 import api
+    G = 128
+    w, g, v = _inputs(8, G, seed=1900)
+    w[0] = 0.0                                   # max |w| = 0
+    v[1] = 0.0; g[1] = 0.0                       # all saliency zero
+    v[2] = 0.0; g[2] = 0.0; v[2, 5] = 1e-6; w[2, 5] = 1e-7   # the only salient element codes to 0
+    w[3] = torch.linspace(-1, 1, G, device="cuda")            # many exact half-levels
+    w_h, g_h, v_h = H._host(w), H._host(g), H._host(v)
+    o = api.recon_int_batch([(w, g, v)], bits=3, group_size=G, clip=CLIP8, codes=True,
+                            symmetric=True)[0]
+    torch.cuda.synchronize()
+    h = oracle.ema(v_h, g_h, 0.999)
+    O = oracle.recon_sym(w_h, h, G, 3, CLIP8)
+    gpu = {"r": H._host(o["r"]), "a": o["a"].cpu().numpy(), "b": o["b"].cpu().numpy(),
+           "codes": o["codes"].cpu().numpy().ravel(), "idx": o["cand_idx"].cpu().numpy()}
+    rep = checker.check_sym(oracle, w_h, h, 3, CLIP8, O, gpu, G, True)
+    assert rep["ok"], json.dumps(rep)
+
+
+def test_sym_paper_shaped_layer(oracle):
+    """A Llama-3.1-8B-shaped layer, INT4 symmetric, group 128."""
+    from paper_2608_13966_gb300 import api
+    w_ = wl.workload("llama_layer_int3")
+    ds = [wl.make_tensor(w_, spec, device="cuda") for spec in w_.tensors]
+    hosts = [tuple(H._host(d[k]) for k in ("w", "g", "v")) for d in ds]
+    outs = api.recon_int_batch([(d["w"], d["g"], d["v"]) for d in ds], bits=4, group_size=128,
+                               clip=list(w_.clip), codes=True, symmetric=True)
+    torch.cuda.synchronize()
+    for spec, o, (w_h, g_h, v_h) in zip(w_.tensors, outs, hosts):
+        h = oracle.ema(v_h, g_h, w_.beta2)
+        O = oracle.recon_sym(w_h, h, 128, 4, list(w_.clip))
+        gpu = {"r": H._host(o["r"]), "a": o["a"].cpu().numpy(), "b": o["b"].cpu().numpy(),
+               "codes": o["codes"].cpu().numpy().ravel(), "idx": o["cand_idx"].cpu().numpy()}
+        rep = checker.check_sym(oracle, w_h, h, 4, list(w_.clip), O, gpu, 128, True)
+        assert rep["ok"], (spec.name, json.dumps(rep))
