@@ -185,9 +185,17 @@ class Step:
                 {"w": d["w"], "g": d["g"], "v": d["v"], "r": d["r"], "codes": None, "a": d["a"],
                  "b": d["b"], "cand_idx": d["idx"], "rows": d["spec"].rows, "cols": d["spec"].cols}
                 for d in model.tensors])
-            args = (ctypes.cast(self.descs, ctypes.c_void_p), len(self.descs), Q.BF16, wlo.beta2,
-                    wlo.bits, wlo.group, self.clip, len(wlo.clip), Q.BF16, self.stream)
-            self.calls.append((self.lib.quasar_recon_int_batch, args, model.elements))
+            if wlo.symmetric:
+                self.opt = Q.options(symmetric=True)
+                args = (ctypes.cast(self.descs, ctypes.c_void_p), len(self.descs), Q.BF16,
+                        wlo.beta2, wlo.bits, wlo.group, self.clip, len(wlo.clip), Q.BF16,
+                        ctypes.cast(ctypes.pointer(self.opt), ctypes.c_void_p), self.stream)
+                self.calls.append((self.lib.quasar_recon_int_batch_ex, args, model.elements))
+            else:
+                args = (ctypes.cast(self.descs, ctypes.c_void_p), len(self.descs), Q.BF16,
+                        wlo.beta2, wlo.bits, wlo.group, self.clip, len(wlo.clip), Q.BF16,
+                        self.stream)
+                self.calls.append((self.lib.quasar_recon_int_batch, args, model.elements))
         else:
             # every tensor in one call (quasar_recon_nvfp4_batch): absmax of
             # every tensor, their scales, one reconstruction launch
@@ -442,7 +450,7 @@ def main():
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--workload", default="llama_int3")
     ap.add_argument("--sweep", default="llama_int2,llama_int4,llama_nvfp4,llama_int3_adamw,"
-                                       "llama_nvfp4_adamw,llama_lut")
+                                       "llama_nvfp4_adamw,llama_lut,llama_int4_sym")
     ap.add_argument("--sweep-steps", type=int, default=10)
     ap.add_argument("--e2e-steps", type=int, default=2)
     ap.add_argument("--cpu-budget", type=float, default=12.0)
