@@ -22,6 +22,8 @@
 // codes), are re-evaluated exactly in float-float arithmetic.
 #pragma once
 
+#include <cuda_fp16.h>
+
 #include "device_common.cuh"
 #include "params.h"
 
@@ -154,15 +156,16 @@ __global__ void __launch_bounds__(256) k_recon_nvfp4(const __grid_constant__ Nvf
     int s_cur = 0;
     uint32_t parity = 0;
 
-    // E2M1 magnitudes of two values y in [0, 6] (ties to even): each is
-    // rounded on the grid spacing of its binade (0.5 below 2, 1 in [2, 4), 2
-    // in [4, 6]) by adding and removing a constant whose ulp is that spacing.
+    // E2M1 magnitudes of two values y >= 0: the hardware conversion rounds
+    // to nearest, ties to the even code, and saturates at 6; converting the
+    // pair back through f16x2 gives their values (a goes to the upper half in
+    // both conversions, so y.y is passed first)
     auto e2m1_2 = [](float2 y) -> float2 {
-        // binade of max(y, 1) (a power of two), times 1.5 * 2^22
-        const float2 B = make_float2(__uint_as_float(__float_as_uint(fmaxf(y.x, 1.0f)) & 0x7F800000u),
-                                     __uint_as_float(__float_as_uint(fmaxf(y.y, 1.0f)) & 0x7F800000u));
-        const float2 M = __fmul2_rn(B, make_float2(6291456.0f, 6291456.0f));
-        return __ffma2_rn(M, make_float2(-1.0f, -1.0f), __fadd2_rn(y, M));
+        uint32_t hh;
+        asm("{\n\t.reg .b8 t;\n\tcvt.rn.satfinite.e2m1x2.f32 t, %1, %2;\n\tcvt.rn.f16x2.e2m1x2 %0, t;\n\t}"
+            : "=r"(hh)
+            : "f"(y.y), "f"(y.x));
+        return __half22float2(*reinterpret_cast<__half2*>(&hh));
     };
 
     for (int64_t it = 0;; ++it) {
@@ -271,8 +274,6 @@ __global__ void __launch_bounds__(256) k_recon_nvfp4(const __grid_constant__ Nvf
 #pragma unroll
             for (int t = 0; t < 8; ++t) {
                 float2 y = __fmul2_rn(aw2[t], P2);
-                y.x = fminf(y.x, 6.0f);
-                y.y = fminf(y.y, 6.0f);
                 q2[t] = e2m1_2(y);
                 const float2 hq = __fmul2_rn(h2[t], q2[t]);
                 S2 = __ffma2_rn(hq, q2[t], S2);
@@ -330,8 +331,6 @@ __global__ void __launch_bounds__(256) k_recon_nvfp4(const __grid_constant__ Nvf
 #pragma unroll
                 for (int t = 0; t < 8; ++t) {
                     float2 y = __fmul2_rn(aw2[t], P2);
-                    y.x = fminf(y.x, 6.0f);
-                    y.y = fminf(y.y, 6.0f);
                     q2[t] = e2m1_2(y);
                     const float2 hq = __fmul2_rn(h2[t], q2[t]);
                     S2 = __ffma2_rn(hq, q2[t], S2);
@@ -395,8 +394,6 @@ __global__ void __launch_bounds__(256) k_recon_nvfp4(const __grid_constant__ Nvf
             for (int hh = 0; hh < 2; ++hh) {
                 const int t = 2 * i + hh;
                 float2 y = __fmul2_rn(aw2[t], Pb2);
-                y.x = fminf(y.x, 6.0f);
-                y.y = fminf(y.y, 6.0f);
                 const float2 q = e2m1_2(y);
                 // the code carries the sign of w (magnitude 0 is stored as +0)
                 const float2 qs = make_float2(q.x > 0.0f ? copysignf(q.x, w2[t].x) : 0.0f,
