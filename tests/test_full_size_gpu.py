@@ -78,3 +78,101 @@ def test_full_model_sampled(oracle, name):
     del model
     torch.cuda.empty_cache()
     assert not bad, bad[:3]
+
+
+@pytest.mark.gpu
+def test_full_model_sampled_symmetric(oracle):
+    """Symmetric INT4 (quasar_options.grid) over the 32-layer model, sampled
+    groups against the oracle's symmetric search."""
+    wl = WL.workload("llama_int4_sym")
+    unit = wl.group
+    model = bench.Model(wl, torch.device("cuda"))
+    samples = _sample(model, unit, seed=4321)
+    stream = torch.cuda.Stream()
+    step = bench.Step(model, wl, stream)
+    with torch.cuda.stream(stream):
+        step.run()
+    torch.cuda.synchronize()
+    bad = []
+    for d, (sel, w_s, g_s, v_s, _) in zip(model.tensors, samples):
+        w = w_s.numpy().ravel()
+        h = oracle.ema(v_s.numpy().ravel(), g_s.numpy().ravel(), wl.beta2)
+        ema = checker.check_ema(h, d["v"].view(-1, unit)[sel].cpu().numpy().ravel())
+        O = oracle.recon_sym(w, h, unit, wl.bits, list(wl.clip))
+        r = d["r"].view(-1, unit)[sel].float().cpu().numpy().ravel()
+        a = d["a"][sel].cpu().numpy()
+        # codes are not written in the timed configuration: read them back from r
+        Q = (1 << (wl.bits - 1)) - 1
+        with np.errstate(divide="ignore", invalid="ignore"):
+            q = np.rint(r.reshape(-1, unit) / a[:, None])
+        q = (np.nan_to_num(q) + Q).astype(np.uint8).ravel()
+        gpu = {"r": r, "a": a, "b": d["b"][sel].cpu().numpy(), "codes": q,
+               "idx": d["idx"][sel].cpu().numpy()}
+        rep = checker.check_sym(oracle, w, h, wl.bits, list(wl.clip), O, gpu, unit, True)
+        if not (rep["ok"] and ema["ok"]):
+            bad.append((d["spec"].name, rep, ema))
+    del model
+    torch.cuda.empty_cache()
+    assert not bad, bad[:3]
+
+
+@pytest.mark.gpu
+def test_full_model_sampled_lut(oracle):
+    """The Rubin INT3 lookup table over the 32-layer model, 48 sampled 8x64
+    blocks per tensor against the oracle's App. B search."""
+    wl = WL.workload("llama_lut")
+    model = bench.Model(wl, torch.device("cuda"))
+    rng = np.random.default_rng(99)
+    picks = []
+    for d in model.tensors:
+        spec = d["spec"]
+        nbr, nbc = spec.rows // 8, spec.cols // 64
+        blocks = np.sort(rng.choice(nbr * nbc, size=min(48, nbr * nbc), replace=False))
+        ws, gs, vs = [], [], []
+        for b in blocks:
+            r0, c0 = (b // nbc) * 8, (b % nbc) * 64
+            ws.append(d["w"][r0:r0 + 8, c0:c0 + 64].cpu().numpy())
+            gs.append(d["g"][r0:r0 + 8, c0:c0 + 64].float().cpu().numpy())
+            vs.append(d["v"][r0:r0 + 8, c0:c0 + 64].cpu().numpy())
+        picks.append((blocks, nbc, ws, gs, vs))
+    stream = torch.cuda.Stream()
+    step = bench.Step(model, wl, stream)
+    with torch.cuda.stream(stream):
+        step.run()
+    torch.cuda.synchronize()
+    bad = []
+    for d, (blocks, nbc, ws, gs, vs) in zip(model.tensors, picks):
+        # the sampled blocks side by side: an 8 x (64 * n) tensor
+        w = np.concatenate(ws, 1)
+        h = oracle.ema(np.concatenate(vs, 1).ravel(), np.concatenate(gs, 1).ravel(),
+                       wl.beta2).reshape(8, -1)
+        O = oracle.recon_lut(w, h, list(wl.clip))
+        r = np.concatenate([d["r"][(b // nbc) * 8:(b // nbc) * 8 + 8,
+                                   (b % nbc) * 64:(b % nbc) * 64 + 64].float().cpu().numpy()
+                            for b in blocks], 1)
+        book = d["book"][torch.as_tensor(blocks, device="cuda")].cpu().numpy()
+        idx = d["idx"][torch.as_tensor(blocks, device="cuda")].cpu().numpy()
+        # indices are not written in the timed configuration: read them back from r
+        vals = np.array([[oracle.e4m3s_value(x) for x in row] for row in book])
+        rb = oracle.lut_blocks(r)
+        qo = oracle.lut_blocks(O["codes"].reshape(w.shape))
+        q = np.zeros_like(rb, dtype=np.uint8)
+        for i in range(rb.shape[0]):
+            hit = rb[i][:, None] == vals[i][None, :]
+            q[i] = np.argmax(hit, 1)
+            # an entry value held by two indices does not name one: where r is
+            # the oracle's entry, that index is as good as the GPU's
+            same = hit[np.arange(hit.shape[0]), qo[i]]
+            q[i][same] = qo[i][same]
+        codes = q.reshape(1, len(blocks), 8, 64).transpose(0, 2, 1, 3).reshape(8, -1)
+        gpu = {"r": r.ravel(), "book": book, "codes": codes, "idx": idx}
+        rep = checker.check_lut(oracle, w, h, list(wl.clip), O, gpu)
+        v_gpu = np.concatenate([d["v"][(b // nbc) * 8:(b // nbc) * 8 + 8,
+                                       (b % nbc) * 64:(b % nbc) * 64 + 64].cpu().numpy()
+                                for b in blocks], 1)
+        ema = checker.check_ema(h.ravel(), v_gpu.ravel())
+        if not (rep["ok"] and ema["ok"]):
+            bad.append((d["spec"].name, rep, ema))
+    del model
+    torch.cuda.empty_cache()
+    assert not bad, bad[:3]
