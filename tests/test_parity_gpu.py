@@ -666,3 +666,31 @@ def test_sym_paper_shaped_layer(oracle):
                "codes": o["codes"].cpu().numpy().ravel(), "idx": o["cand_idx"].cpu().numpy()}
         rep = checker.check_sym(oracle, w_h, h, 4, list(w_.clip), O, gpu, 128, True)
         assert rep["ok"], (spec.name, json.dumps(rep))
+
+
+@pytest.mark.parametrize("path", ["nvfp4", "lut", "sym", "adamw"])
+def test_timeout_path_of_every_kernel(oracle, path):
+    """Each kernel's bounded wait: a barrier nothing arrives at runs out after
+    1 ms, the kernel records the timeout and returns, the status reports it
+    once, and the next call is correct."""
+    from paper_2608_13966_gb300 import api, quasar
+    w, g, v = _inputs(64, 512, seed=2000)
+    assert quasar.quasar_get_device_status() == quasar.QuasarStatus.OK
+    quasar.quasar_debug_force_timeout(1_000_000)
+    try:
+        if path == "nvfp4":
+            api.recon_nvfp4_batch([(w, g, v)], clip=CLIP8)
+        elif path == "lut":
+            api.recon_lut_batch([(w, g, v)], clip=CLIP8)
+        elif path == "sym":
+            api.recon_int_batch([(w, g, v)], bits=3, group_size=128, clip=CLIP8, symmetric=True)
+        else:
+            m = wl.first_moment((64, 512), 2000, device="cuda")
+            api.adamw_recon_int_batch([(w, g, m, v)], lr=1e-5, step=1, bits=3, group_size=128,
+                                      clip=CLIP8)
+    finally:
+        quasar.quasar_debug_force_timeout(0)
+    assert quasar.quasar_get_device_status() == quasar.QuasarStatus.ERR_TIMEOUT
+    assert quasar.quasar_get_device_status() == quasar.QuasarStatus.OK
+    rep, ema = H.run_int(oracle, *_inputs(64, 512, seed=2001), bits=3, group_size=128, clip=CLIP8)
+    _assert(rep, ema)
