@@ -694,3 +694,54 @@ def test_timeout_path_of_every_kernel(oracle, path):
     assert quasar.quasar_get_device_status() == quasar.QuasarStatus.OK
     rep, ema = H.run_int(oracle, *_inputs(64, 512, seed=2001), bits=3, group_size=128, clip=CLIP8)
     _assert(rep, ema)
+
+
+def test_adamw_recon_nvfp4_fp32_gradient_and_options(oracle):
+    """The AdamW + NVFP4 step with an fp32 gradient, h = v'^2 and packed codes."""
+    from paper_2608_13966_gb300 import api
+    hp = dict(wl.ADAMW_NVFP4)
+    w, g, v = _inputs(40, 512, seed=2100, g_dtype=torch.float32)
+    m = wl.first_moment((40, 512), 2100, device="cuda")
+    w_h, g_h, m_h, v_h = (H._host(t) for t in (w, g, m, v))
+    o = api.adamw_recon_nvfp4_batch([(w, g, m, v)], lr=hp["lr"], beta1=hp["beta1"], beta2=0.999,
+                                    eps=hp["eps"], weight_decay=hp["weight_decay"],
+                                    step=hp["step"], clip=CLIP8, codes=True,
+                                    saliency="ema_squared", packed_codes=True,
+                                    r_dtype=torch.float32)[0]
+    torch.cuda.synchronize()
+    hp32 = _hp32(hp, 0.999)
+    w1, m1, v1 = oracle.adamw(w_h, g_h, m_h, v_h, **hp32)
+    st = checker.check_adamw(w_h, g_h, m_h, hp32, w1, m1, v1, H._host(w), H._host(m), H._host(v))
+    assert st["ok"], json.dumps(st)
+    h = oracle.saliency(v1, "ema_squared")
+    _, s_T = oracle.tensor_scale(w1)
+    O = oracle.recon_nvfp4(w1, h, s_T, CLIP8)
+    gpu = {"r": H._host(o["r"]), "scale": o["block_scale"].cpu().numpy(),
+           "tensor_scale": float(o["tensor_scale"].cpu()[0]),
+           "codes": oracle.unpack_nvfp4_codes(o["codes"].cpu().numpy()),
+           "idx": o["cand_idx"].cpu().numpy()}
+    rep = checker.check_nvfp4(oracle, w1, h, CLIP8, s_T, O, gpu, False)
+    assert rep["ok"], json.dumps(rep)
+
+
+def test_more_than_one_launch_of_tensors(oracle):
+    """300 tensors in one batch call: more than a launch holds (256), so the
+    call makes two launches; every tensor matches the oracle."""
+    from paper_2608_13966_gb300 import api
+    items, hosts = [], []
+    for i in range(300):
+        w, g, v = _inputs(2, 128, seed=3000 + i)
+        items.append((w, g, v))
+        hosts.append((H._host(w), H._host(g), H._host(v)))
+    outs = api.recon_int_batch(items, bits=3, group_size=128, clip=CLIP8, codes=True)
+    torch.cuda.synchronize()
+    w_h = np.concatenate([h[0] for h in hosts])
+    hh = np.concatenate([oracle.ema(h[2], h[1], 0.999) for h in hosts])
+    O = oracle.recon_int(w_h, hh, 128, 3, CLIP8)
+    gpu = {"r": np.concatenate([H._host(o["r"]) for o in outs]),
+           "a": np.concatenate([o["a"].cpu().numpy() for o in outs]),
+           "b": np.concatenate([o["b"].cpu().numpy() for o in outs]),
+           "codes": np.concatenate([o["codes"].cpu().numpy().ravel() for o in outs]),
+           "idx": np.concatenate([o["cand_idx"].cpu().numpy() for o in outs])}
+    rep = checker.check_int(oracle, w_h, hh, 3, CLIP8, O, gpu, 128, True)
+    assert rep["ok"], json.dumps(rep)
