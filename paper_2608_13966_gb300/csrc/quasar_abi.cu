@@ -252,7 +252,6 @@ quasar_status launch_persistent(const void* fn, void* params, size_t smem, int64
     return QUASAR_OK;
 }
 
-int g_kind_of(const void* g, quasar_dtype d) { return !g ? 0 : (d == QUASAR_BF16 ? 2 : 1); }
 
 // Variant options of a call (quasar_options; NULL means the defaults).
 struct Opts {
