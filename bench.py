@@ -368,6 +368,35 @@ def timed_steps(step, n_launch_calls, steps, warmup, world):
     return total_ms, kernel_ms
 
 
+def host_link(host, dev, s_in, s_out, reps=3):
+    """Pinned-copy rates of this machine's host link on one layer's e2e buffers:
+    host-to-device (w, g, v), device-to-host (r, v', a, b, index), and both
+    at once on two streams (GB/s)."""
+    def run(inb, outb):
+        torch.cuda.synchronize()
+        t0 = time.perf_counter()
+        for _ in range(reps):
+            if inb:
+                with torch.cuda.stream(s_in):
+                    for h, d in zip(host, dev):
+                        for k in ("w", "g", "v"):
+                            d[k].copy_(h[k], non_blocking=True)
+            if outb:
+                with torch.cuda.stream(s_out):
+                    for h, d in zip(host, dev):
+                        for k in ("r", "v", "a", "b", "idx"):
+                            h[k].copy_(d[k], non_blocking=True)
+        torch.cuda.synchronize()
+        return (time.perf_counter() - t0) / reps
+
+    nin = sum(h[k].numel() * h[k].element_size() for h in host for k in ("w", "g", "v"))
+    nout = sum(h[k].numel() * h[k].element_size() for h in host for k in ("r", "v", "a", "b", "idx"))
+    run(True, True)
+    t_in, t_out, t_both = run(True, False), run(False, True), run(True, True)
+    return {"h2d_gbs": nin / t_in / 1e9, "d2h_gbs": nout / t_out / 1e9,
+            "both_gbs": (nin + nout) / t_both / 1e9}
+
+
 def e2e_rate(wlo, steps, device, stream):
     """Same metric through the C ABI with HOST buffers: every step copies each
     tensor's w, g, v from pinned host memory, reconstructs, and reads r, v',
@@ -437,8 +466,14 @@ def e2e_rate(wlo, steps, device, stream):
     for _ in range(steps):
         one_step()
     dt = (time.perf_counter() - t0) / steps
+    link = host_link(host[0], dev[0], s_in, s_out)
+    # the copies alone need at least this long: in at the one-way rate, out
+    # at its rate, and both over the link's two-way rate
+    bound = max(h2d / link["h2d_gbs"], d2h / link["d2h_gbs"], (h2d + d2h) / link["both_gbs"]) / 1e9
+    link["copy_bound_ms"] = bound * 1e3
+    link["frac_of_copy_bound"] = bound / dt
     return {"value": elements / dt, "unit": "weights/s", "h2d_bytes_per_step": int(h2d),
-            "d2h_bytes_per_step": int(d2h), "ms_per_step": dt * 1e3,
+            "d2h_bytes_per_step": int(d2h), "ms_per_step": dt * 1e3, "host_link": link,
             "how": "one quasar_recon_int_batch call per layer on pinned host buffers: H2D of "
                    "w/g/v, the call, D2H of r/v/a/b/idx, pipelined over three streams with two "
                    "device slots, all inside the timed region"}

@@ -441,6 +441,17 @@ void quasar_debug_force_timeout(int64_t nanoseconds);
  */
 void quasar_debug_set_stats(unsigned int* device_counters);
 
+/*
+ * quasar_debug_set_hoist -- tuning hook.  The integer entry points pick, for
+ * a batch of at most 8 candidates whose factors allow it, a kernel that
+ * clamps |w - c| once per set of 4 candidates instead of every candidate's
+ * code (the codes are the same bit for bit).  While enable is 0 they always
+ * take the per-candidate clamp; 1 (the default, or the environment variable
+ * QUASAR_HOIST at load) restores the automatic choice.  Process-wide; never
+ * needed in normal use.
+ */
+void quasar_debug_set_hoist(int enable);
+
 /* Static, human-readable name of a status code. */
 const char* quasar_status_string(quasar_status status);
 

@@ -26,6 +26,7 @@ UNITS = [
     ("kernels_int.cu", ["-DQUASAR_NCH=1"], "kernels_int_nch1.o"),
     ("kernels_int.cu", ["-DQUASAR_NCH=2"], "kernels_int_nch2.o"),
     ("kernels_int.cu", ["-DQUASAR_NCH=4"], "kernels_int_nch4.o"),
+    ("kernels_int.cu", ["-DQUASAR_NCH=1", "-DQUASAR_HC=1"], "kernels_int_hc.o"),
     ("kernels_nvfp4.cu", [], "kernels_nvfp4.o"),
     ("kernels_lut.cu", [], "kernels_lut.o"),
     ("kernels_sym.cu", [], "kernels_sym.o"),

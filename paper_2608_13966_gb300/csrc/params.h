@@ -60,6 +60,10 @@ struct IntParams {
     unsigned int* stats;  // optional: [0] exact re-evaluations, [1] compensated fits, [2] centred refits
     float f[kMaxClip];     // padded with the last factor
     float invf[kMaxClip];  // fl32(1/f)
+    // hoisted code clamps (the HC kernels): for each set of 4 consecutive
+    // candidate slots, tau / qmax, so that the set's cap on |w - c| is
+    // hcap * range; 0 where no tau exists
+    float hcap[kMaxClip / 4];
     // fused AdamW step: w' = w - (w*lr_wd + step_size * m' / (sqrt(v') * isbc2 + eps))
     float beta1, c1b;      // beta1, 1 - beta1
     float lr_wd;           // lr * weight_decay

@@ -18,6 +18,7 @@ namespace quasar {
 const void* int_kernel_nch1(int epl, bool batch, bool adam, bool var);
 const void* int_kernel_nch2(int epl, bool batch, bool adam, bool var);
 const void* int_kernel_nch4(int epl, bool batch, bool adam, bool var);
+const void* int_kernel_hc(int epl, bool adam);
 const void* nvfp4_kernel(int nch, bool batch);
 const void* amax_kernel(bool batch);
 const void* amax_to_scale_kernel(bool batch);
@@ -45,6 +46,7 @@ constexpr uint64_t kDefaultTimeoutNs = 1000000000ull;  // 1 s per wait
 
 std::atomic<int64_t> g_force_timeout_ns{0};
 std::atomic<unsigned int*> g_stats{nullptr};
+std::atomic<int> g_hoist{-1};  // -1: the environment's choice (tuning().hoist)
 
 struct Tuning {
     int stages = 0;            // 0: chosen from the shared-memory budget
@@ -52,6 +54,7 @@ struct Tuning {
     float tie_kappa = 16.0f;   // NVFP4 tie bound, in ulps
     float tie_scale = 1.0f;    // multiplier of the integer kernel's summation-depth bound
     float fit_ulps = 3.0f;
+    int hoist = 1;             // 0: never the hoisted-clamp integer kernel
 };
 
 const Tuning& tuning()
@@ -63,6 +66,7 @@ const Tuning& tuning()
         if (const char* s = std::getenv("QUASAR_TIE_KAPPA")) x.tie_kappa = (float)std::atof(s);
         if (const char* s = std::getenv("QUASAR_TIE_SCALE")) x.tie_scale = (float)std::atof(s);
         if (const char* s = std::getenv("QUASAR_FIT_ULPS")) x.fit_ulps = (float)std::atof(s);
+        if (const char* s = std::getenv("QUASAR_HOIST")) x.hoist = std::atoi(s);
         return x;
     }();
     return t;
@@ -120,6 +124,27 @@ void fill_clip(const float* clip, int n_clip, float* f, float* invf)
         const float fk = clip[std::min(k, n_clip - 1)];
         f[k] = fk;
         invf[k] = (float)(1.0 / (double)fk);
+    }
+}
+
+// Hoisted code clamps of the integer kernel.  For each set of 4 consecutive
+// candidate slots: a tau with J f_max (1 + 1e-3) <= tau <= (J + 1) f_min
+// (1 - 1e-3), J = (qmax - 1) / 2.  Then min(|d|, tau range / qmax) P_k has
+// the code min(floor(|d| P_k), J) for every slot k of the set: a capped |d|
+// gives cap P_k ~ tau / f_k in [J, J + 1), and below the cap
+// |d| P_k < J + 1.  The margin covers the fp32 roundings of the cap, of R
+// and of P.  Stored as tau / qmax; 0 where no tau exists.
+void fill_hcap(IntParams* p)
+{
+    const int J = p->qmax >> 1;
+    for (int s = 0; s < kMaxClip / 4; ++s) {
+        double fmax = 0.0, fmin = 2.0;
+        for (int k = 4 * s; k < 4 * s + 4; ++k) {
+            fmax = std::max(fmax, (double)p->f[k]);
+            fmin = std::min(fmin, (double)p->f[k]);
+        }
+        const double lo = J * fmax * (1.0 + 1e-3), hi = (J + 1) * fmin * (1.0 - 1e-3);
+        p->hcap[s] = lo < hi ? (float)(0.5 * (lo + hi) / p->qmax) : 0.0f;
     }
 }
 
@@ -356,6 +381,7 @@ quasar_status int_params(quasar_dtype g_dtype, bool has_g, float beta2, int bits
     p->force_timeout_ns = (uint64_t)std::max<int64_t>(0, g_force_timeout_ns.load());
     p->stats = g_stats.load();
     fill_clip(clip, n_clip, p->f, p->invf);
+    fill_hcap(p);
     quasar_status st;
     if ((st = status_ptr(&p->status)) != QUASAR_OK) return st;
     if (adam) {
@@ -395,7 +421,12 @@ quasar_status int_launch(IntLaunch<MAXT>& Lp, int group_size, int n_clip, cudaSt
     const int nch = nch_for(n_clip);
     const bool batch = MAXT > 1;
     const bool var = Lp.p.h_mode != kSalEma || Lp.p.codes_packed;
+    // the hoisted-clamp kernel where both slot sets of the one chunk have a cap
+    const int hoist_on = g_hoist.load() < 0 ? tuning().hoist : g_hoist.load();
+    const bool hoist = batch && !var && nch == 1 && hoist_on && Lp.p.hcap[0] > 0.0f &&
+                       Lp.p.hcap[1] > 0.0f;
     const void* fn = symmetric  ? (MAXT > 1 ? sym_kernel(epl) : nullptr)
+                     : hoist    ? int_kernel_hc(epl, adam)
                      : nch == 1 ? int_kernel_nch1(epl, batch, adam, var)
                      : nch == 2 ? int_kernel_nch2(epl, batch, adam, var)
                                 : int_kernel_nch4(epl, batch, adam, var);
@@ -945,6 +976,8 @@ quasar_status quasar_get_device_status(quasar_stream_t stream)
 void quasar_debug_force_timeout(int64_t nanoseconds) { g_force_timeout_ns.store(nanoseconds); }
 
 void quasar_debug_set_stats(unsigned int* device_counters) { g_stats.store(device_counters); }
+
+void quasar_debug_set_hoist(int enable) { g_hoist.store(enable ? 1 : 0); }
 
 const char* quasar_status_string(quasar_status status)
 {

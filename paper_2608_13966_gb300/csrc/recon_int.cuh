@@ -358,7 +358,14 @@ __device__ void coop_precise(const float* ws, const float* hs, float c, float P,
 // Two CTAs per SM: 8-warp CTAs, 6-warp ones for the AdamW-fused variant.
 // VAR: the variants of the options (a saliency other than v', packed codes);
 // without it they compile out of the common kernel.
-template <int EPL, int NCH, int MAXT, bool ADAM, bool VAR>
+// HC: the code clamp is hoisted out of the candidate loop.  For a set of
+// candidate slots whose factors satisfy J f_max < tau < (J + 1) f_min (with
+// a margin the host checks), clamping |d| once at tau * range / qmax gives
+// every candidate of the set its clamped code: below the cap no code
+// reaches J + 1, above it every code is J.  The codes equal the per-candidate
+// clamp's bit for bit whenever R is finite; the set's cap costs one min per
+// element instead of one per element and candidate.
+template <int EPL, int NCH, int MAXT, bool ADAM, bool VAR, bool HC = false>
 __global__ void __launch_bounds__(ADAM ? 192 : 256, 2)
     k_recon_int(const __grid_constant__ IntLaunch<MAXT> Lp)
 {
@@ -659,6 +666,13 @@ __global__ void __launch_bounds__(ADAM ? 192 : 256, 2)
                     const float2 d = __fadd2_rn(wv, nc2);
                     const float2 ev = __fadd2_rn(wv, nmu2);
                     const float2 ad = abs2(d);
+                    float2 adc[2];
+                    if constexpr (HC) {
+                        // the caps of the chunk's two slot sets
+                        const float cap0 = p.hcap[ch * 2] * range, cap1 = p.hcap[ch * 2 + 1] * range;
+                        adc[0] = make_float2(fminf(ad.x, cap0), fminf(ad.y, cap0));
+                        adc[1] = make_float2(fminf(ad.x, cap1), fminf(ad.y, cap1));
+                    }
                     const float2 hsg = signed_h2(h, d);
                     const float2 sev = make_float2(
                         __uint_as_float(__float_as_uint(ev.x) ^ (__float_as_uint(d.x) & 0x80000000u)),
@@ -670,9 +684,14 @@ __global__ void __launch_bounds__(ADAM ? 192 : 256, 2)
                     }
 #pragma unroll
                     for (int kk = 0; kk < 8; ++kk) {
-                        float2 y = __ffma2_rd(ad, P2[kk], M2);
-                        y.x = fminf(y.x, zcap);
-                        y.y = fminf(y.y, zcap);
+                        float2 y;
+                        if constexpr (HC) {
+                            y = __ffma2_rd(adc[kk >> 2], P2[kk], M2);
+                        } else {
+                            y = __ffma2_rd(ad, P2[kk], M2);
+                            y.x = fminf(y.x, zcap);
+                            y.y = fminf(y.y, zcap);
+                        }
                         const float2 z = __fadd2_rn(y, nhm2);  // |z|
                         const float2 t = __fmul2_rn(h, z);
                         A1[kk] = __ffma2_rn(hsg, z, A1[kk]);

@@ -55,6 +55,7 @@ PROTOTYPES = {
     "quasar_get_device_status": (_I, [_P]),
     "quasar_debug_force_timeout": (None, [_I64]),
     "quasar_debug_set_stats": (None, [_P]),
+    "quasar_debug_set_hoist": (None, [_I]),
     "quasar_status_string": (ctypes.c_char_p, [_I]),
     "quasar_version": (_I, []),
 }
@@ -378,6 +379,10 @@ def quasar_debug_force_timeout(nanoseconds: int) -> None:
 
 def quasar_debug_set_stats(counters) -> None:
     load().quasar_debug_set_stats(_ptr(counters))
+
+
+def quasar_debug_set_hoist(enable: bool) -> None:
+    load().quasar_debug_set_hoist(1 if enable else 0)
 
 
 def quasar_status_string(status) -> str:

@@ -194,6 +194,88 @@ def test_int_batch_matches_oracle_and_single_calls(oracle):
         _assert(rep, ema)
 
 
+def _hoistable(bits, clip):
+    """Whether both slot sets of the one candidate chunk admit a hoisted
+    code clamp: J f_max (1 + 1e-3) < (J + 1) f_min (1 - 1e-3)."""
+    f = [float(np.float32(clip[min(k, len(clip) - 1)])) for k in range(8)]
+    J = ((1 << bits) - 1) >> 1
+    return all(J * max(f[s:s + 4]) * 1.001 < (J + 1) * min(f[s:s + 4]) * 0.999 for s in (0, 4))
+
+
+NARROW8 = [1.0, 0.99, 0.98, 0.97, 0.96, 0.95, 0.94, 0.93]
+
+
+def _edge_inputs(rows, cols, seed):
+    """Ragged t4 weights with the degenerate groups of the edge-case test."""
+    w, g, v = _inputs(rows, cols, seed=seed)
+    if rows >= 6:
+        w[0] = 0.25                                  # zero range
+        v[1] = 0.0; g[1] = 0.0                       # all saliency zero
+        v[2] = 0.0; g[2] = 0.0; v[2, 17] = 1e-6      # one salient element
+        w[3, ::2] = 0.0                              # many exact zeros
+        w[4, 5] = 3.0                                # one outlier
+        w[5] = torch.linspace(-1, 1, cols, device="cuda")  # codes on grid boundaries
+    return w, g, v
+
+
+@pytest.mark.parametrize("bits,clip", [(1, CLIP8), (2, CLIP8), (3, CLIP8), (3, CLIP8[:5]),
+                                       (4, NARROW8)])
+@pytest.mark.parametrize("G", [32, 64, 128, 256])
+def test_int_hoisted_clamp_equals_per_candidate_clamp(bits, clip, G):
+    """The batch kernel that clamps |w - c| once per set of 4 candidates gives
+    bit for bit the outputs of the kernel that clamps every candidate's code
+    (itself checked against the oracle above), on ragged shapes with
+    degenerate groups."""
+    from paper_2608_13966_gb300 import api, quasar
+    assert _hoistable(bits, clip)
+    shapes = [(37, 3 * G), (8, 2 * G), (1, G)]
+    base = [_edge_inputs(r, c, seed=900 + 10 * bits + i) for i, (r, c) in enumerate(shapes)]
+    outs = {}
+    try:
+        for hoist in (True, False):
+            quasar.quasar_debug_set_hoist(hoist)
+            items = [(w.clone(), g.clone(), v.clone()) for w, g, v in base]
+            o = api.recon_int_batch(items, bits=bits, group_size=G, clip=clip, codes=True)
+            torch.cuda.synchronize()
+            outs[hoist] = (o, [v for _, _, v in items])
+    finally:
+        quasar.quasar_debug_set_hoist(True)
+    for i in range(len(shapes)):
+        for key in ("r", "a", "b", "codes", "cand_idx"):
+            assert torch.equal(outs[True][0][i][key], outs[False][0][i][key]), (shapes[i], key)
+        assert torch.equal(outs[True][1][i], outs[False][1][i])
+
+
+def test_adamw_int_hoisted_clamp_equals_per_candidate_clamp():
+    """The fused AdamW + INT3 batch kernel: hoisted and per-candidate clamps
+    give the same w', m', v' and outputs bit for bit."""
+    from paper_2608_13966_gb300 import api, quasar
+    hp = dict(wl.ADAMW_LLAMA_INT3)
+    shapes = [(37, 384), (64, 512)]
+    base = []
+    for i, (rows, cols) in enumerate(shapes):
+        w, g, v = _edge_inputs(rows, cols, seed=950 + i)
+        base.append((w, g, wl.first_moment((rows, cols), 950 + i, device="cuda"), v))
+    outs = {}
+    try:
+        for hoist in (True, False):
+            quasar.quasar_debug_set_hoist(hoist)
+            items = [tuple(t.clone() for t in it) for it in base]
+            o = api.adamw_recon_int_batch(items, lr=hp["lr"], beta1=hp["beta1"], beta2=0.999,
+                                          eps=hp["eps"], weight_decay=hp["weight_decay"],
+                                          step=hp["step"], bits=3, group_size=128, clip=CLIP8,
+                                          codes=True)
+            torch.cuda.synchronize()
+            outs[hoist] = (o, items)
+    finally:
+        quasar.quasar_debug_set_hoist(True)
+    for i in range(len(shapes)):
+        for key in ("r", "a", "b", "codes", "cand_idx"):
+            assert torch.equal(outs[True][0][i][key], outs[False][0][i][key]), (shapes[i], key)
+        for a, b in zip(outs[True][1][i], outs[False][1][i]):
+            assert torch.equal(a, b)
+
+
 def test_nvfp4_batch_matches_oracle_and_single_calls(oracle):
     """One absmax pass, one scale pass and one reconstruction launch over
     tensors of different shapes (one with its amax supplied, a tiny one, an
