@@ -370,27 +370,28 @@ def timed_steps(step, n_launch_calls, steps, warmup, world):
 
 def host_link(host, dev, s_in, s_out, reps=3):
     """Pinned-copy rates of this machine's host link on one layer's e2e buffers:
-    host-to-device (w, g, v), device-to-host (r, v', a, b, index), and both
-    at once on two streams (GB/s)."""
+    host-to-device (w, g, v into slot 0), device-to-host (r, v', a, b, index
+    out of slot 1), and both at once on two streams, as the pipeline overlaps
+    them (GB/s)."""
     def run(inb, outb):
         torch.cuda.synchronize()
         t0 = time.perf_counter()
         for _ in range(reps):
             if inb:
                 with torch.cuda.stream(s_in):
-                    for h, d in zip(host, dev):
+                    for h, d in zip(host[0], dev[0]):
                         for k in ("w", "g", "v"):
                             d[k].copy_(h[k], non_blocking=True)
             if outb:
                 with torch.cuda.stream(s_out):
-                    for h, d in zip(host, dev):
+                    for h, d in zip(host[1], dev[1]):
                         for k in ("r", "v", "a", "b", "idx"):
                             h[k].copy_(d[k], non_blocking=True)
         torch.cuda.synchronize()
         return (time.perf_counter() - t0) / reps
 
-    nin = sum(h[k].numel() * h[k].element_size() for h in host for k in ("w", "g", "v"))
-    nout = sum(h[k].numel() * h[k].element_size() for h in host for k in ("r", "v", "a", "b", "idx"))
+    nin = sum(h[k].numel() * h[k].element_size() for h in host[0] for k in ("w", "g", "v"))
+    nout = sum(h[k].numel() * h[k].element_size() for h in host[1] for k in ("r", "v", "a", "b", "idx"))
     run(True, True)
     t_in, t_out, t_both = run(True, False), run(False, True), run(True, True)
     return {"h2d_gbs": nin / t_in / 1e9, "d2h_gbs": nout / t_out / 1e9,
@@ -466,7 +467,7 @@ def e2e_rate(wlo, steps, device, stream):
     for _ in range(steps):
         one_step()
     dt = (time.perf_counter() - t0) / steps
-    link = host_link(host[0], dev[0], s_in, s_out)
+    link = host_link(host, dev, s_in, s_out)
     # the copies alone need at least this long: in at the one-way rate, out
     # at its rate, and both over the link's two-way rate
     bound = max(h2d / link["h2d_gbs"], d2h / link["d2h_gbs"], (h2d + d2h) / link["both_gbs"]) / 1e9

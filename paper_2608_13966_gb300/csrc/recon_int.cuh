@@ -67,12 +67,6 @@ __device__ __forceinline__ float int_code_z(float d, float P, float zcap)
     return copysignf(__fsub_rn(y, kHalfBelowMagic), d);
 }
 
-__device__ __forceinline__ float2 abs2(float2 x)
-{
-    return make_float2(__uint_as_float(__float_as_uint(x.x) & 0x7FFFFFFFu),
-                       __uint_as_float(__float_as_uint(x.y) & 0x7FFFFFFFu));
-}
-
 // h with the sign of d (h >= 0): the sign survives h = 0 as -0.
 __device__ __forceinline__ float2 signed_h2(float2 h, float2 d)
 {
@@ -665,7 +659,8 @@ __global__ void __launch_bounds__(ADAM ? 192 : 256, 2)
                     const float2 h = pr ? make_float2(h4.z, h4.w) : make_float2(h4.x, h4.y);
                     const float2 d = __fadd2_rn(wv, nc2);
                     const float2 ev = __fadd2_rn(wv, nmu2);
-                    const float2 ad = abs2(d);
+                    // |d| as fabsf: the compiler folds it into the min/FMA operands
+                    const float2 ad = make_float2(fabsf(d.x), fabsf(d.y));
                     float2 adc[2];
                     if constexpr (HC) {
                         // the caps of the chunk's two slot sets
@@ -908,7 +903,7 @@ __global__ void __launch_bounds__(ADAM ? 192 : 256, 2)
                     const float2 wv = pr ? make_float2(w4.z, w4.w) : make_float2(w4.x, w4.y);
                     const float2 h = pr ? make_float2(h4.z, h4.w) : make_float2(h4.x, h4.y);
                     const float2 d = __fadd2_rn(wv, nc2);
-                    float2 y = __ffma2_rd(abs2(d), Pk2, M2);
+                    float2 y = __ffma2_rd(make_float2(fabsf(d.x), fabsf(d.y)), Pk2, M2);
                     y.x = fminf(y.x, zcap);
                     y.y = fminf(y.y, zcap);
                     const float2 z = __fadd2_rn(y, nhm2);
@@ -1027,7 +1022,7 @@ __global__ void __launch_bounds__(ADAM ? 192 : 256, 2)
                         for (int pr = 0; pr < 2; ++pr) {
                             const float2 wv = pr ? make_float2(w4.z, w4.w) : make_float2(w4.x, w4.y);
                             const float2 d = __fadd2_rn(wv, nc2);
-                            float2 y = __ffma2_rd(abs2(d), Pk2, M2);
+                            float2 y = __ffma2_rd(make_float2(fabsf(d.x), fabsf(d.y)), Pk2, M2);
                             y.x = fminf(y.x, zcap);
                             y.y = fminf(y.y, zcap);
                             const float2 z = __fadd2_rn(y, nhm2);
