@@ -368,6 +368,17 @@ def timed_steps(step, n_launch_calls, steps, warmup, world):
     return total_ms, kernel_ms
 
 
+def hoisted_clamp(bits, clip):
+    """Whether the library runs the hoisted-clamp integer kernel for this
+    candidate list (8 or fewer candidates, both slot sets with a cap; the
+    library's own test, restated to name the kernel in the report)."""
+    if len(clip) > 8 or os.environ.get("QUASAR_HOIST", "1") == "0":
+        return False
+    f = [float(np.float32(clip[min(k, len(clip) - 1)])) for k in range(8)]
+    J = ((1 << bits) - 1) >> 1
+    return all(J * max(f[s:s + 4]) * 1.001 < (J + 1) * min(f[s:s + 4]) * 0.999 for s in (0, 4))
+
+
 def host_link(host, dev, s_in, s_out, reps=3):
     """Pinned-copy rates of this machine's host link on one layer's e2e buffers:
     host-to-device (w, g, v into slot 0), device-to-host (r, v', a, b, index
@@ -398,7 +409,7 @@ def host_link(host, dev, s_in, s_out, reps=3):
             "both_gbs": (nin + nout) / t_both / 1e9}
 
 
-def e2e_rate(wlo, steps, device, stream):
+def e2e_rate(wlo, steps, device, stream, n_slots=2):
     """Same metric through the C ABI with HOST buffers: every step copies each
     tensor's w, g, v from pinned host memory, reconstructs, and reads r, v',
     a, b and the kept index back.  Layers are pipelined over three streams
@@ -410,11 +421,11 @@ def e2e_rate(wlo, steps, device, stream):
     lib = Q.load()
     n_layers = len(wlo.tensors) // 7
     specs = wlo.tensors[:7]
-    host, dev = [[], []], [[], []]
+    host, dev = [[] for _ in range(n_slots)], [[] for _ in range(n_slots)]
     for spec in specs:
         d = WL.make_tensor(wlo, spec, device=device)
         n = spec.numel
-        for slot in range(2):
+        for slot in range(n_slots):
             h = {k: v.cpu().pin_memory() for k, v in d.items()}
             h["r"] = torch.empty((spec.rows, spec.cols), dtype=torch.bfloat16).pin_memory()
             h["a"] = torch.empty(n // wlo.group, dtype=torch.float32).pin_memory()
@@ -431,14 +442,14 @@ def e2e_rate(wlo, steps, device, stream):
     descs = [Q.int_tensor_array([
         {"w": d["w"], "g": d["g"], "v": d["v"], "r": d["r"], "codes": None, "a": d["a"],
          "b": d["b"], "cand_idx": d["idx"], "rows": sp.rows, "cols": sp.cols}
-        for d, sp in zip(dev[slot], specs)]) for slot in range(2)]
+        for d, sp in zip(dev[slot], specs)]) for slot in range(n_slots)]
     s_in, s_out = torch.cuda.Stream(), torch.cuda.Stream()
-    ev = {name: [torch.cuda.Event(), torch.cuda.Event()] for name in ("in", "comp", "out")}
-    started = [False, False]
+    ev = {name: [torch.cuda.Event() for _ in range(n_slots)] for name in ("in", "comp", "out")}
+    started = [False] * n_slots
 
     def one_step():
         for layer in range(n_layers):
-            slot = layer & 1
+            slot = layer % n_slots
             with torch.cuda.stream(s_in):
                 if started[slot]:
                     s_in.wait_event(ev["out"][slot])  # the slot's previous layer is out
@@ -516,6 +527,7 @@ def main():
                                        "llama_nvfp4_adamw,llama_lut,llama_int4_sym")
     ap.add_argument("--sweep-steps", type=int, default=10)
     ap.add_argument("--e2e-steps", type=int, default=2)
+    ap.add_argument("--e2e-slots", type=int, default=2)
     ap.add_argument("--cpu-budget", type=float, default=12.0)
     ap.add_argument("--ref-budget", type=float, default=8.0)
     args = ap.parse_args()
@@ -565,7 +577,7 @@ def main():
     if args.e2e_steps > 0 and rank == 0:
         del model
         torch.cuda.empty_cache()
-        e2e = e2e_rate(wlo, args.e2e_steps, device, stream)
+        e2e = e2e_rate(wlo, args.e2e_steps, device, stream, args.e2e_slots)
         e2e["value"] *= world
 
     cpu = None
@@ -579,8 +591,9 @@ def main():
     # differ in size; bytes and time both scale with the weights processed)
     if wlo.fmt == "int":
         tag = "k_recon_int_g%d_k%d%s" % (wlo.group, len(wlo.clip), "_adamw" if wlo.adamw else "")
-        kname = "k_recon_int<%d,1,256,%s> (one launch per step)" % (
-            wlo.group // 8, "true" if wlo.adamw else "false")
+        kname = "k_recon_int<%d,1,256,%s,false,%s> (one launch per step)" % (
+            wlo.group // 8, "true" if wlo.adamw else "false",
+            "true" if hoisted_clamp(wlo.bits, wlo.clip) else "false")
     else:
         tag = ("k_recon_lut_k%d" if wlo.fmt == "lut" else "k_recon_nvfp4_k%d") % len(wlo.clip)
         kname = ("k_recon_lut<256>" if wlo.fmt == "lut" else "k_recon_nvfp4<1,256>") + \
