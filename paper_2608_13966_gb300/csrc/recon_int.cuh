@@ -757,22 +757,42 @@ __global__ void __launch_bounds__(ADAM ? 192 : 256, 2)
         // ---- argmax of E over the group (ties: lowest index)
         float Eb = -INFINITY, dEb = 0.0f;
         int kb = 0x7fff;
+        if constexpr (NCH == 1) {
+            // one candidate a lane: the max of integer keys, E's bits (E >= 0
+            // orders like them) with the low 3 replaced by 7 - k; a candidate
+            // out of the running (E = -inf) has key 0.  Two candidates within
+            // 7 ulps of each other are both within the tie bound below (dE is
+            // at least tie_kappa >= 10 ulps of E), so whichever the key picks,
+            // the exact comparison settles them.
+            uint32_t key = Ek[0] >= 0.0f ? ((__float_as_uint(Ek[0]) & ~7u) | (7u - (uint32_t)sl)) : 0u;
 #pragma unroll
-        for (int ch = 0; ch < NCH; ++ch)
-            if (Ek[ch] > Eb) {  // strict: keeps the lower k of this lane
-                Eb = Ek[ch];
-                dEb = dEk[ch];
-                kb = ch * 8 + sl;
-            }
-#pragma unroll
-        for (int o = 4; o; o >>= 1) {
-            const float Eo = shx(Eb, o);
-            const float dEo = shx(dEb, o);
-            const int ko = __shfl_xor_sync(0xffffffffu, kb, o);
-            if (Eo > Eb || (Eo == Eb && ko < kb)) {
+            for (int o = 4; o; o >>= 1) key = max(key, __shfl_xor_sync(0xffffffffu, key, o));
+            const int kk = 7 - (int)(key & 7u);
+            const float Eo = __shfl_sync(0xffffffffu, Ek[0], (gs * 8) | kk);
+            const float dEo = __shfl_sync(0xffffffffu, dEk[0], (gs * 8) | kk);
+            if (key != 0u) {
                 Eb = Eo;
                 dEb = dEo;
-                kb = ko;
+                kb = kk;
+            }
+        } else {
+#pragma unroll
+            for (int ch = 0; ch < NCH; ++ch)
+                if (Ek[ch] > Eb) {  // strict: keeps the lower k of this lane
+                    Eb = Ek[ch];
+                    dEb = dEk[ch];
+                    kb = ch * 8 + sl;
+                }
+#pragma unroll
+            for (int o = 4; o; o >>= 1) {
+                const float Eo = shx(Eb, o);
+                const float dEo = shx(dEb, o);
+                const int ko = __shfl_xor_sync(0xffffffffu, kb, o);
+                if (Eo > Eb || (Eo == Eb && ko < kb)) {
+                    Eb = Eo;
+                    dEb = dEo;
+                    kb = ko;
+                }
             }
         }
         if (kb > 0x7ff) kb = 0;  // every candidate suspicious: the exact path picks
@@ -930,7 +950,10 @@ __global__ void __launch_bounds__(ADAM ? 192 : 256, 2)
                 // A = sum h (z - m) (small); sum h (w - mu) = Se
                 const float Aq = A * inv_ss;
                 const float Nc = Nr - A * ebar, Dc = Dr - A * Aq;
-                const float an = Nc / Dc;
+                // the quotient from the fast reciprocal and one correction
+                // (the remainder Nc - q Dc is exact by FMA): within an ulp
+                const float q0 = __fdividef(Nc, Dc);
+                const float an = fmaf(fmaf(-q0, Dc, Nc), __fdividef(1.0f, Dc), q0);
                 // Bz = (mu + ebar) - a (m + Aq), as a float pair
                 float p_h, p_l, bh, bl;
                 two_prod(an, m, p_h, p_l);
@@ -940,7 +963,8 @@ __global__ void __launch_bounds__(ADAM ? 192 : 256, 2)
                 a_sel = an;
                 Bz = bh;
                 Bz_lo = bl;
-                kap_sel = __fdividef(sqrtf(Dr * see), fabsf(Nc)) + __fdividef(Dr, Dc);
+                const float dse = fmaxf(Dr * see, 1e-37f);
+                kap_sel = __fdividef(dse * rsqrtf(dse), fabsf(Nc)) + __fdividef(Dr, Dc);
             }
         }
 
