@@ -94,6 +94,23 @@ __device__ __forceinline__ float4 lds128(const void* p)
 
 __device__ __forceinline__ uint2 lds64(const void* p) { return *reinterpret_cast<const uint2*>(p); }
 
+// Minimum / maximum of x over the lanes of `mask` in one warp reduction (used
+// over the whole warp: with a mask per 8-lane segment it ran slower than
+// three shuffle steps).  NaN inputs are ignored, as by fminf / fmaxf.
+__device__ __forceinline__ float lanes_min(float x, unsigned mask)
+{
+    float r;
+    asm volatile("redux.sync.min.f32 %0, %1, %2;" : "=f"(r) : "f"(x), "r"(mask));
+    return r;
+}
+
+__device__ __forceinline__ float lanes_max(float x, unsigned mask)
+{
+    float r;
+    asm volatile("redux.sync.max.f32 %0, %1, %2;" : "=f"(r) : "f"(x), "r"(mask));
+    return r;
+}
+
 __device__ __forceinline__ float bf16lo(uint32_t x) { return __uint_as_float(x << 16); }
 __device__ __forceinline__ float bf16hi(uint32_t x) { return __uint_as_float(x & 0xFFFF0000u); }
 

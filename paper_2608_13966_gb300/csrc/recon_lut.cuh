@@ -300,12 +300,10 @@ __global__ void __launch_bounds__(256, 2) k_recon_lut(const __grid_constant__ Lu
             mx = fmaxf(mx, fmaxf(w2[t].x, w2[t].y));
             ss += h2[t].x + h2[t].y;
         }
+        mn = lanes_min(mn, 0xffffffffu);
+        mx = lanes_max(mx, 0xffffffffu);
 #pragma unroll
-        for (int o = 16; o; o >>= 1) {
-            mn = fminf(mn, __shfl_xor_sync(0xffffffffu, mn, o));
-            mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
-            ss += __shfl_xor_sync(0xffffffffu, ss, o);
-        }
+        for (int o = 16; o; o >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, o);
         if (ss == 0.0f)  // all saliencies zero: h = 1
 #pragma unroll
             for (int t = 0; t < 8; ++t) h2[t] = make_float2(1.0f, 1.0f);
