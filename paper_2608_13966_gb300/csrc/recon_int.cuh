@@ -762,8 +762,9 @@ __global__ void __launch_bounds__(ADAM ? 192 : 256, 2)
             // orders like them) with the low 3 replaced by 7 - k; a candidate
             // out of the running (E = -inf) has key 0.  Two candidates within
             // 7 ulps of each other are both within the tie bound below (dE is
-            // at least tie_kappa >= 10 ulps of E), so whichever the key picks,
-            // the exact comparison settles them.
+            // at least 2 tie_kappa ulps of E, since sqrt(S2 sum h e^2) >= |N|,
+            // and the host's tie_kappa is at least 10), so whichever the key
+            // picks, the exact comparison settles them.
             uint32_t key = Ek[0] >= 0.0f ? ((__float_as_uint(Ek[0]) & ~7u) | (7u - (uint32_t)sl)) : 0u;
 #pragma unroll
             for (int o = 4; o; o >>= 1) key = max(key, __shfl_xor_sync(0xffffffffu, key, o));
