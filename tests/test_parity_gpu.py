@@ -215,6 +215,9 @@ def _edge_inputs(rows, cols, seed):
         w[3, ::2] = 0.0                              # many exact zeros
         w[4, 5] = 3.0                                # one outlier
         w[5] = torch.linspace(-1, 1, cols, device="cuda")  # codes on grid boundaries
+    if rows >= 8:
+        w[6] = w[6] * 1e-30                          # tiny range: R near 1e31
+        w[7] = w[7] * 1e-3 + 1e3                     # small range far from zero
     return w, g, v
 
 
