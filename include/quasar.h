@@ -431,13 +431,14 @@ void quasar_debug_force_timeout(int64_t nanoseconds);
 
 /*
  * quasar_debug_set_stats -- tuning hook.  While device_counters (a device
- * array of at least 3 unsigned ints owned by the caller) is set, the
+ * array of at least 4 unsigned ints owned by the caller) is set, the
  * reconstruction kernels atomically count [0] the groups/blocks whose
  * candidates were re-evaluated exactly because of a near tie, [1] the
  * integer groups whose kept fit was recomputed in compensated (float-float)
- * arithmetic and [2] the integer groups whose kept fit was recomputed about
- * centred codes and weights.  NULL turns counting off.  Process-wide; never
- * needed in normal use.
+ * arithmetic, [2] the integer groups whose kept fit was recomputed about
+ * centred codes and weights and [3] the thread blocks of the integer kernel
+ * with the hoisted code clamp (see quasar_debug_set_hoist).  NULL turns
+ * counting off.  Process-wide; never needed in normal use.
  */
 void quasar_debug_set_stats(unsigned int* device_counters);
 

@@ -57,7 +57,8 @@ struct IntParams {
     uint64_t timeout_ns;
     uint64_t force_timeout_ns;
     unsigned int* status;  // per-device status word
-    unsigned int* stats;  // optional: [0] exact re-evaluations, [1] compensated fits, [2] centred refits
+    unsigned int* stats;  // optional: [0] exact re-evaluations, [1] compensated fits, [2] centred refits,
+                          // [3] CTAs of the hoisted-clamp kernel
     float f[kMaxClip];     // padded with the last factor
     float invf[kMaxClip];  // fl32(1/f)
     // hoisted code clamps (the HC kernels): for each set of 4 consecutive

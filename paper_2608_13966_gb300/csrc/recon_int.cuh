@@ -440,6 +440,9 @@ __global__ void __launch_bounds__(ADAM ? 192 : 256, 2)
             if (u < n_units) issue(u, s);
         }
 
+    if constexpr (HC)  // which kernel ran, for the tuning counters
+        if (p.stats && threadIdx.x == 0) atomicAdd(&p.stats[3], 1u);
+
     if (p.force_timeout_ns && blockIdx.x == 0 && warp == 0) {
         // Failure-path hook: a barrier nothing ever arrives on.
         if (!mbar_wait_bounded(&bars[S], 0, p.force_timeout_ns)) {

@@ -234,14 +234,21 @@ def test_int_hoisted_clamp_equals_per_candidate_clamp(bits, clip, G):
     shapes = [(37, 3 * G), (8, 2 * G), (1, G)]
     base = [_edge_inputs(r, c, seed=900 + 10 * bits + i) for i, (r, c) in enumerate(shapes)]
     outs = {}
+    stats = torch.zeros(8, dtype=torch.int32, device="cuda")
     try:
         for hoist in (True, False):
             quasar.quasar_debug_set_hoist(hoist)
+            stats.zero_()
+            quasar.quasar_debug_set_stats(stats)
             items = [(w.clone(), g.clone(), v.clone()) for w, g, v in base]
             o = api.recon_int_batch(items, bits=bits, group_size=G, clip=clip, codes=True)
             torch.cuda.synchronize()
+            quasar.quasar_debug_set_stats(None)
             outs[hoist] = (o, [v for _, _, v in items])
+            # the hoisted-clamp kernel ran exactly when it was allowed to
+            assert (int(stats[3]) > 0) == hoist, (hoist, stats.tolist())
     finally:
+        quasar.quasar_debug_set_stats(None)
         quasar.quasar_debug_set_hoist(True)
     for i in range(len(shapes)):
         for key in ("r", "a", "b", "codes", "cand_idx"):
