@@ -169,6 +169,10 @@ def workload(name: str) -> Workload:
                         _layer_tensors(LLAMA31_8B_LAYER, 32), "t4", "lognormal",
                         "all linear weights of a 32-layer Llama-3.1-8B-shaped model, symmetric INT4 "
                         "group 128", symmetric=True)
+    if name == "llama_layer_int4_sym":
+        return Workload(name, "int", 4, 128, CLIP_8, 0.999, bf16, bf16, True,
+                        _layer_tensors(LLAMA31_8B_LAYER, 1), "t4", "lognormal",
+                        "one Llama-3.1-8B-shaped layer, symmetric INT4 group 128", symmetric=True)
     if name == "llama_layer_lut":
         return Workload(name, "lut", 3, 512, CLIP_8, 0.999, bf16, bf16, True,
                         _layer_tensors(LLAMA31_8B_LAYER, 1), "t4", "lognormal",
@@ -188,7 +192,7 @@ def workload(name: str) -> Workload:
 WORKLOADS = ("single_int4", "llama_layer_int3", "qwen_layer_int2", "llama_layer_nvfp4",
              "llama_layer_int3_adamw", "llama_layer_nvfp4_adamw", "llama_layer_lut", "llama_int2",
              "llama_int3", "llama_int4", "llama_nvfp4", "llama_int3_adamw", "llama_nvfp4_adamw",
-             "llama_lut", "llama_int4_sym")
+             "llama_lut", "llama_int4_sym", "llama_layer_int4_sym")
 
 
 def _student_t(gen, shape, nu: int, device) -> torch.Tensor:
