@@ -29,7 +29,7 @@ def _sample(model, unit, seed):
 
 
 @pytest.mark.gpu
-@pytest.mark.parametrize("name", ["llama_int3", "llama_nvfp4", "llama_int3_adamw"])
+@pytest.mark.parametrize("name", ["llama_int3", "llama_int2", "llama_int4", "llama_nvfp4", "llama_int3_adamw"])
 def test_full_model_sampled(oracle, name):
     wl = WL.workload(name)
     unit = wl.group if wl.fmt == "int" else 16
