@@ -363,20 +363,30 @@ def timed_steps(step, n_launch_calls, steps, warmup, world):
     end.record()
     torch.cuda.synchronize()
     barrier(world)
+    # a kernel that gave up on a wait leaves its outputs incomplete: such a
+    # run has measured nothing
+    st = Q.quasar_get_device_status(None)
+    if st != Q.QuasarStatus.OK:
+        raise Q.QuasarError(st)
     total_ms = start.elapsed_time(end)
     kernel_ms = sum(s.elapsed_time(e) for ev in events for (s, e) in ev)
     return total_ms, kernel_ms
 
 
-def hoisted_clamp(bits, clip):
-    """Whether the library runs the hoisted-clamp integer kernel for this
-    candidate list (8 or fewer candidates, both slot sets with a cap; the
-    library's own test, restated to name the kernel in the report)."""
-    if len(clip) > 8 or os.environ.get("QUASAR_HOIST", "1") == "0":
-        return False
-    f = [float(np.float32(clip[min(k, len(clip) - 1)])) for k in range(8)]
+def clamp_set_size(bits, clip):
+    """The clamp-set size the library's integer kernel runs with for this
+    candidate list (the largest of 4, 2, 1 consecutive slots whose sets all
+    admit one code clamp; the library's own rule, restated to name the
+    kernel in the report)."""
+    if os.environ.get("QUASAR_HOIST", "1") == "0":
+        return 1
+    f = [float(np.float32(clip[min(k, len(clip) - 1)])) for k in range(32)]
     J = ((1 << bits) - 1) >> 1
-    return all(J * max(f[s:s + 4]) * 1.001 < (J + 1) * min(f[s:s + 4]) * 0.999 for s in (0, 4))
+    for size in (4, 2):
+        if all(J * max(f[s:s + size]) * 1.001 < (J + 1) * min(f[s:s + size]) * 0.999
+               for s in range(0, 32, size)):
+            return size
+    return 1
 
 
 def host_link(host, dev, s_in, s_out, reps=5):
@@ -594,9 +604,11 @@ def main():
     # differ in size; bytes and time both scale with the weights processed)
     if wlo.fmt == "int":
         tag = "k_recon_int_g%d_k%d%s" % (wlo.group, len(wlo.clip), "_adamw" if wlo.adamw else "")
-        kname = "k_recon_int<%d,1,256,%s,false,%s> (one launch per step)" % (
-            wlo.group // 8, "true" if wlo.adamw else "false",
-            "true" if hoisted_clamp(wlo.bits, wlo.clip) else "false")
+        ss = clamp_set_size(wlo.bits, wlo.clip)
+        if wlo.adamw and ss == 2:
+            ss = 1
+        kname = "k_recon_int<%d,%d,256,%s,false,%d> (one launch per step)" % (
+            wlo.group // 8, (len(wlo.clip) + 7) // 8, "true" if wlo.adamw else "false", ss)
     else:
         tag = ("k_recon_lut_k%d" if wlo.fmt == "lut" else "k_recon_nvfp4_k%d") % len(wlo.clip)
         kname = ("k_recon_lut<256>" if wlo.fmt == "lut" else "k_recon_nvfp4<1,256>") + \

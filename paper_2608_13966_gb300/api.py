@@ -1,13 +1,20 @@
 """Convenience layer over the C ABI: allocates the outputs with PyTorch and
 raises ``QuasarError`` on a non-OK status.  The computation itself is the
-library's; this module only allocates and marshals."""
+library's; this module only allocates and marshals.
+
+The calls are asynchronous: the status they return covers argument checks
+and the launch.  A kernel that gives up on a wait (a copy that never lands)
+records that in the device's status word instead, and its outputs are then
+incomplete; ``check_device()`` (or ``quasar_get_device_status``) reads and
+clears that word after synchronising the stream, and callers that must know
+their outputs are whole call it once after their last reconstruction."""
 from __future__ import annotations
 
 import torch
 
 from .quasar import (BF16, F32, QuasarError, QuasarStatus, adamw_nvfp4_tensor_array,
                      adamw_tensor_array, int_tensor_array, lut_tensor_array, nvfp4_tensor_array,
-                     options, quasar_adamw_recon_int_batch, quasar_adamw_recon_nvfp4_batch,
+                     options, quasar_adamw_recon_int_batch, quasar_get_device_status, quasar_adamw_recon_nvfp4_batch,
                      quasar_recon_int, quasar_recon_int_batch_ex, quasar_recon_lut_batch,
                      quasar_recon_nvfp4, quasar_recon_nvfp4_batch_ex, quasar_tensor_amax)
 
@@ -15,6 +22,12 @@ from .quasar import (BF16, F32, QuasarError, QuasarStatus, adamw_nvfp4_tensor_ar
 def _check(st):
     if st != QuasarStatus.OK:
         raise QuasarError(st)
+
+
+def check_device(stream=None):
+    """Synchronise ``stream`` and raise ``QuasarError`` if a kernel of this
+    library timed out on a wait since the last check."""
+    _check(quasar_get_device_status(stream))
 
 
 def _check_2d(w):

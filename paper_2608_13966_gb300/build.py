@@ -23,10 +23,15 @@ NVCC_FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-I" + IN
 # (source, extra flags, object name)
 UNITS = [
     ("quasar_abi.cu", [], "quasar_abi.o"),
-    ("kernels_int.cu", ["-DQUASAR_NCH=1"], "kernels_int_nch1.o"),
-    ("kernels_int.cu", ["-DQUASAR_NCH=2"], "kernels_int_nch2.o"),
-    ("kernels_int.cu", ["-DQUASAR_NCH=4"], "kernels_int_nch4.o"),
-    ("kernels_int.cu", ["-DQUASAR_NCH=1", "-DQUASAR_HC=1"], "kernels_int_hc.o"),
+    ("kernels_int.cu", ["-DQUASAR_NCH=1", "-DQUASAR_SS=4"], "kernels_int_nch1_ss4.o"),
+    ("kernels_int.cu", ["-DQUASAR_NCH=1", "-DQUASAR_SS=2"], "kernels_int_nch1_ss2.o"),
+    ("kernels_int.cu", ["-DQUASAR_NCH=1", "-DQUASAR_SS=1"], "kernels_int_nch1_ss1.o"),
+    ("kernels_int.cu", ["-DQUASAR_NCH=2", "-DQUASAR_SS=4"], "kernels_int_nch2_ss4.o"),
+    ("kernels_int.cu", ["-DQUASAR_NCH=2", "-DQUASAR_SS=2"], "kernels_int_nch2_ss2.o"),
+    ("kernels_int.cu", ["-DQUASAR_NCH=2", "-DQUASAR_SS=1"], "kernels_int_nch2_ss1.o"),
+    ("kernels_int.cu", ["-DQUASAR_NCH=4", "-DQUASAR_SS=4"], "kernels_int_nch4_ss4.o"),
+    ("kernels_int.cu", ["-DQUASAR_NCH=4", "-DQUASAR_SS=2"], "kernels_int_nch4_ss2.o"),
+    ("kernels_int.cu", ["-DQUASAR_NCH=4", "-DQUASAR_SS=1"], "kernels_int_nch4_ss1.o"),
     ("kernels_nvfp4.cu", [], "kernels_nvfp4.o"),
     ("kernels_lut.cu", [], "kernels_lut.o"),
     ("kernels_sym.cu", [], "kernels_sym.o"),

@@ -71,6 +71,16 @@ __device__ __forceinline__ bool mbar_wait_bounded(uint64_t* bar, uint32_t parity
     }
 }
 
+// The bounded wait of a whole warp, with one outcome for all its lanes.  Each
+// lane waits on the barrier itself (so each observes the completed phase and
+// the data the copies delivered), and the warp reports a timeout if any
+// lane's own limit ran out: no lane takes the failure path while others go
+// on to warp-wide shuffles.  Every lane of the warp must call it.
+__device__ __forceinline__ bool warp_wait_bounded(uint64_t* bar, uint32_t parity, uint64_t limit_ns)
+{
+    return __all_sync(0xffffffffu, mbar_wait_bounded(bar, parity, limit_ns));
+}
+
 // 1-D bulk copy global -> shared, completion counted in bytes on `bar`.
 // dst, src and bytes must be multiples of 16.
 __device__ __forceinline__ void bulk_g2s(void* dst, const void* src, uint32_t bytes, uint64_t* bar)

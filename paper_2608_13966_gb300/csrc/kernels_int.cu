@@ -1,63 +1,59 @@
 // Instantiations of the integer-code kernel for one candidate-chunk count
-// (QUASAR_NCH = 1, 2 or 4 chunks of 8 candidates); compiled once per value,
-// and once more with QUASAR_HC for the hoisted-clamp variant (one chunk).
+// (QUASAR_NCH = 1, 2 or 4 chunks of 8 candidates) and one clamp-set size
+// (QUASAR_SS = 4, 2 or 1 candidates); compiled once per pair, in parallel.
 #include "recon_int.cuh"
 
-#ifndef QUASAR_NCH
-#error "QUASAR_NCH must be defined"
+#if !defined(QUASAR_NCH) || !defined(QUASAR_SS)
+#error "QUASAR_NCH and QUASAR_SS must be defined"
 #endif
 
-#define QUASAR_CAT2(a, b) a##b
-#define QUASAR_CAT(a, b) QUASAR_CAT2(a, b)
+#define QUASAR_CAT4(a, b, c, d) a##b##c##d
+#define QUASAR_NAME(n, s) QUASAR_CAT4(int_kernel_nch, n, _ss, s)
 
 namespace quasar {
 
-#ifdef QUASAR_HC
-// Kernel entry of the hoisted-clamp variant (batches of up to kMaxBatch
-// tensors, one chunk of 8 candidates, no option variants); nullptr if not
-// built.
-const void* int_kernel_hc(int epl, bool adam)
-{
-    constexpr int B = kMaxBatch;
-    switch (epl) {
-#define QUASAR_EPL(E)                                                                       \
-    case E:                                                                                 \
-        return adam ? reinterpret_cast<const void*>(&k_recon_int<E, 1, B, true, false, true>) \
-                    : reinterpret_cast<const void*>(&k_recon_int<E, 1, B, false, false, true>);
-    QUASAR_EPL(4)
-    QUASAR_EPL(8)
-    QUASAR_EPL(16)
-    QUASAR_EPL(32)
-#undef QUASAR_EPL
-    default: return nullptr;
-    }
-}
-#else
 // Kernel entry for group size 8*epl: one tensor or a batch of up to
-// kMaxBatch tensors per launch; the AdamW-fused variant and the option
-// variants (var) are built for batches only.  nullptr if not built.
-const void* QUASAR_CAT(int_kernel_nch, QUASAR_NCH)(int epl, bool batch, bool adam, bool var)
+// kMaxBatch tensors per launch.  The AdamW-fused variant is built for batches
+// with sets of 4 or 1 candidates, the option variants (var) for batches with
+// sets of 1; nullptr where not built.
+const void* QUASAR_NAME(QUASAR_NCH, QUASAR_SS)(int epl, bool batch, bool adam, bool var)
 {
     constexpr int C = QUASAR_NCH;
+    constexpr int S = QUASAR_SS;
     constexpr int B = kMaxBatch;
     if ((adam || var) && !batch) return nullptr;
+    if (adam && S == 2) return nullptr;
+    if (var && S != 1) return nullptr;
     switch (epl) {
-#define QUASAR_EPL(E)                                                                          \
-    case E:                                                                                    \
-        if (!batch) return reinterpret_cast<const void*>(&k_recon_int<E, C, 1, false, false>); \
-        if (adam)                                                                              \
-            return var ? reinterpret_cast<const void*>(&k_recon_int<E, C, B, true, true>)      \
-                       : reinterpret_cast<const void*>(&k_recon_int<E, C, B, true, false>);    \
-        return var ? reinterpret_cast<const void*>(&k_recon_int<E, C, B, false, true>)         \
-                   : reinterpret_cast<const void*>(&k_recon_int<E, C, B, false, false>);
+#if QUASAR_SS == 1
+#define QUASAR_VAR(E)                                                                         \
+    if (var)                                                                                  \
+        return adam ? reinterpret_cast<const void*>(&k_recon_int<E, C, B, true, true, S>)     \
+                    : reinterpret_cast<const void*>(&k_recon_int<E, C, B, false, true, S>);
+#else
+#define QUASAR_VAR(E)
+#endif
+#if QUASAR_SS != 2
+#define QUASAR_ADAM(E) \
+    if (adam) return reinterpret_cast<const void*>(&k_recon_int<E, C, B, true, false, S>);
+#else
+#define QUASAR_ADAM(E)
+#endif
+#define QUASAR_EPL(E)                                                                         \
+    case E:                                                                                   \
+        QUASAR_VAR(E)                                                                         \
+        QUASAR_ADAM(E)                                                                        \
+        if (!batch) return reinterpret_cast<const void*>(&k_recon_int<E, C, 1, false, false, S>); \
+        return reinterpret_cast<const void*>(&k_recon_int<E, C, B, false, false, S>);
     QUASAR_EPL(4)
     QUASAR_EPL(8)
     QUASAR_EPL(16)
     QUASAR_EPL(32)
 #undef QUASAR_EPL
+#undef QUASAR_ADAM
+#undef QUASAR_VAR
     default: return nullptr;
     }
 }
-#endif
 
 }  // namespace quasar

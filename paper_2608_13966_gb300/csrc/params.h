@@ -57,14 +57,18 @@ struct IntParams {
     uint64_t timeout_ns;
     uint64_t force_timeout_ns;
     unsigned int* status;  // per-device status word
-    unsigned int* stats;  // optional: [0] exact re-evaluations, [1] compensated fits, [2] centred refits,
-                          // [3] CTAs of the hoisted-clamp kernel
+    unsigned int* stats;  // optional: [0] exact re-evaluations, [1] compensated fits,
+                          // [3] CTAs of kernels whose clamp sets hold more than one candidate
     float f[kMaxClip];     // padded with the last factor
     float invf[kMaxClip];  // fl32(1/f)
-    // hoisted code clamps (the HC kernels): for each set of 4 consecutive
-    // candidate slots, tau / qmax, so that the set's cap on |w - c| is
-    // hcap * range; 0 where no tau exists
-    float hcap[kMaxClip / 4];
+    // code clamps: every candidate slot holds tau / qmax of its clamp set,
+    // so that the set's cap on |w - centre| is cap * range (sets of
+    // set_size consecutive slots; see the integer kernel)
+    float cap[kMaxClip];
+    int set_size;
+    // centre of each 8-candidate chunk's moments: the mean of 1/f over the
+    // chunk's factors
+    float invfc[kMaxClip / 8];
     // fused AdamW step: w' = w - (w*lr_wd + step_size * m' / (sqrt(v') * isbc2 + eps))
     float beta1, c1b;      // beta1, 1 - beta1
     float lr_wd;           // lr * weight_decay

@@ -15,10 +15,12 @@
 #include "quasar.h"
 
 namespace quasar {
-const void* int_kernel_nch1(int epl, bool batch, bool adam, bool var);
-const void* int_kernel_nch2(int epl, bool batch, bool adam, bool var);
-const void* int_kernel_nch4(int epl, bool batch, bool adam, bool var);
-const void* int_kernel_hc(int epl, bool adam);
+// integer-code kernels: one entry per (8-candidate chunks, clamp-set size)
+#define QUASAR_INT_ENTRY(n, s) const void* int_kernel_nch##n##_ss##s(int epl, bool batch, bool adam, bool var);
+QUASAR_INT_ENTRY(1, 4) QUASAR_INT_ENTRY(1, 2) QUASAR_INT_ENTRY(1, 1)
+QUASAR_INT_ENTRY(2, 4) QUASAR_INT_ENTRY(2, 2) QUASAR_INT_ENTRY(2, 1)
+QUASAR_INT_ENTRY(4, 4) QUASAR_INT_ENTRY(4, 2) QUASAR_INT_ENTRY(4, 1)
+#undef QUASAR_INT_ENTRY
 const void* nvfp4_kernel(int nch, bool batch);
 const void* amax_kernel(bool batch);
 const void* amax_to_scale_kernel(bool batch);
@@ -48,24 +50,41 @@ std::atomic<int64_t> g_force_timeout_ns{0};
 std::atomic<unsigned int*> g_stats{nullptr};
 std::atomic<int> g_hoist{-1};  // -1: the environment's choice (tuning().hoist)
 
+// The error bounds' defaults are the smallest values their derivations allow
+// (the summation-depth bound of the candidate errors, the NVFP4 direct-sum
+// bound, the fit error that triggers the compensated fit): an environment
+// value below one is raised to it, so a setting can make the careful paths
+// run more often but never skip one that correctness needs.  Larger values
+// are capped where a float overflow would start to matter.
+constexpr float kTieKappaMin = 16.0f;
+constexpr float kTieScaleMin = 1.0f;
+constexpr float kFitUlpsMin = 3.0f;
+
 struct Tuning {
     int stages = 0;            // 0: chosen from the shared-memory budget
     int smem_budget = 100 * 1024;
-    float tie_kappa = 16.0f;   // NVFP4 tie bound, in ulps
-    float tie_scale = 1.0f;    // multiplier of the integer kernel's summation-depth bound
-    float fit_ulps = 3.0f;
+    float tie_kappa = kTieKappaMin;  // NVFP4 tie bound, in ulps
+    float tie_scale = kTieScaleMin;  // multiplier of the integer kernel's summation-depth bound
+    float fit_ulps = kFitUlpsMin;
     int hoist = 1;             // 0: never the hoisted-clamp integer kernel
 };
+
+// A float from the environment, clamped to [lo, hi] (non-numbers give lo).
+float env_float(const char* s, float lo, float hi)
+{
+    const double x = std::atof(s);
+    return !(x >= lo) ? lo : (x > hi ? hi : (float)x);
+}
 
 const Tuning& tuning()
 {
     static const Tuning t = [] {
         Tuning x;
-        if (const char* s = std::getenv("QUASAR_STAGES")) x.stages = std::atoi(s);
+        if (const char* s = std::getenv("QUASAR_STAGES")) x.stages = std::min(std::max(std::atoi(s), 0), 8);
         if (const char* s = std::getenv("QUASAR_SMEM_BUDGET")) x.smem_budget = std::atoi(s);
-        if (const char* s = std::getenv("QUASAR_TIE_KAPPA")) x.tie_kappa = (float)std::atof(s);
-        if (const char* s = std::getenv("QUASAR_TIE_SCALE")) x.tie_scale = (float)std::atof(s);
-        if (const char* s = std::getenv("QUASAR_FIT_ULPS")) x.fit_ulps = (float)std::atof(s);
+        if (const char* s = std::getenv("QUASAR_TIE_KAPPA")) x.tie_kappa = env_float(s, kTieKappaMin, 1e4f);
+        if (const char* s = std::getenv("QUASAR_TIE_SCALE")) x.tie_scale = env_float(s, kTieScaleMin, 1e3f);
+        if (const char* s = std::getenv("QUASAR_FIT_ULPS")) x.fit_ulps = env_float(s, kFitUlpsMin, 1e4f);
         if (const char* s = std::getenv("QUASAR_HOIST")) x.hoist = std::atoi(s);
         return x;
     }();
@@ -127,24 +146,51 @@ void fill_clip(const float* clip, int n_clip, float* f, float* invf)
     }
 }
 
-// Hoisted code clamps of the integer kernel.  For each set of 4 consecutive
-// candidate slots: a tau with J f_max (1 + 1e-3) <= tau <= (J + 1) f_min
-// (1 - 1e-3), J = (qmax - 1) / 2.  Then min(|d|, tau range / qmax) P_k has
-// the code min(floor(|d| P_k), J) for every slot k of the set: a capped |d|
-// gives cap P_k ~ tau / f_k in [J, J + 1), and below the cap
-// |d| P_k < J + 1.  The margin covers the fp32 roundings of the cap, of R
-// and of P.  Stored as tau / qmax; 0 where no tau exists.
-void fill_hcap(IntParams* p)
+// Code clamps of the integer kernel.  A set of consecutive candidate slots
+// shares one clamp when some tau has J f_max (1 + 1e-3) <= tau <= (J + 1)
+// f_min (1 - 1e-3), J = (qmax - 1) / 2: then min(|d|, tau range / qmax) P_k
+// has the code min(floor(|d| P_k), J) for every slot k of the set (a capped
+// |d| gives cap P_k ~ tau / f_k in [J, J + 1), and below the cap
+// |d| P_k < J + 1).  The margin covers the fp32 roundings of the cap, of R
+// and of P.  The largest set size of 4, 2, 1 whose sets all qualify is taken
+// (a set of one always does), and no larger than max_size; every slot holds
+// its set's tau / qmax.  Also the centre factor of each 8-candidate chunk.
+void fill_caps(IntParams* p, int max_size)
 {
     const int J = p->qmax >> 1;
-    for (int s = 0; s < kMaxClip / 4; ++s) {
+    auto cap_of = [&](int k0, int n, double* tau) {
         double fmax = 0.0, fmin = 2.0;
-        for (int k = 4 * s; k < 4 * s + 4; ++k) {
+        for (int k = k0; k < k0 + n; ++k) {
             fmax = std::max(fmax, (double)p->f[k]);
             fmin = std::min(fmin, (double)p->f[k]);
         }
         const double lo = J * fmax * (1.0 + 1e-3), hi = (J + 1) * fmin * (1.0 - 1e-3);
-        p->hcap[s] = lo < hi ? (float)(0.5 * (lo + hi) / p->qmax) : 0.0f;
+        *tau = 0.5 * (lo + hi);
+        return lo < hi;
+    };
+    int size = 1;
+    for (int cand = std::min(4, max_size); cand > 1; cand >>= 1) {
+        bool ok = true;
+        double tau;
+        for (int k0 = 0; k0 < kMaxClip && ok; k0 += cand) ok = cap_of(k0, cand, &tau);
+        if (ok) {
+            size = cand;
+            break;
+        }
+    }
+    p->set_size = size;
+    for (int k0 = 0; k0 < kMaxClip; k0 += size) {
+        double tau = 0.0;
+        cap_of(k0, size, &tau);
+        for (int k = k0; k < k0 + size; ++k) p->cap[k] = (float)(tau / p->qmax);
+    }
+    for (int c = 0; c < kMaxClip / 8; ++c) {
+        double lo = 1e300, hi = 0.0;
+        for (int k = 8 * c; k < 8 * c + 8 && k < std::max(p->n_clip, 8 * c + 1); ++k) {
+            lo = std::min(lo, 1.0 / (double)p->f[k]);
+            hi = std::max(hi, 1.0 / (double)p->f[k]);
+        }
+        p->invfc[c] = (float)(0.5 * (lo + hi));
     }
 }
 
@@ -197,6 +243,17 @@ struct KernelConfig {
 constexpr int kMaxConfigs = 256;
 KernelConfig g_cfg[kMaxConfigs];
 int g_ncfg = 0;
+// Kernels whose dynamic shared-memory limit was raised, per device.  The
+// limit is always set to the device's opt-in maximum, so it never has to be
+// raised again or lowered for another size (a full table only repeats the
+// same setting).
+struct SmemLimit {
+    const void* fn = nullptr;
+    int dev = -1;
+};
+constexpr int kMaxLimits = 256;
+SmemLimit g_limit[kMaxLimits];
+int g_nlimit = 0;
 
 quasar_status device_info(int* dev_out, const DeviceInfo** info)
 {
@@ -232,24 +289,27 @@ quasar_status status_ptr(unsigned int** p)
 }
 
 // Resident CTAs per SM for (fn, smem) on device dev.  The kernel's dynamic
-// shared-memory limit only ever grows (to the largest size requested so far),
-// so a configuration cached earlier stays launchable.
+// shared-memory limit is set once per device, to the device's opt-in
+// maximum, so every configuration cached earlier stays launchable.
 quasar_status occupancy(const void* fn, size_t smem, int threads, int dev, int* occ)
 {
     std::lock_guard<std::mutex> lock(g_mu);
-    size_t limit = 0;
-    for (int i = 0; i < g_ncfg; ++i) {
-        if (g_cfg[i].fn != fn || g_cfg[i].dev != dev) continue;
-        if (g_cfg[i].smem == smem) {
+    for (int i = 0; i < g_ncfg; ++i)
+        if (g_cfg[i].fn == fn && g_cfg[i].dev == dev && g_cfg[i].smem == smem) {
             *occ = g_cfg[i].occupancy;
             return QUASAR_OK;
         }
-        limit = std::max(limit, g_cfg[i].smem);
+    bool raised = false;
+    for (int i = 0; i < g_nlimit && !raised; ++i) raised = g_limit[i].fn == fn && g_limit[i].dev == dev;
+    if (!raised) {
+        int optin = 0;
+        if (cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev) != cudaSuccess)
+            return QUASAR_ERR_CUDA;
+        if (smem > (size_t)optin) return QUASAR_ERR_UNSUPPORTED;
+        if (cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, optin) != cudaSuccess)
+            return QUASAR_ERR_CUDA;
+        if (g_nlimit < kMaxLimits) g_limit[g_nlimit++] = SmemLimit{fn, dev};
     }
-    if (smem > limit &&
-        cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) !=
-            cudaSuccess)
-        return QUASAR_ERR_CUDA;
     int o = 0;
     if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&o, fn, threads, smem) != cudaSuccess)
         return QUASAR_ERR_CUDA;
@@ -381,7 +441,7 @@ quasar_status int_params(quasar_dtype g_dtype, bool has_g, float beta2, int bits
     p->force_timeout_ns = (uint64_t)std::max<int64_t>(0, g_force_timeout_ns.load());
     p->stats = g_stats.load();
     fill_clip(clip, n_clip, p->f, p->invf);
-    fill_hcap(p);
+    fill_caps(p, 4);
     quasar_status st;
     if ((st = status_ptr(&p->status)) != QUASAR_OK) return st;
     if (adam) {
@@ -421,15 +481,21 @@ quasar_status int_launch(IntLaunch<MAXT>& Lp, int group_size, int n_clip, cudaSt
     const int nch = nch_for(n_clip);
     const bool batch = MAXT > 1;
     const bool var = Lp.p.h_mode != kSalEma || Lp.p.codes_packed;
-    // the hoisted-clamp kernel where both slot sets of the one chunk have a cap
+    // clamp sets: as large as the factors allow, unless switched off (sets of
+    // one); the option variants are built with sets of one, the fused AdamW
+    // step with sets of four or one
     const int hoist_on = g_hoist.load() < 0 ? tuning().hoist : g_hoist.load();
-    const bool hoist = batch && !var && nch == 1 && hoist_on && Lp.p.hcap[0] > 0.0f &&
-                       Lp.p.hcap[1] > 0.0f;
-    const void* fn = symmetric  ? (MAXT > 1 ? sym_kernel(epl) : nullptr)
-                     : hoist    ? int_kernel_hc(epl, adam)
-                     : nch == 1 ? int_kernel_nch1(epl, batch, adam, var)
-                     : nch == 2 ? int_kernel_nch2(epl, batch, adam, var)
-                                : int_kernel_nch4(epl, batch, adam, var);
+    fill_caps(&Lp.p, (!hoist_on || var) ? 1 : 4);
+    if (adam && Lp.p.set_size == 2) fill_caps(&Lp.p, 1);
+    using Entry = const void* (*)(int, bool, bool, bool);
+    static const Entry table[3][3] = {
+        {int_kernel_nch1_ss4, int_kernel_nch1_ss2, int_kernel_nch1_ss1},
+        {int_kernel_nch2_ss4, int_kernel_nch2_ss2, int_kernel_nch2_ss1},
+        {int_kernel_nch4_ss4, int_kernel_nch4_ss2, int_kernel_nch4_ss1}};
+    const int ci = nch == 1 ? 0 : (nch == 2 ? 1 : 2);
+    const int si = Lp.p.set_size == 4 ? 0 : (Lp.p.set_size == 2 ? 1 : 2);
+    const void* fn = symmetric ? (MAXT > 1 ? sym_kernel(epl) : nullptr)
+                               : table[ci][si](epl, batch, adam, var);
     if (!fn) return QUASAR_ERR_UNSUPPORTED;
     return launch_persistent(fn, &Lp, L.smem, units, stream, warps);
 }

@@ -13,29 +13,36 @@
 // The tile stays in shared memory while the unit is processed; the passes
 // below stream it from there.  The grid is persistent.
 //
-// Codes in centred form.  With qmax = 2^bits - 1 odd, H = qmax/2 is a
-// half-integer and Eq. 1's code is q = H + z with
-//     |z| = min(floor(|d| P), J) + 1/2,  sign(z) = sign(d),
-// where d = w - c, P = qmax / (f * range) and J = (qmax - 1)/2.  This equals
-// clamp(round(d P + H), 0, qmax) except at exact rounding ties (t = d P + H a
-// half-integer), which lie inside the checker's margin exemption.  floor is a
-// single FMA rounded toward -inf onto the 2^23 grid (__ffma2_rd), so a code
-// costs one FMA, one min and one add, two elements per instruction.
+// Codes.  With d = (w - min) - rho (the offset from the group's centre,
+// formed without rounding the centre itself: w - min and the half range are
+// exact wherever the group lies far from zero), P = qmax / (f * range) and
+// J = (qmax - 1)/2, Eq. 1's code is q = zeta + J + 1 with
+//     zeta = clamp(floor(d P), -(J+1), J),
+// which equals clamp(round(d P + qmax/2), 0, qmax) except at exact rounding
+// ties (d P an integer), which lie inside the checker's margin exemption.
+// floor is one FMA rounded toward -inf onto the unit grid at 1.5 * 2^23 (the
+// product is exact inside the FMA), so y = M + zeta with M = 1.5 * 2^23.  The
+// clamp is applied to d instead, once per set of candidates: for a set whose
+// factors satisfy J f_max < tau < (J + 1) f_min (with a margin the host
+// checks), clamping |d| at tau * range / qmax gives every candidate of the
+// set its clamped code bit for bit (a set of one always has such a tau).
 //
 // Per group (fp32):
 //   pass A  v' = beta2*v + (1-beta2)*g^2 (written back; kept in the tile as
-//           the saliency h), min/max -> c, range, sum h, sum h w -> mu;
-//   pass B  for 8 candidates at a time, the codes (from d = w - c) and the
-//           moments S1 = sum h z, S2 = sum h z^2, S3 = sum h z e with
+//           the saliency h), min/max -> range, sum h, sum h w -> mu;
+//   pass B  for 4 candidates at a time, the codes and the moments about a
+//           centre zeta0 shared by the candidates of an 8-candidate chunk
+//           (the code of the weighted mean, from mu): S1 = sum h (zeta -
+//           zeta0), S2 = sum h (zeta - zeta0)^2, S3 = sum h (zeta - zeta0) e,
 //           e = w - mu (plus the candidate-independent sum h e, sum h e^2);
 //   reduce  the 8 lanes' partial sums are transposed through shared memory
 //           so that lane sl owns candidate sl of the chunk;
 //   select  D = S2 - S1^2/Ss, N = S3 - S1*Se/Ss: the weighted error of
 //           candidate k is C - N^2/D with C common, so argmin error =
 //           argmax E = N^2/D; the winner's fit is a = N/D with the offset
-//           from the weighted means;
-//   pass C  codes of the kept candidate, r = a*z + Bz, outputs (b = Bz - a*H
-//           is the offset of the paper's r = a*q + b).
+//           from the weighted means, taken from the same centred sums;
+//   pass C  codes of the kept candidate, r = a*zeta + B, outputs (b = B -
+//           a*(J+1) is the offset of the paper's r = a*q + b).
 //
 // Exactness.  E carries fp32 rounding error; candidates whose E lies within
 // an error bound of the best (and candidates whose weighted code variance D
@@ -54,24 +61,21 @@ namespace quasar {
 
 __device__ __forceinline__ float shx(float x, int m) { return __shfl_xor_sync(0xffffffffu, x, m); }
 
-// 2^23: fl_rd(x + 2^23) = 2^23 + floor(x) for 0 <= x < 2^23 (unit spacing).
-constexpr float kFloorMagic = 8388608.0f;
-// 2^23 - 1/2 (exact: spacing 1/2 below 2^23); y - this = floor + 1/2.
-constexpr float kHalfBelowMagic = 8388607.5f;
+// 1.5 * 2^23: in [2^23, 2^24) fp32 values are spaced 1, so fl_rd(x + M) =
+// M + floor(x) for |x| < 2^22.
+constexpr float kGridMagic = 12582912.0f;
 
-// Centred code z = q - qmax/2 of one element for the scale P (see above);
-// zcap = kFloorMagic + J.
-__device__ __forceinline__ float int_code_z(float d, float P, float zcap)
+// Offset of an element from its group's centre, d = (w - mn) - rho.
+__device__ __forceinline__ float centred(float w, float nmn, float nrho)
 {
-    const float y = fminf(__fmaf_rd(fabsf(d), P, kFloorMagic), zcap);
-    return copysignf(__fsub_rn(y, kHalfBelowMagic), d);
+    return __fadd_rn(__fadd_rn(w, nmn), nrho);
 }
 
-// h with the sign of d (h >= 0): the sign survives h = 0 as -0.
-__device__ __forceinline__ float2 signed_h2(float2 h, float2 d)
+// Code q in [0, qmax] of an offset d for the scale P: M + floor(d P) clamped
+// to [ylo, yhi] = [M - J - 1, M + J], minus ylo (exact).
+__device__ __forceinline__ float int_code_q(float d, float P, float ylo, float yhi)
 {
-    return make_float2(__uint_as_float(__float_as_uint(h.x) | (__float_as_uint(d.x) & 0x80000000u)),
-                       __uint_as_float(__float_as_uint(h.y) | (__float_as_uint(d.y) & 0x80000000u)));
+    return __fsub_rn(fminf(fmaxf(__fmaf_rd(d, P, kGridMagic), ylo), yhi), ylo);
 }
 
 // Round x to a multiple of the power of two U (x*invU is exact).
@@ -138,14 +142,14 @@ __device__ __forceinline__ float wsum32(float x)
     return x;
 }
 
-// (hi, lo) + x*H as a renormalised pair: moves an offset between the code
-// origins q = 0 and z = 0 (q = z + H).
-__device__ __forceinline__ void ff_add_prod(float& hi, float& lo, float xh, float xl, float H)
+// (hi, lo) + x*K as a renormalised pair: moves an offset between two code
+// origins (q = 0 and zeta = 0, q = zeta + K).
+__device__ __forceinline__ void ff_add_prod(float& hi, float& lo, float xh, float xl, float K)
 {
     float ph, pl, sh, se;
-    two_prod(xh, H, ph, pl);
+    two_prod(xh, K, ph, pl);
     two_sum(hi, ph, sh, se);
-    lo = __fadd_rn(__fadd_rn(lo, se), fmaf(xl, H, pl));
+    lo = __fadd_rn(__fadd_rn(lo, se), fmaf(xl, K, pl));
     hi = sh;
     ff_norm(hi, lo);
 }
@@ -155,32 +159,45 @@ __device__ __forceinline__ void ff_add_prod(float& hi, float& lo, float xh, floa
 // One group, evaluated by all 32 lanes (lane L takes elements L + 32m) from
 // the tile in shared memory: w at ws, saliency h at hs.
 
+// The code geometry of one group.
+struct GroupGeom {
+    float nmn, nrho;  // -min, -rho: d = (w - min) - rho
+    float ylo, yhi;   // code clamp on the grid M + zeta
+};
+
 // True when candidates with scale factors Pa and Pb give the same codes on
 // every element of the group (whole warp).
 template <int G>
-__device__ bool coop_same_codes(const float* ws, float c, float Pa, float Pb, float zcap)
+__device__ bool coop_same_codes(const float* ws, const GroupGeom& gq, float Pa, float Pb)
 {
     constexpr int M = G / 32;
     const int lane = threadIdx.x & 31;
     bool same = true;
 #pragma unroll
     for (int m = 0; m < M; ++m) {
-        const float d = ws[lane + 32 * m] - c;
-        same &= int_code_z(d, Pa, zcap) == int_code_z(d, Pb, zcap);
+        const float d = centred(ws[lane + 32 * m], gq.nmn, gq.nrho);
+        same &= int_code_q(d, Pa, gq.ylo, gq.yhi) == int_code_q(d, Pb, gq.ylo, gq.yhi);
     }
     return __all_sync(0xffffffffu, same);
 }
 
-// Exact evaluation of one candidate: codes q = z + H, exact degenerate test
-// (all weighted elements on one code), two-pass centred fit, and the direct
-// error sum h (a q + B - w)^2 with (a, B) rounded to a common power-of-two
-// grid U so that a*q + B is exact and only "- w" rounds; lanes combine as a
-// float pair.  Returns the fit as (a, Bz) with r = a z + Bz, and a condition
-// estimate kap of the slope (see the tier-2 trigger in the kernel).
+// Exact evaluation of one candidate: codes q, exact degenerate test (all
+// weighted elements on one code), two-pass centred fit, and the direct error
+// sum h (a q + B - w)^2 with (a, B) rounded to a common power-of-two grid U
+// so that a*q + B is exact and only "- w" rounds; lanes combine as a float
+// pair.  Far from zero (|centre| >= 2 range) the residual is formed about an
+// anchor A at the centre, a q + (B - A) - (w - A), with w - A exact: the grid
+// then follows the group's range rather than its magnitude, and the rounded
+// fit stays a tiny fraction of a level from the optimum (its excess error is
+// second order in that distance).  dbar is the weighted mean of w - cref.
+// Returns the fit as (a, Bz) with r = a zeta + Bz (offset at zeta = 0, i.e.
+// q = J + 1), and a condition estimate kap of the slope (see the tier-2
+// trigger in the kernel).
 template <int G>
-__device__ void coop_exact(const float* ws, const float* hs, float c, float P, float zcap, float H,
-                           float Ss, float dbar, float step, float* err_hi, float* err_lo,
-                           float* a_out, float* Bz_out, float* kap_out, bool* degenerate)
+__device__ void coop_exact(const float* ws, const float* hs, const GroupGeom& gq, float P,
+                           float Jp1, float Ss, float dbar, float step, float cref, float* err_hi,
+                           float* err_lo, float* a_out, float* Bz_out, float* kap_out,
+                           bool* degenerate)
 {
     constexpr int M = G / 32;
     const int lane = threadIdx.x & 31;
@@ -190,7 +207,7 @@ __device__ void coop_exact(const float* ws, const float* hs, float c, float P, f
     for (int m = 0; m < M; ++m) {
         const int e = lane + 32 * m;
         const float h = hs[e];
-        const float q = int_code_z(ws[e] - c, P, zcap) + H;
+        const float q = int_code_q(centred(ws[e], gq.nmn, gq.nrho), P, gq.ylo, gq.yhi);
         s1 = fmaf(h, q, s1);
         if (h > 0.0f) {
             qlo = min(qlo, (int)q);
@@ -215,10 +232,10 @@ __device__ void coop_exact(const float* ws, const float* hs, float c, float P, f
         for (int m = 0; m < M; ++m) {
             const int e = lane + 32 * m;
             const float h = hs[e];
-            const float d = ws[e] - c;
-            const float dq = int_code_z(d, P, zcap) + H - qbar;
+            const float w = ws[e];
+            const float dq = int_code_q(centred(w, gq.nmn, gq.nrho), P, gq.ylo, gq.yhi) - qbar;
             const float hdq = h * dq;
-            const float wd = d - dbar;
+            const float wd = (w - cref) - dbar;
             dd = fmaf(hdq, dq, dd);
             nn = fmaf(hdq, wd, nn);
             ww = fmaf(h * wd, wd, ww);
@@ -230,8 +247,11 @@ __device__ void coop_exact(const float* ws, const float* hs, float c, float P, f
         bc = dbar - a * qbar;
         kap = sqrtf(dd * ww) / fabsf(nn) + 1.0f;
     }
-    const float B = bc + c;
-    const float mr = fmaxf(fabsf(B), fabsf(fmaf(a, 2.0f * H, B))) + fabsf(a);
+    // bc is the offset at q = 0 of w - cref.  Anchor: cref far from zero, else 0.
+    const float range = -2.0f * gq.nrho;
+    const float A = fabsf(cref) >= 2.0f * range ? cref : 0.0f;
+    const float B = bc + (cref - A);  // offset at q = 0 of w - A
+    const float mr = fmaxf(fabsf(B), fabsf(fmaf(a, 2.0f * Jp1, B))) + fabsf(a);
     int er = (int)((__float_as_uint(mr) >> 23) & 0xFF) - 126;  // mr < 2^er
     er = max(er, -100);
     const float U = __uint_as_float((uint32_t)(er - 23 + 127) << 23);
@@ -244,7 +264,8 @@ __device__ void coop_exact(const float* ws, const float* hs, float c, float P, f
         const int e = lane + 32 * m;
         const float h = hs[e];
         const float w = ws[e];
-        const float ev = fmaf(ag, int_code_z(w - c, P, zcap) + H, Bg) - w;
+        const float q = int_code_q(centred(w, gq.nmn, gq.nrho), P, gq.ylo, gq.yhi);
+        const float ev = fmaf(ag, q, Bg) - (w - A);
         t[m] = h * (ev * ev);
     }
 #pragma unroll
@@ -256,7 +277,7 @@ __device__ void coop_exact(const float* ws, const float* hs, float c, float P, f
     *err_hi = eh;
     *err_lo = el;
     *a_out = a;
-    *Bz_out = fmaf(a, H, B);
+    *Bz_out = fmaf(a, Jp1, bc + cref);
     *kap_out = kap;
 }
 
@@ -269,11 +290,11 @@ __device__ void coop_exact(const float* ws, const float* hs, float c, float P, f
 // accumulated and combined across lanes as float pairs (no fp64: its rate on
 // this part is a small fraction of fp32's); the offset is
 // mu - s*mq + mean_h(w - mu - s (q - mq)).  Returns the fit as float pairs,
-// with the offset Bz at the code origin z = 0 (r = a z + Bz).
+// with the offset Bz at the code origin zeta = 0 (q = J + 1, r = a zeta + Bz).
 template <int G>
-__device__ void coop_precise(const float* ws, const float* hs, float c, float P, float zcap,
-                             float H, float Ss, float mu, float* a_hi, float* a_lo, float* Bz_hi,
-                             float* Bz_lo)
+__device__ void coop_precise(const float* ws, const float* hs, const GroupGeom& gq, float P,
+                             float Jp1, float Ss, float mu, float* a_hi, float* a_lo,
+                             float* Bz_hi, float* Bz_lo)
 {
     constexpr int M = G / 32;
     const int lane = threadIdx.x & 31;
@@ -281,7 +302,7 @@ __device__ void coop_precise(const float* ws, const float* hs, float c, float P,
 #pragma unroll
     for (int m = 0; m < M; ++m) {
         const int e = lane + 32 * m;
-        s1 = fmaf(hs[e], int_code_z(ws[e] - c, P, zcap) + H, s1);
+        s1 = fmaf(hs[e], int_code_q(centred(ws[e], gq.nmn, gq.nrho), P, gq.ylo, gq.yhi), s1);
     }
     const float mq = rintf(wsum32(s1) / Ss * 16.0f) * 0.0625f;
 
@@ -291,7 +312,7 @@ __device__ void coop_precise(const float* ws, const float* hs, float c, float P,
         const int e = lane + 32 * m;
         const float h = hs[e];
         const float w = ws[e];
-        const float qd = int_code_z(w - c, P, zcap) + H - mq;
+        const float qd = int_code_q(centred(w, gq.nmn, gq.nrho), P, gq.ylo, gq.yhi) - mq;
         float wh, wl, xh, xl, th, tl, ph, pl;
         two_sum(w, -mu, wh, wl);
         two_prod(h, qd, xh, xl);
@@ -328,16 +349,17 @@ __device__ void coop_precise(const float* ws, const float* hs, float c, float P,
         const int e = lane + 32 * m;
         const float h = hs[e];
         const float w = ws[e];
-        const float qd = int_code_z(w - c, P, zcap) + H - mq;
+        const float qd = int_code_q(centred(w, gq.nmn, gq.nrho), P, gq.ylo, gq.yhi) - mq;
         float wh, wl;
         two_sum(w, -mu, wh, wl);
         Rs = fmaf(h, __fadd_rn(fmaf(-shi, qd, wh), fmaf(-slo, qd, wl)), Rs);
     }
     Rs = wsum32(Rs);
-    // offset at the code origin z = 0, i.e. q = H: mu + s*(H - mq) + mean residual
+    // offset at the code origin zeta = 0, i.e. q = J + 1: mu + s*(J + 1 - mq)
+    // + mean residual
     float ph, pl, zh, zl;
-    two_prod(shi, H - mq, ph, pl);  // H - mq is exact (both multiples of 1/16)
-    pl = fmaf(slo, H - mq, pl);
+    two_prod(shi, Jp1 - mq, ph, pl);  // J + 1 - mq is exact (both multiples of 1/16)
+    pl = fmaf(slo, Jp1 - mq, pl);
     two_sum(mu, ph, zh, zl);
     zl = __fadd_rn(__fadd_rn(zl, pl), Rs / Ss);
     ff_norm(zh, zl);
@@ -352,17 +374,15 @@ __device__ void coop_precise(const float* ws, const float* hs, float c, float P,
 // Two CTAs per SM: 8-warp CTAs, 6-warp ones for the AdamW-fused variant.
 // VAR: the variants of the options (a saliency other than v', packed codes);
 // without it they compile out of the common kernel.
-// HC: the code clamp is hoisted out of the candidate loop.  For a set of
-// candidate slots whose factors satisfy J f_max < tau < (J + 1) f_min (with
-// a margin the host checks), clamping |d| once at tau * range / qmax gives
-// every candidate of the set its clamped code: below the cap no code
-// reaches J + 1, above it every code is J.  The codes equal the per-candidate
-// clamp's bit for bit whenever R is finite; the set's cap costs one min per
-// element instead of one per element and candidate.
-template <int EPL, int NCH, int MAXT, bool ADAM, bool VAR, bool HC = false>
+// SS: candidates per clamp set (4, 2 or 1): the host picks the largest size
+// whose sets all admit a cap (see the header comment); every size gives the
+// same codes.
+template <int EPL, int NCH, int MAXT, bool ADAM, bool VAR, int SS>
 __global__ void __launch_bounds__(ADAM ? 192 : 256, 2)
     k_recon_int(const __grid_constant__ IntLaunch<MAXT> Lp)
 {
+    static_assert(SS == 1 || SS == 2 || SS == 4, "clamp sets of 1, 2 or 4 candidates");
+    constexpr int NS = 4 / SS;  // clamp sets per quad of candidates
     const IntParams& p = Lp.p;
     constexpr int G = EPL * kLanesPerGroup;
     constexpr int UNIT = kGroupsPerUnit * G;
@@ -425,6 +445,8 @@ __global__ void __launch_bounds__(ADAM ? 192 : 256, 2)
     };
 
     // Drain the copies still in flight from iteration `it` on, then leave.
+    // (Each of these waits is bounded too: a copy that never lands is given
+    // up on, and the warp then exits with it still in flight.)
     auto fail = [&](int64_t it) {
         if (lane == 0) record_timeout(p.status);
         for (int j = 0; j < S; ++j) {
@@ -440,22 +462,23 @@ __global__ void __launch_bounds__(ADAM ? 192 : 256, 2)
             if (u < n_units) issue(u, s);
         }
 
-    if constexpr (HC)  // which kernel ran, for the tuning counters
+    if constexpr (SS > 1)  // which kernel ran, for the tuning counters
         if (p.stats && threadIdx.x == 0) atomicAdd(&p.stats[3], 1u);
 
     if (p.force_timeout_ns && blockIdx.x == 0 && warp == 0) {
         // Failure-path hook: a barrier nothing ever arrives on.
-        if (!mbar_wait_bounded(&bars[S], 0, p.force_timeout_ns)) {
+        if (!warp_wait_bounded(&bars[S], 0, p.force_timeout_ns)) {
             fail(0);
             return;
         }
     }
 
     const float qmaxf = (float)p.qmax;
-    const float H = 0.5f * qmaxf;
-    const float zcap = kFloorMagic + (float)(p.qmax >> 1);
-    const float2 M2 = make_float2(kFloorMagic, kFloorMagic);
-    const float2 nhm2 = make_float2(-kHalfBelowMagic, -kHalfBelowMagic);
+    const int J = p.qmax >> 1;
+    const float Jp1 = (float)(J + 1);
+    const float ylo = kGridMagic - Jp1, yhi = kGridMagic + (float)J;
+    const float2 Mg2 = make_float2(kGridMagic, kGridMagic);
+    const float2 nMg2 = make_float2(-kGridMagic, -kGridMagic);
     const float ulp = 5.9604645e-8f * p.tie_kappa;
     const float2 beta22 = make_float2(p.beta2, p.beta2);
     const float2 c12 = make_float2(p.c1, p.c1);
@@ -469,7 +492,7 @@ __global__ void __launch_bounds__(ADAM ? 192 : 256, 2)
     for (int64_t it = 0;; ++it) {
         const int64_t u = first + it * stride;
         if (u >= n_units) break;
-        if (!mbar_wait_bounded(&bars[s_cur], parity, p.timeout_ns)) {
+        if (!warp_wait_bounded(&bars[s_cur], parity, p.timeout_ns)) {
             fail(it);
             return;
         }
@@ -495,7 +518,7 @@ __global__ void __launch_bounds__(ADAM ? 192 : 256, 2)
             float* mout = T.m + gbase + sl * 4;
             auto pass_a = [&](auto gk) {
                 constexpr int GK = decltype(gk)::value;
-                float2 SS = make_float2(0.0f, 0.0f), SW = SS;
+                float2 SS2 = make_float2(0.0f, 0.0f), SW = SS2;
 #pragma unroll
                 for (int i = 0; i < NCHK; ++i) {
                     const int e = gs * G + i * 32 + sl * 4;
@@ -568,11 +591,11 @@ __global__ void __launch_bounds__(ADAM ? 192 : 256, 2)
                     mn = fminf(fminf(fminf(mn, w4.x), fminf(w4.y, w4.z)), w4.w);
                     mx = fmaxf(fmaxf(fmaxf(mx, w4.x), fmaxf(w4.y, w4.z)), w4.w);
                     const float2 hA = make_float2(h4.x, h4.y), hB = make_float2(h4.z, h4.w);
-                    SS = __fadd2_rn(SS, __fadd2_rn(hA, hB));
+                    SS2 = __fadd2_rn(SS2, __fadd2_rn(hA, hB));
                     SW = __ffma2_rn(hA, make_float2(w4.x, w4.y), SW);
                     SW = __ffma2_rn(hB, make_float2(w4.z, w4.w), SW);
                 }
-                ss = SS.x + SS.y;
+                ss = SS2.x + SS2.y;
                 sw = SW.x + SW.y;
             };
             if (p.g_kind == 2) pass_a(std::integral_constant<int, 2>{});
@@ -581,7 +604,7 @@ __global__ void __launch_bounds__(ADAM ? 192 : 256, 2)
             if (VAR && p.h_mode != kSalEma) {
                 // the fit's saliency is v'^2 or 1: rewrite h in the tile (v'
                 // went out already) and take its sums again
-                float2 SS = make_float2(0.0f, 0.0f), SW = SS;
+                float2 SS2 = make_float2(0.0f, 0.0f), SW = SS2;
 #pragma unroll 1
                 for (int i = 0; i < NCHK; ++i) {
                     const int e = gs * G + i * 32 + sl * 4;
@@ -592,11 +615,11 @@ __global__ void __launch_bounds__(ADAM ? 192 : 256, 2)
                              : make_float4(1.0f, 1.0f, 1.0f, 1.0f);
                     *reinterpret_cast<float4*>(hs + e) = h4;
                     const float2 hA = make_float2(h4.x, h4.y), hB = make_float2(h4.z, h4.w);
-                    SS = __fadd2_rn(SS, __fadd2_rn(hA, hB));
+                    SS2 = __fadd2_rn(SS2, __fadd2_rn(hA, hB));
                     SW = __ffma2_rn(hA, make_float2(w4.x, w4.y), SW);
                     SW = __ffma2_rn(hB, make_float2(w4.z, w4.w), SW);
                 }
-                ss = SS.x + SS.y;
+                ss = SS2.x + SS2.y;
                 sw = SW.x + SW.y;
             }
         }
@@ -620,92 +643,98 @@ __global__ void __launch_bounds__(ADAM ? 192 : 256, 2)
         }
         const float range = mx - mn;
         const bool flat = !(range > 0.0f);
-        const float c = 0.5f * (mn + mx);
+        const float rho = 0.5f * range;
+        GroupGeom gq;
+        gq.nmn = -mn;
+        gq.nrho = -rho;
+        gq.ylo = ylo;
+        gq.yhi = yhi;
+        const float cref = mn + rho;  // the centre, rounded (an anchor only)
         if (h_one) ss = (float)G;
         const float inv_ss = __fdividef(1.0f, ss);
         // mu: approximate weighted mean of w (only a centre for the sums)
-        const float mu = h_one ? c : sw * inv_ss;
+        const float mu = h_one ? cref : sw * inv_ss;
         // approximate divisions (<= 2 ulp) are enough here: R scales the code
         // positions (margins are measured against the clipping range), and
         // the accuracy of the kept fit is checked below
         const float R = flat ? 0.0f : __fdividef(qmaxf, range);
-        const float2 nc2 = make_float2(-c, -c), nmu2 = make_float2(-mu, -mu);
+        const float2 nmn2 = make_float2(-mn, -mn), nrho2 = make_float2(-rho, -rho);
+        const float2 nmu2 = make_float2(-mu, -mu);
+        // the weighted mean's offset from the centre, for the chunks' centres
+        const float dmu = centred(mu, -mn, -rho);
 
-        // ---- pass B + reduction + candidate errors, 8 candidates at a time.
-        // Codes use d = w - c; moments use e = w - mu: S1 = sum h z,
-        // S2 = sum h z^2, S3 = sum h z e = sum (h |z|) (sign(d) e).
-        float Ek[NCH], dEk[NCH], T1k[NCH], T2k[NCH], T3k[NCH];
+        // ---- pass B + reduction + candidate errors, 8 candidates a chunk,
+        // 4 a sweep over the tile.  Codes from d = (w - mn) - rho; moments
+        // about the chunk's centre code zeta0 and, for S3, e = w - mu.
+        float Ek[NCH], dEk[NCH], T1k[NCH], T2k[NCH], T3k[NCH], Y0k[NCH];
         bool suspk[NCH];
         float se = 0.0f, see = 0.0f;
 #pragma unroll
         for (int ch = 0; ch < NCH; ++ch) {
-            float2 P2[8];
-#pragma unroll
-            for (int kk = 0; kk < 8; ++kk) {
-                const float P = R * p.invf[ch * 8 + kk];
-                P2[kk] = make_float2(P, P);
-            }
-            float2 A1[8], A2[8], A3[8];
-#pragma unroll
-            for (int kk = 0; kk < 8; ++kk) A1[kk] = A2[kk] = A3[kk] = make_float2(0.0f, 0.0f);
+            // centre: the code of the weighted mean for the chunk's mean 1/f
+            const float y0 = fminf(fmaxf(__fmaf_rd(dmu, R * p.invfc[ch], kGridMagic), ylo), yhi);
+            const float2 nY02 = make_float2(-y0, -y0);
+            Y0k[ch] = y0;
             float2 SE = make_float2(0.0f, 0.0f), SEE = make_float2(0.0f, 0.0f);
+#pragma unroll
+            for (int qd = 0; qd < 2; ++qd) {
+                const int kq = ch * 8 + qd * 4;
+                float2 A1[4], A2[4], A3[4];
+#pragma unroll
+                for (int kk = 0; kk < 4; ++kk) A1[kk] = A2[kk] = A3[kk] = make_float2(0.0f, 0.0f);
+                if ((ch == 0 && qd == 0) || kq < p.n_clip) {
+                    float2 P2[4];
+#pragma unroll
+                    for (int kk = 0; kk < 4; ++kk) {
+                        const float P = R * p.invf[kq + kk];
+                        P2[kk] = make_float2(P, P);
+                    }
+                    float cp[NS];
+#pragma unroll
+                    for (int s = 0; s < NS; ++s) cp[s] = p.cap[kq + s * SS] * range;
 // rolled: a compact unit loop keeps the careful paths' code from evicting it
-// from the instruction cache when they run (the fused AdamW variant, with
-// fewer warps and more registers, gains from two chunks an iteration)
-#pragma unroll(ADAM ? 2 : 1)
-            for (int i = 0; i < NCHK; ++i) {
-                const int e = gs * G + i * 32 + sl * 4;
-                const float4 w4 = lds128(ws + e);
-                const float4 h4 = lds128(hs + e);
+// from the instruction cache when they run
+#pragma unroll 1
+                    for (int i = 0; i < NCHK; ++i) {
+                        const int e = gs * G + i * 32 + sl * 4;
+                        const float4 w4 = lds128(ws + e);
+                        const float4 h4 = lds128(hs + e);
 #pragma unroll
-                for (int pr = 0; pr < 2; ++pr) {
-                    const float2 wv = pr ? make_float2(w4.z, w4.w) : make_float2(w4.x, w4.y);
-                    const float2 h = pr ? make_float2(h4.z, h4.w) : make_float2(h4.x, h4.y);
-                    const float2 d = __fadd2_rn(wv, nc2);
-                    const float2 ev = __fadd2_rn(wv, nmu2);
-                    // |d| as fabsf: the compiler folds it into the min/FMA operands
-                    const float2 ad = make_float2(fabsf(d.x), fabsf(d.y));
-                    float2 adc[2];
-                    if constexpr (HC) {
-                        // the caps of the chunk's two slot sets
-                        const float cap0 = p.hcap[ch * 2] * range, cap1 = p.hcap[ch * 2 + 1] * range;
-                        adc[0] = make_float2(fminf(ad.x, cap0), fminf(ad.y, cap0));
-                        adc[1] = make_float2(fminf(ad.x, cap1), fminf(ad.y, cap1));
-                    }
-                    const float2 hsg = signed_h2(h, d);
-                    const float2 sev = make_float2(
-                        __uint_as_float(__float_as_uint(ev.x) ^ (__float_as_uint(d.x) & 0x80000000u)),
-                        __uint_as_float(__float_as_uint(ev.y) ^ (__float_as_uint(d.y) & 0x80000000u)));
-                    if (ch == 0) {
-                        const float2 he = __fmul2_rn(h, ev);
-                        SE = __fadd2_rn(SE, he);
-                        SEE = __ffma2_rn(he, ev, SEE);
-                    }
+                        for (int pr = 0; pr < 2; ++pr) {
+                            const float2 wv = pr ? make_float2(w4.z, w4.w) : make_float2(w4.x, w4.y);
+                            const float2 h = pr ? make_float2(h4.z, h4.w) : make_float2(h4.x, h4.y);
+                            const float2 d = __fadd2_rn(__fadd2_rn(wv, nmn2), nrho2);
+                            const float2 ev = __fadd2_rn(wv, nmu2);
+                            if (ch == 0 && qd == 0) {
+                                const float2 he = __fmul2_rn(h, ev);
+                                SE = __fadd2_rn(SE, he);
+                                SEE = __ffma2_rn(he, ev, SEE);
+                            }
+                            float2 dc[NS];
 #pragma unroll
-                    for (int kk = 0; kk < 8; ++kk) {
-                        float2 y;
-                        if constexpr (HC) {
-                            y = __ffma2_rd(adc[kk >> 2], P2[kk], M2);
-                        } else {
-                            y = __ffma2_rd(ad, P2[kk], M2);
-                            y.x = fminf(y.x, zcap);
-                            y.y = fminf(y.y, zcap);
+                            for (int s = 0; s < NS; ++s)
+                                dc[s] = make_float2(fminf(fmaxf(d.x, -cp[s]), cp[s]),
+                                                    fminf(fmaxf(d.y, -cp[s]), cp[s]));
+#pragma unroll
+                            for (int kk = 0; kk < 4; ++kk) {
+                                const float2 y = __ffma2_rd(dc[kk / SS], P2[kk], Mg2);
+                                const float2 zc = __fadd2_rn(y, nY02);  // zeta - zeta0, exact
+                                const float2 t = __fmul2_rn(h, zc);
+                                A1[kk] = __ffma2_rn(h, zc, A1[kk]);
+                                A2[kk] = __ffma2_rn(t, zc, A2[kk]);
+                                A3[kk] = __ffma2_rn(t, ev, A3[kk]);
+                            }
                         }
-                        const float2 z = __fadd2_rn(y, nhm2);  // |z|
-                        const float2 t = __fmul2_rn(h, z);
-                        A1[kk] = __ffma2_rn(hsg, z, A1[kk]);
-                        A2[kk] = __ffma2_rn(t, z, A2[kk]);
-                        A3[kk] = __ffma2_rn(t, sev, A3[kk]);
                     }
                 }
-            }
-            // transpose through shared memory: lane L writes row L (its sums
-            // of candidate kk in 16-byte column kk ^ (L & 7)), lane (gs, sl)
-            // sums column sl of the 8 rows of its group (a tree)
+                // transpose through shared memory: lane L writes row L (its sums
+                // of candidate kk in 16-byte column kk ^ (L & 7)), lane (gs, sl)
+                // sums column sl of the 8 rows of its group (a tree)
 #pragma unroll
-            for (int kk = 0; kk < 8; ++kk)
-                *reinterpret_cast<float4*>(red + lane * 32 + ((kk ^ (lane & 7)) << 2)) =
-                    make_float4(A1[kk].x + A1[kk].y, A2[kk].x + A2[kk].y, A3[kk].x + A3[kk].y, 0.0f);
+                for (int kk = 0; kk < 4; ++kk)
+                    *reinterpret_cast<float4*>(red + lane * 32 + (((qd * 4 + kk) ^ (lane & 7)) << 2)) =
+                        make_float4(A1[kk].x + A1[kk].y, A2[kk].x + A2[kk].y, A3[kk].x + A3[kk].y, 0.0f);
+            }
             __syncwarp();
             float4 x[8];
 #pragma unroll
@@ -732,7 +761,7 @@ __global__ void __launch_bounds__(ADAM ? 192 : 256, 2)
             // candidate k = 8 ch + sl: E = N^2/D and a bound dE on its fp32
             // error.  The sums are accumulated over tie_kappa levels at most,
             // so each is within tie_kappa ulps of the sum of its terms'
-            // magnitudes: sum h z^2 = S2, sum |h z e| <= sqrt(S2 * sum h e^2).
+            // magnitudes: sum h zc^2 = S2, sum |h zc e| <= sqrt(S2 * sum h e^2).
             const float ebar = se * inv_ss;
             const float T1 = x[0].x, T2 = x[0].y, T3 = x[0].z;
             const float zbar = T1 * inv_ss;
@@ -802,33 +831,37 @@ __global__ void __launch_bounds__(ADAM ? 192 : 256, 2)
         }
         if (kb > 0x7ff) kb = 0;  // every candidate suspicious: the exact path picks
 
-        // the winner's sums, from its owner lane
-        float T1b = 0.0f, T2b = 0.0f, T3b = 0.0f;
-        {
-            const int owner = (gs * 8) | (kb & 7);
+        // the sums of candidate k, from its owner lane (every lane of a group
+        // names the same k)
+        auto sums_of = [&](int k, float& t1, float& t2, float& t3) {
+            const int owner = (gs * 8) | (k & 7);
 #pragma unroll
             for (int ch = 0; ch < NCH; ++ch) {
-                const float t1 = __shfl_sync(0xffffffffu, T1k[ch], owner);
-                const float t2 = __shfl_sync(0xffffffffu, T2k[ch], owner);
-                const float t3 = __shfl_sync(0xffffffffu, T3k[ch], owner);
-                if ((kb >> 3) == ch) {
-                    T1b = t1;
-                    T2b = t2;
-                    T3b = t3;
+                const float a1 = __shfl_sync(0xffffffffu, T1k[ch], owner);
+                const float a2 = __shfl_sync(0xffffffffu, T2k[ch], owner);
+                const float a3 = __shfl_sync(0xffffffffu, T3k[ch], owner);
+                if ((k >> 3) == ch) {
+                    t1 = a1;
+                    t2 = a2;
+                    t3 = a3;
                 }
             }
-        }
+        };
+        float T1b = 0.0f, T2b = 0.0f, T3b = 0.0f;
+        sums_of(kb, T1b, T2b, T3b);
         // Candidates needing an exact comparison: within the fp32 error bound
-        // of the winner.  Those whose sums equal the winner's bit for bit
-        // ("twins") almost always have the winner's codes -- equal codes give
-        // equal errors, and the lower index is kept, as Algorithm 1's argmin
-        // does -- but an element of tiny saliency can differ without moving the
-        // sums, so twins are first checked code by code (cheaply, deferred).
+        // of the winner.  Those of the winner's chunk (one centre) whose sums
+        // equal the winner's bit for bit ("twins") almost always have the
+        // winner's codes -- equal codes give equal errors, and the lower index
+        // is kept, as Algorithm 1's argmin does -- but an element of tiny
+        // saliency can differ without moving the sums, so twins are first
+        // checked code by code (cheaply, deferred).
         unsigned my_set = 0, my_twin = 0;
 #pragma unroll
         for (int ch = 0; ch < NCH; ++ch) {
             const int k = ch * 8 + sl;
-            const bool twin = T1k[ch] == T1b && T2k[ch] == T2b && T3k[ch] == T3b;
+            const bool twin =
+                ch == (kb >> 3) && T1k[ch] == T1b && T2k[ch] == T2b && T3k[ch] == T3b;
             const bool contender = k != kb && Ek[ch] > -INFINITY && Eb - Ek[ch] <= dEb + dEk[ch];
             if (contender || suspk[ch]) my_set |= 1u << ch;
             if (contender && twin && !suspk[ch]) my_twin |= 1u << ch;
@@ -844,7 +877,7 @@ __global__ void __launch_bounds__(ADAM ? 192 : 256, 2)
         if (Eb == -INFINITY) set = (p.n_clip >= 32) ? 0xFFFFFFFFu : ((1u << p.n_clip) - 1u);
         else if (set) set |= 1u << kb;
 
-        // the kept fit: r = a z + Bz (a = a_sel + a_lo, Bz = Bz + Bz_lo); kap
+        // the kept fit: r = a zeta + Bz (a = a_sel + a_lo, Bz = Bz + Bz_lo); kap
         // estimates the conditioning of its slope
         float a_sel = 0.0f, Bz = 0.0f, kap_sel = 0.0f;
         float Bz_lo = 0.0f, a_lo = 0.0f;
@@ -857,11 +890,17 @@ __global__ void __launch_bounds__(ADAM ? 192 : 256, 2)
             const int g = (__ffs(todo) - 1) >> 3;
             todo &= todo - 1;
             const int src = g * 8;
-            const float gc = __shfl_sync(0xffffffffu, c, src);
+            GroupGeom ggq;
+            ggq.nmn = __shfl_sync(0xffffffffu, gq.nmn, src);
+            ggq.nrho = __shfl_sync(0xffffffffu, gq.nrho, src);
+            ggq.ylo = ylo;
+            ggq.yhi = yhi;
             const float grange = __shfl_sync(0xffffffffu, range, src);
             const float gR = __shfl_sync(0xffffffffu, R, src);
             const float gss = __shfl_sync(0xffffffffu, ss, src);
-            const float gdbar = __shfl_sync(0xffffffffu, (mu + ebar) - c, src);
+            const float gcref = __shfl_sync(0xffffffffu, cref, src);
+            // the weighted mean of w - cref
+            const float gdbar = __shfl_sync(0xffffffffu, (mu - cref) + ebar, src);
             unsigned gset = __shfl_sync(0xffffffffu, set, src);
             const unsigned gtwins = __shfl_sync(0xffffffffu, twins, src);
             const int gkb0 = __shfl_sync(0xffffffffu, kb, src);
@@ -871,7 +910,7 @@ __global__ void __launch_bounds__(ADAM ? 192 : 256, 2)
             while (tw) {
                 const int k = __ffs(tw) - 1;
                 tw &= tw - 1;
-                if (coop_same_codes<G>(gws, gc, gR * p.invf[k], gR * p.invf[gkb0], zcap))
+                if (coop_same_codes<G>(gws, ggq, gR * p.invf[k], gR * p.invf[gkb0]))
                     gset &= ~(1u << k);
             }
             if (gset == (1u << gkb0)) continue;  // only the winner left
@@ -884,8 +923,8 @@ __global__ void __launch_bounds__(ADAM ? 192 : 256, 2)
                 gset &= gset - 1;
                 float eh, el, a_k, B_k, kap_k;
                 bool deg_k;
-                coop_exact<G>(gws, ghs, gc, gR * p.invf[k], zcap, H, gss, gdbar,
-                              p.f[k] * grange / qmaxf, &eh, &el, &a_k, &B_k, &kap_k, &deg_k);
+                coop_exact<G>(gws, ghs, ggq, gR * p.invf[k], Jp1, gss, gdbar,
+                              p.f[k] * grange / qmaxf, gcref, &eh, &el, &a_k, &B_k, &kap_k, &deg_k);
                 if (best_k < 0 || ff_less(eh, el, best_h, best_l)) {
                     best_h = eh;
                     best_l = el;
@@ -905,72 +944,33 @@ __global__ void __launch_bounds__(ADAM ? 192 : 256, 2)
             }
         }
 
-        // ---- pass R: codes of the kept candidate (kept in registers for the
-        // output) and the two sums that the candidate sums only give with
-        // cancellation, now centred: codes about their weighted mean rounded
-        // to a multiple of 1/2 (m), weights about mu.  Then the fit (Eq. 4).
-        constexpr bool kKeepZ = EPL <= 16;
-        float zr[kKeepZ ? EPL : 1];
-        const float Pk = R * p.invf[kb];
-        const float2 Pk2 = make_float2(Pk, Pk);
-        // a multiple of 1/2 (codes z are half-integers, so z - m and (z - m)^2 stay exact)
-        const float m = 0.5f * rintf(2.0f * T1b * inv_ss);
-        {
-            const float2 nm2 = make_float2(-m, -m);
-            float2 D2 = make_float2(0.0f, 0.0f), N2 = D2, A2 = D2;
+        // ---- the fit (Eq. 4) from the kept candidate's centred sums: codes
+        // about its chunk's centre zeta0, weights about mu
+        sums_of(kb, T1b, T2b, T3b);
+        float y0b = Y0k[0];
 #pragma unroll
-            for (int i = 0; i < NCHK; ++i) {
-                const int e = gs * G + i * 32 + sl * 4;
-                const float4 w4 = lds128(ws + e);
-                const float4 h4 = lds128(hs + e);
-#pragma unroll
-                for (int pr = 0; pr < 2; ++pr) {
-                    const float2 wv = pr ? make_float2(w4.z, w4.w) : make_float2(w4.x, w4.y);
-                    const float2 h = pr ? make_float2(h4.z, h4.w) : make_float2(h4.x, h4.y);
-                    const float2 d = __fadd2_rn(wv, nc2);
-                    float2 y = __ffma2_rd(make_float2(fabsf(d.x), fabsf(d.y)), Pk2, M2);
-                    y.x = fminf(y.x, zcap);
-                    y.y = fminf(y.y, zcap);
-                    const float2 z = __fadd2_rn(y, nhm2);
-                    const float2 zs = make_float2(copysignf(z.x, d.x), copysignf(z.y, d.y));
-                    if constexpr (kKeepZ) {
-                        zr[i * 4 + pr * 2] = zs.x;
-                        zr[i * 4 + pr * 2 + 1] = zs.y;
-                    }
-                    const float2 dz = __fadd2_rn(zs, nm2);
-                    const float2 hdz = __fmul2_rn(h, dz);
-                    D2 = __ffma2_rn(hdz, dz, D2);
-                    N2 = __ffma2_rn(hdz, __fadd2_rn(wv, nmu2), N2);
-                    A2 = __fadd2_rn(A2, hdz);
-                }
-            }
-            float Dr = D2.x + D2.y, Nr = N2.x + N2.y, A = A2.x + A2.y;
-#pragma unroll
-            for (int o = 4; o; o >>= 1) {
-                Dr += shx(Dr, o);
-                Nr += shx(Nr, o);
-                A += shx(A, o);
-            }
-            if (!deg_sel) {
-                // A = sum h (z - m) (small); sum h (w - mu) = Se
-                const float Aq = A * inv_ss;
-                const float Nc = Nr - A * ebar, Dc = Dr - A * Aq;
-                // the quotient from the fast reciprocal and one correction
-                // (the remainder Nc - q Dc is exact by FMA): within an ulp
-                const float q0 = __fdividef(Nc, Dc);
-                const float an = fmaf(fmaf(-q0, Dc, Nc), __fdividef(1.0f, Dc), q0);
-                // Bz = (mu + ebar) - a (m + Aq), as a float pair
-                float p_h, p_l, bh, bl;
-                two_prod(an, m, p_h, p_l);
-                two_sum(mu, -p_h, bh, bl);
-                bl = __fadd_rn(bl, __fsub_rn(ebar, fmaf(an, Aq, p_l)));
-                ff_norm(bh, bl);
-                a_sel = an;
-                Bz = bh;
-                Bz_lo = bl;
-                const float dse = fmaxf(Dr * see, 1e-37f);
-                kap_sel = __fdividef(dse * rsqrtf(dse), fabsf(Nc)) + __fdividef(Dr, Dc);
-            }
+        for (int ch = 1; ch < NCH; ++ch)
+            if ((kb >> 3) == ch) y0b = Y0k[ch];
+        if (!deg_sel) {
+            // T1 = sum h (zeta - zeta0) (small); sum h (w - mu) = Se
+            const float Aq = T1b * inv_ss;
+            const float Nc = T3b - T1b * ebar, Dc = T2b - T1b * Aq;
+            // the quotient from the fast reciprocal and one correction
+            // (the remainder Nc - q Dc is exact by FMA): within an ulp
+            const float q0 = __fdividef(Nc, Dc);
+            const float an = fmaf(fmaf(-q0, Dc, Nc), __fdividef(1.0f, Dc), q0);
+            // Bz = (mu + ebar) - a (zeta0 + Aq), as a float pair
+            const float z0 = y0b - kGridMagic;  // exact
+            float p_h, p_l, bh, bl;
+            two_prod(an, z0, p_h, p_l);
+            two_sum(mu, -p_h, bh, bl);
+            bl = __fadd_rn(bl, __fsub_rn(ebar, fmaf(an, Aq, p_l)));
+            ff_norm(bh, bl);
+            a_sel = an;
+            Bz = bh;
+            Bz_lo = bl;
+            const float dse = fmaxf(T2b * see, 1e-37f);
+            kap_sel = __fdividef(dse * rsqrtf(dse), fabsf(Nc)) + __fdividef(T2b, Dc);
         }
 
         // ---- output accuracy check.  The fp32 fit's error at any level is at
@@ -984,8 +984,8 @@ __global__ void __launch_bounds__(ADAM ? 192 : 256, 2)
         bool prec;
         {
             const float est =
-                p.fit_ulps * 5.9604645e-8f * (fabsf(a_sel) * qmaxf * kap_sel + fabsf(c) + range);
-            const float b0 = fmaf(-a_sel, H, Bz);  // offset at q = 0
+                p.fit_ulps * 5.9604645e-8f * (fabsf(a_sel) * qmaxf * kap_sel + fabsf(cref) + range);
+            const float b0 = fmaf(-a_sel, Jp1, Bz);  // offset at q = 0
             prec = est > 1e-7f + 1e-5f * fabsf(b0);
             if (!p.r_bf16) {
                 const float q0 = fminf(fmaxf(rintf(__fdividef(-b0, a_sel)), 0.0f), qmaxf);
@@ -1014,14 +1014,18 @@ __global__ void __launch_bounds__(ADAM ? 192 : 256, 2)
             const int g = (__ffs(todo) - 1) >> 3;
             todo &= todo - 1;
             const int src = g * 8;
-            const float gc = __shfl_sync(0xffffffffu, c, src);
+            GroupGeom ggq;
+            ggq.nmn = __shfl_sync(0xffffffffu, gq.nmn, src);
+            ggq.nrho = __shfl_sync(0xffffffffu, gq.nrho, src);
+            ggq.ylo = ylo;
+            ggq.yhi = yhi;
             const float gR = __shfl_sync(0xffffffffu, R, src);
             const float gss = __shfl_sync(0xffffffffu, ss, src);
             const float gmu = __shfl_sync(0xffffffffu, mu + ebar, src);
             const int gkb = __shfl_sync(0xffffffffu, kb, src);
             if (p.stats && lane == 0) atomicAdd(&p.stats[1], 1u);
             float ga, ga_lo, gB, gB_lo;
-            coop_precise<G>(ws + g * G, hs + g * G, gc, gR * p.invf[gkb], zcap, H, gss, gmu, &ga,
+            coop_precise<G>(ws + g * G, hs + g * G, ggq, gR * p.invf[gkb], Jp1, gss, gmu, &ga,
                             &ga_lo, &gB, &gB_lo);
             if (gs == g) {
                 a_sel = ga;
@@ -1031,32 +1035,30 @@ __global__ void __launch_bounds__(ADAM ? 192 : 256, 2)
             }
         }
 
-        // ---- pass C: outputs of the kept candidate
+        // ---- pass C: outputs of the kept candidate (its codes recomputed
+        // with the clamp of its set, as pass B formed them)
+        const float Pk = R * p.invf[kb];
+        const float capk = p.cap[kb] * range;
         {
             const float2 a2 = make_float2(a_sel, a_sel), B2 = make_float2(Bz, Bz);
             const float2 alo2 = make_float2(a_lo, a_lo), Blo2 = make_float2(Bz_lo, Bz_lo);
+            const float2 Pk2 = make_float2(Pk, Pk);
             const int64_t ebase = gbase + sl * 4;
             // general: codes, fp32 r, zero-range groups (r = w); fast: none
             auto pass_c = [&](auto general) {
                 constexpr bool GEN = decltype(general)::value;
 #pragma unroll
                 for (int i = 0; i < NCHK; ++i) {
-                    float2 zs[2];
-                    if constexpr (kKeepZ) {
-                        zs[0] = make_float2(zr[i * 4], zr[i * 4 + 1]);
-                        zs[1] = make_float2(zr[i * 4 + 2], zr[i * 4 + 3]);
-                    } else {
-                        const float4 w4 = lds128(ws + gs * G + i * 32 + sl * 4);
+                    const float4 w4 = lds128(ws + gs * G + i * 32 + sl * 4);
+                    float2 yv[2], zs[2];
 #pragma unroll
-                        for (int pr = 0; pr < 2; ++pr) {
-                            const float2 wv = pr ? make_float2(w4.z, w4.w) : make_float2(w4.x, w4.y);
-                            const float2 d = __fadd2_rn(wv, nc2);
-                            float2 y = __ffma2_rd(make_float2(fabsf(d.x), fabsf(d.y)), Pk2, M2);
-                            y.x = fminf(y.x, zcap);
-                            y.y = fminf(y.y, zcap);
-                            const float2 z = __fadd2_rn(y, nhm2);
-                            zs[pr] = make_float2(copysignf(z.x, d.x), copysignf(z.y, d.y));
-                        }
+                    for (int pr = 0; pr < 2; ++pr) {
+                        const float2 wv = pr ? make_float2(w4.z, w4.w) : make_float2(w4.x, w4.y);
+                        const float2 d = __fadd2_rn(__fadd2_rn(wv, nmn2), nrho2);
+                        const float2 dc = make_float2(fminf(fmaxf(d.x, -capk), capk),
+                                                      fminf(fmaxf(d.y, -capk), capk));
+                        yv[pr] = __ffma2_rd(dc, Pk2, Mg2);
+                        zs[pr] = __fadd2_rn(yv[pr], nMg2);  // zeta, exact
                     }
                     float2 rv[2];
 #pragma unroll
@@ -1065,19 +1067,19 @@ __global__ void __launch_bounds__(ADAM ? 192 : 256, 2)
                     const int64_t eo = ebase + i * 32;
                     if constexpr (GEN) {
                         if (flat) {
-                            const float4 w4 = lds128(ws + gs * G + i * 32 + sl * 4);
                             rv[0] = make_float2(w4.x, w4.y);
                             rv[1] = make_float2(w4.z, w4.w);
                         }
                         if (T.codes) {
-                            // q = z + qmax/2, an integer in [0, 255]: its bits above 2^23
+                            // q = y - ylo, an integer in [0, 255]: y and ylo share
+                            // a binade, so it is the difference of their bits
+                            const uint32_t b0 = __float_as_uint(ylo);
                             uint32_t cw = 0;
 #pragma unroll
-                            for (int pr = 0; pr < 2; ++pr) {
-                                const float2 qf = __fadd2_rn(__fadd2_rn(zs[pr], make_float2(H, H)), M2);
-                                cw |= ((__float_as_uint(qf.x) & 0xFFu) | ((__float_as_uint(qf.y) & 0xFFu) << 8))
+                            for (int pr = 0; pr < 2; ++pr)
+                                cw |= (((__float_as_uint(yv[pr].x) - b0) & 0xFFu) |
+                                       (((__float_as_uint(yv[pr].y) - b0) & 0xFFu) << 8))
                                       << (16 * pr);
-                            }
                             if (flat) cw = 0;
                             if (!(VAR && p.codes_packed) && valid)
                                 stg_cs(reinterpret_cast<uint32_t*>(T.codes + eo), cw);
@@ -1107,15 +1109,15 @@ __global__ void __launch_bounds__(ADAM ? 192 : 256, 2)
                 // OR-ed into them in the transpose scratch.
                 uint32_t* wsc = reinterpret_cast<uint32_t*>(red) + gs * 8;
                 const uint32_t o = (uint32_t)sl * 4u * (uint32_t)p.bits;
-// (codes recomputed from the tile, as pass R did: kept registers would
+// (codes recomputed from the tile, as pass C forms them: kept registers would
 // raise the pressure of the common path)
 #pragma unroll 1
                 for (int i = 0; i < NCHK; ++i) {
                     uint32_t pk = 0;
 #pragma unroll
                     for (int j = 0; j < 4; ++j) {
-                        const float z = int_code_z(ws[gs * G + i * 32 + sl * 4 + j] - c, Pk, zcap);
-                        const uint32_t q = flat ? 0u : (uint32_t)(int)(z + H);
+                        const float d = centred(ws[gs * G + i * 32 + sl * 4 + j], gq.nmn, gq.nrho);
+                        const uint32_t q = flat ? 0u : (uint32_t)int_code_q(d, Pk, ylo, yhi);
                         pk |= q << (j * p.bits);
                     }
                     const uint64_t f = (uint64_t)pk << (o & 31u);
@@ -1132,11 +1134,11 @@ __global__ void __launch_bounds__(ADAM ? 192 : 256, 2)
                 }
             }
             if (valid && sl == 0) {
-                // b = Bz - a*H: the offset at code 0
+                // b = Bz - a*(J + 1): the offset at code 0
                 float bh = Bz, bl = Bz_lo;
-                ff_add_prod(bh, bl, -a_sel, -a_lo, H);
+                ff_add_prod(bh, bl, -a_sel, -a_lo, Jp1);
                 T.a[grp] = flat ? 0.0f : a_sel;
-                T.b[grp] = flat ? c : __fadd_rn(bh, bl);
+                T.b[grp] = flat ? mn : __fadd_rn(bh, bl);
                 if (T.idx) T.idx[grp] = flat ? 0 : (uint8_t)kb;
             }
         }

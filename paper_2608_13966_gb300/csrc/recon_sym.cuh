@@ -148,7 +148,7 @@ __global__ void __launch_bounds__(256, 2) k_recon_sym(const __grid_constant__ In
             if (u < n_units) issue(u, s);
         }
     if (p.force_timeout_ns && blockIdx.x == 0 && warp == 0) {
-        if (!mbar_wait_bounded(&bars[S], 0, p.force_timeout_ns)) {
+        if (!warp_wait_bounded(&bars[S], 0, p.force_timeout_ns)) {
             fail(0);
             return;
         }
@@ -166,7 +166,7 @@ __global__ void __launch_bounds__(256, 2) k_recon_sym(const __grid_constant__ In
     for (int64_t it = 0;; ++it) {
         const int64_t u = first + it * stride;
         if (u >= n_units) break;
-        if (!mbar_wait_bounded(&bars[s_cur], parity, p.timeout_ns)) {
+        if (!warp_wait_bounded(&bars[s_cur], parity, p.timeout_ns)) {
             fail(it);
             return;
         }

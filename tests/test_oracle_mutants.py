@@ -12,6 +12,7 @@ import subprocess
 import pytest
 
 import oracle as oracle_mod
+from tests import test_oracle_checker_pins as cpins
 from tests import test_oracle_pins as pins
 
 SRC = os.path.join(os.path.dirname(os.path.dirname(os.path.abspath(__file__))),
@@ -74,6 +75,36 @@ MUTANTS = {
     "LUT entry unweighted mean": ("W[q[i] & 7] += hd[i] * (double)w[i];", "W[q[i] & 7] += (double)w[i];"),
     "LUT entry sign dropped": ("return (x < 0.0 && mag != 0) ? (0x80 | mag) : mag;", "return mag;"),
     "LUT empty index at grid offset": ("lo + (double)k * s;", "lo + (double)(k + 1) * s;"),
+    # mistakes in the single-candidate helpers the parity checker calls
+    "refit D3 step over qmax + 1": ("const double step = (mx - mn) * (double)f / (double)qmax;",
+                                    "const double step = (mx - mn) * (double)f / (double)(qmax + 1);"),
+    "refit without the zero-saliency rule": (
+        "group_saliency(h, G, hd);\n    const double step",
+        "for (int i = 0; i < G; ++i) hd[i] = (double)h[i];\n    const double step"),
+    "symmetric refit step over Q + 1": (
+        "const double e = sym_fit(w, hd, code, G, Q, (double)f * amax / (double)Q, s_out);",
+        "const double e = sym_fit(w, hd, code, G, Q, (double)f * amax / (double)(Q + 1), s_out);"),
+    "NVFP4 helper codes keep a negative zero": ("const int neg = (w[i] < 0.0f) && m != 0;",
+                                                "const int neg = (w[i] < 0.0f);"),
+    "NVFP4 helper codes search scale": ("const double sigma = (double)f * amax_b / 6.0;",
+                                        "const double sigma = (double)f * amax_b / 4.0;"),
+    "NVFP4 helper scale fit unweighted": (
+        "s3 += hd[i] * q * (double)w[i];\n    }\n    if (amax_b == 0.0)",
+        "s3 += q * (double)w[i];\n    }\n    if (amax_b == 0.0)"),
+    "NVFP4 helper N4 rule drops the factor": ("((double)f * amax_b / 6.0) / (double)s_T",
+                                              "(amax_b / 6.0) / (double)s_T"),
+    "NVFP4 helper error drops the tensor scale": (
+        "const double alpha = (double)s_T * qo_e4m3_value(scale_bits);",
+        "const double alpha = qo_e4m3_value(scale_bits);"),
+    "LUT helper error reads the next entry": (
+        "const double d = e4m3s_value(book[q[i] & 7]) - (double)w[i];",
+        "const double d = e4m3s_value(book[(q[i] + 1) & 7]) - (double)w[i];"),
+    "LUT helper fit grid origin": (
+        "lut_entries(w, hd, n, c - (double)f * rho, 2.0 * (double)f * rho / 7.0, q, bk, book_margin);",
+        "lut_entries(w, hd, n, c + (double)f * rho, 2.0 * (double)f * rho / 7.0, q, bk, book_margin);"),
+    "LUT helper block ignores the factor": (
+        "e = lut_candidate(w, hd, n, c, rho, (double)f, q, bk, margin, book_margin);",
+        "e = lut_candidate(w, hd, n, c, rho, 1.0, q, bk, margin, book_margin);"),
     "LUT error at the grid point": ("const double d = e4m3s_value(book[q[i]]) - (double)w[i];\n        e += hd[i] * d * d;\n    }\n    return e;\n}\n\n/* Block range",
                                     "const double d = (lo + (double)q[i] * s) - (double)w[i];\n        e += hd[i] * d * d;\n    }\n    return e;\n}\n\n/* Block range"),
 }
@@ -99,6 +130,14 @@ PIN_TESTS = [
     (pins.test_lut_entries_are_the_best_e4m3_values, {}),
     (pins.test_lut_error_and_argmin, {}),
     (pins.test_lut_indices_follow_the_grid, {}),
+    (cpins.test_refit_int_is_weighted_least_squares, {}),
+    (cpins.test_refit_sym_is_least_squares_through_origin, {}),
+    (cpins.test_codes_nvfp4_enumeration_and_kept_codes, {}),
+    (cpins.test_fit_nvfp4_scale_enumerates_e4m3, {}),
+    (cpins.test_eval_nvfp4_is_the_direct_error, {}),
+    (cpins.test_lut_block_matches_app_b_candidates, {}),
+    (cpins.test_lut_fit_is_the_weighted_mean_rounded, {}),
+    (cpins.test_lut_eval_is_the_direct_error, {}),
 ]
 
 
@@ -123,7 +162,8 @@ def test_pins_catch_planted_mistake(oracle, tmp_path, name):
     for sym in ("qo_ema", "qo_adamw", "qo_recon_int", "qo_refit_int", "qo_codes_int", "qo_tensor_scale",
                 "qo_recon_nvfp4", "qo_e2m1_round", "qo_e4m3_round", "qo_e4m3_value",
                 "qo_set_threads", "qo_get_threads", "qo_recon_lut", "qo_lut_block", "qo_lut_eval", "qo_lut_fit",
-                "qo_recon_sym", "qo_codes_sym", "qo_refit_sym"):
+                "qo_recon_sym", "qo_codes_sym", "qo_refit_sym", "qo_codes_nvfp4",
+                "qo_fit_nvfp4_scale", "qo_eval_nvfp4"):
         f_real, f_mut = getattr(real, sym), getattr(lib, sym)
         f_mut.argtypes, f_mut.restype = f_real.argtypes, f_real.restype
     caught = []

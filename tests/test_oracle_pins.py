@@ -187,7 +187,7 @@ def test_fit_brute_force_grid(oracle):
         assert err.min() >= o["err"][0] * (1 - 1e-12)
 
 
-def test_uniform_saliency_is_ordinary_least_squares(oracle):
+def test_uniform_saliency_fit_is_the_polyfit_line(oracle):
     """h = 1: the fit is the ordinary least-squares line of w on q."""
     w, _ = _groups(21, 16, 128)
     h = np.ones_like(w)

@@ -194,12 +194,18 @@ def test_int_batch_matches_oracle_and_single_calls(oracle):
         _assert(rep, ema)
 
 
-def _hoistable(bits, clip):
-    """Whether both slot sets of the one candidate chunk admit a hoisted
-    code clamp: J f_max (1 + 1e-3) < (J + 1) f_min (1 - 1e-3)."""
-    f = [float(np.float32(clip[min(k, len(clip) - 1)])) for k in range(8)]
+def _set_size(bits, clip):
+    """The largest clamp-set size (4, 2 or 1 consecutive candidate slots)
+    whose sets all admit one code clamp: J f_max (1 + 1e-3) < (J + 1) f_min
+    (1 - 1e-3) on every set, J = (qmax - 1) / 2 (the library's own rule,
+    restated to know which kernel should run)."""
+    f = [float(np.float32(clip[min(k, len(clip) - 1)])) for k in range(32)]
     J = ((1 << bits) - 1) >> 1
-    return all(J * max(f[s:s + 4]) * 1.001 < (J + 1) * min(f[s:s + 4]) * 0.999 for s in (0, 4))
+    for size in (4, 2):
+        if all(J * max(f[s:s + size]) * 1.001 < (J + 1) * min(f[s:s + size]) * 0.999
+               for s in range(0, 32, size)):
+            return size
+    return 1
 
 
 NARROW8 = [1.0, 0.99, 0.98, 0.97, 0.96, 0.95, 0.94, 0.93]
@@ -221,16 +227,17 @@ def _edge_inputs(rows, cols, seed):
     return w, g, v
 
 
-@pytest.mark.parametrize("bits,clip", [(1, CLIP8), (2, CLIP8), (3, CLIP8), (3, CLIP8[:5]),
-                                       (4, NARROW8)])
+@pytest.mark.parametrize("bits,clip,size", [(1, CLIP8, 4), (2, CLIP8, 4), (3, CLIP8, 4),
+                                            (3, CLIP8[:5], 4), (4, NARROW8, 4), (4, CLIP8, 2),
+                                            (2, wl.CLIP_16, 4), (5, CLIP8, 1)])
 @pytest.mark.parametrize("G", [32, 64, 128, 256])
-def test_int_hoisted_clamp_equals_per_candidate_clamp(bits, clip, G):
-    """The batch kernel that clamps |w - c| once per set of 4 candidates gives
-    bit for bit the outputs of the kernel that clamps every candidate's code
-    (itself checked against the oracle above), on ragged shapes with
-    degenerate groups."""
+def test_int_hoisted_clamp_equals_per_candidate_clamp(bits, clip, size, G):
+    """The batch kernel that clamps |w - c| once per set of 4 (or 2)
+    candidates gives bit for bit the outputs of the kernel that clamps every
+    candidate on its own (itself checked against the oracle above), on ragged
+    shapes with degenerate groups."""
     from paper_2608_13966_gb300 import api, quasar
-    assert _hoistable(bits, clip)
+    assert _set_size(bits, clip) == size
     shapes = [(37, 3 * G), (8, 2 * G), (1, G)]
     base = [_edge_inputs(r, c, seed=900 + 10 * bits + i) for i, (r, c) in enumerate(shapes)]
     outs = {}
@@ -245,8 +252,8 @@ def test_int_hoisted_clamp_equals_per_candidate_clamp(bits, clip, G):
             torch.cuda.synchronize()
             quasar.quasar_debug_set_stats(None)
             outs[hoist] = (o, [v for _, _, v in items])
-            # the hoisted-clamp kernel ran exactly when it was allowed to
-            assert (int(stats[3]) > 0) == hoist, (hoist, stats.tolist())
+            # a kernel with sets of several candidates ran exactly when allowed
+            assert (int(stats[3]) > 0) == (hoist and size > 1), (hoist, stats.tolist())
     finally:
         quasar.quasar_debug_set_stats(None)
         quasar.quasar_debug_set_hoist(True)
