@@ -608,7 +608,7 @@ def main():
         if wlo.adamw and ss == 2:
             ss = 1
         kname = "k_recon_int<%d,%d,256,%s,false,%d> (one launch per step)" % (
-            wlo.group // 8, (len(wlo.clip) + 7) // 8, "true" if wlo.adamw else "false", ss)
+            wlo.group // 4, (len(wlo.clip) + 7) // 8, "true" if wlo.adamw else "false", ss)
     else:
         tag = ("k_recon_lut_k%d" if wlo.fmt == "lut" else "k_recon_nvfp4_k%d") % len(wlo.clip)
         kname = ("k_recon_lut<256>" if wlo.fmt == "lut" else "k_recon_nvfp4<1,256>") + \

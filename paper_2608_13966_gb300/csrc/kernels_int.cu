@@ -12,7 +12,7 @@
 
 namespace quasar {
 
-// Kernel entry for group size 8*epl: one tensor or a batch of up to
+// Kernel entry for group size 4*epl: one tensor or a batch of up to
 // kMaxBatch tensors per launch.  The AdamW-fused variant is built for batches
 // with sets of 4 or 1 candidates, the option variants (var) for batches with
 // sets of 1; nullptr where not built.
@@ -45,10 +45,10 @@ const void* QUASAR_NAME(QUASAR_NCH, QUASAR_SS)(int epl, bool batch, bool adam, b
         QUASAR_ADAM(E)                                                                        \
         if (!batch) return reinterpret_cast<const void*>(&k_recon_int<E, C, 1, false, false, S>); \
         return reinterpret_cast<const void*>(&k_recon_int<E, C, B, false, false, S>);
-    QUASAR_EPL(4)
     QUASAR_EPL(8)
     QUASAR_EPL(16)
     QUASAR_EPL(32)
+    QUASAR_EPL(64)
 #undef QUASAR_EPL
 #undef QUASAR_ADAM
 #undef QUASAR_VAR

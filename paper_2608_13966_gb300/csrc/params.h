@@ -16,6 +16,14 @@ constexpr uint32_t kIntScratchBytes = 32 * 32 * 4;
 constexpr int kGroupsPerUnit = 4;
 constexpr int kMaxClip = 32;
 
+// The asymmetric integer kernel: 4 lanes a group, 8 groups a unit, and a
+// ring of unit tiles shared by the warps of a CTA.  The candidate sums of a
+// quad of candidates are transposed through the tile's gradient region once
+// the gradient is consumed: at least 2 KB (32 lanes x 4 x 16 bytes).
+constexpr int kIntLanes = 4;
+constexpr int kIntGroups = 8;
+constexpr uint32_t kIntXposeBytes = 2048;
+
 // One tensor of an integer-code launch: its buffers, group count, and the
 // index of its first unit in the launch's sequence of units.
 struct IntTensor {

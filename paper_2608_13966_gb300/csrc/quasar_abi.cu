@@ -408,11 +408,41 @@ struct AdamHp {
     int64_t step;
 };
 
-// Stage bytes of one unit of the integer kernel: w, v, (m,) g.
+// Stage bytes of one unit of the symmetric-code kernel: w, v, g.
 uint32_t int_unit_bytes(int group_size, int g_kind, bool adam)
 {
     const int gbytes = g_kind == 2 ? 2 : (g_kind == 1 ? 4 : 0);
     return (uint32_t)(kGroupsPerUnit * group_size * ((adam ? 12 : 8) + gbytes));
+}
+
+// Shared memory of the asymmetric integer kernel's CTA ring: S slots of one
+// unit tile each (w, v, m for the fused AdamW step, then the gradient
+// region, which is also the transpose scratch and so at least
+// kIntXposeBytes), S + 1 mbarriers and S sequence words.  S is one slot a
+// warp plus `extra` slots in flight (QUASAR_STAGES, default 2).
+Launch plan_ring(int group_size, int g_kind, bool adam, int warps)
+{
+    const uint32_t gbytes = g_kind == 2 ? 2u : (g_kind == 1 ? 4u : 0u);
+    const uint32_t unit = (uint32_t)(kIntGroups * group_size);
+    const uint32_t tile = unit * (adam ? 12u : 8u) + std::max(unit * gbytes, kIntXposeBytes);
+    Launch L;
+    L.stage_bytes = (tile + 127u) & ~127u;
+    auto total = [&](int s) {
+        return (size_t)s * L.stage_bytes + (size_t)(s + 1) * 8 + (size_t)s * 4;
+    };
+    int extra = tuning().stages;
+    if (extra <= 0) {
+        // two slots in flight, one if that keeps two CTAs on an SM (each
+        // CTA's share of the SM's 228 KB, less the 1 KB the system keeps);
+        // one if two would exceed the 227 KB a CTA may have
+        constexpr size_t kTwoCtas = 113 * 1024, kOneCta = 227 * 1024;
+        extra = 2;
+        if ((total(warps + 2) > kTwoCtas && total(warps + 1) <= kTwoCtas) || total(warps + 2) > kOneCta)
+            extra = 1;
+    }
+    L.stages = warps + extra;
+    L.smem = total(L.stages);
+    return L;
 }
 
 // Parameters shared by the tensors of an integer-code call (adam: the
@@ -433,9 +463,11 @@ quasar_status int_params(quasar_dtype g_dtype, bool has_g, float beta2, int bits
     p->n_clip = n_clip;
     p->beta2 = beta2;
     p->c1 = 1.0f - beta2;
-    // each candidate sum is accumulated over at most G/16 (per packed half)
-    // + 1 + 3 (lane tree) additions; a few more roundings form N, D and E
-    p->tie_kappa = tuning().tie_scale * (float)(group_size / 16 + 8);
+    // each candidate sum is accumulated over at most G/8 (asymmetric kernel:
+    // 4 lanes a group) or G/16 (symmetric: 8 lanes) terms a packed half, plus
+    // the halves' sum and the lane tree (2 or 3 levels); the terms' own
+    // roundings and those that form N, D and E make up the rest
+    p->tie_kappa = tuning().tie_scale * (float)(group_size / (opt.symmetric ? 16 : 8) + 8);
     p->fit_ulps = tuning().fit_ulps;
     p->timeout_ns = kDefaultTimeoutNs;
     p->force_timeout_ns = (uint64_t)std::max<int64_t>(0, g_force_timeout_ns.load());
@@ -456,10 +488,6 @@ quasar_status int_params(quasar_dtype g_dtype, bool has_g, float beta2, int bits
         p->isbc2 = (float)(1.0 / std::sqrt(1.0 - std::pow((double)beta2, t)));
         p->eps = adam->eps;
     }
-    const Launch L = plan(int_unit_bytes(group_size, p->g_kind, adam != nullptr), kIntScratchBytes,
-                          adam ? kAdamWarps : kWarps);
-    p->stages = L.stages;
-    p->stage_bytes = L.stage_bytes;
     return QUASAR_OK;
 }
 
@@ -468,16 +496,22 @@ template <int MAXT>
 quasar_status int_launch(IntLaunch<MAXT>& Lp, int group_size, int n_clip, cudaStream_t stream,
                          bool adam = false, bool symmetric = false)
 {
+    // units: 8 groups for the asymmetric kernel, 4 for the symmetric one
+    const int per_unit = symmetric ? kGroupsPerUnit : kIntGroups;
     int64_t units = 0;
     for (int i = 0; i < Lp.n_t; ++i) {
         Lp.t[i].unit0 = units;
-        units += (Lp.t[i].n_groups + kGroupsPerUnit - 1) / kGroupsPerUnit;
+        units += (Lp.t[i].n_groups + per_unit - 1) / per_unit;
     }
     Lp.n_units = units;
     if (units == 0) return QUASAR_OK;
-    const int warps = adam ? kAdamWarps : kWarps;
-    const Launch L = plan(int_unit_bytes(group_size, Lp.p.g_kind, adam), kIntScratchBytes, warps);
-    const int epl = group_size / kLanesPerGroup;
+    int warps = adam ? kAdamWarps : kWarps;
+    if (const char* e = std::getenv("QUASAR_EXP_WARPS")) warps = std::max(1, std::min(8, std::atoi(e)));
+    const Launch L = symmetric ? plan(int_unit_bytes(group_size, Lp.p.g_kind, adam), kIntScratchBytes, warps)
+                               : plan_ring(group_size, Lp.p.g_kind, adam, warps);
+    Lp.p.stages = L.stages;
+    Lp.p.stage_bytes = L.stage_bytes;
+    const int epl = group_size / (symmetric ? kLanesPerGroup : kIntLanes);
     const int nch = nch_for(n_clip);
     const bool batch = MAXT > 1;
     const bool var = Lp.p.h_mode != kSalEma || Lp.p.codes_packed;

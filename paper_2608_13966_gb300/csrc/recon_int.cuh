@@ -181,18 +181,57 @@ __device__ bool coop_same_codes(const float* ws, const GroupGeom& gq, float Pa, 
     return __all_sync(0xffffffffu, same);
 }
 
+// The direct error sum h (a q + B - w)^2 of one candidate for the fit
+// (a, bc), bc the offset at q = 0 of w - cref, with (a, B) rounded to a
+// common power-of-two grid U so that a*q + B is exact and only "- w" rounds;
+// lanes combine as a float pair.  Far from zero (|centre| >= 2 range) the
+// residual is formed about an anchor A at the centre, a q + (B - A) - (w - A),
+// with w - A exact: the grid then follows the group's range rather than its
+// magnitude, and the rounded fit stays a tiny fraction of a level from the
+// given one (the error's excess is second order in that distance).
+template <int G>
+__device__ void coop_error(const float* ws, const float* hs, const GroupGeom& gq, float P,
+                           float Jp1, float cref, float a, float bc, float* err_hi, float* err_lo)
+{
+    constexpr int M = G / 32;
+    const int lane = threadIdx.x & 31;
+    const float range = -2.0f * gq.nrho;
+    const float A = fabsf(cref) >= 2.0f * range ? cref : 0.0f;
+    const float B = bc + (cref - A);  // offset at q = 0 of w - A
+    const float mr = fmaxf(fabsf(B), fabsf(fmaf(a, 2.0f * Jp1, B))) + fabsf(a);
+    int er = (int)((__float_as_uint(mr) >> 23) & 0xFF) - 126;  // mr < 2^er
+    er = max(er, -100);
+    const float U = __uint_as_float((uint32_t)(er - 23 + 127) << 23);
+    const float invU = __uint_as_float((uint32_t)(23 - er + 127) << 23);
+    const float ag = round_to_grid(a, U, invU);
+    const float Bg = round_to_grid(B, U, invU);
+    float t[M];
+#pragma unroll
+    for (int m = 0; m < M; ++m) {
+        const int e = lane + 32 * m;
+        const float h = hs[e];
+        const float w = ws[e];
+        const float q = int_code_q(centred(w, gq.nmn, gq.nrho), P, gq.ylo, gq.yhi);
+        const float ev = fmaf(ag, q, Bg) - (w - A);
+        t[m] = h * (ev * ev);
+    }
+#pragma unroll
+    for (int s = 1; s < M; s <<= 1)
+#pragma unroll
+        for (int m = 0; m + s < M; m += 2 * s) t[m] += t[m + s];
+    float eh = t[0], el = 0.0f;
+    ff_reduce32(eh, el);
+    *err_hi = eh;
+    *err_lo = el;
+}
+
 // Exact evaluation of one candidate: codes q, exact degenerate test (all
 // weighted elements on one code), two-pass centred fit, and the direct error
 // sum h (a q + B - w)^2 with (a, B) rounded to a common power-of-two grid U
 // so that a*q + B is exact and only "- w" rounds; lanes combine as a float
-// pair.  Far from zero (|centre| >= 2 range) the residual is formed about an
-// anchor A at the centre, a q + (B - A) - (w - A), with w - A exact: the grid
-// then follows the group's range rather than its magnitude, and the rounded
-// fit stays a tiny fraction of a level from the optimum (its excess error is
-// second order in that distance).  dbar is the weighted mean of w - cref.
-// Returns the fit as (a, Bz) with r = a zeta + Bz (offset at zeta = 0, i.e.
-// q = J + 1), and a condition estimate kap of the slope (see the tier-2
-// trigger in the kernel).
+// pair (coop_error).  dbar is the weighted mean of w - cref.  Returns the fit
+// as (a, Bz) with r = a zeta + Bz (offset at zeta = 0, i.e. q = J + 1), and a
+// condition estimate kap of the slope (see the tier-2 trigger in the kernel).
 template <int G>
 __device__ void coop_exact(const float* ws, const float* hs, const GroupGeom& gq, float P,
                            float Jp1, float Ss, float dbar, float step, float cref, float* err_hi,
@@ -247,35 +286,7 @@ __device__ void coop_exact(const float* ws, const float* hs, const GroupGeom& gq
         bc = dbar - a * qbar;
         kap = sqrtf(dd * ww) / fabsf(nn) + 1.0f;
     }
-    // bc is the offset at q = 0 of w - cref.  Anchor: cref far from zero, else 0.
-    const float range = -2.0f * gq.nrho;
-    const float A = fabsf(cref) >= 2.0f * range ? cref : 0.0f;
-    const float B = bc + (cref - A);  // offset at q = 0 of w - A
-    const float mr = fmaxf(fabsf(B), fabsf(fmaf(a, 2.0f * Jp1, B))) + fabsf(a);
-    int er = (int)((__float_as_uint(mr) >> 23) & 0xFF) - 126;  // mr < 2^er
-    er = max(er, -100);
-    const float U = __uint_as_float((uint32_t)(er - 23 + 127) << 23);
-    const float invU = __uint_as_float((uint32_t)(23 - er + 127) << 23);
-    const float ag = round_to_grid(a, U, invU);
-    const float Bg = round_to_grid(B, U, invU);
-    float t[M];
-#pragma unroll
-    for (int m = 0; m < M; ++m) {
-        const int e = lane + 32 * m;
-        const float h = hs[e];
-        const float w = ws[e];
-        const float q = int_code_q(centred(w, gq.nmn, gq.nrho), P, gq.ylo, gq.yhi);
-        const float ev = fmaf(ag, q, Bg) - (w - A);
-        t[m] = h * (ev * ev);
-    }
-#pragma unroll
-    for (int s = 1; s < M; s <<= 1)
-#pragma unroll
-        for (int m = 0; m + s < M; m += 2 * s) t[m] += t[m + s];
-    float eh = t[0], el = 0.0f;
-    ff_reduce32(eh, el);
-    *err_hi = eh;
-    *err_lo = el;
+    coop_error<G>(ws, hs, gq, P, Jp1, cref, a, bc, err_hi, err_lo);
     *a_out = a;
     *Bz_out = fmaf(a, Jp1, bc + cref);
     *kap_out = kap;
@@ -371,6 +382,24 @@ __device__ void coop_precise(const float* ws, const float* hs, const GroupGeom& 
 
 // ------------------------------------------------------------------ kernel
 
+// Wait until the tile of sequence number t is the one in flight into a slot
+// (its sequence word, written before the copy is issued), or until limit_ns
+// has passed; the same outcome for every lane of the warp.
+__device__ __forceinline__ bool warp_wait_seq(const volatile int* seq, int t, uint64_t limit_ns)
+{
+    bool ok = *seq == t;
+    if (!__all_sync(0xffffffffu, ok)) {
+        const uint64_t t0 = global_timer_ns();
+        for (;;) {
+#pragma unroll 1
+            for (int i = 0; i < 32 && !ok; ++i) ok = *seq == t;
+            if (ok || global_timer_ns() - t0 > limit_ns) break;
+        }
+        ok = __all_sync(0xffffffffu, ok);
+    }
+    return ok;
+}
+
 // Two CTAs per SM: 8-warp CTAs, 6-warp ones for the AdamW-fused variant.
 // VAR: the variants of the options (a saliency other than v', packed codes);
 // without it they compile out of the common kernel.
@@ -384,57 +413,62 @@ __global__ void __launch_bounds__(ADAM ? 192 : 256, 2)
     static_assert(SS == 1 || SS == 2 || SS == 4, "clamp sets of 1, 2 or 4 candidates");
     constexpr int NS = 4 / SS;  // clamp sets per quad of candidates
     const IntParams& p = Lp.p;
-    constexpr int G = EPL * kLanesPerGroup;
-    constexpr int UNIT = kGroupsPerUnit * G;
+    constexpr int G = EPL * kIntLanes;
+    constexpr int UNIT = kIntGroups * G;
     constexpr int NCHK = EPL / 4;  // 16-byte chunks per lane and group
+    // chunk i of a lane is the group's chunk i ^ (gs & SWZ): the two (or
+    // four) groups a shared-memory access phase covers then hit different
+    // banks
+    constexpr int SWZ = NCHK >= 4 ? 3 : (NCHK >= 2 ? 1 : 0);
     extern __shared__ __align__(128) unsigned char smem[];
 
     const int lane = threadIdx.x & 31;
     const int warp = threadIdx.x >> 5;
     const int nwarps = blockDim.x >> 5;
-    const int gs = lane >> 3;
-    const int sl = lane & 7;
+    const int gs = lane >> 2;
+    const int sl = lane & 3;
+    const int swz = gs & SWZ;
 
+    // the CTA's ring: S tile slots, a full barrier each (and one spare for
+    // the failure hook), and the sequence number of the tile each slot is
+    // loading or holding
     const int S = p.stages;
-    unsigned char* ring = smem + (size_t)warp * S * p.stage_bytes;
-    float* red = reinterpret_cast<float*>(smem + (size_t)nwarps * S * p.stage_bytes +
-                                          (size_t)warp * kIntScratchBytes);
-    uint64_t* bars = reinterpret_cast<uint64_t*>(smem + (size_t)nwarps * S * p.stage_bytes +
-                                                 (size_t)nwarps * kIntScratchBytes) +
-                     warp * (S + 1);
+    unsigned char* ring = smem;
+    uint64_t* bars = reinterpret_cast<uint64_t*>(smem + (size_t)S * p.stage_bytes);
+    volatile int* seq = reinterpret_cast<volatile int*>(bars + S + 1);
 
     const int gbytes = p.g_kind == 2 ? 2 : (p.g_kind == 1 ? 4 : 0);
-    // stage: w | v | m (fused AdamW only) | g
+    // stage: w | v | m (fused AdamW only) | g, then the transpose scratch
     constexpr uint32_t kVOff = UNIT * 4;
     constexpr uint32_t kMOff = UNIT * 8;
     constexpr uint32_t kGOff = UNIT * (ADAM ? 12 : 8);
 
+    // tiles: the CTA takes units blockIdx.x + t * gridDim.x, t = 0 .. nt-1,
+    // and warp w the tiles t = w, w + nwarps, ...; tile t goes to slot t % S
     const int64_t n_units = Lp.n_units;
+    const int nt = n_units > (int64_t)blockIdx.x
+                       ? (int)((n_units - 1 - (int64_t)blockIdx.x) / gridDim.x + 1)
+                       : 0;
+    auto unit_of = [&](int t) { return (int64_t)blockIdx.x + (int64_t)t * gridDim.x; };
     // the tensor of a unit: units are numbered consecutively across the
     // launch's tensors, and each warp meets them in increasing order
     auto tensor_of = [&](int64_t u, int& ti) {
         while (ti + 1 < Lp.n_t && u >= Lp.t[ti + 1].unit0) ++ti;
     };
     int ti = 0;
-    const int64_t first = (int64_t)blockIdx.x * nwarps + warp;
-    const int64_t stride = (int64_t)gridDim.x * nwarps;
 
-    if (lane == 0) {
-        for (int s = 0; s <= S; ++s) mbar_init(&bars[s], 1);
-        mbar_init_fence();
-    }
-    __syncwarp();
-
-    // (the unit issued is at or after the one being processed: its tensor
-    // index is found from ti onwards)
-    auto issue = [&](int64_t u, int s) {
+    // (the unit issued is after the one being processed, or the first ones:
+    // its tensor index is found from ti onwards)
+    auto issue = [&](int t, int s) {
+        const int64_t u = unit_of(t);
         int tj = ti;
         tensor_of(u, tj);
         const IntTensor& T = Lp.t[tj];
-        const int64_t g0 = (u - T.unit0) * kGroupsPerUnit;
-        const int64_t ng = min((int64_t)kGroupsPerUnit, T.n_groups - g0);
+        const int64_t g0 = (u - T.unit0) * kIntGroups;
+        const int64_t ng = min((int64_t)kIntGroups, T.n_groups - g0);
         const uint32_t elems = (uint32_t)(ng * G);
         unsigned char* st = ring + (size_t)s * p.stage_bytes;
+        seq[s] = t;
         mbar_arrive_expect_tx(&bars[s], elems * ((ADAM ? 12u : 8u) + (uint32_t)gbytes));
         bulk_g2s(st, T.w + g0 * G, elems * 4u, &bars[s]);
         bulk_g2s(st + kVOff, T.v + g0 * G, elems * 4u, &bars[s]);
@@ -444,23 +478,24 @@ __global__ void __launch_bounds__(ADAM ? 192 : 256, 2)
                      elems * (uint32_t)gbytes, &bars[s]);
     };
 
-    // Drain the copies still in flight from iteration `it` on, then leave.
-    // (Each of these waits is bounded too: a copy that never lands is given
-    // up on, and the warp then exits with it still in flight.)
-    auto fail = [&](int64_t it) {
+    if (threadIdx.x == 0) {
+        for (int s = 0; s <= S; ++s) mbar_init(&bars[s], 1);
+        for (int s = 0; s < S; ++s) seq[s] = -1;
+        mbar_init_fence();
+        for (int s = 0; s < S && s < nt; ++s) issue(s, s);
+    }
+    __syncthreads();
+
+    // Record the failure and wait (bounded) until every tile issued into
+    // the ring has landed, then leave.  (A copy that never lands is given up
+    // on, and the CTA then exits with it still in flight.)
+    auto fail = [&]() {
         if (lane == 0) record_timeout(p.status);
-        for (int j = 0; j < S; ++j) {
-            const int64_t u = first + (it + j) * stride;
-            if (u >= n_units) break;
-            mbar_wait_bounded(&bars[(it + j) % S], (uint32_t)(((it + j) / S) & 1), p.timeout_ns);
+        for (int s = 0; s < S; ++s) {
+            const int ts = seq[s];
+            if (ts >= 0) mbar_wait_bounded(&bars[s], (uint32_t)((ts / S) & 1), p.timeout_ns);
         }
     };
-
-    if (lane == 0)
-        for (int s = 0; s < S; ++s) {
-            const int64_t u = first + s * stride;
-            if (u < n_units) issue(u, s);
-        }
 
     if constexpr (SS > 1)  // which kernel ran, for the tuning counters
         if (p.stats && threadIdx.x == 0) atomicAdd(&p.stats[3], 1u);
@@ -468,7 +503,7 @@ __global__ void __launch_bounds__(ADAM ? 192 : 256, 2)
     if (p.force_timeout_ns && blockIdx.x == 0 && warp == 0) {
         // Failure-path hook: a barrier nothing ever arrives on.
         if (!warp_wait_bounded(&bars[S], 0, p.force_timeout_ns)) {
-            fail(0);
+            fail();
             return;
         }
     }
@@ -486,26 +521,32 @@ __global__ void __launch_bounds__(ADAM ? 192 : 256, 2)
     const float2 nlrwd2 = make_float2(-p.lr_wd, -p.lr_wd);
     const float2 nstep2 = make_float2(-p.step_size, -p.step_size);
     const float2 isbc22 = make_float2(p.isbc2, p.isbc2), eps2 = make_float2(p.eps, p.eps);
-    int s_cur = 0;
-    uint32_t parity = 0;
+    const unsigned gmask = 0xFu << (gs * kIntLanes);  // this group's lanes
 
-    for (int64_t it = 0;; ++it) {
-        const int64_t u = first + it * stride;
-        if (u >= n_units) break;
-        if (!warp_wait_bounded(&bars[s_cur], parity, p.timeout_ns)) {
-            fail(it);
+    int slot = warp;  // t % S (nwarps < S)
+    uint32_t parity = 0;  // (t / S) & 1
+    for (int t = warp; t < nt; t += nwarps) {
+        if (!warp_wait_seq(seq + slot, t, p.timeout_ns) ||
+            !warp_wait_bounded(&bars[slot], parity, p.timeout_ns)) {
+            fail();
             return;
         }
-        unsigned char* st = ring + (size_t)s_cur * p.stage_bytes;
+        const int64_t u = unit_of(t);
+        unsigned char* st = ring + (size_t)slot * p.stage_bytes;
         float* ws = reinterpret_cast<float*>(st);
         float* hs = reinterpret_cast<float*>(st + kVOff);
         const unsigned char* gsm = st + kGOff;
+        // transpose scratch (the gradient region, free once pass A is done)
+        float* red = reinterpret_cast<float*>(st + kGOff);
 
         tensor_of(u, ti);
         const IntTensor& T = Lp.t[ti];
-        const int64_t grp = (u - T.unit0) * kGroupsPerUnit + gs;
+        const int64_t grp = (u - T.unit0) * kIntGroups + gs;
         const bool valid = grp < T.n_groups;
         const int64_t gbase = grp * (int64_t)G;
+        const float* gws = ws + gs * G;  // this lane's group in the tile
+        float* ghs = hs + gs * G;
+        auto eoff = [&](int i) { return 16 * (i ^ swz) + 4 * sl; };  // chunk i of this lane
 
         // ---- pass A: saliency EMA (h kept in the tile), range, saliency mass
         // and weighted sum of w (a centre for the moments).  The fused variant
@@ -513,15 +554,17 @@ __global__ void __launch_bounds__(ADAM ? 192 : 256, 2)
         // after this pass reconstructs the updated weights.
         float mn = INFINITY, mx = -INFINITY, ss = 0.0f, sw = 0.0f;
         {
-            float* vout = T.v + gbase + sl * 4;
-            float* wout = const_cast<float*>(T.w) + gbase + sl * 4;
-            float* mout = T.m + gbase + sl * 4;
+            float* vout = T.v + gbase;
+            float* wout = const_cast<float*>(T.w) + gbase;
+            float* mout = T.m + gbase;
             auto pass_a = [&](auto gk) {
                 constexpr int GK = decltype(gk)::value;
                 float2 SS2 = make_float2(0.0f, 0.0f), SW = SS2;
-#pragma unroll
+// two chunks an iteration: the loop stays small in the instruction cache
+#pragma unroll 2
                 for (int i = 0; i < NCHK; ++i) {
-                    const int e = gs * G + i * 32 + sl * 4;
+                    const int eo = eoff(i);
+                    const int e = gs * G + eo;
                     float4 w4 = lds128(ws + e);
                     float4 h4 = lds128(hs + e);
                     if constexpr (ADAM) {
@@ -556,18 +599,18 @@ __global__ void __launch_bounds__(ADAM ? 192 : 256, 2)
                                                            __fdividef(mv[pr].y, den.y));
                             // the decrement is formed first and added once, so
                             // w' is w + t rounded a single time
-                            const float2 t = __ffma2_rn(wv[pr], nlrwd2, __fmul2_rn(nstep2, upd));
-                            wv[pr] = __fadd2_rn(wv[pr], t);
+                            const float2 t2 = __ffma2_rn(wv[pr], nlrwd2, __fmul2_rn(nstep2, upd));
+                            wv[pr] = __fadd2_rn(wv[pr], t2);
                         }
                         w4 = make_float4(wv[0].x, wv[0].y, wv[1].x, wv[1].y);
                         h4 = make_float4(hv[0].x, hv[0].y, hv[1].x, hv[1].y);
                         *reinterpret_cast<float4*>(ws + e) = w4;
                         *reinterpret_cast<float4*>(hs + e) = h4;
                         if (valid) {
-                            stg_cs(reinterpret_cast<float4*>(wout + i * 32), w4);
-                            stg_cs(reinterpret_cast<float4*>(mout + i * 32),
+                            stg_cs(reinterpret_cast<float4*>(wout + eo), w4);
+                            stg_cs(reinterpret_cast<float4*>(mout + eo),
                                    make_float4(mv[0].x, mv[0].y, mv[1].x, mv[1].y));
-                            stg_cs(reinterpret_cast<float4*>(vout + i * 32), h4);
+                            stg_cs(reinterpret_cast<float4*>(vout + eo), h4);
                         }
                     } else if constexpr (GK != 0) {
                         float2 gA, gB;
@@ -586,10 +629,10 @@ __global__ void __launch_bounds__(ADAM ? 192 : 256, 2)
                                                      __fmul2_rn(c12, __fmul2_rn(gB, gB)));
                         h4 = make_float4(hA.x, hA.y, hB.x, hB.y);
                         *reinterpret_cast<float4*>(hs + e) = h4;
-                        if (valid) stg_cs(reinterpret_cast<float4*>(vout + i * 32), h4);
+                        if (valid) stg_cs(reinterpret_cast<float4*>(vout + eo), h4);
                     }
-                    mn = fminf(fminf(fminf(mn, w4.x), fminf(w4.y, w4.z)), w4.w);
-                    mx = fmaxf(fmaxf(fmaxf(mx, w4.x), fmaxf(w4.y, w4.z)), w4.w);
+                    mn = fmin3(fmin3(mn, w4.x, w4.y), w4.z, w4.w);
+                    mx = fmax3(fmax3(mx, w4.x, w4.y), w4.z, w4.w);
                     const float2 hA = make_float2(h4.x, h4.y), hB = make_float2(h4.z, h4.w);
                     SS2 = __fadd2_rn(SS2, __fadd2_rn(hA, hB));
                     SW = __ffma2_rn(hA, make_float2(w4.x, w4.y), SW);
@@ -607,7 +650,7 @@ __global__ void __launch_bounds__(ADAM ? 192 : 256, 2)
                 float2 SS2 = make_float2(0.0f, 0.0f), SW = SS2;
 #pragma unroll 1
                 for (int i = 0; i < NCHK; ++i) {
-                    const int e = gs * G + i * 32 + sl * 4;
+                    const int e = gs * G + eoff(i);
                     const float4 w4 = lds128(ws + e);
                     float4 h4 = lds128(hs + e);
                     h4 = p.h_mode == kSalEmaSquared
@@ -624,7 +667,7 @@ __global__ void __launch_bounds__(ADAM ? 192 : 256, 2)
             }
         }
 #pragma unroll
-        for (int o = 4; o; o >>= 1) {
+        for (int o = 2; o; o >>= 1) {
             mn = fminf(mn, shx(mn, o));
             mx = fmaxf(mx, shx(mx, o));
             ss += shx(ss, o);
@@ -637,10 +680,11 @@ __global__ void __launch_bounds__(ADAM ? 192 : 256, 2)
             if (h_one)
 #pragma unroll
                 for (int i = 0; i < NCHK; ++i)
-                    *reinterpret_cast<float4*>(hs + gs * G + i * 32 + sl * 4) =
-                        make_float4(1.0f, 1.0f, 1.0f, 1.0f);
-            __syncwarp();
+                    *reinterpret_cast<float4*>(ghs + eoff(i)) = make_float4(1.0f, 1.0f, 1.0f, 1.0f);
         }
+        // the gradient region becomes the transpose scratch: every lane is
+        // past pass A, and the h rewrites above are visible to all lanes
+        __syncwarp();
         const float range = mx - mn;
         const bool flat = !(range > 0.0f);
         const float rho = 0.5f * range;
@@ -664,10 +708,11 @@ __global__ void __launch_bounds__(ADAM ? 192 : 256, 2)
         const float dmu = centred(mu, -mn, -rho);
 
         // ---- pass B + reduction + candidate errors, 8 candidates a chunk,
-        // 4 a sweep over the tile.  Codes from d = (w - mn) - rho; moments
-        // about the chunk's centre code zeta0 and, for S3, e = w - mu.
-        float Ek[NCH], dEk[NCH], T1k[NCH], T2k[NCH], T3k[NCH], Y0k[NCH];
-        bool suspk[NCH];
+        // 4 (a quad) a sweep over the tile.  Codes from d = (w - mn) - rho;
+        // moments about the chunk's centre code zeta0 and, for S3, e = w - mu.
+        // Lane sl owns candidates 8 ch + 4 qd + sl.
+        float Ek[NCH][2], dEk[NCH][2], T1k[NCH][2], T2k[NCH][2], T3k[NCH][2], Y0k[NCH];
+        bool suspk[NCH][2];
         float se = 0.0f, see = 0.0f;
 #pragma unroll
         for (int ch = 0; ch < NCH; ++ch) {
@@ -676,6 +721,7 @@ __global__ void __launch_bounds__(ADAM ? 192 : 256, 2)
             const float2 nY02 = make_float2(-y0, -y0);
             Y0k[ch] = y0;
             float2 SE = make_float2(0.0f, 0.0f), SEE = make_float2(0.0f, 0.0f);
+            float4 xq[2];
 #pragma unroll
             for (int qd = 0; qd < 2; ++qd) {
                 const int kq = ch * 8 + qd * 4;
@@ -696,9 +742,9 @@ __global__ void __launch_bounds__(ADAM ? 192 : 256, 2)
 // from the instruction cache when they run
 #pragma unroll 1
                     for (int i = 0; i < NCHK; ++i) {
-                        const int e = gs * G + i * 32 + sl * 4;
-                        const float4 w4 = lds128(ws + e);
-                        const float4 h4 = lds128(hs + e);
+                        const int e = eoff(i);
+                        const float4 w4 = lds128(gws + e);
+                        const float4 h4 = lds128(ghs + e);
 #pragma unroll
                         for (int pr = 0; pr < 2; ++pr) {
                             const float2 wv = pr ? make_float2(w4.z, w4.w) : make_float2(w4.x, w4.y);
@@ -719,71 +765,69 @@ __global__ void __launch_bounds__(ADAM ? 192 : 256, 2)
                             for (int kk = 0; kk < 4; ++kk) {
                                 const float2 y = __ffma2_rd(dc[kk / SS], P2[kk], Mg2);
                                 const float2 zc = __fadd2_rn(y, nY02);  // zeta - zeta0, exact
-                                const float2 t = __fmul2_rn(h, zc);
+                                const float2 t2 = __fmul2_rn(h, zc);
                                 A1[kk] = __ffma2_rn(h, zc, A1[kk]);
-                                A2[kk] = __ffma2_rn(t, zc, A2[kk]);
-                                A3[kk] = __ffma2_rn(t, ev, A3[kk]);
+                                A2[kk] = __ffma2_rn(t2, zc, A2[kk]);
+                                A3[kk] = __ffma2_rn(t2, ev, A3[kk]);
                             }
                         }
                     }
                 }
-                // transpose through shared memory: lane L writes row L (its sums
-                // of candidate kk in 16-byte column kk ^ (L & 7)), lane (gs, sl)
-                // sums column sl of the 8 rows of its group (a tree)
+                // transpose through the scratch: lane L writes row L (its sums
+                // of candidate kk in 16-byte column kk ^ ((L >> 1) & 3)), and
+                // lane (gs, sl) sums column sl of its group's 4 rows (each
+                // group starting at another row, so that an access phase's two
+                // groups read rows of both parities: no bank conflicts)
+                __syncwarp();
 #pragma unroll
                 for (int kk = 0; kk < 4; ++kk)
-                    *reinterpret_cast<float4*>(red + lane * 32 + (((qd * 4 + kk) ^ (lane & 7)) << 2)) =
+                    *reinterpret_cast<float4*>(red + lane * 16 + ((kk ^ ((lane >> 1) & 3)) << 2)) =
                         make_float4(A1[kk].x + A1[kk].y, A2[kk].x + A2[kk].y, A3[kk].x + A3[kk].y, 0.0f);
-            }
-            __syncwarp();
-            float4 x[8];
+                __syncwarp();
+                float4 x[4];
 #pragma unroll
-            for (int j = 0; j < 8; ++j)
-                x[j] = *reinterpret_cast<const float4*>(red + (gs * 8 + j) * 32 + ((sl ^ j) << 2));
-#pragma unroll
-            for (int s2 = 1; s2 < 8; s2 <<= 1)
-#pragma unroll
-                for (int j = 0; j + s2 < 8; j += 2 * s2) {
-                    x[j].x += x[j + s2].x;
-                    x[j].y += x[j + s2].y;
-                    x[j].z += x[j + s2].z;
+                for (int j = 0; j < 4; ++j) {
+                    const int row = gs * 4 + ((j + gs) & 3);
+                    x[j] = *reinterpret_cast<const float4*>(red + row * 16 + ((sl ^ ((row >> 1) & 3)) << 2));
                 }
-            __syncwarp();
+                xq[qd] = make_float4((x[0].x + x[1].x) + (x[2].x + x[3].x),
+                                     (x[0].y + x[1].y) + (x[2].y + x[3].y),
+                                     (x[0].z + x[1].z) + (x[2].z + x[3].z), 0.0f);
+            }
             if (ch == 0) {
                 se = SE.x + SE.y;
                 see = SEE.x + SEE.y;
 #pragma unroll
-                for (int o = 4; o; o >>= 1) {
+                for (int o = 2; o; o >>= 1) {
                     se += shx(se, o);
                     see += shx(see, o);
                 }
             }
-            // candidate k = 8 ch + sl: E = N^2/D and a bound dE on its fp32
+            // candidates 8 ch + 4 qd + sl: E = N^2/D and a bound dE on its fp32
             // error.  The sums are accumulated over tie_kappa levels at most,
             // so each is within tie_kappa ulps of the sum of its terms'
             // magnitudes: sum h zc^2 = S2, sum |h zc e| <= sqrt(S2 * sum h e^2).
             const float ebar = se * inv_ss;
-            const float T1 = x[0].x, T2 = x[0].y, T3 = x[0].z;
-            const float zbar = T1 * inv_ss;
-            const float D = T2 - T1 * zbar;
-            const float N = T3 - T1 * ebar;
-            const bool susp = !(D > 1e-3f * T2);
-            const float a = __fdividef(N, D);
-            const float E = susp ? 0.0f : N * a;
-            const float s2e = fmaxf(T2 * see, 1e-37f);
-            const float dN = ulp * (s2e * rsqrtf(s2e) * 1.001f + fabsf(T1 * ebar));
-            const float dD = ulp * (T2 + fabsf(T1 * zbar));
-            const bool real = ch * 8 + sl < p.n_clip;
 #pragma unroll
-            for (int cc = 0; cc < NCH; ++cc)
-                if (cc == ch) {
-                    Ek[cc] = real && !susp ? E : -INFINITY;
-                    dEk[cc] = 2.0f * fabsf(a) * dN + a * a * dD;
-                    suspk[cc] = real && susp;
-                    T1k[cc] = T1;
-                    T2k[cc] = T2;
-                    T3k[cc] = T3;
-                }
+            for (int qd = 0; qd < 2; ++qd) {
+                const float T1 = xq[qd].x, T2 = xq[qd].y, T3 = xq[qd].z;
+                const float zbar = T1 * inv_ss;
+                const float D = T2 - T1 * zbar;
+                const float N = T3 - T1 * ebar;
+                const bool susp = !(D > 1e-3f * T2);
+                const float a = __fdividef(N, D);
+                const float E = susp ? 0.0f : N * a;
+                const float s2e = fmaxf(T2 * see, 1e-37f);
+                const float dN = ulp * (s2e * rsqrtf(s2e) * 1.001f + fabsf(T1 * ebar));
+                const float dD = ulp * (T2 + fabsf(T1 * zbar));
+                const bool real = ch * 8 + qd * 4 + sl < p.n_clip;
+                Ek[ch][qd] = real && !susp ? E : -INFINITY;
+                dEk[ch][qd] = 2.0f * fabsf(a) * dN + a * a * dD;
+                suspk[ch][qd] = real && susp;
+                T1k[ch][qd] = T1;
+                T2k[ch][qd] = T2;
+                T3k[ch][qd] = T3;
+            }
         }
         const float ebar = se * inv_ss;
 
@@ -791,34 +835,45 @@ __global__ void __launch_bounds__(ADAM ? 192 : 256, 2)
         float Eb = -INFINITY, dEb = 0.0f;
         int kb = 0x7fff;
         if constexpr (NCH == 1) {
-            // one candidate a lane: the max of integer keys, E's bits (E >= 0
-            // orders like them) with the low 3 replaced by 7 - k; a candidate
-            // out of the running (E = -inf) has key 0.  Two candidates within
-            // 7 ulps of each other are both within the tie bound below (dE is
-            // at least 2 tie_kappa ulps of E, since sqrt(S2 sum h e^2) >= |N|,
-            // and the host's tie_kappa is at least 10), so whichever the key
-            // picks, the exact comparison settles them.
-            uint32_t key = Ek[0] >= 0.0f ? ((__float_as_uint(Ek[0]) & ~7u) | (7u - (uint32_t)sl)) : 0u;
+            // the max of integer keys, E's bits (E >= 0 orders like them) with
+            // the low 3 replaced by 7 - k; a candidate out of the running
+            // (E = -inf) has key 0.  Two candidates within 7 ulps of each other
+            // are both within the tie bound below (dE is at least 2 tie_kappa
+            // ulps of E, since sqrt(S2 sum h e^2) >= |N|, and the host's
+            // tie_kappa is at least 10), so whichever the key picks, the exact
+            // comparison settles them.
+            uint32_t key = 0;
 #pragma unroll
-            for (int o = 4; o; o >>= 1) key = max(key, __shfl_xor_sync(0xffffffffu, key, o));
+            for (int qd = 0; qd < 2; ++qd) {
+                const uint32_t k = (uint32_t)(qd * 4 + sl);
+                const uint32_t kq = Ek[0][qd] >= 0.0f ? ((__float_as_uint(Ek[0][qd]) & ~7u) | (7u - k)) : 0u;
+                key = max(key, kq);
+            }
+#pragma unroll
+            for (int o = 2; o; o >>= 1) key = max(key, __shfl_xor_sync(0xffffffffu, key, o));
             const int kk = 7 - (int)(key & 7u);
-            const float Eo = __shfl_sync(0xffffffffu, Ek[0], (gs * 8) | kk);
-            const float dEo = __shfl_sync(0xffffffffu, dEk[0], (gs * 8) | kk);
+            const int owner = (gs * 4) | (kk & 3);
+            const float Eo0 = __shfl_sync(0xffffffffu, Ek[0][0], owner);
+            const float Eo1 = __shfl_sync(0xffffffffu, Ek[0][1], owner);
+            const float dEo0 = __shfl_sync(0xffffffffu, dEk[0][0], owner);
+            const float dEo1 = __shfl_sync(0xffffffffu, dEk[0][1], owner);
             if (key != 0u) {
-                Eb = Eo;
-                dEb = dEo;
+                Eb = kk & 4 ? Eo1 : Eo0;
+                dEb = kk & 4 ? dEo1 : dEo0;
                 kb = kk;
             }
         } else {
 #pragma unroll
             for (int ch = 0; ch < NCH; ++ch)
-                if (Ek[ch] > Eb) {  // strict: keeps the lower k of this lane
-                    Eb = Ek[ch];
-                    dEb = dEk[ch];
-                    kb = ch * 8 + sl;
-                }
 #pragma unroll
-            for (int o = 4; o; o >>= 1) {
+                for (int qd = 0; qd < 2; ++qd)
+                    if (Ek[ch][qd] > Eb) {  // strict: keeps the lower k of this lane
+                        Eb = Ek[ch][qd];
+                        dEb = dEk[ch][qd];
+                        kb = ch * 8 + qd * 4 + sl;
+                    }
+#pragma unroll
+            for (int o = 2; o; o >>= 1) {
                 const float Eo = shx(Eb, o);
                 const float dEo = shx(dEb, o);
                 const int ko = __shfl_xor_sync(0xffffffffu, kb, o);
@@ -834,18 +889,20 @@ __global__ void __launch_bounds__(ADAM ? 192 : 256, 2)
         // the sums of candidate k, from its owner lane (every lane of a group
         // names the same k)
         auto sums_of = [&](int k, float& t1, float& t2, float& t3) {
-            const int owner = (gs * 8) | (k & 7);
+            const int owner = (gs * 4) | (k & 3);
 #pragma unroll
-            for (int ch = 0; ch < NCH; ++ch) {
-                const float a1 = __shfl_sync(0xffffffffu, T1k[ch], owner);
-                const float a2 = __shfl_sync(0xffffffffu, T2k[ch], owner);
-                const float a3 = __shfl_sync(0xffffffffu, T3k[ch], owner);
-                if ((k >> 3) == ch) {
-                    t1 = a1;
-                    t2 = a2;
-                    t3 = a3;
+            for (int ch = 0; ch < NCH; ++ch)
+#pragma unroll
+                for (int qd = 0; qd < 2; ++qd) {
+                    const float a1 = __shfl_sync(0xffffffffu, T1k[ch][qd], owner);
+                    const float a2 = __shfl_sync(0xffffffffu, T2k[ch][qd], owner);
+                    const float a3 = __shfl_sync(0xffffffffu, T3k[ch][qd], owner);
+                    if ((k >> 2) == ch * 2 + qd) {
+                        t1 = a1;
+                        t2 = a2;
+                        t3 = a3;
+                    }
                 }
-            }
         };
         float T1b = 0.0f, T2b = 0.0f, T3b = 0.0f;
         sums_of(kb, T1b, T2b, T3b);
@@ -856,24 +913,21 @@ __global__ void __launch_bounds__(ADAM ? 192 : 256, 2)
         // is kept, as Algorithm 1's argmin does -- but an element of tiny
         // saliency can differ without moving the sums, so twins are first
         // checked code by code (cheaply, deferred).
-        unsigned my_set = 0, my_twin = 0;
-#pragma unroll
-        for (int ch = 0; ch < NCH; ++ch) {
-            const int k = ch * 8 + sl;
-            const bool twin =
-                ch == (kb >> 3) && T1k[ch] == T1b && T2k[ch] == T2b && T3k[ch] == T3b;
-            const bool contender = k != kb && Ek[ch] > -INFINITY && Eb - Ek[ch] <= dEb + dEk[ch];
-            if (contender || suspk[ch]) my_set |= 1u << ch;
-            if (contender && twin && !suspk[ch]) my_twin |= 1u << ch;
-        }
         unsigned set = 0, twins = 0;
 #pragma unroll
-        for (int ch = 0; ch < NCH; ++ch) {
-            const unsigned bal = __ballot_sync(0xffffffffu, (my_set >> ch) & 1u);
-            set |= ((bal >> (gs * 8)) & 0xFFu) << (ch * 8);
-            const unsigned balt = __ballot_sync(0xffffffffu, (my_twin >> ch) & 1u);
-            twins |= ((balt >> (gs * 8)) & 0xFFu) << (ch * 8);
-        }
+        for (int ch = 0; ch < NCH; ++ch)
+#pragma unroll
+            for (int qd = 0; qd < 2; ++qd) {
+                const int k = ch * 8 + qd * 4 + sl;
+                const bool twin = ch == (kb >> 3) && T1k[ch][qd] == T1b && T2k[ch][qd] == T2b &&
+                                  T3k[ch][qd] == T3b;
+                const bool contender =
+                    k != kb && Ek[ch][qd] > -INFINITY && Eb - Ek[ch][qd] <= dEb + dEk[ch][qd];
+                const unsigned bal = __ballot_sync(0xffffffffu, contender || suspk[ch][qd]);
+                set |= ((bal >> (gs * 4)) & 0xFu) << (ch * 8 + qd * 4);
+                const unsigned balt = __ballot_sync(0xffffffffu, contender && twin && !suspk[ch][qd]);
+                twins |= ((balt >> (gs * 4)) & 0xFu) << (ch * 8 + qd * 4);
+            }
         if (Eb == -INFINITY) set = (p.n_clip >= 32) ? 0xFFFFFFFFu : ((1u << p.n_clip) - 1u);
         else if (set) set |= 1u << kb;
 
@@ -885,11 +939,10 @@ __global__ void __launch_bounds__(ADAM ? 192 : 256, 2)
 
         // ---- deferred exact comparisons: the whole warp takes one group at a time
         unsigned todo = __ballot_sync(0xffffffffu, valid && !flat && set != 0 && sl == 0);
-        if (todo) __syncwarp();  // h written by other lanes is read below
         while (todo) {
-            const int g = (__ffs(todo) - 1) >> 3;
+            const int g = (__ffs(todo) - 1) >> 2;
             todo &= todo - 1;
-            const int src = g * 8;
+            const int src = g * 4;
             GroupGeom ggq;
             ggq.nmn = __shfl_sync(0xffffffffu, gq.nmn, src);
             ggq.nrho = __shfl_sync(0xffffffffu, gq.nrho, src);
@@ -904,13 +957,13 @@ __global__ void __launch_bounds__(ADAM ? 192 : 256, 2)
             unsigned gset = __shfl_sync(0xffffffffu, set, src);
             const unsigned gtwins = __shfl_sync(0xffffffffu, twins, src);
             const int gkb0 = __shfl_sync(0xffffffffu, kb, src);
-            const float* gws = ws + g * G;
-            const float* ghs = hs + g * G;
+            const float* tws = ws + g * G;
+            const float* ths = hs + g * G;
             unsigned tw = gtwins;
             while (tw) {
                 const int k = __ffs(tw) - 1;
                 tw &= tw - 1;
-                if (coop_same_codes<G>(gws, ggq, gR * p.invf[k], gR * p.invf[gkb0]))
+                if (coop_same_codes<G>(tws, ggq, gR * p.invf[k], gR * p.invf[gkb0]))
                     gset &= ~(1u << k);
             }
             if (gset == (1u << gkb0)) continue;  // only the winner left
@@ -918,13 +971,60 @@ __global__ void __launch_bounds__(ADAM ? 192 : 256, 2)
             float best_h = 0.0f, best_l = 0.0f, ga = 0.0f, gB = 0.0f, gkap = 0.0f;
             int best_k = -1;
             bool gdeg = false;
+            // the quick error pass only where every candidate left shares the
+            // winner's chunk: candidates of different chunks can have equal
+            // codes (their sums, about different centres, differ), and only
+            // the two-pass fit, a function of the codes alone, then gives
+            // them bitwise-equal errors, so that the lower index is kept
+            const bool one_chunk = (gset & ~(0xFFu << ((gkb0 >> 3) * 8))) == 0u;
+            const float gebar = __shfl_sync(0xffffffffu, ebar, src);
+            const float gsee = __shfl_sync(0xffffffffu, see, src);
+            float gy0[NCH];
+#pragma unroll
+            for (int ch = 0; ch < NCH; ++ch) gy0[ch] = __shfl_sync(0xffffffffu, Y0k[ch], src);
             while (gset) {
                 const int k = __ffs(gset) - 1;
                 gset &= gset - 1;
-                float eh, el, a_k, B_k, kap_k;
-                bool deg_k;
-                coop_exact<G>(gws, ghs, ggq, gR * p.invf[k], Jp1, gss, gdbar,
-                              p.f[k] * grange / qmaxf, gcref, &eh, &el, &a_k, &B_k, &kap_k, &deg_k);
+                // the candidate's own fit from its centred sums, where its
+                // fp32 error (fit_ulps ulps times the slope's condition kap)
+                // moves the error sum by less than 1e-9 of itself (second
+                // order: (rel. fit error)^2 times explained over residual
+                // variance): then one error pass settles it; otherwise (and
+                // for nearly degenerate code variance) the two-pass fit
+                float k1 = 0.0f, k2 = 0.0f, k3 = 0.0f, y0k = gy0[0];
+                {
+                    const int owner = src | (k & 3);
+#pragma unroll
+                    for (int ch = 0; ch < NCH; ++ch)
+#pragma unroll
+                        for (int qd = 0; qd < 2; ++qd) {
+                            const float a1 = __shfl_sync(0xffffffffu, T1k[ch][qd], owner);
+                            const float a2 = __shfl_sync(0xffffffffu, T2k[ch][qd], owner);
+                            const float a3 = __shfl_sync(0xffffffffu, T3k[ch][qd], owner);
+                            if ((k >> 2) == ch * 2 + qd) {
+                                k1 = a1;
+                                k2 = a2;
+                                k3 = a3;
+                                y0k = gy0[ch];
+                            }
+                        }
+                }
+                const float Dk = k2 - k1 * (k1 / gss), Nk = k3 - k1 * gebar;
+                const float ak = Nk / Dk, Exk = Nk * ak;
+                const float kapk = sqrtf(k2 * gsee) / fabsf(Nk) + k2 / Dk;
+                const float rel = p.fit_ulps * 5.9604645e-8f * kapk;
+                const bool quick =
+                    one_chunk && Dk > 1e-3f * k2 && rel * rel * Exk < 1e-9f * (gsee - Exk);
+                float eh, el, a_k = 0.0f, B_k = 0.0f, kap_k = 0.0f;
+                bool deg_k = false;
+                if (quick) {
+                    // offset at q = 0 of w - cref: mean(w - cref) - a (mean zeta + J + 1)
+                    const float bck = gdbar - ak * ((y0k - kGridMagic) + k1 / gss + Jp1);
+                    coop_error<G>(tws, ths, ggq, gR * p.invf[k], Jp1, gcref, ak, bck, &eh, &el);
+                } else {
+                    coop_exact<G>(tws, ths, ggq, gR * p.invf[k], Jp1, gss, gdbar,
+                                  p.f[k] * grange / qmaxf, gcref, &eh, &el, &a_k, &B_k, &kap_k, &deg_k);
+                }
                 if (best_k < 0 || ff_less(eh, el, best_h, best_l)) {
                     best_h = eh;
                     best_l = el;
@@ -992,7 +1092,7 @@ __global__ void __launch_bounds__(ADAM ? 192 : 256, 2)
                 const float rmin = fminf(fabsf(b0), fabsf(fmaf(a_sel, q0, b0)));
                 prec |= est > 1e-7f + 1e-5f * rmin;
             } else {
-                for (int q = sl; q <= p.qmax; q += kLanesPerGroup) {
+                for (int q = sl; q <= p.qmax; q += kIntLanes) {
                     const float rq = fmaf(a_sel, (float)q, b0);
                     if (est > 1e-7f + 1e-5f * fabsf(rq)) {
                         const uint32_t bits = __float_as_uint(rq);
@@ -1004,16 +1104,14 @@ __global__ void __launch_bounds__(ADAM ? 192 : 256, 2)
                 }
             }
             prec = prec || est != est;  // NaN sums: take the careful path
-            // one decision per group: any lane of the segment that flagged
-            const unsigned flag = __ballot_sync(0xffffffffu, prec);
-            prec = ((flag >> (gs * kLanesPerGroup)) & 0xFFu) != 0;
+            // one decision per group: any lane of the group that flagged
+            prec = (__ballot_sync(0xffffffffu, prec) & gmask) != 0;
         }
         todo = __ballot_sync(0xffffffffu, valid && refit && prec && sl == 0);
-        if (todo) __syncwarp();
         while (todo) {
-            const int g = (__ffs(todo) - 1) >> 3;
+            const int g = (__ffs(todo) - 1) >> 2;
             todo &= todo - 1;
-            const int src = g * 8;
+            const int src = g * 4;
             GroupGeom ggq;
             ggq.nmn = __shfl_sync(0xffffffffu, gq.nmn, src);
             ggq.nrho = __shfl_sync(0xffffffffu, gq.nrho, src);
@@ -1043,13 +1141,14 @@ __global__ void __launch_bounds__(ADAM ? 192 : 256, 2)
             const float2 a2 = make_float2(a_sel, a_sel), B2 = make_float2(Bz, Bz);
             const float2 alo2 = make_float2(a_lo, a_lo), Blo2 = make_float2(Bz_lo, Bz_lo);
             const float2 Pk2 = make_float2(Pk, Pk);
-            const int64_t ebase = gbase + sl * 4;
+            const int64_t ebase = gbase;
             // general: codes, fp32 r, zero-range groups (r = w); fast: none
             auto pass_c = [&](auto general) {
                 constexpr bool GEN = decltype(general)::value;
-#pragma unroll
+#pragma unroll 2
                 for (int i = 0; i < NCHK; ++i) {
-                    const float4 w4 = lds128(ws + gs * G + i * 32 + sl * 4);
+                    const int eo = eoff(i);
+                    const float4 w4 = lds128(gws + eo);
                     float2 yv[2], zs[2];
 #pragma unroll
                     for (int pr = 0; pr < 2; ++pr) {
@@ -1064,7 +1163,7 @@ __global__ void __launch_bounds__(ADAM ? 192 : 256, 2)
 #pragma unroll
                     for (int pr = 0; pr < 2; ++pr)
                         rv[pr] = __fadd2_rn(__ffma2_rn(a2, zs[pr], B2), __ffma2_rn(alo2, zs[pr], Blo2));
-                    const int64_t eo = ebase + i * 32;
+                    const int64_t ge = ebase + eo;
                     if constexpr (GEN) {
                         if (flat) {
                             rv[0] = make_float2(w4.x, w4.y);
@@ -1082,15 +1181,15 @@ __global__ void __launch_bounds__(ADAM ? 192 : 256, 2)
                                       << (16 * pr);
                             if (flat) cw = 0;
                             if (!(VAR && p.codes_packed) && valid)
-                                stg_cs(reinterpret_cast<uint32_t*>(T.codes + eo), cw);
+                                stg_cs(reinterpret_cast<uint32_t*>(T.codes + ge), cw);
                         }
                     }
                     if (!valid) {
                     } else if (!GEN || p.r_bf16) {
-                        stg_cs(reinterpret_cast<uint2*>(static_cast<__nv_bfloat16*>(T.r) + eo),
+                        stg_cs(reinterpret_cast<uint2*>(static_cast<__nv_bfloat16*>(T.r) + ge),
                                make_uint2(pack_bf16x2(rv[0].x, rv[0].y), pack_bf16x2(rv[1].x, rv[1].y)));
                     } else {
-                        stg_cs(reinterpret_cast<float4*>(static_cast<float*>(T.r) + eo),
+                        stg_cs(reinterpret_cast<float4*>(static_cast<float*>(T.r) + ge),
                                make_float4(rv[0].x, rv[0].y, rv[1].x, rv[1].y));
                     }
                 }
@@ -1104,34 +1203,41 @@ __global__ void __launch_bounds__(ADAM ? 192 : 256, 2)
             }
             if (VAR && T.codes && p.codes_packed) {
                 // the deployment format: the group's codes as one little-endian
-                // bitstream of `bits` bits a code.  Each 32-code chunk fills
-                // `bits` words; the 8 lanes' 4-code fields (4 bits wide) are
-                // OR-ed into them in the transpose scratch.
+                // bitstream of `bits` bits a code.  Each 32-code span fills
+                // `bits` words; in two steps, each of the 4 lanes ORs a 4-code
+                // field (4 bits bits wide) into them in the scratch, and lanes
+                // sl and sl + 4 of the span's words are stored.
                 uint32_t* wsc = reinterpret_cast<uint32_t*>(red) + gs * 8;
-                const uint32_t o = (uint32_t)sl * 4u * (uint32_t)p.bits;
 // (codes recomputed from the tile, as pass C forms them: kept registers would
 // raise the pressure of the common path)
 #pragma unroll 1
-                for (int i = 0; i < NCHK; ++i) {
-                    uint32_t pk = 0;
+                for (int m = 0; m < G / 32; ++m) {
+                    __syncwarp();
+                    wsc[sl] = 0u;
+                    wsc[sl + 4] = 0u;
+                    __syncwarp();
 #pragma unroll
-                    for (int j = 0; j < 4; ++j) {
-                        const float d = centred(ws[gs * G + i * 32 + sl * 4 + j], gq.nmn, gq.nrho);
-                        const uint32_t q = flat ? 0u : (uint32_t)int_code_q(d, Pk, ylo, yhi);
-                        pk |= q << (j * p.bits);
+                    for (int j2 = 0; j2 < 2; ++j2) {
+                        const int c0 = 16 * j2 + 4 * sl;  // first code of the field
+                        uint32_t pk = 0;
+#pragma unroll
+                        for (int j = 0; j < 4; ++j) {
+                            const float d = centred(gws[32 * m + c0 + j], gq.nmn, gq.nrho);
+                            const uint32_t q = flat ? 0u : (uint32_t)int_code_q(d, Pk, ylo, yhi);
+                            pk |= q << (j * p.bits);
+                        }
+                        const uint32_t o = (uint32_t)c0 * (uint32_t)p.bits;
+                        const uint64_t f = (uint64_t)pk << (o & 31u);
+                        atomicOr(&wsc[o >> 5], (uint32_t)f);
+                        if ((uint32_t)(f >> 32)) atomicOr(&wsc[(o >> 5) + 1], (uint32_t)(f >> 32));
                     }
-                    const uint64_t f = (uint64_t)pk << (o & 31u);
-                    if (sl < p.bits) wsc[sl] = 0u;
                     __syncwarp();
-                    atomicOr(&wsc[o >> 5], (uint32_t)f);
-                    if ((uint32_t)(f >> 32)) atomicOr(&wsc[(o >> 5) + 1], (uint32_t)(f >> 32));
-                    __syncwarp();
-                    if (valid && sl < p.bits)
-                        stg_cs(reinterpret_cast<uint32_t*>(T.codes) + grp * (int64_t)(G / 32) * p.bits +
-                                   i * p.bits + sl,
-                               wsc[sl]);
-                    __syncwarp();
+                    uint32_t* dst = reinterpret_cast<uint32_t*>(T.codes) + grp * (int64_t)(G / 32) * p.bits +
+                                    m * p.bits;
+                    if (valid && sl < p.bits) stg_cs(dst + sl, wsc[sl]);
+                    if (valid && sl + 4 < p.bits) stg_cs(dst + sl + 4, wsc[sl + 4]);
                 }
+                __syncwarp();
             }
             if (valid && sl == 0) {
                 // b = Bz - a*(J + 1): the offset at code 0
@@ -1144,17 +1250,16 @@ __global__ void __launch_bounds__(ADAM ? 192 : 256, 2)
         }
 
         // release the tile: all lanes are done with it; order our generic
-        // writes to it before the async-proxy copy that refills it
+        // writes to it before the async-proxy copy that refills it with the
+        // slot's next tile
         __syncwarp();
-        if (lane == 0) {
-            const int64_t un = u + (int64_t)S * stride;
-            if (un < n_units) {
-                asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-                issue(un, s_cur);
-            }
+        if (lane == 0 && t + S < nt) {
+            asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+            issue(t + S, slot);
         }
-        if (++s_cur == S) {
-            s_cur = 0;
+        slot += nwarps;
+        if (slot >= S) {
+            slot -= S;
             parity ^= 1u;
         }
     }
