@@ -58,7 +58,7 @@ std::atomic<int> g_hoist{-1};  // -1: the environment's choice (tuning().hoist)
 // are capped where a float overflow would start to matter.
 constexpr float kTieKappaMin = 16.0f;
 constexpr float kTieScaleMin = 1.0f;
-constexpr float kFitUlpsMin = 3.0f;
+constexpr float kFitUlpsMin = 5.0f;
 
 struct Tuning {
     int stages = 0;            // 0: chosen from the shared-memory budget

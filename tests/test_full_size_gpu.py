@@ -1,9 +1,11 @@
 """Parity at full size: every tensor of the 32-layer Llama-3.1-8B-shaped
 model (6.98e9 weights resident on the device), reconstructed through the
 C-ABI calls and launch configuration that ``bench.py`` times, checked against
-the oracle on a seeded sample of groups (blocks) from every tensor, together
-with the in-place EMA update of those groups (and, for the fused AdamW
-workload, the in-place AdamW step of w and m)."""
+the oracle on every group (block) of layer 0 and on a seeded 1% sample of the
+groups of every other tensor, together with the in-place EMA update of those
+groups (and, for the fused AdamW workload, the in-place AdamW step of w and
+m).  The number of groups the checker took as exempt (an element within 1e-6
+of a code boundary, or a candidate tie within 1e-6) is printed."""
 import numpy as np
 import pytest
 import torch
@@ -12,15 +14,21 @@ import bench
 from paper_2608_13966_gb300 import workloads as WL
 from tests import checker
 
-SAMPLES_PER_TENSOR = 48
+SAMPLE_FRACTION = 0.01   # of the groups of every tensor outside layer 0
+MIN_SAMPLES = 48
 
 
 def _sample(model, unit, seed):
+    """Per tensor: all its groups (blocks) in layer 0, else a seeded 1%."""
     rng = np.random.default_rng(seed)
     out = []
     for d in model.tensors:
         n_units = d["spec"].numel // unit
-        idx = np.sort(rng.choice(n_units, size=min(SAMPLES_PER_TENSOR, n_units), replace=False))
+        if d["spec"].layer == 0:
+            idx = np.arange(n_units)
+        else:
+            k = min(n_units, max(MIN_SAMPLES, int(n_units * SAMPLE_FRACTION)))
+            idx = np.sort(rng.choice(n_units, size=k, replace=False))
         sel = torch.as_tensor(idx, device="cuda")
         m = d["m"].view(-1, unit)[sel].cpu() if "m" in d else None
         out.append((sel, d["w"].view(-1, unit)[sel].cpu(), d["g"].view(-1, unit)[sel].float().cpu(),
@@ -42,6 +50,7 @@ def test_full_model_sampled(oracle, name):
     torch.cuda.synchronize()
 
     bad = []
+    n_checked = n_exempt = 0
     f32 = lambda x: float(np.float32(x))
     for d, (sel, w_s, g_s, v_s, m_s) in zip(model.tensors, samples):
         w = w_s.numpy().ravel()
@@ -73,10 +82,13 @@ def test_full_model_sampled(oracle, name):
                    "tensor_scale": float(d["ts"].cpu()[0]), "codes": None,
                    "idx": d["idx"][sel].cpu().numpy()}
             rep = checker.check_nvfp4(oracle, w, h, list(wl.clip), s_T, O, gpu, True)
+        n_checked += rep["units"]
+        n_exempt += rep["exempt"]
         if not (rep["ok"] and ema["ok"]):
             bad.append((d["spec"].name, rep, ema))
     del model
     torch.cuda.empty_cache()
+    print(f"{name}: {n_checked} groups checked, {n_exempt} exempt")
     assert not bad, bad[:3]
 
 
