@@ -20,6 +20,7 @@ counts.
 from __future__ import annotations
 
 import argparse
+import dataclasses
 import hashlib
 import json
 import os
@@ -79,21 +80,31 @@ def max_over_ranks(x, world):
     return float(t.item())
 
 
-def bytes_per_step(wlo, elements):
-    """Algorithmic HBM bytes of one step: read w (4) + g (2) + v (4), write
-    v (4) + r (2) per weight; per group a, b (fp32) and the kept index (u8)
-    for integer codes; per 16-block the E4M3 scale and index for NVFP4, plus
-    the tensor-absmax pre-pass (one more read of w).  The fused AdamW step
-    also reads m and writes w' and m' (12 more bytes a weight)."""
+DTYPE_NAME = {torch.bfloat16: "bf16", torch.float32: "f32"}
+
+
+def bytes_per_step(wlo, elements, amax_supplied=False):
+    """Algorithmic HBM bytes of one step: read w (4) + g (2 bf16, 4 fp32) +
+    v (4), write v (4) + r (2 bf16, 4 fp32) and the codes (1, where the
+    workload writes them) per weight; per group a, b (fp32) and the kept
+    index (u8) for integer codes; per 16-block the E4M3 scale and index for
+    NVFP4, plus the tensor-absmax pre-pass (one more read of w) unless the
+    caller supplies the amax; per 512-block 8 table bytes and the index for
+    the lookup table.  The fused AdamW step also reads m and writes w' and m'
+    (12 more bytes a weight)."""
+    gb = 2 if wlo.g_dtype == torch.bfloat16 else 4
+    rb = 2 if wlo.r_dtype == torch.bfloat16 else 4
+    cb = 1 if wlo.with_codes else 0
+    core = 4 + gb + 4 + 4 + rb + cb
     if wlo.fmt == "int" and wlo.adamw:
-        return elements * 28 + (elements // wlo.group) * 9
+        return elements * (core + 12) + (elements // wlo.group) * 9
     if wlo.fmt == "nvfp4" and wlo.adamw:  # AdamW + absmax pass, then w', v' -> r
-        return elements * 26 + elements * 10 + (elements // 16) * 2
-    if wlo.fmt == "lut":  # per 512-block: 8 table bytes and the kept index
-        return elements * 16 + (elements // 512) * 9
+        return elements * (12 + gb + 12) + elements * (8 + rb + cb) + (elements // 16) * 2
+    if wlo.fmt == "lut":
+        return elements * core + (elements // 512) * 9
     if wlo.fmt == "int":
-        return elements * 16 + (elements // wlo.group) * 9
-    return elements * 16 + (elements // 16) * 2 + elements * 4
+        return elements * core + (elements // wlo.group) * 9
+    return elements * core + (elements // 16) * 2 + (0 if amax_supplied else elements * 4)
 
 
 class Model:
@@ -108,7 +119,9 @@ class Model:
         for spec in wlo.tensors:
             d = WL.make_tensor(wlo, spec, device=device, seed=shard)
             n = spec.numel
-            d["r"] = torch.empty((spec.rows, spec.cols), dtype=torch.bfloat16, device=device)
+            d["r"] = torch.empty((spec.rows, spec.cols), dtype=wlo.r_dtype, device=device)
+            if wlo.with_codes:
+                d["codes"] = torch.empty(n, dtype=torch.uint8, device=device)
             gsz = min(wlo.group, 128) if wlo.fmt == "int" else 128
             d["a"] = torch.empty(n // gsz, dtype=torch.float32, device=device)
             d["b"] = torch.empty(n // gsz, dtype=torch.float32, device=device)
@@ -123,11 +136,18 @@ class Model:
 class Step:
     """Pre-marshalled C-ABI calls of one step for one format."""
 
-    def __init__(self, model, wlo, stream):
+    def __init__(self, model, wlo, stream, amax_supplied=False):
+        """amax_supplied (NVFP4): every tensor's absmax is handed to the call
+        (taken once here, outside any timing), so the absmax pass is skipped."""
         import ctypes
         self.lib = Q.load()
         self.wlo = wlo
         self.stream = stream.cuda_stream
+        GD = Q.BF16 if wlo.g_dtype == torch.bfloat16 else Q.F32
+        RD = Q.BF16 if wlo.r_dtype == torch.bfloat16 else Q.F32
+        if amax_supplied:
+            for d in model.tensors:
+                d["amax"] = d["w"].abs().max().reshape(1).float()
         self.clip = (ctypes.c_float * len(wlo.clip))(*wlo.clip)
         self.calls = []
         if wlo.adamw and wlo.fmt == "nvfp4":
@@ -139,13 +159,13 @@ class Step:
                                              d["w"].device)
             hp = wlo.adamw
             self.descs = Q.adamw_nvfp4_tensor_array([
-                {"w": d["w"], "g": d["g"], "m": d["m"], "v": d["v"], "r": d["r"], "codes": None,
+                {"w": d["w"], "g": d["g"], "m": d["m"], "v": d["v"], "r": d["r"], "codes": d.get("codes"),
                  "block_scale": d["scale"], "tensor_scale": d["ts"], "cand_idx": d["idx"],
                  "rows": d["spec"].rows, "cols": d["spec"].cols}
                 for d in model.tensors])
-            args = (ctypes.cast(self.descs, ctypes.c_void_p), len(self.descs), Q.BF16, hp["lr"],
+            args = (ctypes.cast(self.descs, ctypes.c_void_p), len(self.descs), GD, hp["lr"],
                     hp["beta1"], wlo.beta2, hp["eps"], hp["weight_decay"], hp["step"], self.clip,
-                    len(wlo.clip), Q.BF16, None, self.stream)
+                    len(wlo.clip), RD, None, self.stream)
             self.calls.append((self.lib.quasar_adamw_recon_nvfp4_batch, args, model.elements))
         elif wlo.adamw:
             # AdamW step + reconstruction of every tensor in one launch
@@ -158,13 +178,13 @@ class Step:
                                              d["w"].device)
             hp = wlo.adamw
             self.descs = Q.adamw_tensor_array([
-                {"w": d["w"], "g": d["g"], "m": d["m"], "v": d["v"], "r": d["r"], "codes": None,
+                {"w": d["w"], "g": d["g"], "m": d["m"], "v": d["v"], "r": d["r"], "codes": d.get("codes"),
                  "a": d["a"], "b": d["b"], "cand_idx": d["idx"], "rows": d["spec"].rows,
                  "cols": d["spec"].cols}
                 for d in model.tensors])
-            args = (ctypes.cast(self.descs, ctypes.c_void_p), len(self.descs), Q.BF16, hp["lr"],
+            args = (ctypes.cast(self.descs, ctypes.c_void_p), len(self.descs), GD, hp["lr"],
                     hp["beta1"], wlo.beta2, hp["eps"], hp["weight_decay"], hp["step"], wlo.bits,
-                    wlo.group, self.clip, len(wlo.clip), Q.BF16, None, self.stream)
+                    wlo.group, self.clip, len(wlo.clip), RD, None, self.stream)
             self.calls.append((self.lib.quasar_adamw_recon_int_batch, args, model.elements))
         elif wlo.fmt == "lut":
             # every tensor in one launch (quasar_recon_lut_batch)
@@ -173,43 +193,44 @@ class Step:
                     d["book"] = torch.empty((d["spec"].numel // 512, 8), dtype=torch.uint8,
                                             device=d["w"].device)
             self.descs = Q.lut_tensor_array([
-                {"w": d["w"], "g": d["g"], "v": d["v"], "r": d["r"], "codes": None, "book": d["book"],
+                {"w": d["w"], "g": d["g"], "v": d["v"], "r": d["r"], "codes": d.get("codes"), "book": d["book"],
                  "cand_idx": d["idx"], "rows": d["spec"].rows, "cols": d["spec"].cols}
                 for d in model.tensors])
-            args = (ctypes.cast(self.descs, ctypes.c_void_p), len(self.descs), Q.BF16, wlo.beta2,
-                    self.clip, len(wlo.clip), Q.BF16, None, self.stream)
+            args = (ctypes.cast(self.descs, ctypes.c_void_p), len(self.descs), GD, wlo.beta2,
+                    self.clip, len(wlo.clip), RD, None, self.stream)
             self.calls.append((self.lib.quasar_recon_lut_batch, args, model.elements))
         elif wlo.fmt == "int":
             # every tensor of the model in one launch (quasar_recon_int_batch)
             self.descs = Q.int_tensor_array([
-                {"w": d["w"], "g": d["g"], "v": d["v"], "r": d["r"], "codes": None, "a": d["a"],
-                 "b": d["b"], "cand_idx": d["idx"], "rows": d["spec"].rows, "cols": d["spec"].cols}
+                {"w": d["w"], "g": d["g"], "v": d["v"], "r": d["r"], "codes": d.get("codes"),
+                 "a": d["a"], "b": d["b"], "cand_idx": d["idx"], "rows": d["spec"].rows,
+                 "cols": d["spec"].cols}
                 for d in model.tensors])
             if wlo.symmetric:
                 self.opt = Q.options(symmetric=True)
-                args = (ctypes.cast(self.descs, ctypes.c_void_p), len(self.descs), Q.BF16,
-                        wlo.beta2, wlo.bits, wlo.group, self.clip, len(wlo.clip), Q.BF16,
+                args = (ctypes.cast(self.descs, ctypes.c_void_p), len(self.descs), GD,
+                        wlo.beta2, wlo.bits, wlo.group, self.clip, len(wlo.clip), RD,
                         ctypes.cast(ctypes.pointer(self.opt), ctypes.c_void_p), self.stream)
                 self.calls.append((self.lib.quasar_recon_int_batch_ex, args, model.elements))
             else:
-                args = (ctypes.cast(self.descs, ctypes.c_void_p), len(self.descs), Q.BF16,
-                        wlo.beta2, wlo.bits, wlo.group, self.clip, len(wlo.clip), Q.BF16,
+                args = (ctypes.cast(self.descs, ctypes.c_void_p), len(self.descs), GD,
+                        wlo.beta2, wlo.bits, wlo.group, self.clip, len(wlo.clip), RD,
                         self.stream)
                 self.calls.append((self.lib.quasar_recon_int_batch, args, model.elements))
         else:
             # every tensor in one call (quasar_recon_nvfp4_batch): absmax of
             # every tensor, their scales, one reconstruction launch
             self.descs = Q.nvfp4_tensor_array([
-                {"w": d["w"], "g": d["g"], "v": d["v"], "tensor_amax": None, "r": d["r"],
-                 "codes": None, "block_scale": d["scale"], "tensor_scale": d["ts"],
+                {"w": d["w"], "g": d["g"], "v": d["v"], "tensor_amax": d.get("amax"), "r": d["r"],
+                 "codes": d.get("codes"), "block_scale": d["scale"], "tensor_scale": d["ts"],
                  "cand_idx": d["idx"], "rows": d["spec"].rows, "cols": d["spec"].cols}
                 for d in model.tensors])
-            args = (ctypes.cast(self.descs, ctypes.c_void_p), len(self.descs), Q.BF16, wlo.beta2,
-                    self.clip, len(wlo.clip), Q.BF16, self.stream)
+            args = (ctypes.cast(self.descs, ctypes.c_void_p), len(self.descs), GD, wlo.beta2,
+                    self.clip, len(wlo.clip), RD, self.stream)
             self.calls.append((self.lib.quasar_recon_nvfp4_batch, args, model.elements))
         # INT: one launch; NVFP4: absmax, scale and reconstruction launches
         # (plus one small memset of the scale slot per tensor)
-        self.launches_per_call = 3 if wlo.fmt == "nvfp4" else 1
+        self.launches_per_call = (2 if amax_supplied else 3) if wlo.fmt == "nvfp4" else 1
 
     def run(self, events=None):
         for i, (fn, args, _) in enumerate(self.calls):
@@ -332,10 +353,11 @@ def kernel_source_hash():
 
 
 def profiled_traffic(kernel_tag):
-    """DRAM bytes per weight (dram__bytes_read.sum + dram__bytes_write.sum of
-    one ncu capture, divided by the weights that launch processed) from the
-    committed summary, if it was taken on the current kernel sources; else
-    None."""
+    """From the committed summary of one ncu capture, if it was taken on the
+    current kernel sources (else None): DRAM bytes per weight
+    (dram__bytes_read.sum + dram__bytes_write.sum over the weights that launch
+    processed) and, where recorded, the issue-slot and FMA-pipe utilisation
+    (smsp__issue_active and sm__pipe_fma_cycles_active, % of peak)."""
     path = os.path.join(ROOT, "profiles", "traffic.txt")
     if not os.path.exists(path):
         return None
@@ -344,7 +366,11 @@ def profiled_traffic(kernel_tag):
         for line in f:
             parts = line.split()
             if len(parts) >= 3 and parts[0] == kernel_tag and parts[1] == want:
-                return float(parts[2])
+                out = {"bytes_per_weight": float(parts[2])}
+                if len(parts) >= 5:
+                    out["issue_active_pct"] = float(parts[3])
+                    out["fma_pipe_pct"] = float(parts[4])
+                return out
     return None
 
 
@@ -521,12 +547,89 @@ def reference_arm(args, world, rank):
             "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
             "ms_per_step": n / value * 1e3, "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-            "config": {"workload": wlo.notes, "elements": n},
+            "config": {"workload": wlo.notes, "elements": n,
+                       "timing": "sampled and extrapolated: each step times the oracle on a "
+                                 "bounded sample of every tensor shape of layer 0 (%s); "
+                                 "ms_per_step is the whole workload at that rate" % desc},
             "cpu_baseline": {"value": value, "unit": "weights/s", "cores": cores, "kind": "oracle",
                              "sample": desc},
             "e2e": {"value": value, "unit": "weights/s", "h2d_bytes_per_step": 0,
                     "d2h_bytes_per_step": 0}}
     print(json.dumps(line), flush=True)
+
+
+# What limits each kernel (from its ncu profiles): the integer kernel is bound
+# by instruction issue -- the candidate loop by the FP32 (FMA) pipe, the
+# per-group selection, fit and output work by dependent latency -- with DRAM
+# well short of its peak; the HBM roofline above is the target's measure.
+LIMITER = {"int": "instruction issue: FMA pipe in the candidate loop, dependent latency in the "
+                  "per-group work; DRAM below its peak (profiles/)",
+           "nvfp4": "instruction issue (E2M1/E4M3 conversions and direct error sums)",
+           "lut": "instruction issue (per-index table sums)"}
+
+
+def alu_roofline(wlo, weights, launch_ms, clk):
+    """The FP32-pipe view of an integer launch: algorithmic FP32 operations
+    (8 per weight and candidate -- code, its clamp, three moment products and
+    their sums -- plus 25 per weight for the EMA, the range, the fixed sums,
+    the output code and r; an FMA counts once) over the launch time, against
+    the SMs' FP32 lanes (128 an SM) at the median SM clock under load."""
+    if wlo.fmt != "int" or launch_ms <= 0:
+        return None
+    props = torch.cuda.get_device_properties(torch.cuda.current_device())
+    mhz = (clk or {}).get("sm_mhz") or 2070.0
+    peak = props.multi_processor_count * 128 * mhz * 1e6 / 1e12
+    ops = 8 * len(wlo.clip) + 25
+    achieved = ops * weights / (launch_ms / 1e3) / 1e12
+    return {"achieved": achieved, "peak": peak, "unit": "T FP32 ops/s", "frac": achieved / peak,
+            "ops_per_weight": ops}
+
+
+# The paper-shaped configurations other than the 32-layer step, each timed
+# on its own: one 256x1024 fp32 matrix (INT4; launch-bound, reported in us,
+# L2 flushed between calls), one Llama-3.1-8B-shaped layer (INT3), one
+# Qwen3-8B-shaped layer (INT2 group 64, 16 candidates), one Llama layer
+# (NVFP4).  Codes are written, as these configurations specify.
+CONFIGS = (("config1_single_int4", "single_int4"), ("config2_llama_layer_int3", "llama_layer_int3"),
+           ("config3_qwen_layer_int2", "qwen_layer_int2"), ("config4_llama_layer_nvfp4", "llama_layer_nvfp4"))
+
+
+def config_entries(device, stream, hbm_peak, reps=20):
+    out = {}
+    flush = torch.empty(256 << 20, dtype=torch.uint8, device=device)  # twice the L2
+    for key, name in CONFIGS:
+        wlo = WL.workload(name)
+        model = Model(wlo, device)
+        st = Step(model, wlo, stream)
+        small = model.elements * 10 < (1 << 28)
+        times = []
+        with torch.cuda.stream(stream):
+            for i in range(3 + reps):
+                if small:
+                    flush.zero_()
+                e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                e0.record()
+                st.run()
+                e1.record()
+                torch.cuda.synchronize()
+                if i >= 3:
+                    times.append(e0.elapsed_time(e1))
+        status = Q.quasar_get_device_status(None)
+        if status != Q.QuasarStatus.OK:
+            raise Q.QuasarError(status)
+        ms = statistics.median(times)
+        b = bytes_per_step(wlo, model.elements)
+        out[key] = {"workload": wlo.notes, "elements": model.elements, "ms_per_call": ms,
+                    "us_per_call": ms * 1e3, "weights_per_s": model.elements / (ms / 1e3),
+                    "hbm_gbs": b / (ms / 1e3) / 1e9, "frac_of_8tbs": b / (ms / 1e3) / 1e9 / NOMINAL_HBM_GBS,
+                    "frac_of_measured": b / (ms / 1e3) / 1e9 / hbm_peak,
+                    "bytes_per_weight": b / model.elements, "calls": reps,
+                    "l2": "flushed between calls" if small else "inputs larger than L2",
+                    "launch_bound": small}
+        del st, model
+        torch.cuda.empty_cache()
+    del flush
+    return out
 
 
 def main():
@@ -536,8 +639,11 @@ def main():
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--workload", default="llama_int3")
-    ap.add_argument("--sweep", default="llama_int2,llama_int4,llama_nvfp4,llama_int3_adamw,"
-                                       "llama_nvfp4_adamw,llama_lut,llama_int4_sym")
+    ap.add_argument("--sweep", default="llama_int2,llama_int4,llama_nvfp4,llama_nvfp4_amax,"
+                                       "llama_int3_adamw,llama_nvfp4_adamw,llama_lut,llama_int4_sym")
+    ap.add_argument("--configs", type=int, default=1, help="time the per-config entries (0: skip)")
+    ap.add_argument("--layers", type=int, default=0,
+                    help="keep only the first N layers of the workload (0: all)")
     ap.add_argument("--sweep-steps", type=int, default=10)
     ap.add_argument("--e2e-steps", type=int, default=2)
     ap.add_argument("--e2e-slots", type=int, default=2)
@@ -554,6 +660,9 @@ def main():
     stream = torch.cuda.Stream()
     hbm_peak, peak_kind = peaks()
     wlo = WL.workload(args.workload)
+    if args.layers > 0:
+        # the first N layers of the workload (small cases for the profiler)
+        wlo = dataclasses.replace(wlo, tensors=tuple(t for t in wlo.tensors if t.layer < args.layers))
     model = Model(wlo, device, shard=rank)
     torch.cuda.synchronize()
     n_el = model.elements
@@ -573,12 +682,15 @@ def main():
 
     sweep = {}
     for name in [s for s in args.sweep.split(",") if s]:
-        sw = WL.workload(name)
-        st = Step(model, sw, stream)
+        # llama_nvfp4_amax: the NVFP4 step with every tensor's absmax supplied
+        # (no absmax pass: 16.125 bytes a weight instead of 20.125)
+        amax_supplied = name == "llama_nvfp4_amax"
+        sw = WL.workload("llama_nvfp4" if amax_supplied else name)
+        st = Step(model, sw, stream, amax_supplied=amax_supplied)
         with torch.cuda.stream(stream):
             t_ms, k_ms = timed_steps(st, len(st.calls), args.sweep_steps, 2, world)
         t_ms = max_over_ranks(t_ms, world)
-        b = bytes_per_step(sw, n_el)
+        b = bytes_per_step(sw, n_el, amax_supplied)
         sweep[name] = {"ms_per_step": t_ms / args.sweep_steps,
                        "weights_per_s": world * n_el / (t_ms / args.sweep_steps / 1e3),
                        "hbm_gbs": b / (t_ms / args.sweep_steps / 1e3) / 1e9,
@@ -587,8 +699,13 @@ def main():
                        "bytes_per_weight": b / n_el}
 
     e2e = None
-    if args.e2e_steps > 0 and rank == 0:
+    configs = None
+    if args.e2e_steps > 0 and rank == 0 or args.configs:
         del model
+        torch.cuda.empty_cache()
+    if args.configs and rank == 0:
+        configs = config_entries(device, stream, hbm_peak)
+    if args.e2e_steps > 0 and rank == 0:
         torch.cuda.empty_cache()
         e2e = e2e_rate(wlo, args.e2e_steps, device, stream, args.e2e_slots)
         e2e["value"] *= world
@@ -613,8 +730,8 @@ def main():
         tag = ("k_recon_lut_k%d" if wlo.fmt == "lut" else "k_recon_nvfp4_k%d") % len(wlo.clip)
         kname = ("k_recon_lut<256>" if wlo.fmt == "lut" else "k_recon_nvfp4<1,256>") + \
             " (one launch per step)"
-    tpw = profiled_traffic(tag)
-    traffic = None if tpw is None else tpw * n_el / len(step.calls)
+    prof = profiled_traffic(tag)
+    traffic = None if prof is None else prof["bytes_per_weight"] * n_el / len(step.calls)
     line = {
         "metric": METRIC, "value": value, "unit": "weights/s", "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_per_step,
@@ -622,7 +739,8 @@ def main():
         "data": "synthetic",
         "config": {"workload": wlo.notes, "elements": n_el, "tensors": len(wlo.tensors),
                    "bits": wlo.bits, "group": wlo.group, "clip_candidates": len(wlo.clip),
-                   "g_dtype": "bf16", "r_dtype": "bf16", "codes": "not written",
+                   "g_dtype": DTYPE_NAME[wlo.g_dtype], "r_dtype": DTYPE_NAME[wlo.r_dtype],
+                   "codes": "written" if wlo.with_codes else "not written",
                    "l2": "inputs larger than L2 (%.0f GB read per step)" % (n_el * 10 / 1e9),
                    "parallelism": "replicas" if world > 1 else "single GPU"},
         "hbm_gbs": hbm_gbs, "frac_of_8tbs": hbm_gbs / NOMINAL_HBM_GBS,
@@ -634,10 +752,17 @@ def main():
                      "bytes_per_weight": step_bytes / n_el,
                      "launch_bytes": step_bytes / len(step.calls),
                      "launch_ms": kernel_ms / args.steps / len(step.calls),
-                     "traffic_tag": tag},
+                     "traffic_tag": tag,
+                     "limiter": LIMITER.get(wlo.fmt),
+                     "ncu_pipes": None if prof is None or "fma_pipe_pct" not in prof else
+                     {"issue_active": prof["issue_active_pct"] / 100,
+                      "fma_pipe": prof["fma_pipe_pct"] / 100,
+                      "source": "profiles/traffic.txt (one ncu capture of one layer)"},
+                     "alu": alu_roofline(wlo, n_el / len(step.calls),
+                                         kernel_ms / args.steps / len(step.calls), clk)},
         "cpu_baseline": cpu, "e2e": e2e,
         "gpu_launches": len(step.calls) * step.launches_per_call * args.steps,
-        "clocks": clk, "sweep": sweep,
+        "clocks": clk, "sweep": sweep, "configs": configs,
     }
     print(json.dumps(line), flush=True)
 

@@ -431,14 +431,17 @@ void quasar_debug_force_timeout(int64_t nanoseconds);
 
 /*
  * quasar_debug_set_stats -- tuning hook.  While device_counters (a device
- * array of at least 4 unsigned ints owned by the caller) is set, the
+ * array of at least 8 unsigned ints owned by the caller) is set, the
  * reconstruction kernels atomically count [0] the groups/blocks whose
  * candidates were re-evaluated exactly because of a near tie, [1] the
  * integer groups whose kept fit was recomputed in compensated (float-float)
- * arithmetic, [2] the integer groups whose kept fit was recomputed about
- * centred codes and weights and [3] the thread blocks of the integer kernel
- * with the hoisted code clamp (see quasar_debug_set_hoist).  NULL turns
- * counting off.  Process-wide; never needed in normal use.
+ * arithmetic, [2] the integer groups with near-tie contenders or
+ * equal-sum candidates, [3] the thread blocks of the integer kernel whose
+ * code-clamp sets hold more than one candidate (see quasar_debug_set_hoist),
+ * [4] the candidates whose error was recomputed from a two-pass fit, [5] those
+ * whose error was recomputed from their own moment sums and [6] the
+ * equal-sum candidates checked code by code.  NULL turns counting off.
+ * Process-wide; never needed in normal use.
  */
 void quasar_debug_set_stats(unsigned int* device_counters);
 

@@ -66,7 +66,9 @@ struct IntParams {
     uint64_t force_timeout_ns;
     unsigned int* status;  // per-device status word
     unsigned int* stats;  // optional: [0] exact re-evaluations, [1] compensated fits,
-                          // [3] CTAs of kernels whose clamp sets hold more than one candidate
+                          // [2] groups with contenders or twins, [3] CTAs of kernels whose
+                          // clamp sets hold more than one candidate, [4] two-pass fits,
+                          // [5] one-pass error sums, [6] twin code checks
     float f[kMaxClip];     // padded with the last factor
     float invf[kMaxClip];  // fl32(1/f)
     // code clamps: every candidate slot holds tau / qmax of its clamp set,
@@ -74,6 +76,10 @@ struct IntParams {
     // set_size consecutive slots; see the integer kernel)
     float cap[kMaxClip];
     int set_size;
+    // 1/f is non-decreasing in k over the real candidates (the factors come
+    // in decreasing order, as the paper's grids do): codes then move
+    // monotonically with k, element by element
+    int monotone;
     // centre of each 8-candidate chunk's moments: the mean of 1/f over the
     // chunk's factors
     float invfc[kMaxClip / 8];

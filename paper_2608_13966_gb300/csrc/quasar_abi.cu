@@ -58,7 +58,7 @@ std::atomic<int> g_hoist{-1};  // -1: the environment's choice (tuning().hoist)
 // are capped where a float overflow would start to matter.
 constexpr float kTieKappaMin = 16.0f;
 constexpr float kTieScaleMin = 1.0f;
-constexpr float kFitUlpsMin = 5.0f;
+constexpr float kFitUlpsMin = 8.0f;
 
 struct Tuning {
     int stages = 0;            // 0: chosen from the shared-memory budget
@@ -474,6 +474,8 @@ quasar_status int_params(quasar_dtype g_dtype, bool has_g, float beta2, int bits
     p->stats = g_stats.load();
     fill_clip(clip, n_clip, p->f, p->invf);
     fill_caps(p, 4);
+    p->monotone = 1;
+    for (int k = 1; k < n_clip; ++k) p->monotone &= p->invf[k] >= p->invf[k - 1] ? 1 : 0;
     quasar_status st;
     if ((st = status_ptr(&p->status)) != QUASAR_OK) return st;
     if (adam) {
@@ -505,8 +507,7 @@ quasar_status int_launch(IntLaunch<MAXT>& Lp, int group_size, int n_clip, cudaSt
     }
     Lp.n_units = units;
     if (units == 0) return QUASAR_OK;
-    int warps = adam ? kAdamWarps : kWarps;
-    if (const char* e = std::getenv("QUASAR_EXP_WARPS")) warps = std::max(1, std::min(8, std::atoi(e)));
+    const int warps = adam ? kAdamWarps : kWarps;
     const Launch L = symmetric ? plan(int_unit_bytes(group_size, Lp.p.g_kind, adam), kIntScratchBytes, warps)
                                : plan_ring(group_size, Lp.p.g_kind, adam, warps);
     Lp.p.stages = L.stages;

@@ -907,19 +907,24 @@ __global__ void __launch_bounds__(ADAM ? 192 : 256, 2)
         float T1b = 0.0f, T2b = 0.0f, T3b = 0.0f;
         sums_of(kb, T1b, T2b, T3b);
         // Candidates needing an exact comparison: within the fp32 error bound
-        // of the winner.  Those of the winner's chunk (one centre) whose sums
-        // equal the winner's bit for bit ("twins") almost always have the
-        // winner's codes -- equal codes give equal errors, and the lower index
-        // is kept, as Algorithm 1's argmin does -- but an element of tiny
+        // of the winner.  Those whose sums, about the winner's centre code
+        // (their chunk's or another chunk's with the same centre), equal the
+        // winner's bit for bit ("twins") almost always have the winner's
+        // codes -- equal codes give equal errors, and the lower index is
+        // kept, as Algorithm 1's argmin does -- but an element of tiny
         // saliency can differ without moving the sums, so twins are first
         // checked code by code (cheaply, deferred).
+        float y0w = Y0k[0];
+#pragma unroll
+        for (int ch = 1; ch < NCH; ++ch)
+            if ((kb >> 3) == ch) y0w = Y0k[ch];
         unsigned set = 0, twins = 0;
 #pragma unroll
         for (int ch = 0; ch < NCH; ++ch)
 #pragma unroll
             for (int qd = 0; qd < 2; ++qd) {
                 const int k = ch * 8 + qd * 4 + sl;
-                const bool twin = ch == (kb >> 3) && T1k[ch][qd] == T1b && T2k[ch][qd] == T2b &&
+                const bool twin = Y0k[ch] == y0w && T1k[ch][qd] == T1b && T2k[ch][qd] == T2b &&
                                   T3k[ch][qd] == T3b;
                 const bool contender =
                     k != kb && Ek[ch][qd] > -INFINITY && Eb - Ek[ch][qd] <= dEb + dEk[ch][qd];
@@ -956,32 +961,91 @@ __global__ void __launch_bounds__(ADAM ? 192 : 256, 2)
             const float gdbar = __shfl_sync(0xffffffffu, (mu - cref) + ebar, src);
             unsigned gset = __shfl_sync(0xffffffffu, set, src);
             const unsigned gtwins = __shfl_sync(0xffffffffu, twins, src);
-            const int gkb0 = __shfl_sync(0xffffffffu, kb, src);
+            int gw = __shfl_sync(0xffffffffu, kb, src);  // the winner
             const float* tws = ws + g * G;
             const float* ths = hs + g * G;
+            float gy0[NCH];
+#pragma unroll
+            for (int ch = 0; ch < NCH; ++ch) gy0[ch] = __shfl_sync(0xffffffffu, Y0k[ch], src);
+            if (p.stats && lane == 0) atomicAdd(&p.stats[2], 1u);
+            auto same_codes = [&](int k) {
+                if (p.stats && lane == 0) atomicAdd(&p.stats[6], 1u);
+                return coop_same_codes<G>(tws, ggq, gR * p.invf[k], gR * p.invf[gw]);
+            };
+            // Codes move monotonically with 1/f, element by element (the
+            // factors decrease with k), so two candidates with equal codes
+            // share them with every candidate between them: the highest twin
+            // settles all twins when its codes are the winner's.
+            const bool mono = p.monotone != 0;
             unsigned tw = gtwins;
+            if (tw && mono) {
+                const int khi = 31 - __clz(tw);
+                tw &= ~(1u << khi);
+                if (same_codes(khi)) {
+                    gset &= ~((2u << khi) - (2u << gw));  // (gw, khi]
+                    tw = 0;
+                }
+            }
             while (tw) {
                 const int k = __ffs(tw) - 1;
                 tw &= tw - 1;
-                if (coop_same_codes<G>(tws, ggq, gR * p.invf[k], gR * p.invf[gkb0]))
-                    gset &= ~(1u << k);
+                if (same_codes(k)) gset &= ~(1u << k);
             }
-            if (gset == (1u << gkb0)) continue;  // only the winner left
+            // Contenders about another centre code (their sums are not
+            // comparable with the winner's): first whether they share the
+            // winner's codes -- below the winner, lowest first, such a
+            // candidate becomes the winner; above it, highest first, it
+            // drops out (with monotone codes, so does everything between it
+            // and the winner).
+            auto other_centres = [&]() {
+                float y0g = gy0[0];
+#pragma unroll
+                for (int ch = 1; ch < NCH; ++ch)
+                    if ((gw >> 3) == ch) y0g = gy0[ch];
+                unsigned m = 0;
+#pragma unroll
+                for (int ch = 0; ch < NCH; ++ch)
+                    if (gy0[ch] != y0g) m |= 0xFFu << (8 * ch);
+                return m;
+            };
+            if (NCH > 1) {
+                const unsigned cmask = other_centres();
+                unsigned lo = gset & cmask & ((1u << gw) - 1u);
+                while (lo) {
+                    const int k = __ffs(lo) - 1;
+                    lo &= lo - 1;
+                    if (same_codes(k)) {
+                        gset &= ~(mono ? (2u << gw) - (2u << k) : 1u << gw);  // (k, gw]
+                        gw = k;
+                        break;
+                    }
+                }
+                unsigned hi = gset & cmask & ~((2u << gw) - 1u);
+                while (hi) {
+                    const int k = 31 - __clz(hi);
+                    hi &= ~(1u << k);
+                    if (same_codes(k)) {
+                        gset &= ~(mono ? (2u << k) - (2u << gw) : 1u << k);  // (gw, k]
+                        if (mono) break;
+                    }
+                }
+            }
+            if (gset == (1u << gw)) {  // only the winner left
+                if (gs == g) kb = gw;
+                continue;
+            }
             if (p.stats && lane == 0) atomicAdd(&p.stats[0], 1u);
             float best_h = 0.0f, best_l = 0.0f, ga = 0.0f, gB = 0.0f, gkap = 0.0f;
             int best_k = -1;
             bool gdeg = false;
-            // the quick error pass only where every candidate left shares the
-            // winner's chunk: candidates of different chunks can have equal
-            // codes (their sums, about different centres, differ), and only
-            // the two-pass fit, a function of the codes alone, then gives
-            // them bitwise-equal errors, so that the lower index is kept
-            const bool one_chunk = (gset & ~(0xFFu << ((gkb0 >> 3) * 8))) == 0u;
+            // the quick error pass only where every candidate left has the
+            // winner's centre code: candidates about different centres can
+            // have equal codes with unequal sums, and only the two-pass fit, a
+            // function of the codes alone, then gives them bitwise-equal
+            // errors, so that the lower index is kept
+            const bool one_chunk = (gset & other_centres()) == 0u;
             const float gebar = __shfl_sync(0xffffffffu, ebar, src);
             const float gsee = __shfl_sync(0xffffffffu, see, src);
-            float gy0[NCH];
-#pragma unroll
-            for (int ch = 0; ch < NCH; ++ch) gy0[ch] = __shfl_sync(0xffffffffu, Y0k[ch], src);
             while (gset) {
                 const int k = __ffs(gset) - 1;
                 gset &= gset - 1;
@@ -1017,6 +1081,7 @@ __global__ void __launch_bounds__(ADAM ? 192 : 256, 2)
                     one_chunk && Dk > 1e-3f * k2 && rel * rel * Exk < 1e-9f * (gsee - Exk);
                 float eh, el, a_k = 0.0f, B_k = 0.0f, kap_k = 0.0f;
                 bool deg_k = false;
+                if (p.stats && lane == 0) atomicAdd(&p.stats[quick ? 5 : 4], 1u);
                 if (quick) {
                     // offset at q = 0 of w - cref: mean(w - cref) - a (mean zeta + J + 1)
                     const float bck = gdbar - ak * ((y0k - kGridMagic) + k1 / gss + Jp1);
@@ -1073,28 +1138,36 @@ __global__ void __launch_bounds__(ADAM ? 192 : 256, 2)
             kap_sel = __fdividef(dse * rsqrtf(dse), fabsf(Nc)) + __fdividef(T2b, Dc);
         }
 
-        // ---- output accuracy check.  The fp32 fit's error at any level is at
-        // most about est = fit_ulps * ulp * (|a| qmax kap + |c| + range)
-        // (fit_ulps calibrated against the oracle with a margin).  The offset
-        // b (fp32) and a level written in fp32 must meet tol(x) = 1e-7 +
-        // 1e-5|x|.  A level written in bf16 is exact when no bf16 rounding
-        // midpoint lies within est of it, and within the tolerance band when
-        // est <= tol.  Groups that could miss get the compensated fit.
+        // ---- output accuracy check.  The fp32 fit's error at level q is at
+        // most about est(q) = fit_ulps * ulp * (|a| kap (|q - qbar| + 1) + |c|
+        // + |mu| + sqrt(see / Ss)): the slope's relative error (kap ulps)
+        // times the level's distance from the weighted mean code qbar, plus
+        // the error of the weighted mean itself, of the order of ulps of the
+        // weighted mean |w| (at most |mu| + sqrt(see / Ss)) or, far from
+        // zero, of the centre c.  fit_ulps is calibrated against the oracle
+        // with a margin.  The slope a, the offset b (fp32) and a level
+        // written in fp32 must meet tol(x) = 1e-7 + 1e-5|x|.  A level written
+        // in bf16 is exact when no bf16 rounding midpoint lies within est of
+        // it, and within the tolerance band when est <= tol.  Groups that
+        // could miss get the compensated fit.
         const bool refit = !flat && !deg_sel;
         bool prec;
         {
-            const float est =
-                p.fit_ulps * 5.9604645e-8f * (fabsf(a_sel) * qmaxf * kap_sel + fabsf(cref) + range);
+            const float uf = p.fit_ulps * 5.9604645e-8f;
+            const float ea = uf * fabsf(a_sel) * kap_sel;
+            const float ec = uf * (fabsf(cref) + fabsf(mu) + sqrtf(see * inv_ss));
+            // the weighted mean code (q = zeta + J + 1)
+            const float qbar = (y0b - kGridMagic) + T1b * inv_ss + Jp1;
             const float b0 = fmaf(-a_sel, Jp1, Bz);  // offset at q = 0
-            prec = est > 1e-7f + 1e-5f * fabsf(b0);
-            if (!p.r_bf16) {
-                const float q0 = fminf(fmaxf(rintf(__fdividef(-b0, a_sel)), 0.0f), qmaxf);
-                const float rmin = fminf(fabsf(b0), fabsf(fmaf(a_sel, q0, b0)));
-                prec |= est > 1e-7f + 1e-5f * rmin;
-            } else {
-                for (int q = sl; q <= p.qmax; q += kIntLanes) {
-                    const float rq = fmaf(a_sel, (float)q, b0);
-                    if (est > 1e-7f + 1e-5f * fabsf(rq)) {
+            prec = fmaf(ea, fabsf(qbar) + 1.0f, ec) > 1e-7f + 1e-5f * fabsf(b0);
+            prec |= ea > 1e-7f + 1e-5f * fabsf(a_sel);
+            for (int q = sl; q <= p.qmax; q += kIntLanes) {
+                const float rq = fmaf(a_sel, (float)q, b0);
+                const float est = fmaf(ea, fabsf((float)q - qbar) + 1.0f, ec);
+                if (est > 1e-7f + 1e-5f * fabsf(rq)) {
+                    if (!p.r_bf16) {
+                        prec = true;
+                    } else {
                         const uint32_t bits = __float_as_uint(rq);
                         const int dmid = abs((int)(bits & 0xFFFFu) - 0x8000);  // fp32 ulps to the midpoint
                         const float ulp32 =
@@ -1103,7 +1176,8 @@ __global__ void __launch_bounds__(ADAM ? 192 : 256, 2)
                     }
                 }
             }
-            prec = prec || est != est;  // NaN sums: take the careful path
+            const float esum = ea + ec + qbar;
+            prec = prec || esum != esum;  // NaN sums: take the careful path
             // one decision per group: any lane of the group that flagged
             prec = (__ballot_sync(0xffffffffu, prec) & gmask) != 0;
         }
