@@ -383,8 +383,9 @@ quasar_status quasar_adamw_recon_nvfp4_batch(const quasar_adamw_nvfp4_tensor* te
  *             (options), 192 bytes a block: the block's 512 indices in
  *             row-major block order, 3 bits each, little-endian.
  *   cand_idx  [rows/8 * cols/64] uint8, or NULL.
- * rows % 8 == 0 and cols % 64 == 0, else QUASAR_ERR_INVALID_ARG.  Other
- * rules, options and returns as quasar_recon_int_batch_ex.
+ * rows % 8 == 0 and cols % 64 == 0, and fewer than 2^32 blocks a tensor,
+ * else QUASAR_ERR_INVALID_ARG.  Other rules, options and returns as
+ * quasar_recon_int_batch_ex.
  */
 typedef struct {
     const float* w;

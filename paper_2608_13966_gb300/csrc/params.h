@@ -143,10 +143,12 @@ struct Nvfp4Params {
 constexpr int kLutRows = 8;
 constexpr int kLutCols = 64;
 constexpr int kLutBlock = kLutRows * kLutCols;
-// Per-warp scratch of the LUT kernel: the transpose of 24 per-code sums
-// (rows padded to 33 floats), and per candidate its table (8 bytes), error,
-// error bound and whether an entry's rounding was undecided.
-constexpr uint32_t kLutSumsBytes = 24 * 33 * 4;
+// Per-warp scratch of the LUT kernel: the transpose of 12 per-threshold
+// sums of each of two candidates (rows of 36 floats: 16-byte aligned, readers
+// of rows r and r + 8 share banks), and per candidate its table (8 bytes), error, error bound and which
+// entries' roundings were undecided.
+constexpr int kLutRow = 36;
+constexpr uint32_t kLutSumsBytes = 24 * kLutRow * 4;
 constexpr uint32_t kLutCandBytes = kMaxClip * 20;
 constexpr uint32_t kLutScratchBytes = kLutSumsBytes + kLutCandBytes + 64;
 
@@ -177,7 +179,9 @@ struct LutParams {
     uint64_t timeout_ns;
     uint64_t force_timeout_ns;
     unsigned int* status;
-    unsigned int* stats;  // optional: [0] blocks compared exactly, [1] entries rounded exactly
+    unsigned int* stats;  // optional: [0] blocks compared exactly, [1] candidates evaluated
+                          // exactly, [2] blocks whose fast winner had an undecided entry,
+                          // [3] blocks whose near ties took direct fp32 errors
     float f[kMaxClip];
     float invf[kMaxClip];
 };

@@ -905,6 +905,7 @@ quasar_status quasar_recon_lut_batch(const quasar_lut_tensor* tensors, int n_ten
         if (s1 != QUASAR_OK) return s1;
         if (x.rows % kLutRows != 0 || x.cols % kLutCols != 0) return QUASAR_ERR_INVALID_ARG;
         const int64_t n_blocks = n / kLutBlock;
+        if (n_blocks > (int64_t)UINT32_MAX) return QUASAR_ERR_INVALID_ARG;  // 32-bit block indices
         if (n > 0) {
             if (!x.book || !aligned16(x.book)) return QUASAR_ERR_INVALID_ARG;
             if (x.codes && !aligned16(x.codes)) return QUASAR_ERR_INVALID_ARG;

@@ -9,15 +9,20 @@
 //
 // One warp owns one block: lane L holds block elements 16 L .. 16 L + 15
 // (row L / 4, columns 16 (L % 4) ..), read once from a per-warp TMA ring.
-// Per candidate each lane accumulates, for every index j, H_j = sum h and
-// W_j = sum h (w - g_j) about the index's grid point g_j (one-hot masks,
-// packed f32x2), and Q = sum h (w - g_q)^2 over all elements; the 17 sums are
-// transposed through shared memory, lane j forms entry j, and the error is
-//   sum_j (H_j d_j^2 - 2 d_j W_j) + Q,   d_j = C_j - g_j.
-// Both the entry's rounding and the error carry an fp32 bound.  Candidates
-// within the bound of the best, and undecided roundings, are settled exactly
-// (float-float sums, whole warp), so indices, tables and the kept candidate
-// equal the exact computation's.
+// An index is a sign s of d = w - c and a magnitude level m = min(floor(|d|
+// P), 3).  Per candidate each lane accumulates, for each sign and threshold
+// t = 1, 2, 3, the sums of h and of h |d| over its elements with m >= t
+// (packed f32x2; the masks [m >= t] come from saturated adds on the floor,
+// so no per-index one-hot work); the 12 sums are transposed through shared
+// memory, and with the block's per-sign totals they give every index's H_j =
+// sum h and X_j = sum h |d|.  Index j's entry is the E4M3 rounding of its
+// weighted mean c + s X_j / H_j, and the error is
+//   sum h d^2 - sum_j X_j^2 / H_j + sum_j H_j (C_j - mean_j)^2
+// (the within-index scatter plus each entry's offset from its mean).  Both
+// the entry's rounding and the error carry an fp32 bound.  Candidates within
+// the bound of the best, and undecided roundings, are settled exactly
+// (float-float sums over the codes, whole warp), so indices, tables and the
+// kept candidate equal the exact computation's.
 #pragma once
 
 #include <cuda_bf16.h>
@@ -104,6 +109,15 @@ __device__ __forceinline__ float code_z(float d, float P)
     return copysignf(__fsub_rn(y, kHalfBelow), d);
 }
 
+// [x + b >= 1] for x + b an integer (x on the 2^23 grid): the sum saturated
+// to [0, 1]
+__device__ __forceinline__ float add_sat(float x, float b)
+{
+    float r;
+    asm("add.rn.sat.f32 %0, %1, %2;" : "=f"(r) : "f"(x), "f"(b));
+    return r;
+}
+
 // The E4M3 value nearest the float-float x = xh + xl (ties to the even
 // mantissa): the rounding of xh, or one of its neighbours.
 __device__ __forceinline__ uint32_t e4m3_round_ff(float xh, float xl)
@@ -159,6 +173,8 @@ __global__ void __launch_bounds__(256, 2) k_recon_lut(const __grid_constant__ Lu
     float* cbnd = cerr + kMaxClip;                                        // [32]
     uint32_t* camb = reinterpret_cast<uint32_t*>(cbnd + kMaxClip);      // [32]
     float* table = reinterpret_cast<float*>(scr + kLutSumsBytes + kLutCandBytes);  // [8]
+    // the block's per-sign sums of h and h |d|, and sum h d^2
+    float* bconst = table + 8;  // [5]
     uint64_t* bars = reinterpret_cast<uint64_t*>(smem + (size_t)nwarps * S * p.stage_bytes +
                                                  (size_t)nwarps * kLutScratchBytes) +
                      warp * (S + 1);
@@ -188,9 +204,11 @@ __global__ void __launch_bounds__(256, 2) k_recon_lut(const __grid_constant__ Lu
         int tj = ti;
         tensor_of(u, tj);
         const LutTensor& T = Lp.t[tj];
-        const int64_t b = u - T.unit0;
-        const int64_t nbc = T.cols / kLutCols;
-        const int64_t base = (b / nbc) * kLutRows * T.cols + (b % nbc) * kLutCols;
+        // block row and column (a tensor holds fewer than 2^32 blocks)
+        const uint32_t b = (uint32_t)(u - T.unit0);
+        const uint32_t nbc = (uint32_t)(T.cols / kLutCols);
+        const uint32_t brow = b / nbc;
+        const int64_t base = (int64_t)brow * kLutRows * T.cols + (int64_t)(b - brow * nbc) * kLutCols;
         unsigned char* st = ring + (size_t)s * p.stage_bytes;
         if (lane == 0) mbar_arrive_expect_tx(&bars[s], (uint32_t)kLutBlock * (8u + (uint32_t)gbytes));
         __syncwarp();
@@ -228,8 +246,6 @@ __global__ void __launch_bounds__(256, 2) k_recon_lut(const __grid_constant__ Lu
     const float2 beta22 = make_float2(p.beta2, p.beta2);
     const float2 c12 = make_float2(p.c1, p.c1);
     const float2 M2 = make_float2(kMagic, kMagic);
-    const float2 cap2 = make_float2(kMagic + 3.0f, kMagic + 3.0f);
-    const float2 nmh2 = make_float2(-kHalfBelow, -kHalfBelow);
     const float gam = kU * p.tie_kappa;
     int s_cur = 0;
     uint32_t parity = 0;
@@ -244,11 +260,12 @@ __global__ void __launch_bounds__(256, 2) k_recon_lut(const __grid_constant__ Lu
         const unsigned char* st = ring + (size_t)s_cur * p.stage_bytes;
         tensor_of(u, ti);
         const LutTensor& T = Lp.t[ti];
-        const int64_t b = u - T.unit0;
-        const int64_t nbc = T.cols / kLutCols;
+        const uint32_t b = (uint32_t)(u - T.unit0);
+        const uint32_t nbc = (uint32_t)(T.cols / kLutCols);
+        const uint32_t brow = b / nbc;
         // the lane's 16 elements: row lane/4 of the block, columns 16 (lane % 4) ..
-        const int64_t gofs =
-            ((b / nbc) * kLutRows + (lane >> 2)) * T.cols + (b % nbc) * kLutCols + (lane & 3) * 16;
+        const int64_t gofs = ((int64_t)brow * kLutRows + (lane >> 2)) * T.cols +
+                             (int64_t)(b - brow * nbc) * kLutCols + (lane & 3) * 16;
 
         // ---- pass A: w, the saliency EMA (v' out), the fit's saliency h
         float2 w2[8], h2[8];
@@ -312,109 +329,191 @@ __global__ void __launch_bounds__(256, 2) k_recon_lut(const __grid_constant__ Lu
         const float c = 0.5f * (mn + mx);
         const float R = flat ? 0.0f : __fdividef(7.0f, range);
         const float2 nc2 = make_float2(-c, -c);
-        // the fp32 error of a centred value w - g: two roundings of magnitude
-        // at most |w - c| + |c|, plus the grid point's own
-        const float eps_e = 4.0f * kU * (range + fabsf(c));
+
+        // candidate-independent: |d| = |w - c| and the saliency split by the
+        // sign of d (a negative zero counts as negative, as the index does);
+        // w itself is read again from memory only by the exact look
+        float2 ad2[8], hp2[8], hn2[8];
+        uint32_t negm = 0;  // bit i: element i has d < 0 (or -0)
+        {
+            float tp, tn, up, un, sd;
+            float2 Tp = make_float2(0.0f, 0.0f), Tn = Tp, Up = Tp, Un = Tp, Sd = Tp;
+#pragma unroll
+            for (int t = 0; t < 8; ++t) {
+                const float2 d = __fadd2_rn(w2[t], nc2);
+                const bool nx = signbit(d.x), ny = signbit(d.y);
+                negm |= (nx ? 1u : 0u) << (2 * t);
+                negm |= (ny ? 1u : 0u) << (2 * t + 1);
+                ad2[t] = make_float2(fabsf(d.x), fabsf(d.y));
+                hp2[t] = make_float2(nx ? 0.0f : h2[t].x, ny ? 0.0f : h2[t].y);
+                hn2[t] = make_float2(nx ? h2[t].x : 0.0f, ny ? h2[t].y : 0.0f);
+                Tp = __fadd2_rn(Tp, hp2[t]);
+                Tn = __fadd2_rn(Tn, hn2[t]);
+                const float2 hd = __fmul2_rn(h2[t], ad2[t]);
+                Up = __fadd2_rn(Up, make_float2(nx ? 0.0f : hd.x, ny ? 0.0f : hd.y));
+                Un = __fadd2_rn(Un, make_float2(nx ? hd.x : 0.0f, ny ? hd.y : 0.0f));
+                Sd = __ffma2_rn(hd, ad2[t], Sd);
+            }
+            tp = Tp.x + Tp.y;
+            tn = Tn.x + Tn.y;
+            up = Up.x + Up.y;
+            un = Un.x + Un.y;
+            sd = Sd.x + Sd.y;
+#pragma unroll
+            for (int o = 16; o; o >>= 1) {
+                tp += __shfl_xor_sync(0xffffffffu, tp, o);
+                tn += __shfl_xor_sync(0xffffffffu, tn, o);
+                up += __shfl_xor_sync(0xffffffffu, up, o);
+                un += __shfl_xor_sync(0xffffffffu, un, o);
+                sd += __shfl_xor_sync(0xffffffffu, sd, o);
+            }
+            // one value for every lane, kept in the scratch until the
+            // candidates' entries need them
+            if (lane == 0) {
+                bconst[0] = tp;
+                bconst[1] = tn;
+                bconst[2] = up;
+                bconst[3] = un;
+                bconst[4] = sd;
+            }
+        }
 
         int kb = 0;
         if (!flat) {
-            // ---- candidates: indices, per-index sums, entries, error
+            // ---- candidates, two a pass: per-index sums of each (12 rows of
+            // the scratch a candidate), then entries and errors of both at
+            // once (lanes 0..7 the first, 8..15 the second)
 #pragma unroll 1
-            for (int k = 0; k < K; ++k) {
-                const float P = R * p.invf[k];
-                const float sg = __fdividef(1.0f, P);  // the grid step
-                const float2 P2 = make_float2(P, P), nsg2 = make_float2(-sg, -sg);
-                float2 Hs[8], Ws[8], Qt = make_float2(0.0f, 0.0f);
+            for (int k0 = 0; k0 < K; k0 += 2) {
+                const int nk = min(2, K - k0);
+#pragma unroll 1
+                for (int kk = 0; kk < nk; ++kk) {
+                    const float P = R * p.invf[k0 + kk];
+                    const float2 P2 = make_float2(P, P);
+                    // [l]: threshold m >= l + 1; sums of h (A) and h |d| (X),
+                    // by sign.  The masked saliency h [m >= t] is exact, and
+                    // so is its product with |d| inside the FMA: every term
+                    // is exact.
+                    float2 Ap[3], An[3], Xp[3], Xn[3];
 #pragma unroll
-                for (int j = 0; j < 8; ++j) Hs[j] = Ws[j] = make_float2(0.0f, 0.0f);
+                    for (int l = 0; l < 3; ++l) Ap[l] = An[l] = Xp[l] = Xn[l] = make_float2(0.0f, 0.0f);
 #pragma unroll
-                for (int t = 0; t < 8; ++t) {
-                    const float2 d = __fadd2_rn(w2[t], nc2);
-                    const float2 ad = make_float2(fabsf(d.x), fabsf(d.y));
-                    float2 y = __ffma2_rd(ad, P2, M2);
-                    y.x = fminf(y.x, cap2.x);
-                    y.y = fminf(y.y, cap2.y);
-                    const float2 za = __fadd2_rn(y, nmh2);
-                    const float2 z = make_float2(copysignf(za.x, d.x), copysignf(za.y, d.y));
-                    const float2 e = __ffma2_rn(z, nsg2, d);  // w - g_j, g_j = c + z sg
-                    const float2 he = __fmul2_rn(h2[t], e);
-                    Qt = __ffma2_rn(he, e, Qt);
+                    for (int t = 0; t < 8; ++t) {
+                        const float2 y = __ffma2_rd(ad2[t], P2, M2);  // 2^23 + floor(|d| P)
 #pragma unroll
-                    for (int j = 0; j < 8; ++j) {
-                        const float zj = (float)j - 3.5f;
-                        const float2 m = make_float2(z.x == zj ? 1.0f : 0.0f, z.y == zj ? 1.0f : 0.0f);
-                        Hs[j] = __ffma2_rn(m, h2[t], Hs[j]);
-                        Ws[j] = __ffma2_rn(m, he, Ws[j]);
+                        for (int l = 0; l < 3; ++l) {
+                            const float nb = -(kMagic + (float)l);
+                            const float2 mk = make_float2(add_sat(y.x, nb), add_sat(y.y, nb));
+                            const float2 mp = __fmul2_rn(hp2[t], mk);
+                            const float2 mq = __fmul2_rn(hn2[t], mk);
+                            Ap[l] = __fadd2_rn(Ap[l], mp);
+                            An[l] = __fadd2_rn(An[l], mq);
+                            Xp[l] = __ffma2_rn(mp, ad2[t], Xp[l]);
+                            Xn[l] = __ffma2_rn(mq, ad2[t], Xn[l]);
+                        }
+                    }
+                    // rows (of this candidate's 12): A+ 0..2, A- 3..5, X+ 6..8,
+                    // X- 9..11
+                    float* rows = sums + kk * 12 * kLutRow + lane;
+#pragma unroll
+                    for (int l = 0; l < 3; ++l) {
+                        rows[l * kLutRow] = Ap[l].x + Ap[l].y;
+                        rows[(3 + l) * kLutRow] = An[l].x + An[l].y;
+                        rows[(6 + l) * kLutRow] = Xp[l].x + Xp[l].y;
+                        rows[(9 + l) * kLutRow] = Xn[l].x + Xn[l].y;
                     }
                 }
-                // transpose: row q of the scratch holds sum q of every lane
-#pragma unroll
-                for (int j = 0; j < 8; ++j) {
-                    sums[j * 33 + lane] = Hs[j].x + Hs[j].y;
-                    sums[(8 + j) * 33 + lane] = Ws[j].x + Ws[j].y;
-                }
-                sums[16 * 33 + lane] = Qt.x + Qt.y;
                 __syncwarp();
+                // lane r < 12 nk sums row r
                 float tot = 0.0f;
-                if (lane < 17) {
+                if (lane < 12 * nk) {
                     float a0 = 0.0f, a1 = 0.0f, a2 = 0.0f, a3 = 0.0f;
 #pragma unroll
-                    for (int i = 0; i < 32; i += 4) {
-                        a0 += sums[lane * 33 + i];
-                        a1 += sums[lane * 33 + i + 1];
-                        a2 += sums[lane * 33 + i + 2];
-                        a3 += sums[lane * 33 + i + 3];
+                    for (int i = 0; i < 8; ++i) {
+                        const float4 v = *reinterpret_cast<const float4*>(sums + lane * kLutRow + 4 * i);
+                        a0 += v.x;
+                        a1 += v.y;
+                        a2 += v.z;
+                        a3 += v.w;
                     }
                     tot = (a0 + a1) + (a2 + a3);
                 }
                 __syncwarp();
-                // lane j < 8: entry j
+                // lane j < 8 of each half: index j, sign s (j >= 4: d >= 0),
+                // level m; its H = A_m - A_(m+1) and X = X_m - X_(m+1) (A_0,
+                // X_0: the sign's totals; A_4 = X_4 = 0)
+                const int half = (lane >> 3) & 1;
+                const int rb = half * 12;  // the candidate's first row
+                const float P = R * p.invf[min(k0 + half, K - 1)];
+                const float sg = __fdividef(1.0f, P);
                 const int j = lane & 7;
-                const float Hj = tot;
-                const float Wj = __shfl_sync(0xffffffffu, tot, j + 8);
-                const float Qt1 = __shfl_sync(0xffffffffu, tot, 16);
-                const float gj = fmaf((float)j - 3.5f, sg, c);
-                // A >= sum over index j of h |w - g_j|: |w - g_j| <= sg/2 inside
-                // the range, and up to (1 - f) rho + sg/2 for the clamped ends
-                const float emax = (j == 0 || j == 7)
-                                       ? fmaf(0.5f * range, fmaxf(1.0f - p.f[k], 0.0f), 0.5f * sg)
-                                       : 0.5f * sg;
-                const float A = Hj * (emax * (1.0f + 8.0f * kU) + eps_e);
-                float mean = gj, dm = 4.0f * kU * fabsf(gj);
-                if (Hj > 0.0f) {
-                    const float q = __fdividef(Wj, Hj);
-                    mean = gj + q;
-                    dm = gam * (A + fabsf(Wj)) / Hj + eps_e + 4.0f * kU * (fabsf(mean) + fabsf(q));
+                const bool pos = j >= 4;
+                const int m = pos ? j - 4 : 3 - j;
+                const int r0 = rb + (pos ? 0 : 3);
+                const float sA0 = __shfl_sync(0xffffffffu, tot, r0 + max(m - 1, 0));
+                const float sA1 = __shfl_sync(0xffffffffu, tot, r0 + min(m, 2));
+                const float sX0 = __shfl_sync(0xffffffffu, tot, 6 + r0 + max(m - 1, 0));
+                const float sX1 = __shfl_sync(0xffffffffu, tot, 6 + r0 + min(m, 2));
+                const float Am = m == 0 ? bconst[pos ? 0 : 1] : sA0;
+                const float Am1 = m == 3 ? 0.0f : sA1;
+                const float Xm = m == 0 ? bconst[pos ? 2 : 3] : sX0;
+                const float Xm1 = m == 3 ? 0.0f : sX1;
+                const float H = Am - Am1, X = fmaxf(Xm - Xm1, 0.0f);
+                const float sgn = pos ? 1.0f : -1.0f;
+                const float gj = fmaf((float)j - 3.5f, sg, c);  // the grid point
+                // errors: the cumulative sums are sums of exact nonnegative
+                // terms over at most tie_kappa levels (the per-sign totals of
+                // h |d| carry one more rounding a term)
+                const float dA = gam * (Am + Am1) + kU * H;
+                const float dX = (gam + kU) * (Xm + Xm1) + kU * X;
+                float mean = gj, q = 0.0f, dq = 0.0f, dm = 4.0f * kU * fabsf(gj);
+                if (H > 0.0f) {
+                    q = __fdividef(X, H);
+                    mean = fmaf(sgn, q, c);
+                    dq = __fdividef(dX + q * dA, H) + 2.0f * kU * q;
+                    // plus the roundings of w - c (relative u each), of the
+                    // quotient's use and of the mean's sum
+                    dm = dq + 3.0f * kU * q + 2.0f * kU * fabsf(mean);
                 }
                 const uint32_t cb = e4m3_encode(mean);
                 const bool amb = e4m3_encode(mean - dm) != e4m3_encode(mean + dm);
-                const float dd = e4m3_decode(cb) - gj;
-                const float Sj = fmaf(Hj * dd, dd, -2.0f * dd * Wj);
-                float bj = (gam + 4.0f * kU) * (Hj * dd * dd + 2.0f * fabsf(dd) * A) +
-                           2.0f * eps_e * (fabsf(dd) * Hj + 2.0f * A);
-                if (amb)  // the other rounding differs by at most this much
-                    bj += 2.0f * Hj * dm *
-                          fabsf(e4m3_decode(e4m3_encode(mean + dm)) - e4m3_decode(e4m3_encode(mean - dm)));
-                float E = lane < 8 ? Sj : 0.0f, dE = lane < 8 ? bj : 0.0f;
-                uint32_t wb = lane < 8 ? cb << (8 * (lane & 3)) : 0u;
+                const float dc = e4m3_decode(cb) - mean;
+                // the index's error: H (C - mean)^2 - X^2 / H (the scatter
+                // term sum h d^2 is added once below)
+                const float Sj = H > 0.0f ? fmaf(H * dc, dc, -X * q) : 0.0f;
+                float bj = dA * dc * dc + 2.0f * H * fabsf(dc) * dm + 3.0f * kU * H * dc * dc + dX * q +
+                           X * dq + 2.0f * kU * X * q;
+                if (amb) {  // the other rounding moves the entry by at most this much
+                    const float c1 = e4m3_decode(e4m3_encode(mean - dm)) - mean;
+                    const float c2 = e4m3_decode(e4m3_encode(mean + dm)) - mean;
+                    bj += H * fabsf(c2 - c1) * (fabsf(c1) + fabsf(c2) + 2.0f * dm);
+                }
+                const bool live = lane < 16;
+                float E = live ? Sj : 0.0f, dE = live ? bj : 0.0f, aE = live ? fabsf(Sj) : 0.0f;
+                uint32_t wb = live ? cb << (8 * (lane & 3)) : 0u;
 #pragma unroll
                 for (int o = 4; o; o >>= 1) {
                     E += __shfl_xor_sync(0xffffffffu, E, o);
                     dE += __shfl_xor_sync(0xffffffffu, dE, o);
+                    aE += __shfl_xor_sync(0xffffffffu, aE, o);
                 }
-                E += Qt1;
-                dE += (gam + 4.0f * kU) * Qt1 + 4.0f * kU * fabsf(E);
+                const float sd = bconst[4];
+                E += sd;
+                // sum h d^2: its terms' roundings (|d|^2, h times it) and sum
+                dE += (gam + 3.0f * kU) * sd + 4.0f * kU * (sd + aE);
 #pragma unroll
                 for (int o = 2; o; o >>= 1) wb |= __shfl_xor_sync(0xffffffffu, wb, o);
-                const uint32_t wb1 = __shfl_sync(0xffffffffu, wb, 4);
-                const uint32_t ambm = __ballot_sync(0xffffffffu, amb && lane < 8) & 0xFFu;
-                if (lane == 0) {
+                const uint32_t wb1 = __shfl_sync(0xffffffffu, wb, (lane & 8) | 4);
+                const uint32_t ambm = __ballot_sync(0xffffffffu, amb && live);
+                if (lane == 0 || (lane == 8 && nk == 2)) {
+                    const int k = k0 + half;
                     cbook[2 * k] = wb;
                     cbook[2 * k + 1] = wb1;
                     cerr[k] = E;
                     cbnd[k] = dE;
-                    camb[k] = ambm;
+                    camb[k] = (ambm >> (8 * half)) & 0xFFu;
                 }
+                __syncwarp();  // the scratch rows are rewritten by the next pass
             }
             __syncwarp();
 
@@ -435,11 +534,146 @@ __global__ void __launch_bounds__(256, 2) k_recon_lut(const __grid_constant__ Lu
             kb = kk;
             const float dEb = __shfl_sync(0xffffffffu, dEk, kb);
             unsigned set = __ballot_sync(0xffffffffu, lane < K && lane != kb && Ek - Eb <= dEk + dEb);
-            if (set || camb[kb]) set |= 1u << kb;
+            if (p.stats && lane == 0 && camb[kb]) atomicAdd(&p.stats[2], 1u);
+
+            // index (0..7) of element i for the grid of P
+            auto index_of = [&](int i, float P) {
+                const float a = (i & 1) ? ad2[i >> 1].y : ad2[i >> 1].x;
+                const float mf = fminf(__fmaf_rd(a, P, kMagic) - kMagic, 3.0f);
+                const int mi = (int)mf;
+                return ((negm >> i) & 1u) ? 3 - mi : 4 + mi;
+            };
+            // Undecided entries of candidate k from direct per-index sums
+            // (fp32, nonnegative exact terms, 16 + 5 levels: relative error
+            // within 24 ulps): settled (table updated) unless a rounding is
+            // still undecided.
+            auto refine = [&](int k) -> bool {
+                const float P = R * p.invf[k];
+                uint32_t und = camb[k];
+                uint32_t w0 = cbook[2 * k], w1 = cbook[2 * k + 1];
+                while (und) {
+                    const int j = __ffs(und) - 1;
+                    und &= und - 1;
+                    float Hs = 0.0f, Xs = 0.0f;
+#pragma unroll
+                    for (int i = 0; i < 16; ++i) {
+                        if (index_of(i, P) == j) {
+                            const float hv = (i & 1) ? hp2[i >> 1].y + hn2[i >> 1].y : hp2[i >> 1].x + hn2[i >> 1].x;
+                            const float av = (i & 1) ? ad2[i >> 1].y : ad2[i >> 1].x;
+                            Hs += hv;
+                            Xs = fmaf(hv, av, Xs);
+                        }
+                    }
+#pragma unroll
+                    for (int o = 16; o; o >>= 1) {
+                        Hs += __shfl_xor_sync(0xffffffffu, Hs, o);
+                        Xs += __shfl_xor_sync(0xffffffffu, Xs, o);
+                    }
+                    Hs = __shfl_sync(0xffffffffu, Hs, 0);
+                    Xs = __shfl_sync(0xffffffffu, Xs, 0);
+                    if (!(Hs > 0.0f)) return false;
+                    const float q = Xs / Hs;
+                    const float mean = fmaf(j >= 4 ? 1.0f : -1.0f, q, c);
+                    // two sums (24 ulps each), the quotient, w - c (an ulp a
+                    // term), the mean's sum
+                    const float dm = 52.0f * kU * q + 2.0f * kU * fabsf(mean);
+                    if (e4m3_encode(mean - dm) != e4m3_encode(mean + dm)) return false;
+                    const uint32_t cbj = e4m3_encode(mean);
+                    if (j < 4) w0 = (w0 & ~(0xFFu << (8 * j))) | (cbj << (8 * j));
+                    else w1 = (w1 & ~(0xFFu << (8 * (j - 4)))) | (cbj << (8 * (j - 4)));
+                }
+                __syncwarp();
+                if (lane == 0) {
+                    cbook[2 * k] = w0;
+                    cbook[2 * k + 1] = w1;
+                    camb[k] = 0u;
+                }
+                __syncwarp();
+                return true;
+            };
+
+            if (set == 0u) {
+                // the winner alone: its table must be decided
+                if (camb[kb] && !refine(kb)) set = 1u << kb;
+            } else {
+                set |= 1u << kb;
+                bool decided = true;
+                for (unsigned s2 = set; s2; s2 &= s2 - 1) {
+                    const int k = __ffs(s2) - 1;
+                    if (camb[k] && !refine(k)) decided = false;
+                }
+                if (decided) {
+                    // direct fp32 errors sum h (C_q - w)^2 of the candidates
+                    // left (terms within 3 ulps, 21 levels: 32 ulps in all)
+                    if (p.stats && lane == 0) atomicAdd(&p.stats[3], 1u);
+                    float xwv[16];
+#pragma unroll
+                    for (int i = 0; i < 4; ++i) {
+                        const float4 w4 = __ldg(reinterpret_cast<const float4*>(T.w + gofs + i * 4));
+                        xwv[4 * i] = w4.x;
+                        xwv[4 * i + 1] = w4.y;
+                        xwv[4 * i + 2] = w4.z;
+                        xwv[4 * i + 3] = w4.w;
+                    }
+                    for (unsigned s2 = set; s2; s2 &= s2 - 1) {
+                        const int k = __ffs(s2) - 1;
+                        const float P = R * p.invf[k];
+                        if (lane < 8)
+                            table[lane] = e4m3_decode((cbook[2 * k + (lane >> 2)] >> (8 * (lane & 3))) & 0xFFu);
+                        __syncwarp();
+                        float acc = 0.0f;
+#pragma unroll
+                        for (int i = 0; i < 16; ++i) {
+                            const float hv = (i & 1) ? hp2[i >> 1].y + hn2[i >> 1].y : hp2[i >> 1].x + hn2[i >> 1].x;
+                            const float df = table[index_of(i, P)] - xwv[i];
+                            acc = fmaf(hv * df, df, acc);
+                        }
+#pragma unroll
+                        for (int o = 16; o; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
+                        acc = __shfl_sync(0xffffffffu, acc, 0);
+                        __syncwarp();
+                        if (lane == 0) {
+                            cerr[k] = acc;
+                            cbnd[k] = 32.0f * kU * acc;
+                        }
+                    }
+                    __syncwarp();
+                    // the argmin again, over the set
+                    const bool in = lane < K && ((set >> lane) & 1u);
+                    float Ed = in ? cerr[lane] : INFINITY;
+                    const float dEd = in ? cbnd[lane] : 0.0f;
+                    float Edb = Ed;
+                    int kd = lane;
+#pragma unroll
+                    for (int o = 16; o; o >>= 1) {
+                        const float Eo = __shfl_xor_sync(0xffffffffu, Edb, o);
+                        const int ko = __shfl_xor_sync(0xffffffffu, kd, o);
+                        if (Eo < Edb || (Eo == Edb && ko < kd)) {
+                            Edb = Eo;
+                            kd = ko;
+                        }
+                    }
+                    kb = kd;
+                    const float dEdb = __shfl_sync(0xffffffffu, dEd, kb);
+                    set = __ballot_sync(0xffffffffu, in && lane != kb && Ed - Edb <= dEd + dEdb);
+                    if (set) set |= 1u << kb;
+                }
+            }
+
 
             // ---- exact look: float-float sums, exact roundings, direct error
             if (set) {
                 if (p.stats && lane == 0) atomicAdd(&p.stats[0], 1u);
+                // the lane's w again (from memory: this path is rare) and h
+                float2 xw[8], xh[8];
+#pragma unroll
+                for (int i = 0; i < 4; ++i) {
+                    const float4 w4 = __ldg(reinterpret_cast<const float4*>(T.w + gofs + i * 4));
+                    xw[2 * i] = make_float2(w4.x, w4.y);
+                    xw[2 * i + 1] = make_float2(w4.z, w4.w);
+                }
+#pragma unroll
+                for (int t = 0; t < 8; ++t) xh[t] = __fadd2_rn(hp2[t], hn2[t]);  // one of the two is 0
                 float best_h = 0.0f, best_l = 0.0f;
                 int best_k = -1;
                 uint32_t best_w0 = 0, best_w1 = 0;
@@ -452,8 +686,8 @@ __global__ void __launch_bounds__(256, 2) k_recon_lut(const __grid_constant__ Lu
                     float zz[16];
 #pragma unroll
                     for (int t = 0; t < 8; ++t) {
-                        zz[2 * t] = code_z(w2[t].x - c, P);
-                        zz[2 * t + 1] = code_z(w2[t].y - c, P);
+                        zz[2 * t] = code_z(xw[t].x - c, P);
+                        zz[2 * t + 1] = code_z(xw[t].y - c, P);
                     }
                     uint32_t w0 = 0, w1 = 0;
 #pragma unroll 1
@@ -464,8 +698,8 @@ __global__ void __launch_bounds__(256, 2) k_recon_lut(const __grid_constant__ Lu
 #pragma unroll
                         for (int i = 0; i < 16; ++i) {
                             if (zz[i] == zj) {
-                                const float hv = (i & 1) ? h2[i >> 1].y : h2[i >> 1].x;
-                                const float wv = (i & 1) ? w2[i >> 1].y : w2[i >> 1].x;
+                                const float hv = (i & 1) ? xh[i >> 1].y : xh[i >> 1].x;
+                                const float wv = (i & 1) ? xw[i >> 1].y : xw[i >> 1].x;
                                 float eh, el, ph, pl;
                                 two_sum(wv, -gj, eh, el);
                                 two_prod(hv, eh, ph, pl);
@@ -502,8 +736,8 @@ __global__ void __launch_bounds__(256, 2) k_recon_lut(const __grid_constant__ Lu
                     for (int i = 0; i < 16; ++i) {
                         const int q = (int)(zz[i] + 3.5f);
                         const uint32_t cb = ((q < 4 ? w0 : w1) >> (8 * (q & 3))) & 0xFFu;
-                        const float hv = (i & 1) ? h2[i >> 1].y : h2[i >> 1].x;
-                        const float wv = (i & 1) ? w2[i >> 1].y : w2[i >> 1].x;
+                        const float hv = (i & 1) ? xh[i >> 1].y : xh[i >> 1].x;
+                        const float wv = (i & 1) ? xw[i >> 1].y : xw[i >> 1].x;
                         float dh, dl, sh, sl;
                         two_sum(e4m3_decode(cb), -wv, dh, dl);
                         two_prod(dh, dh, sh, sl);
@@ -547,8 +781,9 @@ __global__ void __launch_bounds__(256, 2) k_recon_lut(const __grid_constant__ Lu
         float rv[16];
 #pragma unroll
         for (int i = 0; i < 16; ++i) {
-            const float wv = (i & 1) ? w2[i >> 1].y : w2[i >> 1].x;
-            const uint32_t q = flat ? 0u : (uint32_t)(int)(code_z(wv - c, P) + 3.5f);
+            const float adv = (i & 1) ? ad2[i >> 1].y : ad2[i >> 1].x;
+            const float dv = ((negm >> i) & 1u) ? -adv : adv;  // w - c
+            const uint32_t q = flat ? 0u : (uint32_t)(int)(code_z(dv, P) + 3.5f);
             q4[i >> 2] |= q << (8 * (i & 3));
             rv[i] = table[q];
         }
@@ -580,7 +815,7 @@ __global__ void __launch_bounds__(256, 2) k_recon_lut(const __grid_constant__ Lu
                 const uint32_t olo = __shfl_down_sync(0xffffffffu, lo, 1);
                 const uint32_t ohi = __shfl_down_sync(0xffffffffu, hi, 1);
                 if ((lane & 1) == 0) {
-                    uint32_t* dst = reinterpret_cast<uint32_t*>(T.codes) + b * 48 + (lane >> 1) * 3;
+                    uint32_t* dst = reinterpret_cast<uint32_t*>(T.codes) + (size_t)b * 48 + (lane >> 1) * 3;
                     stg_cs(dst, lo);
                     stg_cs(dst + 1, (hi & 0xFFFFu) | (olo << 16));
                     stg_cs(dst + 2, (olo >> 16) | (ohi << 16));
@@ -588,7 +823,7 @@ __global__ void __launch_bounds__(256, 2) k_recon_lut(const __grid_constant__ Lu
             }
         }
         if (lane == 0) {
-            stg_cs(reinterpret_cast<uint2*>(T.book + b * 8), make_uint2(bw0, bw1));
+            stg_cs(reinterpret_cast<uint2*>(T.book + (size_t)b * 8), make_uint2(bw0, bw1));
             if (T.idx) T.idx[b] = (uint8_t)kb;
         }
         __syncwarp();  // table and scratch are reused by the next block
