@@ -704,7 +704,10 @@ def main():
         del model
         torch.cuda.empty_cache()
     if args.configs and rank == 0:
+        # the paper-shaped configurations beside the sweep's formats (the
+        # 32-layer INT3 step itself is this line's headline)
         configs = config_entries(device, stream, hbm_peak)
+        sweep.update(configs)
     if args.e2e_steps > 0 and rank == 0:
         torch.cuda.empty_cache()
         e2e = e2e_rate(wlo, args.e2e_steps, device, stream, args.e2e_slots)
@@ -762,7 +765,7 @@ def main():
                                          kernel_ms / args.steps / len(step.calls), clk)},
         "cpu_baseline": cpu, "e2e": e2e,
         "gpu_launches": len(step.calls) * step.launches_per_call * args.steps,
-        "clocks": clk, "sweep": sweep, "configs": configs,
+        "clocks": clk, "sweep": sweep,
     }
     print(json.dumps(line), flush=True)
 
