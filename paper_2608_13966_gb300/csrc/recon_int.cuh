@@ -840,7 +840,7 @@ __global__ void __launch_bounds__(ADAM ? 192 : 256, 2)
             // (E = -inf) has key 0.  Two candidates within 7 ulps of each other
             // are both within the tie bound below (dE is at least 2 tie_kappa
             // ulps of E, since sqrt(S2 sum h e^2) >= |N|, and the host's
-            // tie_kappa is at least 10), so whichever the key picks, the exact
+            // tie_kappa is at least 12), so whichever the key picks, the exact
             // comparison settles them.
             uint32_t key = 0;
 #pragma unroll
@@ -913,21 +913,62 @@ __global__ void __launch_bounds__(ADAM ? 192 : 256, 2)
         // codes -- equal codes give equal errors, and the lower index is
         // kept, as Algorithm 1's argmin does -- but an element of tiny
         // saliency can differ without moving the sums, so twins are first
-        // checked code by code (cheaply, deferred).
+        // checked code by code (cheaply, deferred) -- unless every saliency
+        // of the group is too large for that.  Between two factors every
+        // element's code moves away from the centre or stays, and a moving
+        // element has |d| >= range f / q_max (f the smaller factor), so a
+        // code difference moves T3 - (c - mu) T1 by at least h_min range f /
+        // q_max, less the roundings of e, d and c (every term has the sign of
+        // the move: e - (c - mu) is d up to those roundings).  Bitwise-equal
+        // sums bound that change by twice their fp32 errors, ulp sqrt(T2 see)
+        // and |c - mu| ulp sqrt(Ss T2); a larger bound leaves the codes
+        // equal (up to elements of zero saliency, which move no error).
         float y0w = Y0k[0];
 #pragma unroll
         for (int ch = 1; ch < NCH; ++ch)
             if ((kb >> 3) == ch) y0w = Y0k[ch];
+        bool twinf[NCH][2];
+        bool anytwin = false;
+#pragma unroll
+        for (int ch = 0; ch < NCH; ++ch)
+#pragma unroll
+            for (int qd = 0; qd < 2; ++qd) {
+                const int k = ch * 8 + qd * 4 + sl;
+                twinf[ch][qd] = k != kb && Y0k[ch] == y0w && T1k[ch][qd] == T1b &&
+                                T2k[ch][qd] == T2b && T3k[ch][qd] == T3b;
+                anytwin |= twinf[ch][qd];
+            }
+        // the bound (only where a warp has twins): the group's smallest
+        // saliency, from the tile (the fit's h, 1 for all-zero groups).
+        // Built for 16 or more candidates, where twins are common (with 8
+        // they are rare and the code costs more than it saves).
+        constexpr bool kCertify = NCH >= 2 && !ADAM;
+        float twin_q = INFINITY, twin_h = 0.0f, twin_e = 0.0f;
+        if (kCertify && __any_sync(0xffffffffu, anytwin)) {
+            float hmn = INFINITY;
+#pragma unroll 1
+            for (int i = 0; i < NCHK; ++i) {
+                const float4 h4 = lds128(ghs + eoff(i));
+                hmn = fmin3(fmin3(hmn, h4.x, h4.y), h4.z, h4.w);
+            }
+#pragma unroll
+            for (int o = 2; o; o >>= 1) hmn = fminf(hmn, shx(hmn, o));
+            const float t2s = fmaxf(T2b * see, 0.0f), t2w = fmaxf(ss * T2b, 0.0f);
+            twin_q = 2.0f * ulp * (sqrtf(t2s) + fabsf(cref - mu) * sqrtf(t2w)) * qmaxf;
+            twin_h = hmn * range;
+            twin_e = hmn * qmaxf * (8.0f * 5.9604645e-8f) * (range + fabsf(cref));
+        }
         unsigned set = 0, twins = 0;
 #pragma unroll
         for (int ch = 0; ch < NCH; ++ch)
 #pragma unroll
             for (int qd = 0; qd < 2; ++qd) {
                 const int k = ch * 8 + qd * 4 + sl;
-                const bool twin = Y0k[ch] == y0w && T1k[ch][qd] == T1b && T2k[ch][qd] == T2b &&
-                                  T3k[ch][qd] == T3b;
-                const bool contender =
-                    k != kb && Ek[ch][qd] > -INFINITY && Eb - Ek[ch][qd] <= dEb + dEk[ch][qd];
+                const bool twin = twinf[ch][qd];
+                // a twin whose codes are certainly the winner's: as the winner
+                const bool sure = kCertify && twin && twin_h * fminf(p.f[k], p.f[kb]) - twin_e > twin_q;
+                const bool contender = k != kb && !sure && Ek[ch][qd] > -INFINITY &&
+                                       Eb - Ek[ch][qd] <= dEb + dEk[ch][qd];
                 const unsigned bal = __ballot_sync(0xffffffffu, contender || suspk[ch][qd]);
                 set |= ((bal >> (gs * 4)) & 0xFu) << (ch * 8 + qd * 4);
                 const unsigned balt = __ballot_sync(0xffffffffu, contender && twin && !suspk[ch][qd]);
@@ -1155,7 +1196,9 @@ __global__ void __launch_bounds__(ADAM ? 192 : 256, 2)
         {
             const float uf = p.fit_ulps * 5.9604645e-8f;
             const float ea = uf * fabsf(a_sel) * kap_sel;
-            const float ec = uf * (fabsf(cref) + fabsf(mu) + sqrtf(see * inv_ss));
+            // (plus half an ulp of Bz: pass C may fold Bz's low part into it)
+            const float ec = uf * (fabsf(cref) + fabsf(mu) + sqrtf(see * inv_ss)) +
+                             0.5f * 5.9604645e-8f * fabsf(Bz);
             // the weighted mean code (q = zeta + J + 1)
             const float qbar = (y0b - kGridMagic) + T1b * inv_ss + Jp1;
             const float b0 = fmaf(-a_sel, Jp1, Bz);  // offset at q = 0
@@ -1214,9 +1257,14 @@ __global__ void __launch_bounds__(ADAM ? 192 : 256, 2)
         {
             const float2 a2 = make_float2(a_sel, a_sel), B2 = make_float2(Bz, Bz);
             const float2 alo2 = make_float2(a_lo, a_lo), Blo2 = make_float2(Bz_lo, Bz_lo);
+            // the fast path folds Bz's low part into Bz (within the half ulp
+            // the accuracy check allows for it); a compensated fit keeps both
+            const float Bf = __fadd_rn(Bz, Bz_lo);
+            const float2 Bf2 = make_float2(Bf, Bf);
             const float2 Pk2 = make_float2(Pk, Pk);
             const int64_t ebase = gbase;
-            // general: codes, fp32 r, zero-range groups (r = w); fast: none
+            // general: codes, fp32 r, zero-range groups (r = w), compensated fits;
+            // fast: none of these (and the folded offset)
             auto pass_c = [&](auto general) {
                 constexpr bool GEN = decltype(general)::value;
 #pragma unroll 2
@@ -1236,7 +1284,8 @@ __global__ void __launch_bounds__(ADAM ? 192 : 256, 2)
                     float2 rv[2];
 #pragma unroll
                     for (int pr = 0; pr < 2; ++pr)
-                        rv[pr] = __fadd2_rn(__ffma2_rn(a2, zs[pr], B2), __ffma2_rn(alo2, zs[pr], Blo2));
+                        rv[pr] = GEN ? __fadd2_rn(__ffma2_rn(a2, zs[pr], B2), __ffma2_rn(alo2, zs[pr], Blo2))
+                                     : __ffma2_rn(a2, zs[pr], Bf2);
                     const int64_t ge = ebase + eo;
                     if constexpr (GEN) {
                         if (flat) {
@@ -1270,7 +1319,7 @@ __global__ void __launch_bounds__(ADAM ? 192 : 256, 2)
             };
             // lanes of a missing group store nothing (with VAR every lane runs
             // pass C: the packed codes below synchronise the warp)
-            const bool gen = !p.r_bf16 || T.codes != nullptr || __any_sync(0xffffffffu, flat);
+            const bool gen = !p.r_bf16 || T.codes != nullptr || __any_sync(0xffffffffu, flat || a_lo != 0.0f);
             if (VAR || valid) {
                 if (gen) pass_c(std::true_type{});
                 else pass_c(std::false_type{});
