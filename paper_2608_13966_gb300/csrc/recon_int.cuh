@@ -128,6 +128,11 @@ __device__ __forceinline__ void ff_reduce32(float& hi, float& lo)
         ff_acc(hi, lo, oh, ol);
         ff_norm(hi, lo);
     }
+    // the float-pair sum is not symmetric in its operands, so lanes can end
+    // one rounding apart: every lane takes lane 0's pair, so that decisions
+    // taken from it are the same across the warp
+    hi = __shfl_sync(0xffffffffu, hi, 0);
+    lo = __shfl_sync(0xffffffffu, lo, 0);
 }
 
 __device__ __forceinline__ bool ff_less(float ah, float al, float bh, float bl)

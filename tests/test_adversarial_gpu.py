@@ -7,7 +7,9 @@ estimate that decides the compensated fit):
 * ranges of a few ulps of the centre (a handful of distinct values);
 * saliencies spanning 1e-30 .. 1e3 inside one group;
 * exact duplicate weights (two or three distinct values a group);
-* 8-bit codes, groups of 256 and 32 candidates on Student-t(2) weights.
+* 8-bit codes, groups of 256 and 32 candidates on Student-t(2) weights;
+* INT2, groups of 64 and 16 candidates (where candidates with the winner's
+  sums are certified by the saliency floor or checked code by code).
 
 Every case runs through the C ABI (single-tensor and batch calls) and is
 checked with the same acceptance as the other parity tests (Algorithm 1,
@@ -22,6 +24,7 @@ from tests import checker
 from tests import gpu_harness as H
 
 CLIP8 = list(WL.CLIP_8)
+CLIP16 = list(WL.CLIP_16)
 CLIP32 = [round(1.0 - 0.025 * i, 3) for i in range(32)]
 
 
@@ -87,6 +90,13 @@ CASES = {
     "bits8_g256_k32_t2": (heavy_t2, 8, 256, CLIP32),
     "bits2_g64_k32_t2": (heavy_t2, 2, 64, CLIP32),
     "bits4_g32_k8_far": (far_from_zero, 4, 32, CLIP8),
+    # 16 candidates: equal-sum candidates are taken as the winner's without a
+    # code check when the group's smallest saliency allows it; these inputs
+    # have tiny saliencies (the check runs) and repeated values (many equal
+    # codes)
+    "bits2_g64_k16_span": (saliency_span, 2, 64, CLIP16),
+    "bits2_g64_k16_dup": (duplicates, 2, 64, CLIP16),
+    "bits2_g64_k16_t2": (heavy_t2, 2, 64, CLIP16),
 }
 
 
