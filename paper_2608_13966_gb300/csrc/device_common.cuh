@@ -157,4 +157,23 @@ __device__ __forceinline__ void stg_cs(uint32_t* p, uint32_t v)
 // integer (round-to-nearest-even) in the low mantissa bits.
 constexpr float kRoundMagic = 12582912.0f;
 
+// Saliency sums near the bottom of fp32's range: the reconstruction is
+// invariant to a common scale of h (Algorithm 1's argmin and Eq. 4's fit), so
+// a group (or block) whose sum of h is below 2^-40 is fitted with h scaled by a
+// power of two s = s1 s2, exactly, chosen so that x s lies in [1, 2) for the
+// sum x: the products of its moment sums then stay normal.  Two factors,
+// because s can exceed the largest float power of two 2^127.
+constexpr float kTinySaliency = 9.094947e-13f;  // 2^-40
+
+__device__ __forceinline__ void tiny_scale(float x, float& s1, float& s2)
+{
+    s1 = 1.0f;
+    if (x < 1.17549435e-38f) {  // denormal: first 2^64
+        s1 = 18446744073709551616.0f;
+        x *= s1;
+    }
+    const int e = (int)((__float_as_uint(x) >> 23) & 0xFFu) - 127;  // x = 1.f 2^e
+    s2 = __uint_as_float((uint32_t)(127 - e) << 23);
+}
+
 }  // namespace quasar

@@ -687,6 +687,37 @@ __global__ void __launch_bounds__(ADAM ? 192 : 256, 2)
                 for (int i = 0; i < NCHK; ++i)
                     *reinterpret_cast<float4*>(ghs + eoff(i)) = make_float4(1.0f, 1.0f, 1.0f, 1.0f);
         }
+        // a sum of saliencies near the bottom of the fp32 range: h scaled by
+        // a power of two in the tile, and its sums taken again
+        const bool h_tiny = !h_one && ss < kTinySaliency;
+        if (__any_sync(0xffffffffu, h_tiny)) {
+            float s1 = 1.0f, s2 = 1.0f;
+            tiny_scale(ss, s1, s2);
+            float2 SS2 = make_float2(0.0f, 0.0f), SW = SS2;
+            if (h_tiny) {
+#pragma unroll 1
+                for (int i = 0; i < NCHK; ++i) {
+                    const float4 w4 = lds128(gws + eoff(i));
+                    float4 h4 = lds128(ghs + eoff(i));
+                    h4 = make_float4(h4.x * s1 * s2, h4.y * s1 * s2, h4.z * s1 * s2, h4.w * s1 * s2);
+                    *reinterpret_cast<float4*>(ghs + eoff(i)) = h4;
+                    const float2 hA = make_float2(h4.x, h4.y), hB = make_float2(h4.z, h4.w);
+                    SS2 = __fadd2_rn(SS2, __fadd2_rn(hA, hB));
+                    SW = __ffma2_rn(hA, make_float2(w4.x, w4.y), SW);
+                    SW = __ffma2_rn(hB, make_float2(w4.z, w4.w), SW);
+                }
+            }
+            float ss2 = SS2.x + SS2.y, sw2 = SW.x + SW.y;
+#pragma unroll
+            for (int o = 2; o; o >>= 1) {
+                ss2 += shx(ss2, o);
+                sw2 += shx(sw2, o);
+            }
+            if (h_tiny) {
+                ss = ss2;
+                sw = sw2;
+            }
+        }
         // the gradient region becomes the transpose scratch: every lane is
         // past pass A, and the h rewrites above are visible to all lanes
         __syncwarp();
@@ -819,8 +850,10 @@ __global__ void __launch_bounds__(ADAM ? 192 : 256, 2)
                 const float zbar = T1 * inv_ss;
                 const float D = T2 - T1 * zbar;
                 const float N = T3 - T1 * ebar;
-                const bool susp = !(D > 1e-3f * T2);
                 const float a = __fdividef(N, D);
+                // a near-degenerate code variance, or a non-finite E (sums
+                // near the denormal range): left to the exact comparison
+                const bool susp = !(D > 1e-3f * T2) || !(N * a < INFINITY);
                 const float E = susp ? 0.0f : N * a;
                 const float s2e = fmaxf(T2 * see, 1e-37f);
                 const float dN = ulp * (s2e * rsqrtf(s2e) * 1.001f + fabsf(T1 * ebar));

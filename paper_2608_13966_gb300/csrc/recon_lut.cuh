@@ -179,7 +179,7 @@ __global__ void __launch_bounds__(256, 2) k_recon_lut(const __grid_constant__ Lu
     uint32_t* camb = reinterpret_cast<uint32_t*>(cbnd + kMaxClip);      // [32]
     float* table = reinterpret_cast<float*>(scr + kLutSumsBytes + kLutCandBytes);  // [8]
     // the block's per-sign sums of h and h |d|, and sum h d^2
-    float* bconst = table + 8;  // [5]
+    float* bconst = table + 8;  // [7]: also the block's sum of h and its range
     uint64_t* bars = reinterpret_cast<uint64_t*>(smem + (size_t)nwarps * S * p.stage_bytes +
                                                  (size_t)nwarps * kLutScratchBytes) +
                      warp * (S + 1);
@@ -380,6 +380,8 @@ __global__ void __launch_bounds__(256, 2) k_recon_lut(const __grid_constant__ Lu
                 bconst[2] = up;
                 bconst[3] = un;
                 bconst[4] = sd;
+                bconst[5] = ss;
+                bconst[6] = range;
             }
         }
 
@@ -481,11 +483,16 @@ __global__ void __launch_bounds__(256, 2) k_recon_lut(const __grid_constant__ Lu
                     dm = dq + 3.0f * kU * q + 2.0f * kU * fabsf(mean);
                 }
                 const uint32_t cb = e4m3_encode(mean);
-                const bool amb = e4m3_encode(mean - dm) != e4m3_encode(mean + dm);
+                // an index whose H is not clearly above its error bound may be
+                // empty or may hold weights of tiny saliency lost to the
+                // differences: its entry is undecided unless nothing on its
+                // side reaches its level, and its whole term is bounded below
+                const bool thin = !(H > dA) && Am + Am1 > 0.0f;
+                const bool amb = thin || e4m3_encode(mean - dm) != e4m3_encode(mean + dm);
                 const float dc = e4m3_decode(cb) - mean;
                 // the index's error: H (C - mean)^2 - X^2 / H (the scatter
                 // term sum h d^2 is added once below)
-                const float Sj = H > 0.0f ? fmaf(H * dc, dc, -X * q) : 0.0f;
+                const float Sj = H > 0.0f && !thin ? fmaf(H * dc, dc, -X * q) : 0.0f;
                 float bj = dA * dc * dc + 2.0f * H * fabsf(dc) * dm + 3.0f * kU * H * dc * dc + dX * q +
                            X * dq + 2.0f * kU * X * q;
                 if (amb) {  // the other rounding moves the entry by at most this much
@@ -493,6 +500,7 @@ __global__ void __launch_bounds__(256, 2) k_recon_lut(const __grid_constant__ Lu
                     const float c2 = e4m3_decode(e4m3_encode(mean + dm)) - mean;
                     bj += H * fabsf(c2 - c1) * (fabsf(c1) + fabsf(c2) + 2.0f * dm);
                 }
+                bj = thin ? 2.0f * (dA + fabsf(H)) * bconst[6] * bconst[6] : bj;
                 const bool live = lane < 16;
                 float E = live ? Sj : 0.0f, dE = live ? bj : 0.0f, aE = live ? fabsf(Sj) : 0.0f;
                 uint32_t wb = live ? cb << (8 * (lane & 3)) : 0u;
@@ -541,6 +549,19 @@ __global__ void __launch_bounds__(256, 2) k_recon_lut(const __grid_constant__ Lu
             unsigned set = __ballot_sync(0xffffffffu, lane < K && lane != kb && Ek - Eb <= dEk + dEb);
             if (p.stats && lane == 0 && camb[kb]) atomicAdd(&p.stats[2], 1u);
 
+            // a block whose sum of saliencies is near the bottom of the fp32
+            // range: its fast sums are not to be trusted; h is scaled by a
+            // power of two and every candidate and entry is settled below
+            // (ts1 ts2: that power of two, applied where the settling steps
+            // read h; 1 otherwise)
+            float ts1 = 1.0f, ts2 = 1.0f;
+            if (bconst[5] > 0.0f && bconst[5] < kTinySaliency) {
+                tiny_scale(bconst[5], ts1, ts2);
+                set = (K >= 32) ? 0xFFFFFFFFu : ((1u << K) - 1u);
+                if (lane < K) camb[lane] = 0xFFu;
+                __syncwarp();
+            }
+
             // index (0..7) of element i for the grid of P
             auto index_of = [&](int i, float P) {
                 const float a = (i & 1) ? ad2[i >> 1].y : ad2[i >> 1].x;
@@ -563,7 +584,7 @@ __global__ void __launch_bounds__(256, 2) k_recon_lut(const __grid_constant__ Lu
 #pragma unroll
                     for (int i = 0; i < 16; ++i) {
                         if (index_of(i, P) == j) {
-                            const float hv = (i & 1) ? hp2[i >> 1].y + hn2[i >> 1].y : hp2[i >> 1].x + hn2[i >> 1].x;
+                            const float hv = ((i & 1) ? hp2[i >> 1].y + hn2[i >> 1].y : hp2[i >> 1].x + hn2[i >> 1].x) * ts1 * ts2;
                             const float av = (i & 1) ? ad2[i >> 1].y : ad2[i >> 1].x;
                             Hs += hv;
                             Xs = fmaf(hv, av, Xs);
@@ -576,14 +597,19 @@ __global__ void __launch_bounds__(256, 2) k_recon_lut(const __grid_constant__ Lu
                     }
                     Hs = __shfl_sync(0xffffffffu, Hs, 0);
                     Xs = __shfl_sync(0xffffffffu, Xs, 0);
-                    if (!(Hs > 0.0f)) return false;
-                    const float q = Xs / Hs;
-                    const float mean = fmaf(j >= 4 ? 1.0f : -1.0f, q, c);
-                    // two sums (24 ulps each), the quotient, w - c (an ulp a
-                    // term), the mean's sum
-                    const float dm = 52.0f * kU * q + 2.0f * kU * fabsf(mean);
-                    if (e4m3_encode(mean - dm) != e4m3_encode(mean + dm)) return false;
-                    const uint32_t cbj = e4m3_encode(mean);
+                    uint32_t cbj;
+                    if (!(Hs > 0.0f)) {
+                        // no weight of nonzero saliency: the grid point
+                        cbj = e4m3_encode(fmaf((float)j - 3.5f, __fdividef(1.0f, P), c));
+                    } else {
+                        const float q = Xs / Hs;
+                        const float mean = fmaf(j >= 4 ? 1.0f : -1.0f, q, c);
+                        // two sums (24 ulps each), the quotient, w - c (an ulp
+                        // a term), the mean's sum
+                        const float dm = 52.0f * kU * q + 2.0f * kU * fabsf(mean);
+                        if (e4m3_encode(mean - dm) != e4m3_encode(mean + dm)) return false;
+                        cbj = e4m3_encode(mean);
+                    }
                     if (j < 4) w0 = (w0 & ~(0xFFu << (8 * j))) | (cbj << (8 * j));
                     else w1 = (w1 & ~(0xFFu << (8 * (j - 4)))) | (cbj << (8 * (j - 4)));
                 }
@@ -629,7 +655,7 @@ __global__ void __launch_bounds__(256, 2) k_recon_lut(const __grid_constant__ Lu
                         float acc = 0.0f;
 #pragma unroll
                         for (int i = 0; i < 16; ++i) {
-                            const float hv = (i & 1) ? hp2[i >> 1].y + hn2[i >> 1].y : hp2[i >> 1].x + hn2[i >> 1].x;
+                            const float hv = ((i & 1) ? hp2[i >> 1].y + hn2[i >> 1].y : hp2[i >> 1].x + hn2[i >> 1].x) * ts1 * ts2;
                             const float df = table[index_of(i, P)] - xwv[i];
                             acc = fmaf(hv * df, df, acc);
                         }
@@ -678,7 +704,9 @@ __global__ void __launch_bounds__(256, 2) k_recon_lut(const __grid_constant__ Lu
                     xw[2 * i + 1] = make_float2(w4.z, w4.w);
                 }
 #pragma unroll
-                for (int t = 0; t < 8; ++t) xh[t] = __fadd2_rn(hp2[t], hn2[t]);  // one of the two is 0
+                for (int t = 0; t < 8; ++t)  // one of the two is 0
+                    xh[t] = __fmul2_rn(__fmul2_rn(__fadd2_rn(hp2[t], hn2[t]), make_float2(ts1, ts1)),
+                                       make_float2(ts2, ts2));
                 float best_h = 0.0f, best_l = 0.0f;
                 int best_k = -1;
                 uint32_t best_w0 = 0, best_w1 = 0;

@@ -251,9 +251,19 @@ __global__ void __launch_bounds__(256) k_recon_nvfp4(const __grid_constant__ Nvf
             amax_b = fmaxf(amax_b, fmaxf(aw2[t].x, aw2[t].y));
             SS = __fadd2_rn(SS, h2[t]);
         }
-        if (SS.x + SS.y == 0.0f) {  // all saliencies zero: h = 1
+        const float ssb = SS.x + SS.y;
+        if (__any_sync(0xffffffffu, ssb < kTinySaliency)) {
+            if (ssb == 0.0f) {  // all saliencies zero: h = 1
 #pragma unroll
-            for (int t = 0; t < 8; ++t) h2[t] = make_float2(1.0f, 1.0f);
+                for (int t = 0; t < 8; ++t) h2[t] = make_float2(1.0f, 1.0f);
+            } else if (ssb < kTinySaliency) {
+                // near the bottom of the fp32 range: h scaled by a power of two
+                float s1, s2;
+                tiny_scale(ssb, s1, s2);
+                const float2 s12 = make_float2(s1, s1), s22 = make_float2(s2, s2);
+#pragma unroll
+                for (int t = 0; t < 8; ++t) h2[t] = __fmul2_rn(__fmul2_rn(h2[t], s12), s22);
+            }
         }
         const bool zero = !(amax_b > 0.0f);
         const float P1 = zero ? 0.0f : __fdiv_rn(6.0f, amax_b);  // 1/sigma at f = 1

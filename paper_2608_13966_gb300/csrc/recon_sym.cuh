@@ -228,6 +228,21 @@ __global__ void __launch_bounds__(256, 2) k_recon_sym(const __grid_constant__ In
                 for (int i = 0; i < NCHK; ++i)
                     *reinterpret_cast<float4*>(hs + gs * G + i * 32 + sl * 4) = make_float4(1.0f, 1.0f, 1.0f, 1.0f);
         }
+        // a sum of saliencies near the bottom of the fp32 range: h scaled by
+        // a power of two
+        const bool h_tiny = ss > 0.0f && ss < kTinySaliency;
+        if (__any_sync(0xffffffffu, h_tiny)) {
+            if (h_tiny) {
+                float s1, s2;
+                tiny_scale(ss, s1, s2);
+#pragma unroll 1
+                for (int i = 0; i < NCHK; ++i) {
+                    float4* hp = reinterpret_cast<float4*>(hs + gs * G + i * 32 + sl * 4);
+                    const float4 h4 = *hp;
+                    *hp = make_float4(h4.x * s1 * s2, h4.y * s1 * s2, h4.z * s1 * s2, h4.w * s1 * s2);
+                }
+            }
+        }
         __syncwarp();
         const bool flat = !(amax > 0.0f);
         const float R = flat ? 0.0f : __fdividef(Q, amax);  // P = R / f

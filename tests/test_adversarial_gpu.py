@@ -66,6 +66,16 @@ def saliency_span(seed, n_groups, G):
     return w, h
 
 
+def denormal_saliency(seed, n_groups, G):
+    """t4 weights; saliency 10^u, u uniform in [-45, -38]: denormal and
+    barely normal fp32 values, every group's sum far below the normal range
+    of its squares (an EMA of squared gradients that decayed for long)."""
+    rng = np.random.default_rng(seed)
+    w = (0.02 * rng.standard_t(4, n_groups * G)).astype(np.float32)
+    h = (10.0 ** rng.uniform(-45.0, -38.0, n_groups * G)).astype(np.float32)
+    return w, h
+
+
 def duplicates(seed, n_groups, G):
     """Two or three distinct values a group, each repeated."""
     rng = np.random.default_rng(seed)
@@ -97,6 +107,8 @@ CASES = {
     "bits2_g64_k16_span": (saliency_span, 2, 64, CLIP16),
     "bits2_g64_k16_dup": (duplicates, 2, 64, CLIP16),
     "bits2_g64_k16_t2": (heavy_t2, 2, 64, CLIP16),
+    "bits3_g128_k8_denorm": (denormal_saliency, 3, 128, CLIP8),
+    "bits2_g64_k16_denorm": (denormal_saliency, 2, 64, CLIP16),
 }
 
 
@@ -135,9 +147,10 @@ def test_int_adversarial(oracle, case, r_dtype):
 
 
 @pytest.mark.gpu
-@pytest.mark.parametrize("case", ["saliency_span", "duplicates", "heavy_t2"])
+@pytest.mark.parametrize("case", ["saliency_span", "duplicates", "heavy_t2", "denormal_saliency"])
 def test_nvfp4_adversarial(oracle, case):
-    gen = {"saliency_span": saliency_span, "duplicates": duplicates, "heavy_t2": heavy_t2}[case]
+    gen = {"saliency_span": saliency_span, "duplicates": duplicates, "heavy_t2": heavy_t2,
+           "denormal_saliency": denormal_saliency}[case]
     n_rows = 40
     w, h = gen(23, n_rows, 256)
     w_t = torch.tensor(w, device="cuda").reshape(n_rows, 256)
@@ -145,3 +158,41 @@ def test_nvfp4_adversarial(oracle, case):
     rep, ema = H.run_nvfp4(oracle, w_t, None, v_t, clip=CLIP8)
     _assert(rep, case)
     _assert(ema, case)
+
+
+@pytest.mark.gpu
+@pytest.mark.parametrize("case", ["saliency_span", "duplicates", "denormal_saliency"])
+def test_lut_adversarial(oracle, case):
+    """The Rubin lookup table (App. B) on 8x64 blocks of the same inputs."""
+    gen = {"saliency_span": saliency_span, "duplicates": duplicates,
+           "denormal_saliency": denormal_saliency}[case]
+    rows, cols = 24, 320  # 15 blocks
+    w, h = gen(29, rows * cols // 64, 64)
+    w_t = torch.tensor(w, device="cuda").reshape(rows, cols)
+    v_t = torch.tensor(h, device="cuda").reshape(rows, cols)
+    out = api.recon_lut_batch([(w_t, None, v_t)], clip=CLIP8, codes=True, r_dtype=torch.float32)[0]
+    torch.cuda.synchronize()
+    w2, h2 = w.reshape(rows, cols), h.reshape(rows, cols)
+    O = oracle.recon_lut(w2, h2, CLIP8)
+    gpu = {"r": H._host(out["r"]), "book": out["book"].cpu().numpy(),
+           "codes": out["codes"].cpu().numpy(), "idx": out["cand_idx"].cpu().numpy()}
+    _assert(checker.check_lut(oracle, w2, h2, CLIP8, O, gpu), case)
+
+
+@pytest.mark.gpu
+@pytest.mark.parametrize("case", ["saliency_span", "denormal_saliency", "far_from_zero"])
+def test_sym_adversarial(oracle, case):
+    """Symmetric codes (Sec. 4.1.2's closed form) on the same inputs."""
+    gen = {"saliency_span": saliency_span, "denormal_saliency": denormal_saliency,
+           "far_from_zero": far_from_zero}[case]
+    n_groups, G, bits = 149, 128, 4
+    w, h = gen(31, n_groups, G)
+    w_t = torch.tensor(w, device="cuda").reshape(n_groups, G)
+    v_t = torch.tensor(h, device="cuda").reshape(n_groups, G)
+    out = api.recon_int_batch([(w_t, None, v_t)], bits=bits, group_size=G, clip=CLIP8, codes=True,
+                              symmetric=True, r_dtype=torch.float32)[0]
+    torch.cuda.synchronize()
+    O = oracle.recon_sym(w, h, G, bits, CLIP8)
+    gpu = {"r": H._host(out["r"]), "a": out["a"].cpu().numpy(), "b": out["b"].cpu().numpy(),
+           "codes": out["codes"].cpu().numpy().ravel(), "idx": out["cand_idx"].cpu().numpy()}
+    _assert(checker.check_sym(oracle, w, h, bits, CLIP8, O, gpu, G, False), case)
