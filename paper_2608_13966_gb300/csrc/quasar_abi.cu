@@ -66,7 +66,7 @@ struct Tuning {
     float tie_kappa = kTieKappaMin;  // NVFP4 tie bound, in ulps
     float tie_scale = kTieScaleMin;  // multiplier of the integer kernel's summation-depth bound
     float fit_ulps = kFitUlpsMin;
-    int hoist = 1;             // 0: never the hoisted-clamp integer kernel
+    int hoist = 1;             // 0: the integer kernel's code-clamp sets hold one candidate
 };
 
 // A float from the environment, clamped to [lo, hi] (non-numbers give lo).

@@ -2,16 +2,19 @@
 // code assignment, Eq. 4 weighted least-squares dequantizer, Eq. 3 weighted
 // error; saliency EMA of Sec. 4.1.1 / App. A.2), one fused pass over HBM.
 //
-// Work decomposition.  A "unit" is 4 consecutive groups; one warp owns a unit
-// at a time, 8 lanes per group, EPL = G/8 elements per lane.  Lane sl of a
-// group handles elements {32*i + 4*sl + j : i < EPL/4, j < 4}, so every
-// 16-byte shared-memory access of the warp is bank-conflict free and every
-// global store covers whole 128-byte segments.  Each warp runs its own ring
-// of `stages` shared-memory tiles filled by 1-D TMA bulk copies
-// (cp.async.bulk + mbarrier), so w, g and v are read from HBM exactly once,
-// and the loads of later units overlap the arithmetic of the current one.
-// The tile stays in shared memory while the unit is processed; the passes
-// below stream it from there.  The grid is persistent.
+// Work decomposition.  A "unit" is 8 consecutive groups; one warp owns a unit
+// at a time, 4 lanes per group, EPL = G/4 elements per lane.  Lane sl of
+// group gs holds the group's 16-byte chunks {i ^ swz : i < EPL/4} at element
+// offset 4 sl within each 16-element span (swz a per-group XOR, so that the
+// groups one shared-memory access phase covers hit different banks).  The
+// CTA runs one ring of tile slots (one unit each) filled by 1-D TMA bulk
+// copies (cp.async.bulk + mbarrier); each slot carries the sequence number of
+// the unit loading into it, warp j takes the CTA's units j, j + warps, ...
+// and, done with a tile, issues the copy of the unit that many slots ahead
+// into the same slot.  w, g and v are read from HBM exactly once, and the
+// loads of later units overlap the arithmetic of the current ones.  After
+// pass A the tile's gradient region is the warp's transpose scratch.  The
+// grid is persistent.
 //
 // Codes.  With d = (w - min) - rho (the offset from the group's centre,
 // formed without rounding the centre itself: w - min and the half range are
@@ -35,8 +38,8 @@
 //           (the code of the weighted mean, from mu): S1 = sum h (zeta -
 //           zeta0), S2 = sum h (zeta - zeta0)^2, S3 = sum h (zeta - zeta0) e,
 //           e = w - mu (plus the candidate-independent sum h e, sum h e^2);
-//   reduce  the 8 lanes' partial sums are transposed through shared memory
-//           so that lane sl owns candidate sl of the chunk;
+//   reduce  the 4 lanes' partial sums are transposed through the scratch so
+//           that lane sl owns candidate sl of each 4-candidate quad;
 //   select  D = S2 - S1^2/Ss, N = S3 - S1*Se/Ss: the weighted error of
 //           candidate k is C - N^2/D with C common, so argmin error =
 //           argmax E = N^2/D; the winner's fit is a = N/D with the offset
@@ -49,7 +52,7 @@
 // is too small to trust) are re-evaluated exactly, and fits whose fp32
 // rounding could miss the output tolerance are recomputed in compensated
 // (float-float) arithmetic.  Both are rare; they are deferred to the end of
-// the unit and done by the whole warp on one group at a time.
+// the unit's selection and done by the whole warp on one group at a time.
 #pragma once
 
 #include <type_traits>
