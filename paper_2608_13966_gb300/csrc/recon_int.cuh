@@ -419,7 +419,10 @@ __global__ void __launch_bounds__(ADAM ? 192 : 256, 2)
     k_recon_int(const __grid_constant__ IntLaunch<MAXT> Lp)
 {
     static_assert(SS == 1 || SS == 2 || SS == 4, "clamp sets of 1, 2 or 4 candidates");
-    constexpr int NS = 4 / SS;  // clamp sets per quad of candidates
+    // candidates a sweep of pass B over the tile: all 8 of the chunk with
+    // one chunk (the loads, offsets and loop shared by 8), a quad with more
+    // (whose other live state leaves no room for 8 sets of sums)
+    constexpr int QW = NCH == 1 ? 8 : 4;
     const IntParams& p = Lp.p;
     constexpr int G = EPL * kIntLanes;
     constexpr int UNIT = kIntGroups * G;
@@ -747,9 +750,9 @@ __global__ void __launch_bounds__(ADAM ? 192 : 256, 2)
         const float dmu = centred(mu, -mn, -rho);
 
         // ---- pass B + reduction + candidate errors, 8 candidates a chunk,
-        // 4 (a quad) a sweep over the tile.  Codes from d = (w - mn) - rho;
-        // moments about the chunk's centre code zeta0 and, for S3, e = w - mu.
-        // Lane sl owns candidates 8 ch + 4 qd + sl.
+        // QW a sweep over the tile.  Codes from d = (w - mn) - rho; moments
+        // about the chunk's centre code zeta0 and, for S3, e = w - mu.  Lane
+        // sl owns candidates 8 ch + 4 qd + sl.
         float Ek[NCH][2], dEk[NCH][2], T1k[NCH][2], T2k[NCH][2], T3k[NCH][2], Y0k[NCH];
         bool suspk[NCH][2];
         float se = 0.0f, see = 0.0f;
@@ -762,21 +765,21 @@ __global__ void __launch_bounds__(ADAM ? 192 : 256, 2)
             float2 SE = make_float2(0.0f, 0.0f), SEE = make_float2(0.0f, 0.0f);
             float4 xq[2];
 #pragma unroll
-            for (int qd = 0; qd < 2; ++qd) {
-                const int kq = ch * 8 + qd * 4;
-                float2 A1[4], A2[4], A3[4];
+            for (int sw = 0; sw < 8 / QW; ++sw) {
+                const int kq = ch * 8 + sw * QW;
+                float2 A1[QW], A2[QW], A3[QW];
 #pragma unroll
-                for (int kk = 0; kk < 4; ++kk) A1[kk] = A2[kk] = A3[kk] = make_float2(0.0f, 0.0f);
-                if ((ch == 0 && qd == 0) || kq < p.n_clip) {
-                    float2 P2[4];
+                for (int kk = 0; kk < QW; ++kk) A1[kk] = A2[kk] = A3[kk] = make_float2(0.0f, 0.0f);
+                if ((ch == 0 && sw == 0) || kq < p.n_clip) {
+                    float2 P2[QW];
 #pragma unroll
-                    for (int kk = 0; kk < 4; ++kk) {
+                    for (int kk = 0; kk < QW; ++kk) {
                         const float P = R * p.invf[kq + kk];
                         P2[kk] = make_float2(P, P);
                     }
-                    float cp[NS];
+                    float cp[QW / SS];
 #pragma unroll
-                    for (int s = 0; s < NS; ++s) cp[s] = p.cap[kq + s * SS] * range;
+                    for (int s = 0; s < QW / SS; ++s) cp[s] = p.cap[kq + s * SS] * range;
 // rolled: a compact unit loop keeps the careful paths' code from evicting it
 // from the instruction cache when they run
 #pragma unroll 1
@@ -790,18 +793,18 @@ __global__ void __launch_bounds__(ADAM ? 192 : 256, 2)
                             const float2 h = pr ? make_float2(h4.z, h4.w) : make_float2(h4.x, h4.y);
                             const float2 d = __fadd2_rn(__fadd2_rn(wv, nmn2), nrho2);
                             const float2 ev = __fadd2_rn(wv, nmu2);
-                            if (ch == 0 && qd == 0) {
+                            if (ch == 0 && sw == 0) {
                                 const float2 he = __fmul2_rn(h, ev);
                                 SE = __fadd2_rn(SE, he);
                                 SEE = __ffma2_rn(he, ev, SEE);
                             }
-                            float2 dc[NS];
+                            float2 dc[QW / SS];
 #pragma unroll
-                            for (int s = 0; s < NS; ++s)
+                            for (int s = 0; s < QW / SS; ++s)
                                 dc[s] = make_float2(fminf(fmaxf(d.x, -cp[s]), cp[s]),
                                                     fminf(fmaxf(d.y, -cp[s]), cp[s]));
 #pragma unroll
-                            for (int kk = 0; kk < 4; ++kk) {
+                            for (int kk = 0; kk < QW; ++kk) {
                                 const float2 y = __ffma2_rd(dc[kk / SS], P2[kk], Mg2);
                                 const float2 zc = __fadd2_rn(y, nY02);  // zeta - zeta0, exact
                                 const float2 t2 = __fmul2_rn(h, zc);
@@ -812,26 +815,32 @@ __global__ void __launch_bounds__(ADAM ? 192 : 256, 2)
                         }
                     }
                 }
-                // transpose through the scratch: lane L writes row L (its sums
-                // of candidate kk in 16-byte column kk ^ ((L >> 1) & 3)), and
-                // lane (gs, sl) sums column sl of its group's 4 rows (each
-                // group starting at another row, so that an access phase's two
-                // groups read rows of both parities: no bank conflicts)
-                __syncwarp();
+                // transpose each quad through the scratch: lane L writes row L
+                // (its sums of candidate kk in 16-byte column kk ^ ((L >> 1) &
+                // 3)), and lane (gs, sl) sums column sl of its group's 4 rows
+                // (each group starting at another row, so that an access
+                // phase's two groups read rows of both parities: no bank
+                // conflicts)
 #pragma unroll
-                for (int kk = 0; kk < 4; ++kk)
-                    *reinterpret_cast<float4*>(red + lane * 16 + ((kk ^ ((lane >> 1) & 3)) << 2)) =
-                        make_float4(A1[kk].x + A1[kk].y, A2[kk].x + A2[kk].y, A3[kk].x + A3[kk].y, 0.0f);
-                __syncwarp();
-                float4 x[4];
+                for (int q4 = 0; q4 < QW / 4; ++q4) {
+                    __syncwarp();
 #pragma unroll
-                for (int j = 0; j < 4; ++j) {
-                    const int row = gs * 4 + ((j + gs) & 3);
-                    x[j] = *reinterpret_cast<const float4*>(red + row * 16 + ((sl ^ ((row >> 1) & 3)) << 2));
+                    for (int kk = 0; kk < 4; ++kk) {
+                        const int c = q4 * 4 + kk;
+                        *reinterpret_cast<float4*>(red + lane * 16 + ((kk ^ ((lane >> 1) & 3)) << 2)) =
+                            make_float4(A1[c].x + A1[c].y, A2[c].x + A2[c].y, A3[c].x + A3[c].y, 0.0f);
+                    }
+                    __syncwarp();
+                    float4 x[4];
+#pragma unroll
+                    for (int j = 0; j < 4; ++j) {
+                        const int row = gs * 4 + ((j + gs) & 3);
+                        x[j] = *reinterpret_cast<const float4*>(red + row * 16 + ((sl ^ ((row >> 1) & 3)) << 2));
+                    }
+                    xq[sw * (QW / 4) + q4] = make_float4((x[0].x + x[1].x) + (x[2].x + x[3].x),
+                                                         (x[0].y + x[1].y) + (x[2].y + x[3].y),
+                                                         (x[0].z + x[1].z) + (x[2].z + x[3].z), 0.0f);
                 }
-                xq[qd] = make_float4((x[0].x + x[1].x) + (x[2].x + x[3].x),
-                                     (x[0].y + x[1].y) + (x[2].y + x[3].y),
-                                     (x[0].z + x[1].z) + (x[2].z + x[3].z), 0.0f);
             }
             if (ch == 0) {
                 se = SE.x + SE.y;
@@ -1000,21 +1009,46 @@ __global__ void __launch_bounds__(ADAM ? 192 : 256, 2)
             twin_e = hmn * qmaxf * (8.0f * 5.9604645e-8f) * (range + fabsf(cref));
         }
         unsigned set = 0, twins = 0;
+        if constexpr (!kCertify) {
+            // contenders first; the twins among them only where a warp has any
+            bool cont[NCH][2];
 #pragma unroll
-        for (int ch = 0; ch < NCH; ++ch)
+            for (int ch = 0; ch < NCH; ++ch)
 #pragma unroll
-            for (int qd = 0; qd < 2; ++qd) {
-                const int k = ch * 8 + qd * 4 + sl;
-                const bool twin = twinf[ch][qd];
-                // a twin whose codes are certainly the winner's: as the winner
-                const bool sure = kCertify && twin && twin_h * fminf(p.f[k], p.f[kb]) - twin_e > twin_q;
-                const bool contender = k != kb && !sure && Ek[ch][qd] > -INFINITY &&
-                                       Eb - Ek[ch][qd] <= dEb + dEk[ch][qd];
-                const unsigned bal = __ballot_sync(0xffffffffu, contender || suspk[ch][qd]);
-                set |= ((bal >> (gs * 4)) & 0xFu) << (ch * 8 + qd * 4);
-                const unsigned balt = __ballot_sync(0xffffffffu, contender && twin && !suspk[ch][qd]);
-                twins |= ((balt >> (gs * 4)) & 0xFu) << (ch * 8 + qd * 4);
+                for (int qd = 0; qd < 2; ++qd) {
+                    const int k = ch * 8 + qd * 4 + sl;
+                    cont[ch][qd] = k != kb && Ek[ch][qd] > -INFINITY &&
+                                   Eb - Ek[ch][qd] <= dEb + dEk[ch][qd];
+                    const unsigned bal = __ballot_sync(0xffffffffu, cont[ch][qd] || suspk[ch][qd]);
+                    set |= ((bal >> (gs * 4)) & 0xFu) << (ch * 8 + qd * 4);
+                }
+            if (__any_sync(0xffffffffu, set != 0u)) {
+#pragma unroll
+                for (int ch = 0; ch < NCH; ++ch)
+#pragma unroll
+                    for (int qd = 0; qd < 2; ++qd) {
+                        const unsigned balt =
+                            __ballot_sync(0xffffffffu, cont[ch][qd] && twinf[ch][qd] && !suspk[ch][qd]);
+                        twins |= ((balt >> (gs * 4)) & 0xFu) << (ch * 8 + qd * 4);
+                    }
             }
+        } else {
+#pragma unroll
+            for (int ch = 0; ch < NCH; ++ch)
+#pragma unroll
+                for (int qd = 0; qd < 2; ++qd) {
+                    const int k = ch * 8 + qd * 4 + sl;
+                    const bool twin = twinf[ch][qd];
+                    // a twin whose codes are certainly the winner's: as the winner
+                    const bool sure = twin && twin_h * fminf(p.f[k], p.f[kb]) - twin_e > twin_q;
+                    const bool contender = k != kb && !sure && Ek[ch][qd] > -INFINITY &&
+                                           Eb - Ek[ch][qd] <= dEb + dEk[ch][qd];
+                    const unsigned bal = __ballot_sync(0xffffffffu, contender || suspk[ch][qd]);
+                    set |= ((bal >> (gs * 4)) & 0xFu) << (ch * 8 + qd * 4);
+                    const unsigned balt = __ballot_sync(0xffffffffu, contender && twin && !suspk[ch][qd]);
+                    twins |= ((balt >> (gs * 4)) & 0xFu) << (ch * 8 + qd * 4);
+                }
+        }
         if (Eb == -INFINITY) set = (p.n_clip >= 32) ? 0xFFFFFFFFu : ((1u << p.n_clip) - 1u);
         else if (set) set |= 1u << kb;
 
