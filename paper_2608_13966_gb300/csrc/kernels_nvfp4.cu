@@ -26,6 +26,12 @@ const void* amax_kernel(bool batch)
 
 const void* adamw_amax_kernel() { return reinterpret_cast<const void*>(&k_adamw_amax<kMaxBatch>); }
 
+const void* amax_init_kernel(bool batch)
+{
+    return batch ? reinterpret_cast<const void*>(&k_amax_init<kMaxBatch>)
+                 : reinterpret_cast<const void*>(&k_amax_init<1>);
+}
+
 const void* amax_to_scale_kernel(bool batch)
 {
     return batch ? reinterpret_cast<const void*>(&k_amax_to_scale<kMaxBatch>)

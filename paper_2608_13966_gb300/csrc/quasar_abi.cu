@@ -23,6 +23,7 @@ QUASAR_INT_ENTRY(4, 4) QUASAR_INT_ENTRY(4, 2) QUASAR_INT_ENTRY(4, 1)
 #undef QUASAR_INT_ENTRY
 const void* nvfp4_kernel(int nch, bool batch);
 const void* amax_kernel(bool batch);
+const void* amax_init_kernel(bool batch);
 const void* amax_to_scale_kernel(bool batch);
 const void* lut_kernel();
 const void* adamw_amax_kernel();
@@ -587,6 +588,18 @@ quasar_status nvfp4_params(bool has_g, quasar_dtype g_dtype, float beta2, const 
     return status_ptr(&p->status);
 }
 
+// The absmax slots of a batch set to 0 (those of the tensors whose amax is
+// computed, or all of them), in one launch.
+template <int MAXT>
+quasar_status zero_amax_slots(const AmaxBatch<MAXT>& B, bool all, cudaStream_t s)
+{
+    int flag = all ? 1 : 0;
+    void* args[] = {(void*)&B, (void*)&flag};
+    if (cudaLaunchKernel(amax_init_kernel(MAXT > 1), dim3(1), dim3(256), args, 0, s) != cudaSuccess)
+        return QUASAR_ERR_CUDA;
+    return QUASAR_OK;
+}
+
 // Absmax of the tensors whose amax is not supplied, into their scale slots
 // (zeroed first by the caller of each slot), then every slot := s_T.
 template <int MAXT>
@@ -619,10 +632,9 @@ quasar_status nvfp4_run(Nvfp4Launch<MAXT>& Lp, AmaxBatch<MAXT>& B, int n_clip, c
     quasar_status st;
     if (!amax_done) {
         // scale slots of tensors whose amax is computed start at 0
-        for (int i = 0; i < B.n_t; ++i)
-            if (!B.t[i].amax_in &&
-                cudaMemsetAsync(B.t[i].slot, 0, sizeof(float), s) != cudaSuccess)
-                return QUASAR_ERR_CUDA;
+        bool any = false;
+        for (int i = 0; i < B.n_t; ++i) any |= !B.t[i].amax_in;
+        if (any && (st = zero_amax_slots(B, false, s)) != QUASAR_OK) return st;
         if ((st = launch_amax(B, s)) != QUASAR_OK) return st;
     }
     {
@@ -1044,9 +1056,8 @@ quasar_status quasar_adamw_recon_nvfp4_batch(const quasar_adamw_nvfp4_tensor* te
         for (int i = 0; i < Lp.n_t; ++i) {
             describe(tensors[i0 + i], &Lp.t[i], &B.t[i], &Ad.t[i]);
             nmax = std::max(nmax, Ad.t[i].n);
-            if (cudaMemsetAsync(B.t[i].slot, 0, sizeof(float), s) != cudaSuccess)
-                return QUASAR_ERR_CUDA;
         }
+        if ((st = zero_amax_slots(B, true, s)) != QUASAR_OK) return st;
         if (nmax > 0) {
             const int64_t want = (nmax / 4 + kThreads - 1) / kThreads;
             const int64_t per = std::max<int64_t>(1, (int64_t)info->nsm * 8 / Ad.n_t);

@@ -473,6 +473,15 @@ __global__ void __launch_bounds__(256) k_amax(const __grid_constant__ AmaxBatch<
     }
 }
 
+// Zero the absmax slots of a batch before k_amax: those of the tensors whose
+// amax is computed, or every slot (all != 0), in one launch.
+template <int MAXT>
+__global__ void k_amax_init(const __grid_constant__ AmaxBatch<MAXT> B, int all)
+{
+    for (int i = threadIdx.x; i < B.n_t; i += blockDim.x)
+        if (all || !B.t[i].amax_in) *B.t[i].slot = 0.0f;
+}
+
 // *slot := s_T of the supplied amax, or of the amax the slot holds.
 template <int MAXT>
 __global__ void k_amax_to_scale(const __grid_constant__ AmaxBatch<MAXT> B)
