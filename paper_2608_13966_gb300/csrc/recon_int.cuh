@@ -1271,17 +1271,20 @@ __global__ void __launch_bounds__(ADAM ? 192 : 256, 2)
         {
             const float uf = p.fit_ulps * 5.9604645e-8f;
             const float ea = uf * fabsf(a_sel) * kap_sel;
-            // (plus half an ulp of Bz: pass C may fold Bz's low part into it)
-            const float ec = uf * (fabsf(cref) + fabsf(mu) + sqrtf(see * inv_ss)) +
+            // (plus half an ulp of Bz: pass C may fold Bz's low part into it;
+            // the square root as x rsqrt(x), within 2 ulps: immaterial beside
+            // the margin in fit_ulps)
+            const float sv = fmaxf(see * inv_ss, 1e-37f);
+            const float ec = uf * (fabsf(cref) + fabsf(mu) + sv * rsqrtf(sv)) +
                              0.5f * 5.9604645e-8f * fabsf(Bz);
             // the weighted mean code (q = zeta + J + 1)
             const float qbar = (y0b - kGridMagic) + T1b * inv_ss + Jp1;
             const float b0 = fmaf(-a_sel, Jp1, Bz);  // offset at q = 0
             prec = fmaf(ea, fabsf(qbar) + 1.0f, ec) > 1e-7f + 1e-5f * fabsf(b0);
             prec |= ea > 1e-7f + 1e-5f * fabsf(a_sel);
-            for (int q = sl; q <= p.qmax; q += kIntLanes) {
-                const float rq = fmaf(a_sel, (float)q, b0);
-                const float est = fmaf(ea, fabsf((float)q - qbar) + 1.0f, ec);
+            for (float qf = (float)sl; qf <= qmaxf; qf += (float)kIntLanes) {
+                const float rq = fmaf(a_sel, qf, b0);
+                const float est = fmaf(ea, fabsf(qf - qbar) + 1.0f, ec);
                 if (est > 1e-7f + 1e-5f * fabsf(rq)) {
                     if (!p.r_bf16) {
                         prec = true;
