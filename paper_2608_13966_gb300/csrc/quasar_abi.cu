@@ -17,7 +17,7 @@
 namespace quasar {
 // integer-code kernels: one entry per (8-candidate chunks, clamp-set size)
 #define QUASAR_INT_ENTRY(n, s) const void* int_kernel_nch##n##_ss##s(int epl, bool batch, bool adam, bool var);
-QUASAR_INT_ENTRY(1, 4) QUASAR_INT_ENTRY(1, 2) QUASAR_INT_ENTRY(1, 1)
+QUASAR_INT_ENTRY(1, 4) QUASAR_INT_ENTRY(1, 3) QUASAR_INT_ENTRY(1, 2) QUASAR_INT_ENTRY(1, 1)
 QUASAR_INT_ENTRY(2, 4) QUASAR_INT_ENTRY(2, 2) QUASAR_INT_ENTRY(2, 1)
 QUASAR_INT_ENTRY(4, 4) QUASAR_INT_ENTRY(4, 2) QUASAR_INT_ENTRY(4, 1)
 #undef QUASAR_INT_ENTRY
@@ -156,9 +156,13 @@ void fill_clip(const float* clip, int n_clip, float* f, float* invf)
 // and of P.  The largest set size of 4, 2, 1 whose sets all qualify is taken
 // (a set of one always does), and no larger than max_size; every slot holds
 // its set's tau / qmax.  Also the centre factor of each 8-candidate chunk.
-void fill_caps(IntParams* p, int max_size)
+void fill_caps(IntParams* p, int max_size, bool allow3 = false)
 {
     const int J = p->qmax >> 1;
+    // the sets of a size: consecutive runs of `size` slots; 3: the runs 3, 3,
+    // 2 of every 8 slots (used with a single chunk only)
+    auto first_of = [](int size, int k) { return size == 3 ? 8 * (k / 8) + 3 * ((k % 8) / 3) : k - k % size; };
+    auto len_of = [](int size, int k0) { return size == 3 ? (k0 % 8 == 6 ? 2 : 3) : size; };
     auto cap_of = [&](int k0, int n, double* tau) {
         double fmax = 0.0, fmin = 2.0;
         for (int k = k0; k < k0 + n; ++k) {
@@ -170,20 +174,22 @@ void fill_caps(IntParams* p, int max_size)
         return lo < hi;
     };
     int size = 1;
-    for (int cand = std::min(4, max_size); cand > 1; cand >>= 1) {
+    for (int cand : {4, 3, 2}) {
+        if (cand > max_size || (cand == 3 && !allow3)) continue;
         bool ok = true;
         double tau;
-        for (int k0 = 0; k0 < kMaxClip && ok; k0 += cand) ok = cap_of(k0, cand, &tau);
+        for (int k0 = 0; k0 < kMaxClip && ok; k0 += len_of(cand, k0)) ok = cap_of(k0, len_of(cand, k0), &tau);
         if (ok) {
             size = cand;
             break;
         }
     }
     p->set_size = size;
-    for (int k0 = 0; k0 < kMaxClip; k0 += size) {
+    for (int k = 0; k < kMaxClip; ++k) {
+        const int k0 = first_of(size, k);
         double tau = 0.0;
-        cap_of(k0, size, &tau);
-        for (int k = k0; k < k0 + size; ++k) p->cap[k] = (float)(tau / p->qmax);
+        cap_of(k0, len_of(size, k0), &tau);
+        p->cap[k] = (float)(tau / p->qmax);
     }
     for (int c = 0; c < kMaxClip / 8; ++c) {
         double lo = 1e300, hi = 0.0;
@@ -521,15 +527,17 @@ quasar_status int_launch(IntLaunch<MAXT>& Lp, int group_size, int n_clip, cudaSt
     // one); the option variants are built with sets of one, the fused AdamW
     // step with sets of four or one
     const int hoist_on = g_hoist.load() < 0 ? tuning().hoist : g_hoist.load();
-    fill_caps(&Lp.p, (!hoist_on || var) ? 1 : 4);
+    // (sets 3-3-2 with a single chunk, not for the fused AdamW step)
+    fill_caps(&Lp.p, (!hoist_on || var) ? 1 : 4, nch == 1 && !adam);
     if (adam && Lp.p.set_size == 2) fill_caps(&Lp.p, 1);
     using Entry = const void* (*)(int, bool, bool, bool);
-    static const Entry table[3][3] = {
-        {int_kernel_nch1_ss4, int_kernel_nch1_ss2, int_kernel_nch1_ss1},
-        {int_kernel_nch2_ss4, int_kernel_nch2_ss2, int_kernel_nch2_ss1},
-        {int_kernel_nch4_ss4, int_kernel_nch4_ss2, int_kernel_nch4_ss1}};
+    static const Entry table[3][4] = {
+        {int_kernel_nch1_ss4, int_kernel_nch1_ss3, int_kernel_nch1_ss2, int_kernel_nch1_ss1},
+        {int_kernel_nch2_ss4, nullptr, int_kernel_nch2_ss2, int_kernel_nch2_ss1},
+        {int_kernel_nch4_ss4, nullptr, int_kernel_nch4_ss2, int_kernel_nch4_ss1}};
     const int ci = nch == 1 ? 0 : (nch == 2 ? 1 : 2);
-    const int si = Lp.p.set_size == 4 ? 0 : (Lp.p.set_size == 2 ? 1 : 2);
+    const int si = Lp.p.set_size == 4 ? 0 : (Lp.p.set_size == 3 ? 1 : (Lp.p.set_size == 2 ? 2 : 3));
+    if (!table[ci][si]) return QUASAR_ERR_UNSUPPORTED;
     const void* fn = symmetric ? (MAXT > 1 ? sym_kernel(epl) : nullptr)
                                : table[ci][si](epl, batch, adam, var);
     if (!fn) return QUASAR_ERR_UNSUPPORTED;

@@ -411,18 +411,23 @@ __device__ __forceinline__ bool warp_wait_seq(const volatile int* seq, int t, ui
 // Two CTAs per SM: 8-warp CTAs, 6-warp ones for the AdamW-fused variant.
 // VAR: the variants of the options (a saliency other than v', packed codes);
 // without it they compile out of the common kernel.
-// SS: candidates per clamp set (4, 2 or 1): the host picks the largest size
-// whose sets all admit a cap (see the header comment); every size gives the
-// same codes.
+// SS: candidates per clamp set (4, 2 or 1; 3: the sets 0-2, 3-5 and 6-7 of a
+// single chunk): the host picks the largest size whose sets all admit a cap
+// (see the header comment); every size gives the same codes.
 template <int EPL, int NCH, int MAXT, bool ADAM, bool VAR, int SS>
 __global__ void __launch_bounds__(ADAM ? 192 : 256, 2)
     k_recon_int(const __grid_constant__ IntLaunch<MAXT> Lp)
 {
-    static_assert(SS == 1 || SS == 2 || SS == 4, "clamp sets of 1, 2 or 4 candidates");
+    static_assert(SS == 1 || SS == 2 || SS == 4 || (SS == 3 && NCH == 1),
+                  "clamp sets of 1, 2 or 4 candidates, or 3-3-2 in a single chunk");
     // candidates a sweep of pass B over the tile: all 8 of the chunk with
     // one chunk (the loads, offsets and loop shared by 8), a quad with more
     // (whose other live state leaves no room for 8 sets of sums)
     constexpr int QW = NCH == 1 ? 8 : 4;
+    // clamp sets a sweep, and the set of the sweep's candidate kk (its first
+    // slot is kq + set * SS)
+    constexpr int NSETS = SS == 3 ? 3 : QW / SS;
+    auto set_of = [](int kk) { return SS == 3 ? (kk < 3 ? 0 : (kk < 6 ? 1 : 2)) : kk / SS; };
     const IntParams& p = Lp.p;
     constexpr int G = EPL * kIntLanes;
     constexpr int UNIT = kIntGroups * G;
@@ -777,9 +782,9 @@ __global__ void __launch_bounds__(ADAM ? 192 : 256, 2)
                         const float P = R * p.invf[kq + kk];
                         P2[kk] = make_float2(P, P);
                     }
-                    float cp[QW / SS];
+                    float cp[NSETS];
 #pragma unroll
-                    for (int s = 0; s < QW / SS; ++s) cp[s] = p.cap[kq + s * SS] * range;
+                    for (int s = 0; s < NSETS; ++s) cp[s] = p.cap[kq + s * SS] * range;
 // rolled: a compact unit loop keeps the careful paths' code from evicting it
 // from the instruction cache when they run
 #pragma unroll 1
@@ -798,14 +803,14 @@ __global__ void __launch_bounds__(ADAM ? 192 : 256, 2)
                                 SE = __fadd2_rn(SE, he);
                                 SEE = __ffma2_rn(he, ev, SEE);
                             }
-                            float2 dc[QW / SS];
+                            float2 dc[NSETS];
 #pragma unroll
-                            for (int s = 0; s < QW / SS; ++s)
+                            for (int s = 0; s < NSETS; ++s)
                                 dc[s] = make_float2(fminf(fmaxf(d.x, -cp[s]), cp[s]),
                                                     fminf(fmaxf(d.y, -cp[s]), cp[s]));
 #pragma unroll
                             for (int kk = 0; kk < QW; ++kk) {
-                                const float2 y = __ffma2_rd(dc[kk / SS], P2[kk], Mg2);
+                                const float2 y = __ffma2_rd(dc[set_of(kk)], P2[kk], Mg2);
                                 const float2 zc = __fadd2_rn(y, nY02);  // zeta - zeta0, exact
                                 const float2 t2 = __fmul2_rn(h, zc);
                                 A1[kk] = __ffma2_rn(h, zc, A1[kk]);

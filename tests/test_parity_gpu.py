@@ -201,14 +201,21 @@ def _set_size(bits, clip):
     restated to know which kernel should run)."""
     f = [float(np.float32(clip[min(k, len(clip) - 1)])) for k in range(32)]
     J = ((1 << bits) - 1) >> 1
-    for size in (4, 2):
-        if all(J * max(f[s:s + size]) * 1.001 < (J + 1) * min(f[s:s + size]) * 0.999
-               for s in range(0, 32, size)):
-            return size
+    ok = lambda s, n: J * max(f[s:s + n]) * 1.001 < (J + 1) * min(f[s:s + n]) * 0.999
+    if all(ok(s, 4) for s in range(0, 32, 4)):
+        return 4
+    # runs of 3, 3 and 2 of every 8 slots, with a single chunk of candidates
+    if len(clip) <= 8 and all(ok(s + o, n) for s in range(0, 32, 8) for o, n in ((0, 3), (3, 3), (6, 2))):
+        return 3
+    if all(ok(s, 2) for s in range(0, 32, 2)):
+        return 2
     return 1
 
 
 NARROW8 = [1.0, 0.99, 0.98, 0.97, 0.96, 0.95, 0.94, 0.93]
+# 16 factors whose INT4 clamp sets hold 2 candidates (4 do not fit; 3-3-2 is
+# for a single chunk only)
+CLIP16_W = [round(1.0 - 0.03 * i, 4) for i in range(16)]
 
 
 def _edge_inputs(rows, cols, seed):
@@ -228,11 +235,11 @@ def _edge_inputs(rows, cols, seed):
 
 
 @pytest.mark.parametrize("bits,clip,size", [(1, CLIP8, 4), (2, CLIP8, 4), (3, CLIP8, 4),
-                                            (3, CLIP8[:5], 4), (4, NARROW8, 4), (4, CLIP8, 2),
-                                            (2, wl.CLIP_16, 4), (5, CLIP8, 1)])
+                                            (3, CLIP8[:5], 4), (4, NARROW8, 4), (4, CLIP8, 3),
+                                            (4, CLIP16_W, 2), (2, wl.CLIP_16, 4), (5, CLIP8, 1)])
 @pytest.mark.parametrize("G", [32, 64, 128, 256])
 def test_int_hoisted_clamp_equals_per_candidate_clamp(bits, clip, size, G):
-    """The batch kernel that clamps |w - c| once per set of 4 (or 2)
+    """The batch kernel that clamps |w - c| once per set of 4 (or 3, or 2)
     candidates gives bit for bit the outputs of the kernel that clamps every
     candidate on its own (itself checked against the oracle above), on ragged
     shapes with degenerate groups."""
