@@ -594,7 +594,7 @@ CONFIGS = (("config1_single_int4", "single_int4"), ("config2_llama_layer_int3", 
            ("config3_qwen_layer_int2", "qwen_layer_int2"), ("config4_llama_layer_nvfp4", "llama_layer_nvfp4"))
 
 
-def config_entries(device, stream, hbm_peak, reps=20):
+def config_entries(device, stream, hbm_peak, reps=20, warm=10):
     out = {}
     flush = torch.empty(256 << 20, dtype=torch.uint8, device=device)  # twice the L2
     for key, name in CONFIGS:
@@ -604,7 +604,7 @@ def config_entries(device, stream, hbm_peak, reps=20):
         small = model.elements * 10 < (1 << 28)
         times = []
         with torch.cuda.stream(stream):
-            for i in range(3 + reps):
+            for i in range(warm + reps):
                 if small:
                     flush.zero_()
                 e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
@@ -612,7 +612,7 @@ def config_entries(device, stream, hbm_peak, reps=20):
                 st.run()
                 e1.record()
                 torch.cuda.synchronize()
-                if i >= 3:
+                if i >= warm:
                     times.append(e0.elapsed_time(e1))
         status = Q.quasar_get_device_status(None)
         if status != Q.QuasarStatus.OK:

@@ -24,6 +24,7 @@ NVCC_FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-I" + IN
 UNITS = [
     ("quasar_abi.cu", [], "quasar_abi.o"),
     ("kernels_int.cu", ["-DQUASAR_NCH=1", "-DQUASAR_SS=4"], "kernels_int_nch1_ss4.o"),
+    ("kernels_int.cu", ["-DQUASAR_NCH=1", "-DQUASAR_SS=8"], "kernels_int_nch1_ss8.o"),
     ("kernels_int.cu", ["-DQUASAR_NCH=1", "-DQUASAR_SS=3"], "kernels_int_nch1_ss3.o"),
     ("kernels_int.cu", ["-DQUASAR_NCH=1", "-DQUASAR_SS=2"], "kernels_int_nch1_ss2.o"),
     ("kernels_int.cu", ["-DQUASAR_NCH=1", "-DQUASAR_SS=1"], "kernels_int_nch1_ss1.o"),

@@ -1,7 +1,7 @@
 // Instantiations of the integer-code kernel for one candidate-chunk count
 // (QUASAR_NCH = 1, 2 or 4 chunks of 8 candidates) and one clamp-set size
-// (QUASAR_SS = 4, 2 or 1 candidates, or 3 for the sets 3-3-2 of a single
-// chunk); compiled once per pair, in parallel.
+// (QUASAR_SS = 4, 2 or 1 candidates; with a single chunk also 8, or 3 for
+// the sets 3-3-2); compiled once per pair, in parallel.
 #include "recon_int.cuh"
 
 #if !defined(QUASAR_NCH) || !defined(QUASAR_SS)
@@ -23,7 +23,7 @@ const void* QUASAR_NAME(QUASAR_NCH, QUASAR_SS)(int epl, bool batch, bool adam, b
     constexpr int S = QUASAR_SS;
     constexpr int B = kMaxBatch;
     if ((adam || var) && !batch) return nullptr;
-    if (adam && (S == 2 || S == 3)) return nullptr;
+    if (adam && (S == 2 || S == 3 || S == 8)) return nullptr;
     if (var && S != 1) return nullptr;
     switch (epl) {
 #if QUASAR_SS == 1

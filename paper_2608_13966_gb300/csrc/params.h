@@ -73,8 +73,9 @@ struct IntParams {
     float invf[kMaxClip];  // fl32(1/f)
     // code clamps: every candidate slot holds tau / qmax of its clamp set,
     // so that the set's cap on |w - centre| is cap * range (sets of
-    // set_size consecutive slots, or with set_size 3 the runs of 3, 3 and 2
-    // slots of each 8; see the integer kernel)
+    // set_size consecutive slots (8 and 3 with a single chunk only), or with
+    // set_size 3 the runs of 3, 3 and 2 slots of each 8; see the integer
+    // kernel)
     float cap[kMaxClip];
     int set_size;
     // 1/f is non-decreasing in k over the real candidates (the factors come

@@ -17,7 +17,8 @@
 namespace quasar {
 // integer-code kernels: one entry per (8-candidate chunks, clamp-set size)
 #define QUASAR_INT_ENTRY(n, s) const void* int_kernel_nch##n##_ss##s(int epl, bool batch, bool adam, bool var);
-QUASAR_INT_ENTRY(1, 4) QUASAR_INT_ENTRY(1, 3) QUASAR_INT_ENTRY(1, 2) QUASAR_INT_ENTRY(1, 1)
+QUASAR_INT_ENTRY(1, 8) QUASAR_INT_ENTRY(1, 4) QUASAR_INT_ENTRY(1, 3) QUASAR_INT_ENTRY(1, 2)
+QUASAR_INT_ENTRY(1, 1)
 QUASAR_INT_ENTRY(2, 4) QUASAR_INT_ENTRY(2, 2) QUASAR_INT_ENTRY(2, 1)
 QUASAR_INT_ENTRY(4, 4) QUASAR_INT_ENTRY(4, 2) QUASAR_INT_ENTRY(4, 1)
 #undef QUASAR_INT_ENTRY
@@ -156,11 +157,11 @@ void fill_clip(const float* clip, int n_clip, float* f, float* invf)
 // and of P.  The largest set size of 4, 2, 1 whose sets all qualify is taken
 // (a set of one always does), and no larger than max_size; every slot holds
 // its set's tau / qmax.  Also the centre factor of each 8-candidate chunk.
-void fill_caps(IntParams* p, int max_size, bool allow3 = false)
+void fill_caps(IntParams* p, int max_size, bool single_chunk = false)
 {
     const int J = p->qmax >> 1;
     // the sets of a size: consecutive runs of `size` slots; 3: the runs 3, 3,
-    // 2 of every 8 slots (used with a single chunk only)
+    // 2 of every 8 slots (3 and 8: with a single chunk only)
     auto first_of = [](int size, int k) { return size == 3 ? 8 * (k / 8) + 3 * ((k % 8) / 3) : k - k % size; };
     auto len_of = [](int size, int k0) { return size == 3 ? (k0 % 8 == 6 ? 2 : 3) : size; };
     auto cap_of = [&](int k0, int n, double* tau) {
@@ -174,8 +175,8 @@ void fill_caps(IntParams* p, int max_size, bool allow3 = false)
         return lo < hi;
     };
     int size = 1;
-    for (int cand : {4, 3, 2}) {
-        if (cand > max_size || (cand == 3 && !allow3)) continue;
+    for (int cand : {8, 4, 3, 2}) {
+        if ((cand == 3 || cand == 8) ? (!single_chunk || max_size < 4) : cand > max_size) continue;
         bool ok = true;
         double tau;
         for (int k0 = 0; k0 < kMaxClip && ok; k0 += len_of(cand, k0)) ok = cap_of(k0, len_of(cand, k0), &tau);
@@ -527,16 +528,17 @@ quasar_status int_launch(IntLaunch<MAXT>& Lp, int group_size, int n_clip, cudaSt
     // one); the option variants are built with sets of one, the fused AdamW
     // step with sets of four or one
     const int hoist_on = g_hoist.load() < 0 ? tuning().hoist : g_hoist.load();
-    // (sets 3-3-2 with a single chunk, not for the fused AdamW step)
+    // (sets of 8 or 3-3-2 with a single chunk, not for the fused AdamW step)
     fill_caps(&Lp.p, (!hoist_on || var) ? 1 : 4, nch == 1 && !adam);
     if (adam && Lp.p.set_size == 2) fill_caps(&Lp.p, 1);
     using Entry = const void* (*)(int, bool, bool, bool);
-    static const Entry table[3][4] = {
-        {int_kernel_nch1_ss4, int_kernel_nch1_ss3, int_kernel_nch1_ss2, int_kernel_nch1_ss1},
-        {int_kernel_nch2_ss4, nullptr, int_kernel_nch2_ss2, int_kernel_nch2_ss1},
-        {int_kernel_nch4_ss4, nullptr, int_kernel_nch4_ss2, int_kernel_nch4_ss1}};
+    static const Entry table[3][5] = {
+        {int_kernel_nch1_ss8, int_kernel_nch1_ss4, int_kernel_nch1_ss3, int_kernel_nch1_ss2, int_kernel_nch1_ss1},
+        {nullptr, int_kernel_nch2_ss4, nullptr, int_kernel_nch2_ss2, int_kernel_nch2_ss1},
+        {nullptr, int_kernel_nch4_ss4, nullptr, int_kernel_nch4_ss2, int_kernel_nch4_ss1}};
     const int ci = nch == 1 ? 0 : (nch == 2 ? 1 : 2);
-    const int si = Lp.p.set_size == 4 ? 0 : (Lp.p.set_size == 3 ? 1 : (Lp.p.set_size == 2 ? 2 : 3));
+    const int ss = Lp.p.set_size;
+    const int si = ss == 8 ? 0 : (ss == 4 ? 1 : (ss == 3 ? 2 : (ss == 2 ? 3 : 4)));
     if (!table[ci][si]) return QUASAR_ERR_UNSUPPORTED;
     const void* fn = symmetric ? (MAXT > 1 ? sym_kernel(epl) : nullptr)
                                : table[ci][si](epl, batch, adam, var);

@@ -411,15 +411,15 @@ __device__ __forceinline__ bool warp_wait_seq(const volatile int* seq, int t, ui
 // Two CTAs per SM: 8-warp CTAs, 6-warp ones for the AdamW-fused variant.
 // VAR: the variants of the options (a saliency other than v', packed codes);
 // without it they compile out of the common kernel.
-// SS: candidates per clamp set (4, 2 or 1; 3: the sets 0-2, 3-5 and 6-7 of a
-// single chunk): the host picks the largest size whose sets all admit a cap
-// (see the header comment); every size gives the same codes.
+// SS: candidates per clamp set (4, 2 or 1; with a single chunk also 8, or 3:
+// the sets 0-2, 3-5 and 6-7): the host picks the largest size whose sets all
+// admit a cap (see the header comment); every size gives the same codes.
 template <int EPL, int NCH, int MAXT, bool ADAM, bool VAR, int SS>
 __global__ void __launch_bounds__(ADAM ? 192 : 256, 2)
     k_recon_int(const __grid_constant__ IntLaunch<MAXT> Lp)
 {
-    static_assert(SS == 1 || SS == 2 || SS == 4 || (SS == 3 && NCH == 1),
-                  "clamp sets of 1, 2 or 4 candidates, or 3-3-2 in a single chunk");
+    static_assert(SS == 1 || SS == 2 || SS == 4 || ((SS == 3 || SS == 8) && NCH == 1),
+                  "clamp sets of 1, 2 or 4 candidates, or of 8 or 3-3-2 in a single chunk");
     // candidates a sweep of pass B over the tile: all 8 of the chunk with
     // one chunk (the loads, offsets and loop shared by 8), a quad with more
     // (whose other live state leaves no room for 8 sets of sums)

@@ -202,6 +202,9 @@ def _set_size(bits, clip):
     f = [float(np.float32(clip[min(k, len(clip) - 1)])) for k in range(32)]
     J = ((1 << bits) - 1) >> 1
     ok = lambda s, n: J * max(f[s:s + n]) * 1.001 < (J + 1) * min(f[s:s + n]) * 0.999
+    # one set of 8 (every slot of each 8) with a single chunk of candidates
+    if len(clip) <= 8 and all(ok(s, 8) for s in range(0, 32, 8)):
+        return 8
     if all(ok(s, 4) for s in range(0, 32, 4)):
         return 4
     # runs of 3, 3 and 2 of every 8 slots, with a single chunk of candidates
@@ -234,12 +237,12 @@ def _edge_inputs(rows, cols, seed):
     return w, g, v
 
 
-@pytest.mark.parametrize("bits,clip,size", [(1, CLIP8, 4), (2, CLIP8, 4), (3, CLIP8, 4),
-                                            (3, CLIP8[:5], 4), (4, NARROW8, 4), (4, CLIP8, 3),
+@pytest.mark.parametrize("bits,clip,size", [(1, CLIP8, 8), (2, CLIP8, 8), (3, CLIP8, 4),
+                                            (3, CLIP8[:5], 8), (4, NARROW8, 8), (4, CLIP8, 3),
                                             (4, CLIP16_W, 2), (2, wl.CLIP_16, 4), (5, CLIP8, 1)])
 @pytest.mark.parametrize("G", [32, 64, 128, 256])
 def test_int_hoisted_clamp_equals_per_candidate_clamp(bits, clip, size, G):
-    """The batch kernel that clamps |w - c| once per set of 4 (or 3, or 2)
+    """The batch kernel that clamps |w - c| once per set of 8, 4, 3 or 2
     candidates gives bit for bit the outputs of the kernel that clamps every
     candidate on its own (itself checked against the oracle above), on ragged
     shapes with degenerate groups."""
