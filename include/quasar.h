@@ -447,11 +447,12 @@ void quasar_debug_force_timeout(int64_t nanoseconds);
 void quasar_debug_set_stats(unsigned int* device_counters);
 
 /*
- * quasar_debug_set_hoist -- tuning hook.  The integer entry points pick, for
- * a batch of at most 8 candidates whose factors allow it, a kernel that
- * clamps |w - c| once per set of 4 candidates instead of every candidate's
- * code (the codes are the same bit for bit).  While enable is 0 they always
- * take the per-candidate clamp; 1 (the default, or the environment variable
+ * quasar_debug_set_hoist -- tuning hook.  Where the clip factors allow it,
+ * the integer entry points pick a kernel that clamps |w - c| once per set of
+ * consecutive candidates instead of every candidate's code: sets of 4 or 2,
+ * and with at most 8 candidates also one set of 8 or the runs 3, 3 and 2
+ * (the codes are the same bit for bit).  While enable is 0 they always take
+ * the per-candidate clamp; 1 (the default, or the environment variable
  * QUASAR_HOIST at load) restores the automatic choice.  Process-wide; never
  * needed in normal use.
  */

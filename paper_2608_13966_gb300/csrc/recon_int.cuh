@@ -33,7 +33,8 @@
 // Per group (fp32):
 //   pass A  v' = beta2*v + (1-beta2)*g^2 (written back; kept in the tile as
 //           the saliency h), min/max -> range, sum h, sum h w -> mu;
-//   pass B  for 4 candidates at a time, the codes and the moments about a
+//   pass B  for the 8 candidates of a single chunk at once (4 at a time with
+//           more chunks), the codes and the moments about a
 //           centre zeta0 shared by the candidates of an 8-candidate chunk
 //           (the code of the weighted mean, from mu): S1 = sum h (zeta -
 //           zeta0), S2 = sum h (zeta - zeta0)^2, S3 = sum h (zeta - zeta0) e,
