@@ -387,80 +387,93 @@ __global__ void __launch_bounds__(256, 2) k_recon_lut(const __grid_constant__ Lu
 
         int kb = 0;
         if (!flat) {
-            // ---- candidates, two a pass: per-index sums of each (12 rows of
-            // the scratch a candidate), then entries and errors of both at
-            // once (lanes 0..7 the first, 8..15 the second)
+            // ---- candidates, four a pass: in two rounds of two, the
+            // per-index sums of each (12 rows of the scratch a candidate)
+            // summed across lanes, then entries and errors of all four at
+            // once (lanes 8 q .. 8 q + 7 candidate k0 + q)
 #pragma unroll 1
-            for (int k0 = 0; k0 < K; k0 += 2) {
-                const int nk = min(2, K - k0);
+            for (int k0 = 0; k0 < K; k0 += 4) {
+                float tot_a = 0.0f, tot_b = 0.0f;  // the two rounds' row sums
 #pragma unroll 1
-                for (int kk = 0; kk < nk; ++kk) {
-                    const float P = R * p.invf[k0 + kk];
-                    const float2 P2 = make_float2(P, P);
-                    // [l]: threshold m >= l + 1; sums of h (A) and h |d| (X),
-                    // by sign.  The masked saliency h [m >= t] is exact, and
-                    // so is its product with |d| inside the FMA: every term
-                    // is exact.
-                    float2 Ap[3], An[3], Xp[3], Xn[3];
+                for (int kr = k0; kr < min(k0 + 4, K); kr += 2) {
+                    const int nk = min(2, K - kr);
+#pragma unroll 1
+                    for (int kk = 0; kk < nk; ++kk) {
+                        const float P = R * p.invf[kr + kk];
+                        const float2 P2 = make_float2(P, P);
+                        // [l]: threshold m >= l + 1; sums of h (A) and h |d| (X),
+                        // by sign.  The masked saliency h [m >= t] is exact, and
+                        // so is its product with |d| inside the FMA: every term
+                        // is exact.
+                        float2 Ap[3], An[3], Xp[3], Xn[3];
 #pragma unroll
-                    for (int l = 0; l < 3; ++l) Ap[l] = An[l] = Xp[l] = Xn[l] = make_float2(0.0f, 0.0f);
+                        for (int l = 0; l < 3; ++l) Ap[l] = An[l] = Xp[l] = Xn[l] = make_float2(0.0f, 0.0f);
 #pragma unroll
-                    for (int t = 0; t < 8; ++t) {
-                        const float2 y = __ffma2_rd(ad2[t], P2, M2);  // 2^23 + floor(|d| P)
+                        for (int t = 0; t < 8; ++t) {
+                            const float2 y = __ffma2_rd(ad2[t], P2, M2);  // 2^23 + floor(|d| P)
+#pragma unroll
+                            for (int l = 0; l < 3; ++l) {
+                                const float nb = -(kMagic + (float)l);
+                                const float2 mk = make_float2(add_sat(y.x, nb), add_sat(y.y, nb));
+                                const float2 mp = __fmul2_rn(hp2[t], mk);
+                                const float2 mq = __fmul2_rn(hn2[t], mk);
+                                Ap[l] = __fadd2_rn(Ap[l], mp);
+                                An[l] = __fadd2_rn(An[l], mq);
+                                Xp[l] = __ffma2_rn(mp, ad2[t], Xp[l]);
+                                Xn[l] = __ffma2_rn(mq, ad2[t], Xn[l]);
+                            }
+                        }
+                        // rows (of this candidate's 12): A+ 0..2, A- 3..5, X+ 6..8,
+                        // X- 9..11
+                        float* rows = sums + kk * 12 * kLutRow + lane;
 #pragma unroll
                         for (int l = 0; l < 3; ++l) {
-                            const float nb = -(kMagic + (float)l);
-                            const float2 mk = make_float2(add_sat(y.x, nb), add_sat(y.y, nb));
-                            const float2 mp = __fmul2_rn(hp2[t], mk);
-                            const float2 mq = __fmul2_rn(hn2[t], mk);
-                            Ap[l] = __fadd2_rn(Ap[l], mp);
-                            An[l] = __fadd2_rn(An[l], mq);
-                            Xp[l] = __ffma2_rn(mp, ad2[t], Xp[l]);
-                            Xn[l] = __ffma2_rn(mq, ad2[t], Xn[l]);
+                            rows[l * kLutRow] = Ap[l].x + Ap[l].y;
+                            rows[(3 + l) * kLutRow] = An[l].x + An[l].y;
+                            rows[(6 + l) * kLutRow] = Xp[l].x + Xp[l].y;
+                            rows[(9 + l) * kLutRow] = Xn[l].x + Xn[l].y;
                         }
                     }
-                    // rows (of this candidate's 12): A+ 0..2, A- 3..5, X+ 6..8,
-                    // X- 9..11
-                    float* rows = sums + kk * 12 * kLutRow + lane;
+                    __syncwarp();
+                    // lane r < 12 nk sums row r
+                    if (lane < 12 * nk) {
+                        float a0 = 0.0f, a1 = 0.0f, a2 = 0.0f, a3 = 0.0f;
 #pragma unroll
-                    for (int l = 0; l < 3; ++l) {
-                        rows[l * kLutRow] = Ap[l].x + Ap[l].y;
-                        rows[(3 + l) * kLutRow] = An[l].x + An[l].y;
-                        rows[(6 + l) * kLutRow] = Xp[l].x + Xp[l].y;
-                        rows[(9 + l) * kLutRow] = Xn[l].x + Xn[l].y;
+                        for (int i = 0; i < 8; ++i) {
+                            const float4 v = *reinterpret_cast<const float4*>(sums + lane * kLutRow + 4 * i);
+                            a0 += v.x;
+                            a1 += v.y;
+                            a2 += v.z;
+                            a3 += v.w;
+                        }
+                        const float tot = (a0 + a1) + (a2 + a3);
+                        if (kr == k0) tot_a = tot;
+                        else tot_b = tot;
                     }
+                    __syncwarp();  // the scratch rows are rewritten by the next round
                 }
-                __syncwarp();
-                // lane r < 12 nk sums row r
-                float tot = 0.0f;
-                if (lane < 12 * nk) {
-                    float a0 = 0.0f, a1 = 0.0f, a2 = 0.0f, a3 = 0.0f;
-#pragma unroll
-                    for (int i = 0; i < 8; ++i) {
-                        const float4 v = *reinterpret_cast<const float4*>(sums + lane * kLutRow + 4 * i);
-                        a0 += v.x;
-                        a1 += v.y;
-                        a2 += v.z;
-                        a3 += v.w;
-                    }
-                    tot = (a0 + a1) + (a2 + a3);
-                }
-                __syncwarp();
-                // lane j < 8 of each half: index j, sign s (j >= 4: d >= 0),
-                // level m; its H = A_m - A_(m+1) and X = X_m - X_(m+1) (A_0,
-                // X_0: the sign's totals; A_4 = X_4 = 0)
-                const int half = (lane >> 3) & 1;
-                const int rb = half * 12;  // the candidate's first row
-                const float P = R * p.invf[min(k0 + half, K - 1)];
+                // lane j < 8 of each group q of 8: index j, sign s (j >= 4:
+                // d >= 0), level m; its H = A_m - A_(m+1) and X = X_m - X_(m+1)
+                // (A_0, X_0: the sign's totals; A_4 = X_4 = 0)
+                const int q4 = lane >> 3;   // candidate k0 + q4
+                const int half = q4 & 1;
+                const int rb = half * 12;  // the candidate's first row in its round
+                const float P = R * p.invf[min(k0 + q4, K - 1)];
                 const float sg = __fdividef(1.0f, P);
                 const int j = lane & 7;
                 const bool pos = j >= 4;
                 const int m = pos ? j - 4 : 3 - j;
                 const int r0 = rb + (pos ? 0 : 3);
-                const float sA0 = __shfl_sync(0xffffffffu, tot, r0 + max(m - 1, 0));
-                const float sA1 = __shfl_sync(0xffffffffu, tot, r0 + min(m, 2));
-                const float sX0 = __shfl_sync(0xffffffffu, tot, 6 + r0 + max(m - 1, 0));
-                const float sX1 = __shfl_sync(0xffffffffu, tot, 6 + r0 + min(m, 2));
+                // a row sum of this lane's round (q4 < 2: the first)
+                auto row = [&](int r) {
+                    const float va = __shfl_sync(0xffffffffu, tot_a, r);
+                    const float vb = __shfl_sync(0xffffffffu, tot_b, r);
+                    return q4 < 2 ? va : vb;
+                };
+                const float sA0 = row(r0 + max(m - 1, 0));
+                const float sA1 = row(r0 + min(m, 2));
+                const float sX0 = row(6 + r0 + max(m - 1, 0));
+                const float sX1 = row(6 + r0 + min(m, 2));
                 const float Am = m == 0 ? bconst[pos ? 0 : 1] : sA0;
                 const float Am1 = m == 3 ? 0.0f : sA1;
                 const float Xm = m == 0 ? bconst[pos ? 2 : 3] : sX0;
@@ -501,7 +514,7 @@ __global__ void __launch_bounds__(256, 2) k_recon_lut(const __grid_constant__ Lu
                     bj += H * fabsf(c2 - c1) * (fabsf(c1) + fabsf(c2) + 2.0f * dm);
                 }
                 bj = thin ? 2.0f * (dA + fabsf(H)) * bconst[6] * bconst[6] : bj;
-                const bool live = lane < 16;
+                const bool live = k0 + q4 < K;
                 float E = live ? Sj : 0.0f, dE = live ? bj : 0.0f, aE = live ? fabsf(Sj) : 0.0f;
                 uint32_t wb = live ? cb << (8 * (lane & 3)) : 0u;
 #pragma unroll
@@ -516,17 +529,17 @@ __global__ void __launch_bounds__(256, 2) k_recon_lut(const __grid_constant__ Lu
                 dE += (gam + 3.0f * kU) * sd + 4.0f * kU * (sd + aE);
 #pragma unroll
                 for (int o = 2; o; o >>= 1) wb |= __shfl_xor_sync(0xffffffffu, wb, o);
-                const uint32_t wb1 = __shfl_sync(0xffffffffu, wb, (lane & 8) | 4);
+                const uint32_t wb1 = __shfl_sync(0xffffffffu, wb, (lane & 24) | 4);
                 const uint32_t ambm = __ballot_sync(0xffffffffu, amb && live);
-                if (lane == 0 || (lane == 8 && nk == 2)) {
-                    const int k = k0 + half;
+                if ((lane & 7) == 0 && live) {
+                    const int k = k0 + q4;
                     cbook[2 * k] = wb;
                     cbook[2 * k + 1] = wb1;
                     cerr[k] = E;
                     cbnd[k] = dE;
-                    camb[k] = (ambm >> (8 * half)) & 0xFFu;
+                    camb[k] = (ambm >> (8 * q4)) & 0xFFu;
                 }
-                __syncwarp();  // the scratch rows are rewritten by the next pass
+                __syncwarp();
             }
             __syncwarp();
 
